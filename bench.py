@@ -1,0 +1,440 @@
+"""Benchmark of the hybrid packed-CKKS linear layer on GB300.
+
+One step = one evaluation of the whole layer (every signed sum, shared signed
+sum, scale PMult, raw PMult-MAC and the final reduction) through the C ABI
+(fiona_linear_eval), on synthetic residues already resident in HBM.
+
+  value        nonzero ciphertext terms per second (raw + signed terms with
+               t != 0) of the whole job, all ranks
+  roofline     minimal HBM bytes per launch (each used input, plaintext and
+               output limb moved once) / average kernel time, against the
+               measured copy bandwidth
+  e2e          the same metric through fiona_linear_eval_host: host inputs
+               (pinned) -> device -> kernel -> host outputs every step; the
+               plaintexts (the model's weights) stay resident on the device
+  cpu_baseline the CPU oracle on a bounded sample of the same layer, on every
+               host core (one spawn process per core)
+
+--impl reference times the CPU oracle as the reference arm.
+Multi-GPU (torchrun): every rank evaluates its own replica of the layer
+(independent queries, weak scaling, no data-path collective).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2609_35352_gb300 import workloads as W  # noqa: E402
+
+METRIC = "hybrid linear layer ciphertext-terms/s and HBM GB/s (% of GB300 peak), N=2^16"
+UNIT = "ciphertext-terms/s"
+DEFAULT_WORKLOAD = "wsum-hybrid"
+WORKLOAD_TEXT = {
+    "wsum-pmult": "64-ciphertext weighted sum -> 1 output, all PMult",
+    "wsum-ternary": "64-ciphertext weighted sum -> 1 output, all ternary (one scale PMult)",
+    "wsum-hybrid": "64-ciphertext weighted sum -> 1 output, 50/50 hybrid (32 raw, 32 signed)",
+    "vgg": "VGG11-style conv layer, 144 rotated inputs -> 16 outputs, 79% ternary",
+    "vit": "ViT-B-style BSGS projection, 32 -> 24, 65% ternary, 25% shared sums",
+    "bert": "BERT-base-style FFN column packing, 96 -> 96, 53% ternary, 30% shared sums",
+}
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ----------------------------------------------------------------------------
+# CPU oracle on a sample (spawned workers; never forked after CUDA init)
+# ----------------------------------------------------------------------------
+def _oracle_worker(task):
+    name, limb, coefs = task
+    import oracle
+    wl = W.make_workload(name)
+    p = wl.plan
+    k = np.asarray(coefs, dtype=np.uint64)
+    X = wl.input_values(np.arange(p.n_in).reshape(-1, 1, 1), np.arange(2).reshape(1, -1, 1),
+                        limb, k.reshape(1, 1, -1)).reshape(p.n_in, 2, 1, -1)
+    P = wl.plaintext_values(np.arange(p.n_pt).reshape(-1, 1), limb, k.reshape(1, -1))
+    P = P.reshape(p.n_pt, 1, -1)
+    t0 = time.perf_counter()
+    oracle.linear_eval(p, [wl.moduli[limb]], X, P)
+    return time.perf_counter() - t0, len(coefs)
+
+
+class OracleSampler:
+    """Runs the oracle over `positions` sampled (limb, coefficient) positions
+    per step, split over `cores` spawned processes."""
+
+    def __init__(self, name: str, cores: int, budget_s: float):
+        import oracle
+        oracle.build()
+        self.name = name
+        self.wl = W.make_workload(name)
+        self.cores = cores
+        self.pool = mp.get_context("spawn").Pool(cores)
+        # calibrate: one worker, a few positions
+        dt, n = self.pool.apply(_oracle_worker, ((name, 0, list(range(8))),))
+        per_pos = dt / n
+        total = int(budget_s * cores / per_pos)
+        full = self.wl.L * self.wl.N
+        self.positions = max(cores, min(total, full))
+        self.per_core = max(1, self.positions // cores)
+        self.positions = self.per_core * cores
+        self.step_no = 0
+
+    def tasks(self):
+        wl = self.wl
+        out = []
+        base = self.step_no * self.positions
+        for c in range(self.cores):
+            start = (base + c * self.per_core) % (wl.L * wl.N)
+            flat = (start + np.arange(self.per_core)) % (wl.L * wl.N)
+            limb = int(flat[0] // wl.N)
+            # keep each task inside one limb
+            coefs = [int(x % wl.N) for x in flat if int(x // wl.N) == limb]
+            out.append((self.name, limb, coefs))
+        self.step_no += 1
+        return out
+
+    def step(self):
+        res = self.pool.map(_oracle_worker, self.tasks())
+        wall = max(r[0] for r in res)
+        pos = sum(r[1] for r in res)
+        return wall, pos
+
+    def throughput(self, wall: float, pos: int) -> float:
+        frac = pos / (self.wl.L * self.wl.N)
+        return frac * self.wl.plan.counts()["nonzero"] / wall
+
+    def sample_text(self, pos: int) -> str:
+        return ("oracle on %d sampled (limb, coefficient) positions of %d per step "
+                "(all outputs, both polys), %d spawned processes; terms/s scaled by the "
+                "sampled fraction" % (pos, self.wl.L * self.wl.N, self.cores))
+
+    def close(self):
+        self.pool.terminate()
+        self.pool.join()
+
+
+# ----------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device: int):
+        self.device = device
+        self.proc = None
+        self.file = None
+
+    def start(self):
+        try:
+            self.file = tempfile.TemporaryFile(mode="w+")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.device), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"],
+                    "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.seek(0)
+        sm, smax, power = [], [], []
+        reasons = set()
+        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        for line in self.file.read().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for n, v in zip(names[1:], parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": max(power)}
+
+
+# ----------------------------------------------------------------------------
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_35352_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh", ".h", ".cpp")) and not f.startswith("workload"):
+            with open(os.path.join(csrc, f), "rb") as fh:
+                h.update(f.encode() + b"\0" + fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources; None otherwise."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+    except (OSError, ValueError):
+        return None
+    ent = d.get(workload)
+    if not ent or ent.get("kernel_src_sha") != kernel_source_hash():
+        return None
+    return ent.get("dram_bytes_per_launch")
+
+
+def workload_config(wl: W.Workload, name: str, stats: dict) -> dict:
+    return {
+        "workload": "%s (%s): N=2^%d, L=%d RNS limbs of %d-bit primes, %d inputs -> %d outputs"
+                    % (name, WORKLOAD_TEXT.get(name, name), wl.N.bit_length() - 1, wl.L,
+                       max(wl.moduli).bit_length(), wl.plan.n_in, wl.plan.n_out),
+        "N": wl.N, "L": wl.L, "n_in": wl.plan.n_in, "n_out": wl.plan.n_out,
+        "nonzero_terms": stats["n_nonzero_terms"], "raw_terms": stats["n_raw_terms"],
+        "signed_terms": stats["n_signed_terms"], "shared_sums": stats["n_nodes"],
+        "bytes_min_per_step": stats["bytes_min"],
+        "l2": "inputs larger than L2 (%.2f GB read per step, L2 129 MB)" % (stats["bytes_min"] / 1e9),
+    }
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def run_reference(args, rank: int, world: int) -> None:
+    if rank != 0:
+        return
+    cores = host_cores()
+    wl = W.make_workload(args.workload)
+    # sized so that warmup + steps stay within about two minutes
+    budget = max(0.5, min(5.0, 120.0 / max(1, args.steps + args.warmup)))
+    smp = OracleSampler(args.workload, cores, budget)
+    for _ in range(args.warmup):
+        smp.step()
+    walls, poss = [], []
+    for _ in range(args.steps):
+        w, p = smp.step()
+        walls.append(w)
+        poss.append(p)
+    smp.close()
+    wall = sum(walls)
+    frac = sum(poss) / (wl.L * wl.N)
+    value = frac * wl.plan.counts()["nonzero"] / wall
+    stats = {"n_nonzero_terms": wl.plan.counts()["nonzero"], "n_raw_terms": wl.plan.counts()["raw"],
+             "n_signed_terms": wl.plan.counts()["plus"] + wl.plan.counts()["minus"],
+             "n_nodes": wl.plan.n_nodes,
+             "bytes_min_per_step": None,
+             "bytes_min": 0}
+    cfg = workload_config(wl, args.workload, stats)
+    cfg.pop("l2")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * wall / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u64", "data": "synthetic", "config": cfg,
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": smp.sample_text(poss[0] if poss else 0)},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, rank: int, world: int, local_rank: int) -> None:
+    import torch
+
+    from paper_2609_35352_gb300 import build as B
+    from paper_2609_35352_gb300 import fiona as F
+
+    if rank == 0:
+        B.build()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.set_device(local_rank)
+    dev = local_rank
+    name = args.workload
+    wl = W.make_workload(name)
+    p = wl.plan
+
+    # CPU baseline first (rank 0, N = 1): spawned workers, before heavy GPU use
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cores = host_cores()
+        smp = OracleSampler(name, cores, args.cpu_budget)
+        w, pos = smp.step()
+        cpu = {"value": smp.throughput(w, pos), "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": smp.sample_text(pos)}
+        smp.close()
+
+    ctx = F.Context(wl.N, wl.moduli, device=dev)
+    plan = F.Plan(ctx, p)
+    stats = plan.stats()
+    n_in = 2 * p.n_in * wl.L * wl.N
+    n_pt = p.n_pt * wl.L * wl.N
+    n_out = 2 * p.n_out * wl.L * wl.N
+    d_in = torch.empty(max(n_in, 2), dtype=torch.int64, device="cuda")
+    d_pt = torch.empty(max(n_pt, 2), dtype=torch.int64, device="cuda")
+    d_out = torch.empty(max(n_out, 2), dtype=torch.int64, device="cuda")
+    stream = torch.cuda.Stream()
+    F.device_fill(d_in, 2 * p.n_in, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_INPUTS), 0, stream)
+    F.device_fill(d_pt, p.n_pt, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_PLAINTEXTS), 0, stream)
+    stream.synchronize()
+
+    for _ in range(args.warmup):
+        plan.eval(d_in, d_pt, d_out, stream=stream)
+    stream.synchronize()
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = ClockSampler(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_begin = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_begin.record(stream)
+    for s in range(args.steps):
+        starts[s].record(stream)
+        plan.eval(d_in, d_pt, d_out, stream=stream)
+        stops[s].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    elapsed_ms = t_begin.elapsed_time(t_end)
+    kernel_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    ms_per_step = elapsed_ms / args.steps
+    terms = stats["n_nonzero_terms"]
+    value = world * terms * args.steps / (elapsed_ms / 1e3)
+
+    avg_kernel_s = statistics.mean(kernel_ms) / 1e3
+    peak, peak_kind = measured_peak()
+    achieved = stats["bytes_min"] / avg_kernel_s / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": profiled_traffic(name),
+                "peak_kind": peak_kind,
+                "algorithmic_bytes_per_launch": stats["bytes_min"],
+                "kernel_ms_median": statistics.median(kernel_ms)}
+
+    # end to end: host inputs -> result on the host, plaintexts resident
+    e2e = None
+    if not args.no_e2e:
+        h_in = torch.empty(max(n_in, 2), dtype=torch.int64, pin_memory=True)
+        h_out = torch.empty(max(n_out, 2), dtype=torch.int64, pin_memory=True)
+        h_in.copy_(d_in.cpu())
+        e2e_steps = max(3, min(args.steps, args.e2e_steps))
+        for _ in range(2):
+            plan.eval_host(h_in, d_pt, h_out, d_in, d_out, stream=stream)
+        if world > 1:
+            torch.distributed.barrier()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            plan.eval_host(h_in, d_pt, h_out, d_in, d_out, stream=stream)
+        dt = time.perf_counter() - t0
+        if world > 1:
+            t = torch.tensor([dt], device="cuda")
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            dt = float(t.item())
+        e2e = {"value": world * terms * e2e_steps / dt, "unit": UNIT,
+               "h2d_bytes_per_step": n_in * 8, "d2h_bytes_per_step": n_out * 8,
+               "ms_per_step": 1e3 * dt / e2e_steps, "steps": e2e_steps}
+
+    if rank == 0:
+        cfg = workload_config(wl, name, stats)
+        cfg["parallelism"] = "replicas x%d (independent layer per GPU)" % world
+        cfg["kernel"] = "tiled" if stats["smem_bytes"] else "direct"
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
+            "data": "synthetic (seeded SplitMix64 residues, filled on the device)",
+            "config": cfg,
+            "hbm_gbs": achieved, "hbm_frac": achieved / peak,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "clocks": clk, "gpu_launches": args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    plan.close()
+    ctx.close()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(WORKLOAD_TEXT))
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--cpu-budget", type=float, default=2.0,
+                    help="seconds of oracle work per host core for cpu_baseline")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,217 @@
+/*
+ * fiona.h -- C ABI of the GB300 evaluator for hybrid packed-CKKS linear layers.
+ *
+ * The operation (Sec. 4.2 of "Fiona: Accelerating FHE Inference with
+ * Packing-Aware Ternary Weights", "Exact Compilation of Routed Linear
+ * Operators"): every packed output ciphertext y_j of a linear layer is a sum
+ * of signed terms and raw terms over input ciphertexts A_i that are already
+ * rotated into place (Sec. 2.3, "Packed Evaluation of a Linear Layer"):
+ *
+ *   y_j = sum_{scale groups g of j} gamma_g * ( sum_{t=+1} A_i - sum_{t=-1} A_i )
+ *       + sum_{raw terms e of j}    P_e * A_{i_e}
+ *
+ * evaluated in RNS, NTT (evaluation) form, where PMult is the element-wise
+ * product of residues in each limb and Add/Sub the element-wise modular
+ * sum/difference (Sec. 2.2, "Homomorphic Operations").  Terms with t = 0 are
+ * skipped (Sec. 4.1, "Packing-Aware Weight Representation").  Each scale
+ * group applies its reconstruction-factor plaintext gamma_g once to its signed
+ * sum ("Grouping Reconstruction Operations"); signed sums shared by several
+ * outputs are formed once and reused with sign +1 or -1 ("Sharing Signed
+ * Sums", Eq. "shared-example"); signed and raw products of an output are
+ * added before any rescale, so the output is left at scale
+ * Delta_ct * Delta_pt and is not rescaled ("Combining the Signed and Raw
+ * Routes").  All plaintexts of one layer must be encoded at the same scale
+ * and every input must be at the same level and slot arrangement.
+ *
+ * Memory layouts (row-major uint64 residues in [0, q_l); every buffer must
+ * start on a 16-byte boundary, FIONA_ERR_ARG otherwise):
+ *   inputs      [n_in ][2][L][N]   c0, c1 of each input ciphertext
+ *   plaintexts  [n_pt ][L][N]      raw-group and scale (gamma) plaintexts
+ *   outputs     [n_out][2][L][N]   overwritten, canonical residues in [0, q_l)
+ *
+ * Ownership: fiona_ctx and fiona_plan objects are created and freed by the
+ * library (the matching _destroy call).  Every data buffer is owned by the
+ * caller; the library neither frees nor retains it after a call returns.
+ *
+ * Errors: every function that can fail returns a fiona_status (0 = success,
+ * negative = failure) and leaves its out-arguments untouched on failure.
+ * fiona_last_error() returns a one-line description of the most recent
+ * failure in the calling thread.  No entry point synchronises the device,
+ * except where stated.
+ */
+#ifndef FIONA_H
+#define FIONA_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define FIONA_ABI_VERSION 1
+
+typedef struct fiona_ctx fiona_ctx;   /* N, RNS moduli, per-limb constants on one device */
+typedef struct fiona_plan fiona_plan; /* one validated, lowered linear layer */
+
+typedef enum fiona_status {
+    FIONA_OK = 0,
+    FIONA_ERR_ARG = -1,     /* null pointer, size out of range, misaligned buffer */
+    FIONA_ERR_MODULUS = -2, /* a modulus is not an odd prime < 2^60 with q = 1 mod 2N */
+    FIONA_ERR_PLAN = -3,    /* the layer description is malformed (see fiona_plan_create) */
+    FIONA_ERR_NOMEM = -4,   /* host or device allocation failed */
+    FIONA_ERR_CUDA = -5,    /* a CUDA runtime call failed (launch, copy, device) */
+    FIONA_ERR_RANGE = -6,   /* fiona_check_residues found a residue >= q_l */
+    FIONA_ERR_NODEVICE = -7 /* evaluation requested on a validation-only context */
+} fiona_status;
+
+/* Pass as `device` to fiona_ctx_create for a validation-only context: plans
+ * can be created, validated and inspected with fiona_plan_stats, nothing
+ * touches a GPU, and fiona_linear_eval returns FIONA_ERR_NODEVICE. */
+#define FIONA_DEVICE_NONE (-1)
+
+/* Route of one term (Sec. 4.1: a pure group takes the signed route, every
+ * other group the raw route). */
+enum { FIONA_TERM_RAW = 0, FIONA_TERM_TERNARY = 1 };
+
+/* One term = one execution group g_{j,i}: the weights of output j applied to
+ * input A_i through one plaintext operand (Sec. 2.3 "Packing Layout and
+ * Execution Groups"; Sec. 4.2 notation g_{j,i}).  16 bytes. */
+typedef struct fiona_term {
+    uint32_t input;   /* i, index of the input ciphertext, < n_in                     */
+    uint32_t pt;      /* RAW: index of the raw-group plaintext, < n_pt; TERNARY: 0     */
+    uint32_t group;   /* TERNARY: scale group, < n_groups, owned by this output; RAW: 0 */
+    int8_t kind;      /* FIONA_TERM_RAW or FIONA_TERM_TERNARY                          */
+    int8_t sign;      /* TERNARY: h_g in {-1, 0, +1}; RAW: 0                           */
+    uint16_t reserved;/* must be 0                                                      */
+} fiona_term;
+
+/* Child of a shared signed sum U_k: an input ciphertext or an earlier shared
+ * sum, with sign +1 or -1 (Sec. 4.2 "Sharing Signed Sums").  8 bytes. */
+typedef struct fiona_sum_child {
+    uint32_t ref;     /* input index (< n_in) or node index (< this node's index) */
+    int8_t is_node;   /* 0: ref is an input; 1: ref is a node                      */
+    int8_t sign;      /* +1 or -1                                                   */
+    uint16_t reserved;/* must be 0                                                  */
+} fiona_sum_child;
+
+/* Output `output` takes sign * U_node into the signed sum of its scale group
+ * `group`, in place of the signed terms U_node stands for (a sum can be
+ * reused with all signs reversed, Sec. 4.2).  16 bytes. */
+typedef struct fiona_sum_use {
+    uint32_t output;
+    uint32_t group;
+    uint32_t node;
+    int8_t sign;      /* +1 or -1 */
+    uint8_t reserved[3];
+} fiona_sum_use;
+
+/* Operation counts in the paper's units (Sec. 6 "Measurements" counts weight
+ * PMults, Add/Sub and rescales; Table "eval-linear-compilation") and sizes. */
+typedef struct fiona_plan_stats_t {
+    uint64_t n_terms;             /* all terms, t = 0 included                             */
+    uint64_t n_nonzero_terms;     /* raw + signed terms with t != 0 (the unit of terms/s)  */
+    uint64_t n_raw_terms;
+    uint64_t n_signed_terms;      /* TERNARY terms with t = +1 or -1                        */
+    uint64_t n_skipped_terms;     /* TERNARY terms with t = 0                               */
+    uint64_t n_scale_groups_used; /* scale groups with at least one signed term            */
+    uint64_t n_nodes;
+    uint64_t n_uses;
+    uint64_t pmult_per_term;      /* term by term: one PMult per raw or signed term        */
+    uint64_t pmult_grouped;       /* grouped: one PMult per raw term and per used group    */
+    uint64_t addsub_flat;         /* grouped, no sharing: n-1 Add/Sub to combine n operands */
+    uint64_t addsub_shared;       /* with each shared sum formed once                       */
+    uint64_t rescale_separate;    /* one rescale per route (signed, raw) per output         */
+    uint64_t rescale_combined;    /* one rescale per output with any nonzero term           */
+    uint64_t n_inputs_used;       /* inputs read by at least one nonzero term               */
+    uint64_t n_plaintexts_used;   /* distinct plaintexts read                               */
+    uint64_t bytes_min;           /* each used input, plaintext and each output moved once  */
+    uint64_t wide_products;       /* 64x64->128-bit products per evaluation                 */
+    uint32_t N;
+    uint32_t L;
+    uint32_t n_in, n_out, n_pt, n_groups;
+    uint32_t tile_coeffs;         /* coefficients per CTA tile chosen by the lowering       */
+    uint32_t warps_per_cta;
+    uint32_t smem_bytes;          /* dynamic shared memory per CTA                          */
+    uint32_t ctas_per_sm;         /* occupancy the lowering planned for                     */
+    uint32_t reserved[6];
+} fiona_plan_stats_t;
+
+/* Create a context for ring dimension N (a power of two, 2^10 <= N <= 2^17)
+ * and L RNS moduli (1 <= L <= 64) on CUDA device `device` (or
+ * FIONA_DEVICE_NONE).  Each modulus must be an odd prime below 2^60 with
+ * q = 1 (mod 2N) (an NTT-friendly CKKS prime, Sec. 2.2; the paper's setting
+ * is N = 2^16, Sec. 5 "Execution Environment"); the check is a deterministic
+ * Miller-Rabin test.  Moduli must be distinct.  The moduli are copied.
+ * Errors: FIONA_ERR_ARG, FIONA_ERR_MODULUS, FIONA_ERR_NOMEM, FIONA_ERR_CUDA. */
+int fiona_ctx_create(uint32_t N, const uint64_t *moduli, uint32_t L, int device,
+                     fiona_ctx **out);
+void fiona_ctx_destroy(fiona_ctx *ctx); /* NULL is a no-op; destroy plans first */
+
+/* Validate and lower one linear layer (Sec. 4.2).
+ *   terms[term_offsets[j] .. term_offsets[j+1]) are the terms of output j
+ *   (CSR, term_offsets has n_out+1 entries, term_offsets[0] = 0).  The term
+ *   list is the ground truth of what each output computes.
+ *   group_scale_pt[g] is the plaintext holding gamma_g; group_output[g] the
+ *   output that owns group g (a scale group belongs to one output).
+ *   Nodes k = 0..n_nodes-1 are shared signed sums with children
+ *   children[node_offsets[k] .. node_offsets[k+1]); a child node must have a
+ *   smaller index (children first), so the DAG is acyclic by construction.
+ *   uses[] say which signed terms are evaluated through a shared sum.
+ * FIONA_ERR_PLAN if: an index is out of range; a RAW term has sign != 0 or a
+ * TERNARY term a sign outside {-1,0,+1}; a reserved field is nonzero; a
+ * group's terms belong to another output than group_output[g]; a node has no
+ * child, a child sign not +/-1, a child node index >= its own, or expands to
+ * the same input twice; a use's node, expanded with its sign, is not matched
+ * by the output's TERNARY terms in that group with the same inputs and signs;
+ * two uses in one output cover the same term ("at most one of any two
+ * overlapping candidates", Sec. 4.2).  Arrays are copied; the caller may free
+ * them on return.  The plan keeps a pointer to ctx: destroy it first.
+ * The device schedule is uploaded with a synchronous copy. */
+int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out, uint32_t n_pt,
+                      const uint32_t *term_offsets, const fiona_term *terms,
+                      uint32_t n_groups, const uint32_t *group_scale_pt,
+                      const uint32_t *group_output,
+                      uint32_t n_nodes, const uint32_t *node_offsets,
+                      const fiona_sum_child *children,
+                      uint32_t n_uses, const fiona_sum_use *uses, fiona_plan **out);
+void fiona_plan_destroy(fiona_plan *plan); /* NULL is a no-op */
+
+int fiona_plan_stats(const fiona_plan *plan, fiona_plan_stats_t *out);
+
+/* Evaluate the layer on the GPU: enqueue the fused kernel on `cuda_stream`
+ * (a cudaStream_t; NULL = the legacy default stream) and return at once.
+ * `inputs`, `plaintexts`, `outputs` are device pointers of the ctx's device
+ * in the layouts above; outputs must not overlap the other two.  Residues
+ * must be < q_l (undefined results otherwise; fiona_check_residues checks).
+ * Errors: FIONA_ERR_ARG (null or misaligned pointer), FIONA_ERR_NODEVICE,
+ * FIONA_ERR_CUDA (launch failure, reported from cudaGetLastError). */
+int fiona_linear_eval(const fiona_plan *plan, void *cuda_stream, const uint64_t *inputs,
+                      const uint64_t *plaintexts, uint64_t *outputs);
+
+/* End-to-end evaluation from host memory: copies `h_inputs` (host, layout
+ * [n_in][2][L][N], pinned for overlap) to the caller's device buffer
+ * `d_inputs`, evaluates with the device-resident `d_plaintexts` (the model's
+ * weights stay on the GPU), and copies the result through `d_outputs` to
+ * `h_outputs` (host, [n_out][2][L][N]).  The work is split into limb chunks
+ * so the copies of one chunk overlap the kernel of another (RNS limbs are
+ * independent).  Synchronous: returns when h_outputs holds the result.
+ * Errors as fiona_linear_eval. */
+int fiona_linear_eval_host(const fiona_plan *plan, void *cuda_stream, const uint64_t *h_inputs,
+                           const uint64_t *d_plaintexts, uint64_t *h_outputs,
+                           uint64_t *d_inputs, uint64_t *d_outputs);
+
+/* Debug check of the precondition residue < q_l: scans `count` ciphertext
+ * polys or plaintexts ([count][L][N], pass n_in*2 for inputs) on the device
+ * and returns FIONA_OK, or FIONA_ERR_RANGE if any residue is >= q_l.
+ * Synchronous. */
+int fiona_check_residues(const fiona_ctx *ctx, void *cuda_stream, const uint64_t *data,
+                         uint64_t count);
+
+const char *fiona_status_str(int status);
+const char *fiona_last_error(void); /* thread-local; "" if none */
+int fiona_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FIONA_H */

@@ -1,0 +1,682 @@
+// fiona_host.cpp -- C ABI entry points: contexts, plan validation, operation
+// statistics, schedule upload and evaluation dispatch (host side).
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <new>
+
+#include "fiona_internal.h"
+
+typedef unsigned __int128 u128;
+
+// ---------------------------------------------------------------------------
+// errors
+// ---------------------------------------------------------------------------
+static thread_local char g_last_error[512];
+
+int set_error(int code, const char *fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+static int cuda_fail(cudaError_t e, const char *what)
+{
+    return set_error(FIONA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+extern "C" const char *fiona_last_error(void) { return g_last_error; }
+
+extern "C" int fiona_abi_version(void) { return FIONA_ABI_VERSION; }
+
+extern "C" const char *fiona_status_str(int status)
+{
+    switch (status) {
+    case FIONA_OK: return "ok";
+    case FIONA_ERR_ARG: return "invalid argument";
+    case FIONA_ERR_MODULUS: return "invalid RNS modulus";
+    case FIONA_ERR_PLAN: return "invalid plan";
+    case FIONA_ERR_NOMEM: return "out of memory";
+    case FIONA_ERR_CUDA: return "CUDA error";
+    case FIONA_ERR_RANGE: return "residue out of range";
+    case FIONA_ERR_NODEVICE: return "context has no device";
+    default: return "unknown status";
+    }
+}
+
+// Sets the context's device for the duration of a call and restores the
+// caller's device afterwards.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev)
+    {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard()
+    {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+// ---------------------------------------------------------------------------
+// moduli
+// ---------------------------------------------------------------------------
+static uint64_t mulmod_u64(uint64_t a, uint64_t b, uint64_t n) { return (uint64_t)((u128)a * b % n); }
+
+static uint64_t powmod_u64(uint64_t a, uint64_t e, uint64_t n)
+{
+    uint64_t r = 1 % n;
+    a %= n;
+    while (e) {
+        if (e & 1) r = mulmod_u64(r, a, n);
+        a = mulmod_u64(a, a, n);
+        e >>= 1;
+    }
+    return r;
+}
+
+// Deterministic Miller-Rabin; the first twelve primes as bases are exact for
+// every n < 3.3e24 (Sorenson and Webster, 2015), so for every 64-bit n.
+static bool is_prime_u64(uint64_t n)
+{
+    static const uint64_t bases[] = {2, 3, 5, 7, 11, 13, 17, 19, 23, 29, 31, 37};
+    if (n < 2) return false;
+    for (uint64_t p : bases)
+        if (n % p == 0) return n == p;
+    uint64_t d = n - 1;
+    int s = 0;
+    while ((d & 1) == 0) {
+        d >>= 1;
+        ++s;
+    }
+    for (uint64_t a : bases) {
+        uint64_t x = powmod_u64(a, d, n);
+        if (x == 1 || x == n - 1) continue;
+        bool composite = true;
+        for (int r = 1; r < s; ++r) {
+            x = mulmod_u64(x, x, n);
+            if (x == n - 1) {
+                composite = false;
+                break;
+            }
+        }
+        if (composite) return false;
+    }
+    return true;
+}
+
+static LimbConst limb_constants(uint64_t q)
+{
+    LimbConst c;
+    c.q = q;
+    const u128 mu = ~(u128)0 / q;  // floor((2^128 - 1) / q) = floor(2^128 / q) for odd q
+    c.mu_hi = (uint64_t)(mu >> 64);
+    c.mu_lo = (uint64_t)mu;
+    c.mu64 = ~(uint64_t)0 / q;     // floor(2^64 / q) for odd q
+    return c;
+}
+
+extern "C" int fiona_ctx_create(uint32_t N, const uint64_t *moduli, uint32_t L, int device,
+                                fiona_ctx **out)
+{
+    if (!out || !moduli) return set_error(FIONA_ERR_ARG, "ctx_create: null argument");
+    if (N < 1024 || N > 131072 || (N & (N - 1)))
+        return set_error(FIONA_ERR_ARG, "ctx_create: N=%u is not a power of two in [2^10, 2^17]", N);
+    if (L < 1 || L > FIONA_MAX_LIMBS)
+        return set_error(FIONA_ERR_ARG, "ctx_create: L=%u outside [1, %d]", L, FIONA_MAX_LIMBS);
+    for (uint32_t l = 0; l < L; ++l) {
+        const uint64_t q = moduli[l];
+        if (q >= (1ull << 60) || q < 3 || !(q & 1))
+            return set_error(FIONA_ERR_MODULUS, "modulus %u (%llu) is not odd and below 2^60", l,
+                             (unsigned long long)q);
+        if ((q - 1) % (2ull * N) != 0)
+            return set_error(FIONA_ERR_MODULUS, "modulus %u (%llu) is not 1 mod 2N", l,
+                             (unsigned long long)q);
+        if (!is_prime_u64(q))
+            return set_error(FIONA_ERR_MODULUS, "modulus %u (%llu) is not prime", l,
+                             (unsigned long long)q);
+        for (uint32_t m = 0; m < l; ++m)
+            if (moduli[m] == q)
+                return set_error(FIONA_ERR_MODULUS, "moduli %u and %u are equal", m, l);
+    }
+    fiona_ctx *ctx = new (std::nothrow) fiona_ctx;
+    if (!ctx) return set_error(FIONA_ERR_NOMEM, "ctx_create: host allocation");
+    ctx->N = N;
+    ctx->L = L;
+    ctx->device = device;
+    ctx->moduli.assign(moduli, moduli + L);
+    for (uint32_t l = 0; l < L; ++l) {
+        ctx->limbs.push_back(limb_constants(moduli[l]));
+        ctx->q_max = std::max(ctx->q_max, moduli[l]);
+    }
+    if (device != FIONA_DEVICE_NONE) {
+        int count = 0;
+        cudaError_t e = cudaGetDeviceCount(&count);
+        if (e != cudaSuccess || device < 0 || device >= count) {
+            delete ctx;
+            return set_error(FIONA_ERR_CUDA, "ctx_create: device %d unavailable (%s)", device,
+                             e == cudaSuccess ? "no such device" : cudaGetErrorString(e));
+        }
+        DeviceGuard g(device);
+        int smem = 0;
+        cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount, device);
+        cudaDeviceGetAttribute(&smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, device);
+        ctx->smem_optin = (size_t)smem;
+        e = cudaMalloc(&ctx->d_limbs, sizeof(LimbConst) * L);
+        if (e == cudaSuccess) e = cudaMalloc(&ctx->d_flag, sizeof(int));
+        if (e == cudaSuccess)
+            e = cudaMemcpy(ctx->d_limbs, ctx->limbs.data(), sizeof(LimbConst) * L,
+                           cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) {
+            cudaFree(ctx->d_limbs);
+            cudaFree(ctx->d_flag);
+            delete ctx;
+            return e == cudaErrorMemoryAllocation
+                       ? set_error(FIONA_ERR_NOMEM, "ctx_create: device allocation")
+                       : cuda_fail(e, "ctx_create");
+        }
+    }
+    *out = ctx;
+    return FIONA_OK;
+}
+
+extern "C" void fiona_ctx_destroy(fiona_ctx *ctx)
+{
+    if (!ctx) return;
+    if (ctx->device != FIONA_DEVICE_NONE) {
+        DeviceGuard g(ctx->device);
+        cudaFree(ctx->d_limbs);
+        cudaFree(ctx->d_flag);
+    }
+    delete ctx;
+}
+
+// ---------------------------------------------------------------------------
+// plan validation (the rules of Sec. 4.2 as stated in fiona.h)
+// ---------------------------------------------------------------------------
+static int validate(const fiona_ctx *ctx, HostPlan &hp)
+{
+    const uint32_t n_out = hp.n_out;
+    if (hp.term_offsets.size() != (size_t)n_out + 1 || hp.term_offsets[0] != 0)
+        return set_error(FIONA_ERR_PLAN, "term_offsets[0] must be 0");
+    for (uint32_t j = 0; j < n_out; ++j)
+        if (hp.term_offsets[j + 1] < hp.term_offsets[j])
+            return set_error(FIONA_ERR_PLAN, "term_offsets decrease at output %u", j);
+    for (uint32_t g = 0; g < hp.n_groups; ++g) {
+        if (hp.group_scale_pt[g] >= hp.n_pt)
+            return set_error(FIONA_ERR_PLAN, "group %u: scale plaintext %u >= n_pt", g,
+                             hp.group_scale_pt[g]);
+        if (hp.group_output[g] >= n_out)
+            return set_error(FIONA_ERR_PLAN, "group %u: output %u >= n_out", g, hp.group_output[g]);
+    }
+    for (uint32_t j = 0; j < n_out; ++j)
+        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
+            const fiona_term &t = hp.terms[e];
+            if (t.input >= hp.n_in)
+                return set_error(FIONA_ERR_PLAN, "term %u: input %u >= n_in", e, t.input);
+            if (t.reserved != 0) return set_error(FIONA_ERR_PLAN, "term %u: reserved != 0", e);
+            if (t.kind == FIONA_TERM_RAW) {
+                if (t.pt >= hp.n_pt)
+                    return set_error(FIONA_ERR_PLAN, "term %u: plaintext %u >= n_pt", e, t.pt);
+                if (t.sign != 0 || t.group != 0)
+                    return set_error(FIONA_ERR_PLAN, "term %u: raw term with sign or group", e);
+            } else if (t.kind == FIONA_TERM_TERNARY) {
+                if (t.sign < -1 || t.sign > 1)
+                    return set_error(FIONA_ERR_PLAN, "term %u: sign %d not in {-1,0,1}", e, t.sign);
+                if (t.group >= hp.n_groups)
+                    return set_error(FIONA_ERR_PLAN, "term %u: group %u >= n_groups", e, t.group);
+                if (hp.group_output[t.group] != j)
+                    return set_error(FIONA_ERR_PLAN, "term %u: group %u belongs to output %u, not %u",
+                                     e, t.group, hp.group_output[t.group], j);
+                if (t.pt != 0) return set_error(FIONA_ERR_PLAN, "term %u: ternary term with pt", e);
+            } else {
+                return set_error(FIONA_ERR_PLAN, "term %u: unknown kind %d", e, t.kind);
+            }
+        }
+    // shared signed sums: expand each node to its leaves (children first)
+    if (hp.node_offsets.size() != (size_t)hp.n_nodes + 1 || hp.node_offsets[0] != 0)
+        return set_error(FIONA_ERR_PLAN, "node_offsets[0] must be 0");
+    hp.node_leaves.assign(hp.n_nodes, {});
+    std::vector<int> acc(hp.n_in, 0);
+    for (uint32_t k = 0; k < hp.n_nodes; ++k) {
+        if (hp.node_offsets[k + 1] <= hp.node_offsets[k])
+            return set_error(FIONA_ERR_PLAN, "node %u has no child", k);
+        std::vector<uint32_t> touched;
+        for (uint32_t c = hp.node_offsets[k]; c < hp.node_offsets[k + 1]; ++c) {
+            const fiona_sum_child &ch = hp.children[c];
+            if (ch.reserved != 0 || (ch.sign != 1 && ch.sign != -1) ||
+                (ch.is_node != 0 && ch.is_node != 1))
+                return set_error(FIONA_ERR_PLAN, "node %u child %u: bad sign/flag", k, c);
+            if (ch.is_node) {
+                if (ch.ref >= k)
+                    return set_error(FIONA_ERR_PLAN, "node %u: child node %u not listed before it",
+                                     k, ch.ref);
+                for (auto &lv : hp.node_leaves[ch.ref]) {
+                    if (acc[lv.first] != 0)
+                        return set_error(FIONA_ERR_PLAN, "node %u: input %u appears twice", k,
+                                         lv.first);
+                    acc[lv.first] = lv.second * ch.sign;
+                    touched.push_back(lv.first);
+                }
+            } else {
+                if (ch.ref >= hp.n_in)
+                    return set_error(FIONA_ERR_PLAN, "node %u: input %u >= n_in", k, ch.ref);
+                if (acc[ch.ref] != 0)
+                    return set_error(FIONA_ERR_PLAN, "node %u: input %u appears twice", k, ch.ref);
+                acc[ch.ref] = ch.sign;
+                touched.push_back(ch.ref);
+            }
+        }
+        std::sort(touched.begin(), touched.end());
+        for (uint32_t i : touched) {
+            hp.node_leaves[k].push_back({i, acc[i]});
+            acc[i] = 0;
+        }
+    }
+    // uses: each must match uncovered signed terms of its output's group
+    hp.term_use.assign(hp.terms.size(), -1);
+    for (uint32_t u = 0; u < hp.n_uses; ++u) {
+        const fiona_sum_use &us = hp.uses[u];
+        if (us.output >= n_out || us.group >= hp.n_groups || us.node >= hp.n_nodes ||
+            (us.sign != 1 && us.sign != -1) || us.reserved[0] || us.reserved[1] || us.reserved[2])
+            return set_error(FIONA_ERR_PLAN, "use %u: index out of range or bad sign", u);
+        if (hp.group_output[us.group] != us.output)
+            return set_error(FIONA_ERR_PLAN, "use %u: group %u does not belong to output %u", u,
+                             us.group, us.output);
+        for (auto &lv : hp.node_leaves[us.node]) {
+            const int want = lv.second * us.sign;
+            bool found = false;
+            for (uint32_t e = hp.term_offsets[us.output]; e < hp.term_offsets[us.output + 1]; ++e) {
+                const fiona_term &t = hp.terms[e];
+                if (t.kind == FIONA_TERM_TERNARY && t.group == us.group && t.input == lv.first &&
+                    t.sign == want) {
+                    if (hp.term_use[e] >= 0) continue;
+                    hp.term_use[e] = (int32_t)u;
+                    found = true;
+                    break;
+                }
+            }
+            if (!found) {
+                // distinguish overlap from a plain mismatch for the message
+                for (uint32_t e = hp.term_offsets[us.output]; e < hp.term_offsets[us.output + 1];
+                     ++e) {
+                    const fiona_term &t = hp.terms[e];
+                    if (t.kind == FIONA_TERM_TERNARY && t.group == us.group &&
+                        t.input == lv.first && t.sign == want && hp.term_use[e] >= 0)
+                        return set_error(FIONA_ERR_PLAN,
+                                         "use %u overlaps use %d in output %u (input %u)", u,
+                                         hp.term_use[e], us.output, lv.first);
+                }
+                return set_error(FIONA_ERR_PLAN,
+                                 "use %u: output %u group %u has no term (input %u, sign %d)", u,
+                                 us.output, us.group, lv.first, want);
+            }
+        }
+    }
+    (void)ctx;
+    return FIONA_OK;
+}
+
+// ---------------------------------------------------------------------------
+// statistics in the paper's units
+// ---------------------------------------------------------------------------
+static void compute_stats(const fiona_ctx *ctx, const HostPlan &hp, fiona_plan_stats_t &s)
+{
+    memset(&s, 0, sizeof s);
+    s.N = ctx->N;
+    s.L = ctx->L;
+    s.n_in = hp.n_in;
+    s.n_out = hp.n_out;
+    s.n_pt = hp.n_pt;
+    s.n_groups = hp.n_groups;
+    s.n_nodes = hp.n_nodes;
+    s.n_uses = hp.n_uses;
+    std::vector<uint8_t> in_used(hp.n_in, 0), pt_used(hp.n_pt, 0), grp_used(hp.n_groups, 0);
+    for (uint32_t j = 0; j < hp.n_out; ++j) {
+        uint64_t S = 0, R = 0, ops_direct = 0;
+        std::map<uint32_t, uint64_t> uses_in_group;
+        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
+            const fiona_term &t = hp.terms[e];
+            ++s.n_terms;
+            if (t.kind == FIONA_TERM_RAW) {
+                ++R;
+                in_used[t.input] = 1;
+                pt_used[t.pt] = 1;
+            } else if (t.sign == 0) {
+                ++s.n_skipped_terms;
+            } else {
+                ++S;
+                in_used[t.input] = 1;
+                if (!grp_used[t.group]) {
+                    grp_used[t.group] = 1;
+                    pt_used[hp.group_scale_pt[t.group]] = 1;
+                }
+                if (hp.term_use[e] < 0) ++ops_direct;
+            }
+        }
+        for (uint32_t u = 0; u < hp.n_uses; ++u)
+            if (hp.uses[u].output == j) ++ops_direct;  // each use is one operand
+        s.n_raw_terms += R;
+        s.n_signed_terms += S;
+        if (S + R > 0) {
+            s.addsub_flat += S + R - 1;
+            s.addsub_shared += ops_direct + R - 1;
+            s.rescale_combined += 1;
+        }
+        s.rescale_separate += (S > 0) + (R > 0);
+    }
+    for (uint32_t k = 0; k < hp.n_nodes; ++k)
+        s.addsub_shared += hp.node_offsets[k + 1] - hp.node_offsets[k] - 1;
+    for (uint32_t g = 0; g < hp.n_groups; ++g) s.n_scale_groups_used += grp_used[g];
+    for (uint8_t v : in_used) s.n_inputs_used += v;
+    for (uint8_t v : pt_used) s.n_plaintexts_used += v;
+    s.n_nonzero_terms = s.n_raw_terms + s.n_signed_terms;
+    s.pmult_per_term = s.n_raw_terms + s.n_signed_terms;
+    s.pmult_grouped = s.n_raw_terms + s.n_scale_groups_used;
+    const uint64_t limb_poly = (uint64_t)ctx->N * ctx->L * 8;
+    s.bytes_min = limb_poly * (2 * s.n_inputs_used + s.n_plaintexts_used + 2ull * hp.n_out);
+    s.wide_products = 2ull * ctx->L * ctx->N * s.pmult_grouped;
+}
+
+// ---------------------------------------------------------------------------
+// direct schedule: per output, its used scale groups (signed operands) and
+// its raw terms, evaluated term by term without the DAG
+// ---------------------------------------------------------------------------
+static int upload(fiona_plan *p, const std::vector<std::pair<const void *, size_t>> &parts,
+                  std::vector<size_t> &offsets)
+{
+    size_t total = 0;
+    offsets.clear();
+    for (auto &pr : parts) {
+        offsets.push_back(total);
+        total += (pr.second + 255) & ~(size_t)255;
+    }
+    if (total == 0) total = 256;
+    std::vector<uint8_t> host(total, 0);
+    for (size_t i = 0; i < parts.size(); ++i)
+        if (parts[i].second) memcpy(host.data() + offsets[i], parts[i].first, parts[i].second);
+    cudaError_t e = cudaMalloc(&p->sched.blob, total);
+    if (e != cudaSuccess) return set_error(FIONA_ERR_NOMEM, "schedule upload: %s", cudaGetErrorString(e));
+    p->sched.bytes = total;
+    e = cudaMemcpy(p->sched.blob, host.data(), total, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "schedule upload");
+    return FIONA_OK;
+}
+
+static int lower_direct(fiona_plan *p)
+{
+    const HostPlan &hp = p->hp;
+    std::vector<DirOut> outs(hp.n_out);
+    std::vector<DirSeg> segs;
+    std::vector<uint32_t> ops, raw_in, raw_pt;
+    for (uint32_t j = 0; j < hp.n_out; ++j) {
+        DirOut &o = outs[j];
+        o.seg_begin = (uint32_t)segs.size();
+        std::vector<uint32_t> seen;
+        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
+            const fiona_term &t = hp.terms[e];
+            if (t.kind != FIONA_TERM_TERNARY || t.sign == 0) continue;
+            if (std::find(seen.begin(), seen.end(), t.group) != seen.end()) continue;
+            seen.push_back(t.group);
+            DirSeg sg{};
+            sg.scale_pt = hp.group_scale_pt[t.group];
+            sg.op_begin = (uint32_t)ops.size();
+            for (uint32_t f = e; f < hp.term_offsets[j + 1]; ++f) {
+                const fiona_term &u = hp.terms[f];
+                if (u.kind == FIONA_TERM_TERNARY && u.group == t.group && u.sign != 0)
+                    ops.push_back(u.input | (u.sign < 0 ? 0x80000000u : 0u));
+            }
+            sg.op_end = (uint32_t)ops.size();
+            segs.push_back(sg);
+        }
+        o.seg_end = (uint32_t)segs.size();
+        o.raw_begin = (uint32_t)raw_in.size();
+        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
+            const fiona_term &t = hp.terms[e];
+            if (t.kind != FIONA_TERM_RAW) continue;
+            raw_in.push_back(t.input);
+            raw_pt.push_back(t.pt);
+        }
+        o.raw_end = (uint32_t)raw_in.size();
+    }
+    std::vector<size_t> off;
+    int rc = upload(p, {{outs.data(), outs.size() * sizeof(DirOut)},
+                        {segs.data(), segs.size() * sizeof(DirSeg)},
+                        {ops.data(), ops.size() * 4},
+                        {raw_in.data(), raw_in.size() * 4},
+                        {raw_pt.data(), raw_pt.size() * 4}},
+                    off);
+    if (rc) return rc;
+    uint8_t *b = (uint8_t *)p->sched.blob;
+    p->d_dir_out = (const DirOut *)(b + off[0]);
+    p->d_dir_seg = (const DirSeg *)(b + off[1]);
+    p->d_sig_ops = (const uint32_t *)(b + off[2]);
+    p->d_raw_input = (const uint32_t *)(b + off[3]);
+    p->d_raw_pt = (const uint32_t *)(b + off[4]);
+    return FIONA_OK;
+}
+
+static void release_device(fiona_plan *p)
+{
+    if (!p->ctx || p->ctx->device == FIONA_DEVICE_NONE) return;
+    DeviceGuard g(p->ctx->device);
+    if (p->tiled) free_tiled(p);
+    cudaFree(p->sched.blob);
+    p->sched.blob = nullptr;
+    if (p->copy_in_stream) cudaStreamDestroy((cudaStream_t)p->copy_in_stream);
+    if (p->copy_out_stream) cudaStreamDestroy((cudaStream_t)p->copy_out_stream);
+    p->copy_in_stream = p->copy_out_stream = nullptr;
+}
+
+extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out,
+                                 uint32_t n_pt, const uint32_t *term_offsets,
+                                 const fiona_term *terms, uint32_t n_groups,
+                                 const uint32_t *group_scale_pt, const uint32_t *group_output,
+                                 uint32_t n_nodes, const uint32_t *node_offsets,
+                                 const fiona_sum_child *children, uint32_t n_uses,
+                                 const fiona_sum_use *uses, fiona_plan **out)
+{
+    if (!ctx || !out || !term_offsets) return set_error(FIONA_ERR_ARG, "plan_create: null argument");
+    if (n_in > 65535 || n_out > 65535 || n_pt >= (1u << 24) || n_groups >= (1u << 24) ||
+        n_nodes > 65535 || n_uses >= (1u << 24))
+        return set_error(FIONA_ERR_ARG, "plan_create: size limit exceeded");
+    if ((n_groups && (!group_scale_pt || !group_output)) || (n_uses && !uses) ||
+        (n_nodes && (!node_offsets || !children)))
+        return set_error(FIONA_ERR_ARG, "plan_create: null array with nonzero count");
+    const uint64_t n_terms = term_offsets[n_out];
+    if (n_terms && !terms) return set_error(FIONA_ERR_ARG, "plan_create: null terms");
+    if (n_terms >= (1u << 28)) return set_error(FIONA_ERR_ARG, "plan_create: too many terms");
+
+    fiona_plan *p = new (std::nothrow) fiona_plan;
+    if (!p) return set_error(FIONA_ERR_NOMEM, "plan_create: host allocation");
+    p->ctx = ctx;
+    HostPlan &hp = p->hp;
+    hp.n_in = n_in;
+    hp.n_out = n_out;
+    hp.n_pt = n_pt;
+    hp.n_groups = n_groups;
+    hp.n_nodes = n_nodes;
+    hp.n_uses = n_uses;
+    hp.term_offsets.assign(term_offsets, term_offsets + n_out + 1);
+    if (hp.term_offsets[0] != 0) {
+        delete p;
+        return set_error(FIONA_ERR_PLAN, "term_offsets[0] must be 0");
+    }
+    hp.terms.assign(terms, terms + n_terms);
+    if (n_groups) {
+        hp.group_scale_pt.assign(group_scale_pt, group_scale_pt + n_groups);
+        hp.group_output.assign(group_output, group_output + n_groups);
+    }
+    if (n_nodes) {
+        hp.node_offsets.assign(node_offsets, node_offsets + n_nodes + 1);
+        if (hp.node_offsets[0] != 0 || hp.node_offsets[n_nodes] > (1u << 24)) {
+            delete p;
+            return set_error(FIONA_ERR_PLAN, "node_offsets malformed");
+        }
+        hp.children.assign(children, children + hp.node_offsets[n_nodes]);
+    } else {
+        hp.node_offsets.assign(1, 0);
+    }
+    if (n_uses) hp.uses.assign(uses, uses + n_uses);
+
+    int rc = validate(ctx, hp);
+    if (rc) {
+        delete p;
+        return rc;
+    }
+    compute_stats(ctx, hp, p->stats);
+    // lazy-reduction budgets from the largest modulus
+    const u128 qm1 = ctx->q_max - 1;
+    const u128 mb = (~(u128)0) / (qm1 * qm1);
+    p->mac_budget = (uint32_t)std::min<u128>(mb, 1u << 30);
+    const uint64_t sb = ~(uint64_t)0 / (ctx->q_max - 1);
+    p->signed_budget = (uint32_t)std::min<uint64_t>(sb, 1u << 30);
+
+    if (ctx->device != FIONA_DEVICE_NONE) {
+        DeviceGuard g(ctx->device);
+        if (!g.ok) {
+            delete p;
+            return set_error(FIONA_ERR_CUDA, "plan_create: cannot select device %d", ctx->device);
+        }
+        rc = lower_direct(p);
+        if (rc == FIONA_OK) {
+            cudaError_t e = cudaStreamCreateWithFlags((cudaStream_t *)&p->copy_in_stream,
+                                                      cudaStreamNonBlocking);
+            if (e == cudaSuccess)
+                e = cudaStreamCreateWithFlags((cudaStream_t *)&p->copy_out_stream,
+                                              cudaStreamNonBlocking);
+            if (e != cudaSuccess) rc = cuda_fail(e, "plan_create: stream");
+        }
+        if (rc) {
+            release_device(p);
+            delete p;
+            return rc;
+        }
+    }
+    p->stats.tile_coeffs = 256;
+    p->stats.warps_per_cta = 4;
+    p->stats.smem_bytes = 0;
+    p->stats.ctas_per_sm = 0;
+    *out = p;
+    return FIONA_OK;
+}
+
+extern "C" void fiona_plan_destroy(fiona_plan *p)
+{
+    if (!p) return;
+    release_device(p);
+    delete p;
+}
+
+extern "C" int fiona_plan_stats(const fiona_plan *p, fiona_plan_stats_t *out)
+{
+    if (!p || !out) return set_error(FIONA_ERR_ARG, "plan_stats: null argument");
+    *out = p->stats;
+    return FIONA_OK;
+}
+
+// ---------------------------------------------------------------------------
+// evaluation
+// ---------------------------------------------------------------------------
+static int check_eval_args(const fiona_plan *p, const void *in, const void *pt, const void *out)
+{
+    if (!p) return set_error(FIONA_ERR_ARG, "linear_eval: null plan");
+    if (p->ctx->device == FIONA_DEVICE_NONE)
+        return set_error(FIONA_ERR_NODEVICE, "linear_eval: validation-only context");
+    if (!out) return set_error(FIONA_ERR_ARG, "linear_eval: null outputs");
+    if ((p->hp.n_in && !in) || (p->hp.n_pt && !pt))
+        return set_error(FIONA_ERR_ARG, "linear_eval: null inputs or plaintexts");
+    if (((uintptr_t)in | (uintptr_t)pt | (uintptr_t)out) & 15)
+        return set_error(FIONA_ERR_ARG, "linear_eval: buffers must be 16-byte aligned");
+    return FIONA_OK;
+}
+
+static int launch_range(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
+                        uint64_t *out, uint32_t l0, uint32_t l1)
+{
+    if (p->kernel == 1) return launch_tiled(p, stream, in, pt, out, l0, l1);
+    return launch_direct(p, stream, in, pt, out, l0, l1);
+}
+
+extern "C" int fiona_linear_eval(const fiona_plan *p, void *stream, const uint64_t *in,
+                                 const uint64_t *pt, uint64_t *out)
+{
+    int rc = check_eval_args(p, in, pt, out);
+    if (rc) return rc;
+    if (p->hp.n_out == 0) return FIONA_OK;
+    DeviceGuard g(p->ctx->device);
+    return launch_range(p, stream, in, pt, out, 0, p->ctx->L);
+}
+
+extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const uint64_t *h_in,
+                                      const uint64_t *d_pt, uint64_t *h_out, uint64_t *d_in,
+                                      uint64_t *d_out)
+{
+    int rc = check_eval_args(p, d_in, d_pt, d_out);
+    if (rc) return rc;
+    if ((p->hp.n_in && !h_in) || !h_out)
+        return set_error(FIONA_ERR_ARG, "linear_eval_host: null host buffer");
+    if (p->hp.n_out == 0) return FIONA_OK;
+    DeviceGuard g(p->ctx->device);
+    const uint32_t L = p->ctx->L, N = p->ctx->N;
+    const size_t pitch = (size_t)L * N * 8;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaStream_t sin = (cudaStream_t)p->copy_in_stream, sout = (cudaStream_t)p->copy_out_stream;
+    const uint32_t chunks = std::min<uint32_t>(L, 4);
+    cudaEvent_t ev[2 * 4 + 1];
+    int made = 0;
+    cudaError_t e = cudaSuccess;
+    for (int i = 0; i < 2 * (int)chunks + 1 && e == cudaSuccess; ++i, ++made)
+        e = cudaEventCreateWithFlags(&ev[i], cudaEventDisableTiming);
+    // the copy streams must not run ahead of work already queued on `stream`
+    if (e == cudaSuccess) e = cudaEventRecord(ev[2 * chunks], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(sin, ev[2 * chunks], 0);
+    for (uint32_t c = 0; c < chunks && e == cudaSuccess && rc == FIONA_OK; ++c) {
+        const uint32_t l0 = L * c / chunks, l1 = L * (c + 1) / chunks;
+        const size_t width = (size_t)(l1 - l0) * N * 8;
+        if (p->hp.n_in) {
+            e = cudaMemcpy2DAsync(d_in + (size_t)l0 * N, pitch, h_in + (size_t)l0 * N, pitch, width,
+                                  (size_t)p->hp.n_in * 2, cudaMemcpyHostToDevice, sin);
+            if (e != cudaSuccess) break;
+        }
+        if ((e = cudaEventRecord(ev[2 * c], sin)) != cudaSuccess) break;
+        if ((e = cudaStreamWaitEvent(s, ev[2 * c], 0)) != cudaSuccess) break;
+        rc = launch_range(p, s, d_in, d_pt, d_out, l0, l1);
+        if (rc) break;
+        if ((e = cudaEventRecord(ev[2 * c + 1], s)) != cudaSuccess) break;
+        if ((e = cudaStreamWaitEvent(sout, ev[2 * c + 1], 0)) != cudaSuccess) break;
+        e = cudaMemcpy2DAsync(h_out + (size_t)l0 * N, pitch, d_out + (size_t)l0 * N, pitch, width,
+                              (size_t)p->hp.n_out * 2, cudaMemcpyDeviceToHost, sout);
+    }
+    cudaError_t e2 = cudaStreamSynchronize(sout);
+    cudaError_t e3 = cudaStreamSynchronize(sin);
+    for (int i = 0; i < made; ++i) cudaEventDestroy(ev[i]);
+    if (rc) return rc;
+    if (e != cudaSuccess) return cuda_fail(e, "linear_eval_host");
+    if (e2 != cudaSuccess) return cuda_fail(e2, "linear_eval_host: sync");
+    if (e3 != cudaSuccess) return cuda_fail(e3, "linear_eval_host: sync");
+    return FIONA_OK;
+}
+
+extern "C" int fiona_check_residues(const fiona_ctx *ctx, void *stream, const uint64_t *data,
+                                    uint64_t count)
+{
+    if (!ctx) return set_error(FIONA_ERR_ARG, "check_residues: null ctx");
+    if (ctx->device == FIONA_DEVICE_NONE)
+        return set_error(FIONA_ERR_NODEVICE, "check_residues: validation-only context");
+    if (count == 0) return FIONA_OK;
+    if (!data || ((uintptr_t)data & 15))
+        return set_error(FIONA_ERR_ARG, "check_residues: null or misaligned data");
+    DeviceGuard g(ctx->device);
+    return launch_check_residues(ctx, stream, data, count);
+}

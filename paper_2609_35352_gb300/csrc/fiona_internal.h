@@ -1,0 +1,100 @@
+// fiona_internal.h -- structures shared by the host library code and the
+// CUDA kernels (not part of the public ABI).
+#pragma once
+#include <stddef.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/fiona.h"
+#include "rns.cuh"
+
+#define FIONA_MAX_LIMBS 64
+
+// ---------------------------------------------------------------------------
+// Direct schedule (one thread per coefficient pair and output): a flat list of
+// scale-group segments and raw terms per output.
+// ---------------------------------------------------------------------------
+struct DirOut {
+    uint32_t seg_begin, seg_end;  // into DirSeg[]
+    uint32_t raw_begin, raw_end;  // into raw_input[] / raw_pt[]
+};
+struct DirSeg {
+    uint32_t scale_pt;
+    uint32_t op_begin, op_end;    // into sig_ops[]: input | (sign < 0) << 31
+    uint32_t pad;
+};
+
+// ---------------------------------------------------------------------------
+// Tiled schedule (one CTA per limb x coefficient tile; inputs staged in shared
+// memory by TMA bulk copies; shared signed sums formed once per tile; each
+// warp owns a job list).  Defined in lower_tiled.cpp / kernel_tiled.cu.
+// ---------------------------------------------------------------------------
+struct TiledSchedule;
+
+struct DeviceSchedule {
+    void *blob = nullptr;  // one device allocation holding every array below
+    size_t bytes = 0;
+};
+
+struct fiona_ctx {
+    uint32_t N = 0, L = 0;
+    int device = FIONA_DEVICE_NONE;
+    std::vector<uint64_t> moduli;
+    std::vector<LimbConst> limbs;
+    uint64_t q_max = 0;
+    LimbConst *d_limbs = nullptr;   // device copy of limbs
+    int *d_flag = nullptr;          // scratch flag for fiona_check_residues
+    int sm_count = 0;
+    size_t smem_optin = 0;
+};
+
+struct HostPlan {
+    uint32_t n_in = 0, n_out = 0, n_pt = 0, n_groups = 0, n_nodes = 0, n_uses = 0;
+    std::vector<uint32_t> term_offsets;
+    std::vector<fiona_term> terms;
+    std::vector<uint32_t> group_scale_pt, group_output;
+    std::vector<uint32_t> node_offsets;
+    std::vector<fiona_sum_child> children;
+    std::vector<fiona_sum_use> uses;
+    // derived by validation
+    std::vector<std::vector<std::pair<uint32_t, int>>> node_leaves;  // (input, sign)
+    std::vector<int32_t> term_use;  // use index covering term e, or -1
+};
+
+struct fiona_plan {
+    const fiona_ctx *ctx = nullptr;
+    HostPlan hp;
+    fiona_plan_stats_t stats{};
+    uint32_t mac_budget = 0;     // products a 128-bit accumulator may take before a reduction
+    uint32_t signed_budget = 0;  // residues a 64-bit signed accumulator may take
+    int kernel = 0;              // 0 = direct, 1 = tiled
+    // direct schedule (device pointers into sched.blob)
+    DeviceSchedule sched;
+    const DirOut *d_dir_out = nullptr;
+    const DirSeg *d_dir_seg = nullptr;
+    const uint32_t *d_sig_ops = nullptr;
+    const uint32_t *d_raw_input = nullptr;
+    const uint32_t *d_raw_pt = nullptr;
+    // tiled schedule
+    TiledSchedule *tiled = nullptr;
+    // streams for fiona_linear_eval_host
+    void *copy_in_stream = nullptr;
+    void *copy_out_stream = nullptr;
+};
+
+// kernels.cu
+int launch_direct(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
+                  uint64_t *out, uint32_t limb_begin, uint32_t limb_end);
+int launch_check_residues(const fiona_ctx *ctx, void *stream, const uint64_t *data,
+                          uint64_t count);
+
+// lower_tiled.cpp / kernel_tiled.cu
+int lower_tiled(fiona_plan *p);
+void free_tiled(fiona_plan *p);
+int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
+                 uint64_t *out, uint32_t limb_begin, uint32_t limb_end);
+
+// fiona_host.cpp
+int set_error(int code, const char *fmt, ...);

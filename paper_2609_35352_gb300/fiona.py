@@ -1,0 +1,251 @@
+"""Thin ctypes binding of the C ABI in include/fiona.h (argument marshalling
+only: every step of the evaluation runs in libfiona.so's CUDA kernels).
+
+Buffers are passed as torch tensors (their ``data_ptr()``; int64 storage is
+read as uint64 residues) or as raw integer addresses.  The library must have
+been built (``paper_2609_35352_gb300.build.build()``); importing this module
+without it raises, there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Any, Dict, Optional
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libfiona.so")
+WORKLOAD_LIB_PATH = os.path.join(_HERE, "_build", "libfiona_workload.so")
+
+FIONA_OK = 0
+FIONA_ERR_ARG = -1
+FIONA_ERR_MODULUS = -2
+FIONA_ERR_PLAN = -3
+FIONA_ERR_NOMEM = -4
+FIONA_ERR_CUDA = -5
+FIONA_ERR_RANGE = -6
+FIONA_ERR_NODEVICE = -7
+FIONA_DEVICE_NONE = -1
+
+EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona_plan_destroy",
+            "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host",
+            "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version")
+
+
+class FionaError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        super().__init__("%s failed: %s (%d): %s" % (where, status_str(status), status, detail))
+        self.status = status
+
+
+class PlanStats(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_uint64) for n in (
+        "n_terms", "n_nonzero_terms", "n_raw_terms", "n_signed_terms", "n_skipped_terms",
+        "n_scale_groups_used", "n_nodes", "n_uses", "pmult_per_term", "pmult_grouped",
+        "addsub_flat", "addsub_shared", "rescale_separate", "rescale_combined",
+        "n_inputs_used", "n_plaintexts_used", "bytes_min", "wide_products")] + \
+        [(n, ctypes.c_uint32) for n in (
+            "N", "L", "n_in", "n_out", "n_pt", "n_groups", "tile_coeffs", "warps_per_cta",
+            "smem_bytes", "ctas_per_sm")] + [("reserved", ctypes.c_uint32 * 6)]
+
+    def as_dict(self) -> Dict[str, int]:
+        return {n: int(getattr(self, n)) for n, _ in self._fields_ if n != "reserved"}
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libfiona.so is not built (%s); run "
+                               "paper_2609_35352_gb300.build.build()" % LIB_PATH)
+        L = ctypes.CDLL(LIB_PATH)
+        p, u32, i32 = ctypes.c_void_p, ctypes.c_uint32, ctypes.c_int
+        L.fiona_ctx_create.argtypes = [u32, p, u32, i32, ctypes.POINTER(p)]
+        L.fiona_ctx_create.restype = i32
+        L.fiona_ctx_destroy.argtypes = [p]
+        L.fiona_ctx_destroy.restype = None
+        L.fiona_plan_create.argtypes = [p, u32, u32, u32, p, p, u32, p, p, u32, p, p, u32, p,
+                                        ctypes.POINTER(p)]
+        L.fiona_plan_create.restype = i32
+        L.fiona_plan_destroy.argtypes = [p]
+        L.fiona_plan_destroy.restype = None
+        L.fiona_plan_stats.argtypes = [p, ctypes.POINTER(PlanStats)]
+        L.fiona_plan_stats.restype = i32
+        L.fiona_linear_eval.argtypes = [p, p, p, p, p]
+        L.fiona_linear_eval.restype = i32
+        L.fiona_linear_eval_host.argtypes = [p, p, p, p, p, p, p]
+        L.fiona_linear_eval_host.restype = i32
+        L.fiona_check_residues.argtypes = [p, p, p, ctypes.c_uint64]
+        L.fiona_check_residues.restype = i32
+        L.fiona_status_str.argtypes = [i32]
+        L.fiona_status_str.restype = ctypes.c_char_p
+        L.fiona_last_error.argtypes = []
+        L.fiona_last_error.restype = ctypes.c_char_p
+        L.fiona_abi_version.argtypes = []
+        L.fiona_abi_version.restype = i32
+        _lib = L
+    return _lib
+
+
+def status_str(status: int) -> str:
+    return lib().fiona_status_str(status).decode()
+
+
+def last_error() -> str:
+    return lib().fiona_last_error().decode()
+
+
+def _check(status: int, where: str) -> None:
+    if status != FIONA_OK:
+        raise FionaError(status, where, last_error())
+
+
+def addr(x: Any) -> int:
+    """Device or host address of a torch tensor, numpy array or integer."""
+    if x is None:
+        return 0
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return int(x.data_ptr())
+    if isinstance(x, np.ndarray):
+        return int(x.ctypes.data)
+    raise TypeError("cannot take the address of %r" % type(x))
+
+
+def stream_handle(stream: Any) -> int:
+    if stream is None:
+        return 0
+    if isinstance(stream, int):
+        return stream
+    return int(stream.cuda_stream)
+
+
+class Context:
+    """fiona_ctx: ring dimension N and RNS moduli on one device."""
+
+    def __init__(self, N: int, moduli, device: int = 0):
+        q = np.ascontiguousarray(np.asarray(moduli, dtype=np.uint64))
+        self._q = q
+        h = ctypes.c_void_p()
+        _check(lib().fiona_ctx_create(N, q.ctypes.data, q.shape[0], device, ctypes.byref(h)),
+               "fiona_ctx_create")
+        self.handle = h
+        self.N, self.L, self.device = N, int(q.shape[0]), device
+
+    def check_residues(self, data, count: int, stream=None) -> int:
+        """FIONA_OK or FIONA_ERR_RANGE (raises on other errors)."""
+        rc = lib().fiona_check_residues(self.handle, stream_handle(stream), addr(data), count)
+        if rc not in (FIONA_OK, FIONA_ERR_RANGE):
+            _check(rc, "fiona_check_residues")
+        return rc
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            lib().fiona_ctx_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def _arr(a, dtype) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a), dtype=dtype)
+
+
+class Plan:
+    """fiona_plan: one validated, lowered layer.  ``desc`` provides n_in,
+    n_out, n_pt, term_offsets, terms, group_scale_pt, group_output,
+    node_offsets, children and uses (see workloads.Plan)."""
+
+    def __init__(self, ctx: Context, desc):
+        self.ctx = ctx
+        self._keep = []
+
+        def ptr(a):
+            self._keep.append(a)
+            return a.ctypes.data if a.size else None
+
+        offs = _arr(desc.term_offsets, np.uint32)
+        terms = np.ascontiguousarray(desc.terms)
+        gsp = _arr(desc.group_scale_pt, np.uint32)
+        gout = _arr(desc.group_output, np.uint32)
+        noffs = _arr(desc.node_offsets, np.uint32)
+        ch = np.ascontiguousarray(desc.children)
+        us = np.ascontiguousarray(desc.uses)
+        n_nodes = max(int(noffs.shape[0]) - 1, 0)
+        h = ctypes.c_void_p()
+        rc = lib().fiona_plan_create(ctx.handle, desc.n_in, desc.n_out, desc.n_pt, ptr(offs),
+                                     ptr(terms), int(gsp.shape[0]), ptr(gsp), ptr(gout),
+                                     n_nodes, ptr(noffs) if n_nodes else None, ptr(ch),
+                                     int(us.shape[0]), ptr(us), ctypes.byref(h))
+        self._keep = []
+        _check(rc, "fiona_plan_create")
+        self.handle = h
+        self.n_in, self.n_out, self.n_pt = desc.n_in, desc.n_out, desc.n_pt
+
+    def stats(self) -> Dict[str, int]:
+        s = PlanStats()
+        _check(lib().fiona_plan_stats(self.handle, ctypes.byref(s)), "fiona_plan_stats")
+        return s.as_dict()
+
+    def eval(self, inputs, plaintexts, outputs, stream=None) -> None:
+        """Enqueue fiona_linear_eval on `stream` (device buffers)."""
+        _check(lib().fiona_linear_eval(self.handle, stream_handle(stream), addr(inputs),
+                                       addr(plaintexts), addr(outputs)), "fiona_linear_eval")
+
+    def eval_status(self, inputs, plaintexts, outputs, stream=None) -> int:
+        return lib().fiona_linear_eval(self.handle, stream_handle(stream), addr(inputs),
+                                       addr(plaintexts), addr(outputs))
+
+    def eval_host(self, h_inputs, d_plaintexts, h_outputs, d_inputs, d_outputs,
+                  stream=None) -> None:
+        """fiona_linear_eval_host: host inputs -> host outputs (synchronous)."""
+        _check(lib().fiona_linear_eval_host(self.handle, stream_handle(stream), addr(h_inputs),
+                                            addr(d_plaintexts), addr(h_outputs), addr(d_inputs),
+                                            addr(d_outputs)), "fiona_linear_eval_host")
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            lib().fiona_plan_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+# -- device filler for synthetic inputs (libfiona_workload.so) ---------------
+_wlib: Optional[ctypes.CDLL] = None
+
+
+def workload_lib() -> ctypes.CDLL:
+    global _wlib
+    if _wlib is None:
+        if not os.path.exists(WORKLOAD_LIB_PATH):
+            raise RuntimeError("libfiona_workload.so is not built")
+        W = ctypes.CDLL(WORKLOAD_LIB_PATH)
+        W.fiona_workload_fill.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint64,
+                                          ctypes.c_uint32, ctypes.c_uint32, ctypes.c_void_p,
+                                          ctypes.c_uint64, ctypes.c_int]
+        W.fiona_workload_fill.restype = ctypes.c_int
+        _wlib = W
+    return _wlib
+
+
+def device_fill(dst, outer: int, L: int, N: int, moduli, key: int, mode: int = 0,
+                stream=None) -> None:
+    q = _arr(moduli, np.uint64)
+    rc = workload_lib().fiona_workload_fill(stream_handle(stream), addr(dst), outer, L, N,
+                                            q.ctypes.data, key, mode)
+    if rc != 0:
+        raise RuntimeError("fiona_workload_fill failed (%d)" % rc)

@@ -1,0 +1,167 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the CPU
+oracle on the same seeded inputs.  The bar is bit-exact equality of every
+residue (integer arithmetic mod q, a unique canonical result)."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+pytestmark = pytest.mark.gpu
+
+import oracle  # noqa: E402
+from paper_2609_35352_gb300 import build as B  # noqa: E402
+from paper_2609_35352_gb300 import fiona as F  # noqa: E402
+from paper_2609_35352_gb300 import workloads as W  # noqa: E402
+
+from gpu_util import DeviceLayer, oracle_at, to_device, to_host  # noqa: E402
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    B.build()
+
+
+# Reduced sizes: the same plan structure, N and L small enough for the oracle
+# to finish in seconds, still many coefficient tiles per limb.
+SMALL = [
+    ("tiny", None, None),
+    ("tiny-dag", None, None),
+    ("worked-example", None, None),
+    ("wsum-pmult", 1024, 3),
+    ("wsum-ternary", 1024, 3),
+    ("wsum-hybrid", 2048, 2),
+    ("vgg", 1024, 2),
+    ("vit", 2048, 2),
+    ("bert", 1024, 1),
+    ("overflow60", None, None),
+]
+
+
+@pytest.mark.parametrize("name,N,L", SMALL)
+def test_elementwise_parity_small(name, N, L):
+    wl = W.make_workload(name, N=N, L=L)
+    dl = DeviceLayer(wl)
+    dl.run()
+    got = dl.outputs()
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    mism = np.argwhere(got != want)
+    assert mism.shape[0] == 0, "first mismatches (j, c, l, k): %s" % mism[:5].tolist()
+    # a second launch on a dirty output buffer gives the same result
+    dl.run()
+    assert np.array_equal(dl.outputs(), want)
+
+
+def test_edge_plans():
+    R, T = W.TERM_RAW, W.TERM_TERNARY
+    qs = W.ntt_primes(1024, 50, 3)
+    plans = [
+        W.build_plan(0, 1, [[]], 0, [], [], [], []),                          # no terms
+        W.build_plan(2, 2, [[(0, T, 0, 0, 0), (1, T, 0, 0, 0)], [(1, R, 0, 0, 0)]], 2, [1], [0],
+                     [], []),                                                  # only t = 0
+        W.build_plan(1, 1, [[(0, R, 0, 0, 0), (0, R, 0, 0, 0), (0, T, 1, 0, 0)]], 2, [1], [0],
+                     [], []),                                                  # duplicate pair
+        W.build_plan(3, 3, [[(2, T, -1, 0, 0)], [(0, T, 1, 0, 1), (1, T, 1, 0, 1)], []], 3,
+                     [2, 2], [0, 1], [], []),                                  # ragged outputs
+    ]
+    for i, p in enumerate(plans):
+        wl = W.Workload("edge%d" % i, 1024, qs, p, 1000 + i)
+        dl = DeviceLayer(wl)
+        dl.run()
+        want = oracle.linear_eval(p, qs, dl.X if dl.X.size else np.zeros((0, 2, 3, 1024), np.uint64),
+                                  dl.P if dl.P.size else np.zeros((0, 3, 1024), np.uint64))
+        assert np.array_equal(dl.outputs(), want), i
+
+
+def test_boundary_residues():
+    """Residues 0, 1, q-1 and random, on 60-bit primes (widest accepted)."""
+    qs = W.ntt_primes(1024, 60, 2)
+    wl = W.make_workload("tiny", N=1024)
+    wl = W.Workload("tiny60", 1024, qs, wl.plan, wl.seed)
+    dl = DeviceLayer(wl)
+    X, P = dl.X.copy(), dl.P.copy()
+    q = wl.moduli_np.reshape(1, 1, -1, 1)
+    X[..., 0:8] = 0
+    X[..., 8:16] = 1
+    X[..., 16:64] = (q - 1)
+    P[..., 32:64] = q.reshape(1, -1, 1) - 1
+    P[..., 64:72] = 0
+    dl.d_in.copy_(to_device(X))
+    dl.d_pt.copy_(to_device(P))
+    dl.run()
+    assert np.array_equal(dl.outputs(), oracle.linear_eval(wl.plan, qs, X, P))
+
+
+FULL = ["wsum-pmult", "wsum-ternary", "wsum-hybrid", "vgg", "vit", "bert"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled_parity(name):
+    """Full N = 2^16 layer, inputs filled on the device; outputs compared with
+    the oracle at sampled (limb, coefficient) coordinates, every output."""
+    wl = W.make_workload(name)
+    dl = DeviceLayer(wl, host_inputs=False)
+    dl.run()
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(42)
+    n_s = 24 if name == "bert" else 64
+    limbs = rng.integers(0, wl.L, n_s)
+    coefs = rng.integers(0, wl.N, n_s)
+    coefs[:2] = [0, wl.N - 1]
+    want = oracle_at(wl, limbs, coefs)
+    out = dl.d_out.view(wl.plan.n_out, 2, wl.L, wl.N)
+    got = to_host(out[:, :, torch.from_numpy(limbs).cuda(), torch.from_numpy(coefs).cuda()].contiguous())
+    assert np.array_equal(got.reshape(want.shape), want)
+    # every residue canonical
+    assert dl.ctx.check_residues(dl.d_out, wl.plan.n_out * 2) == F.FIONA_OK
+
+
+def test_device_fill_matches_host_generator():
+    wl = W.make_workload("vit")
+    dl = DeviceLayer(wl, host_inputs=False)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(3)
+    for _ in range(4):
+        i, c, l = int(rng.integers(32)), int(rng.integers(2)), int(rng.integers(16))
+        k = rng.integers(0, wl.N, 50)
+        dev = to_host(dl.d_in.view(32, 2, 16, wl.N)[i, c, l].contiguous())[k]
+        assert np.array_equal(dev, wl.input_values(i, c, l, k))
+        p = int(rng.integers(wl.plan.n_pt))
+        devp = to_host(dl.d_pt.view(wl.plan.n_pt, 16, wl.N)[p, l].contiguous())[k]
+        assert np.array_equal(devp, wl.plaintext_values(p, l, k))
+
+
+def test_host_buffer_path_matches_device_path():
+    wl = W.make_workload("vit", N=4096, L=5)
+    dl = DeviceLayer(wl)
+    dl.run()
+    want = dl.outputs()
+    h_in = torch.from_numpy(dl.X.view(np.int64)).pin_memory()
+    h_out = torch.zeros(want.size, dtype=torch.int64).pin_memory()
+    d_in2 = torch.zeros_like(dl.d_in)
+    d_out2 = torch.zeros_like(dl.d_out)
+    dl.plan.eval_host(h_in, dl.d_pt, h_out, d_in2, d_out2)
+    assert np.array_equal(h_out.numpy().view(np.uint64).reshape(want.shape), want)
+
+
+def test_stream_and_alignment_errors():
+    wl = W.make_workload("tiny")
+    dl = DeviceLayer(wl)
+    s = torch.cuda.Stream()
+    dl.d_out.fill_(0)
+    dl.run(stream=s)
+    s.synchronize()
+    assert np.array_equal(dl.outputs(), oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P))
+    # misaligned pointers are refused before any launch
+    assert dl.plan.eval_status(dl.d_in.data_ptr() + 8, dl.d_pt, dl.d_out) == F.FIONA_ERR_ARG
+
+
+def test_check_residues_detects_out_of_range():
+    wl = W.make_workload("tiny")
+    dl = DeviceLayer(wl)
+    assert dl.ctx.check_residues(dl.d_in, 2 * wl.plan.n_in) == F.FIONA_OK
+    X = dl.X.copy()
+    X[3, 1, 2, 77] = wl.moduli[2]  # residue == q
+    dl.d_in.copy_(to_device(X))
+    assert dl.ctx.check_residues(dl.d_in, 2 * wl.plan.n_in) == F.FIONA_ERR_RANGE
