@@ -195,27 +195,31 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash() -> str:
+KERNEL_FILES = {"direct": ["kernel_direct.cu", "rns.cuh"],
+                "tiled": ["kernel_tiled.cu", "rns.cuh"]}
+
+
+def kernel_source_hash(kernel: str) -> str:
+    """Hash of the device code of one kernel variant."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_35352_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        if f.endswith((".cu", ".cuh", ".h", ".cpp")) and not f.startswith("workload"):
-            with open(os.path.join(csrc, f), "rb") as fh:
-                h.update(f.encode() + b"\0" + fh.read())
+    for f in KERNEL_FILES[kernel]:
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + b"\0" + fh.read())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str):
+def profiled_traffic(workload: str, kernel: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel sources; None otherwise."""
+    on the current sources of this kernel; None otherwise."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
             d = json.load(f)
     except (OSError, ValueError):
         return None
-    ent = d.get(workload)
-    if not ent or ent.get("kernel_src_sha") != kernel_source_hash():
+    ent = d.get("%s/%s" % (kernel, workload))
+    if not ent or ent.get("kernel_src_sha") != kernel_source_hash(kernel):
         return None
     return ent.get("dram_bytes_per_launch")
 
@@ -354,8 +358,10 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     avg_kernel_s = statistics.mean(kernel_ms) / 1e3
     peak, peak_kind = measured_peak()
     achieved = stats["bytes_min"] / avg_kernel_s / 1e9
+    kernel = "tiled" if stats["kernel"] == 2 else "direct"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": profiled_traffic(name),
+                "frac": achieved / peak, "traffic": profiled_traffic(name, kernel),
+                "kernel": kernel,
                 "peak_kind": peak_kind,
                 "algorithmic_bytes_per_launch": stats["bytes_min"],
                 "kernel_ms_median": statistics.median(kernel_ms)}
@@ -386,7 +392,10 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     if rank == 0:
         cfg = workload_config(wl, name, stats)
         cfg["parallelism"] = "replicas x%d (independent layer per GPU)" % world
-        cfg["kernel"] = "tiled" if stats["smem_bytes"] else "direct"
+        cfg["kernel"] = kernel
+        cfg["tile_coeffs"] = stats["tile_coeffs"]
+        cfg["warps_per_cta"] = stats["warps_per_cta"]
+        cfg["ctas_per_sm"] = stats["ctas_per_sm"]
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,

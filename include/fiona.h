@@ -61,8 +61,18 @@ typedef enum fiona_status {
     FIONA_ERR_NOMEM = -4,   /* host or device allocation failed */
     FIONA_ERR_CUDA = -5,    /* a CUDA runtime call failed (launch, copy, device) */
     FIONA_ERR_RANGE = -6,   /* fiona_check_residues found a residue >= q_l */
-    FIONA_ERR_NODEVICE = -7 /* evaluation requested on a validation-only context */
+    FIONA_ERR_NODEVICE = -7,/* evaluation requested on a validation-only context */
+    FIONA_ERR_TIMEOUT = -8  /* a kernel gave up waiting for its own copies (see fiona_device_check) */
 } fiona_status;
+
+/* Kernel variants (fiona_plan_select_kernel).  DIRECT: one thread per output
+ * and coefficient pair, inputs read through L2 for every output.  TILED: one
+ * CTA per limb and coefficient tile; the tile of every input is copied once
+ * into shared memory (bulk asynchronous copies), shared signed sums are
+ * formed once per tile, and the warps split the outputs.  AUTO (the default
+ * after fiona_plan_create): TILED for layers with more than one output whose
+ * tile fits in shared memory, DIRECT otherwise. */
+enum { FIONA_KERNEL_AUTO = 0, FIONA_KERNEL_DIRECT = 1, FIONA_KERNEL_TILED = 2 };
 
 /* Pass as `device` to fiona_ctx_create for a validation-only context: plans
  * can be created, validated and inspected with fiona_plan_stats, nothing
@@ -133,7 +143,8 @@ typedef struct fiona_plan_stats_t {
     uint32_t warps_per_cta;
     uint32_t smem_bytes;          /* dynamic shared memory per CTA                          */
     uint32_t ctas_per_sm;         /* occupancy the lowering planned for                     */
-    uint32_t reserved[6];
+    uint32_t kernel;              /* variant in use: FIONA_KERNEL_DIRECT or FIONA_KERNEL_TILED */
+    uint32_t reserved[5];
 } fiona_plan_stats_t;
 
 /* Create a context for ring dimension N (a power of two, 2^10 <= N <= 2^17)
@@ -178,6 +189,13 @@ void fiona_plan_destroy(fiona_plan *plan); /* NULL is a no-op */
 
 int fiona_plan_stats(const fiona_plan *plan, fiona_plan_stats_t *out);
 
+/* Choose the kernel variant used by later evaluations of `plan`
+ * (FIONA_KERNEL_AUTO, _DIRECT or _TILED).  Both compute the same residues.
+ * FIONA_ERR_ARG if the variant cannot run this plan (TILED needs the tile of
+ * every input and shared sum to fit in shared memory).  Not thread-safe
+ * against concurrent evaluations of the same plan. */
+int fiona_plan_select_kernel(fiona_plan *plan, int kernel);
+
 /* Evaluate the layer on the GPU: enqueue the fused kernel on `cuda_stream`
  * (a cudaStream_t; NULL = the legacy default stream) and return at once.
  * `inputs`, `plaintexts`, `outputs` are device pointers of the ctx's device
@@ -206,6 +224,13 @@ int fiona_linear_eval_host(const fiona_plan *plan, void *cuda_stream, const uint
  * Synchronous. */
 int fiona_check_residues(const fiona_ctx *ctx, void *cuda_stream, const uint64_t *data,
                          uint64_t count);
+
+/* Report kernel-side failures of earlier evaluations on this context:
+ * synchronises `cuda_stream`, then returns FIONA_ERR_TIMEOUT (and clears the
+ * flag) if a tiled kernel gave up waiting for its bulk copies (every such
+ * wait is bounded; the CTA then leaves its tile unwritten), FIONA_ERR_CUDA on
+ * a CUDA error, FIONA_OK otherwise. */
+int fiona_device_check(const fiona_ctx *ctx, void *cuda_stream);
 
 const char *fiona_status_str(int status);
 const char *fiona_last_error(void); /* thread-local; "" if none */

@@ -78,7 +78,7 @@ def linear_eval(plan, moduli, inputs: np.ndarray, plaintexts: np.ndarray,
     L = q.shape[0]
     inputs = _c(inputs, np.uint64)
     plaintexts = _c(plaintexts, np.uint64)
-    n = inputs.shape[-1] if inputs.size else (plaintexts.shape[-1] if plaintexts.size else 0)
+    n = inputs.shape[-1] if inputs.ndim == 4 else plaintexts.shape[-1]
     assert inputs.shape == (plan.n_in, 2, L, n), inputs.shape
     assert plaintexts.shape == (plan.n_pt, L, n), plaintexts.shape
     out = np.zeros((plan.n_out, 2, L, n), dtype=np.uint64)

@@ -10,6 +10,7 @@
 #include <new>
 
 #include "fiona_internal.h"
+#include "tiled.h"
 
 typedef unsigned __int128 u128;
 
@@ -47,6 +48,7 @@ extern "C" const char *fiona_status_str(int status)
     case FIONA_ERR_CUDA: return "CUDA error";
     case FIONA_ERR_RANGE: return "residue out of range";
     case FIONA_ERR_NODEVICE: return "context has no device";
+    case FIONA_ERR_TIMEOUT: return "kernel wait timed out";
     default: return "unknown status";
     }
 }
@@ -174,12 +176,15 @@ extern "C" int fiona_ctx_create(uint32_t N, const uint64_t *moduli, uint32_t L, 
         ctx->smem_optin = (size_t)smem;
         e = cudaMalloc(&ctx->d_limbs, sizeof(LimbConst) * L);
         if (e == cudaSuccess) e = cudaMalloc(&ctx->d_flag, sizeof(int));
+        if (e == cudaSuccess) e = cudaMalloc(&ctx->d_kerr, sizeof(int));
+        if (e == cudaSuccess) e = cudaMemset(ctx->d_kerr, 0, sizeof(int));
         if (e == cudaSuccess)
             e = cudaMemcpy(ctx->d_limbs, ctx->limbs.data(), sizeof(LimbConst) * L,
                            cudaMemcpyHostToDevice);
         if (e != cudaSuccess) {
             cudaFree(ctx->d_limbs);
             cudaFree(ctx->d_flag);
+            cudaFree(ctx->d_kerr);
             delete ctx;
             return e == cudaErrorMemoryAllocation
                        ? set_error(FIONA_ERR_NOMEM, "ctx_create: device allocation")
@@ -197,6 +202,7 @@ extern "C" void fiona_ctx_destroy(fiona_ctx *ctx)
         DeviceGuard g(ctx->device);
         cudaFree(ctx->d_limbs);
         cudaFree(ctx->d_flag);
+        cudaFree(ctx->d_kerr);
     }
     delete ctx;
 }
@@ -478,6 +484,62 @@ static void release_device(fiona_plan *p)
     p->copy_in_stream = p->copy_out_stream = nullptr;
 }
 
+// Kernel choice: TILED for layers with more than one output whose tile fits
+// in shared memory (every input is then read from HBM once), DIRECT otherwise
+// (a single output has no input reuse to exploit).
+static int select_kernel(fiona_plan *p, int which)
+{
+    int k;
+    if (which == FIONA_KERNEL_DIRECT)
+        k = 0;
+    else if (which == FIONA_KERNEL_TILED)
+        k = 1;
+    else if (which == FIONA_KERNEL_AUTO)
+        k = (p->tiled && p->hp.n_out > 1) ? 1 : 0;
+    else
+        return set_error(FIONA_ERR_ARG, "select_kernel: unknown variant %d", which);
+    if (k == 1 && !p->tiled && p->ctx->device != FIONA_DEVICE_NONE)
+        return set_error(FIONA_ERR_ARG, "select_kernel: the tiled kernel cannot run this plan");
+    p->kernel = k;
+    fiona_plan_stats_t &s = p->stats;
+    if (k == 1 && p->tiled) {
+        s.kernel = FIONA_KERNEL_TILED;
+        s.tile_coeffs = p->tiled->tile;
+        s.warps_per_cta = p->tiled->warps;
+        s.smem_bytes = (uint32_t)p->tiled->smem;
+        s.ctas_per_sm = p->tiled->ctas_per_sm;
+    } else {
+        s.kernel = FIONA_KERNEL_DIRECT;
+        s.tile_coeffs = 256;
+        s.warps_per_cta = 4;
+        s.smem_bytes = 0;
+        s.ctas_per_sm = 0;
+    }
+    return FIONA_OK;
+}
+
+extern "C" int fiona_plan_select_kernel(fiona_plan *p, int which)
+{
+    if (!p) return set_error(FIONA_ERR_ARG, "select_kernel: null plan");
+    return select_kernel(p, which);
+}
+
+extern "C" int fiona_device_check(const fiona_ctx *ctx, void *stream)
+{
+    if (!ctx) return set_error(FIONA_ERR_ARG, "device_check: null ctx");
+    if (ctx->device == FIONA_DEVICE_NONE)
+        return set_error(FIONA_ERR_NODEVICE, "device_check: validation-only context");
+    DeviceGuard g(ctx->device);
+    cudaStream_t s = (cudaStream_t)stream;
+    int flag = 0;
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess) e = cudaMemcpy(&flag, ctx->d_kerr, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && flag) e = cudaMemset(ctx->d_kerr, 0, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "device_check");
+    return flag ? set_error(FIONA_ERR_TIMEOUT, "a kernel gave up waiting for its bulk copies")
+                : FIONA_OK;
+}
+
 extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out,
                                  uint32_t n_pt, const uint32_t *term_offsets,
                                  const fiona_term *terms, uint32_t n_groups,
@@ -549,6 +611,12 @@ extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n
             return set_error(FIONA_ERR_CUDA, "plan_create: cannot select device %d", ctx->device);
         }
         rc = lower_direct(p);
+        if (rc == FIONA_OK && hp.n_out > 0) {
+            // the tiled schedule is optional: a plan whose tile does not fit
+            // in shared memory runs on the direct kernel
+            if (lower_tiled(p) != FIONA_OK) p->tiled = nullptr;
+            set_error(FIONA_OK, "");
+        }
         if (rc == FIONA_OK) {
             cudaError_t e = cudaStreamCreateWithFlags((cudaStream_t *)&p->copy_in_stream,
                                                       cudaStreamNonBlocking);
@@ -563,10 +631,7 @@ extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n
             return rc;
         }
     }
-    p->stats.tile_coeffs = 256;
-    p->stats.warps_per_cta = 4;
-    p->stats.smem_bytes = 0;
-    p->stats.ctas_per_sm = 0;
+    select_kernel(p, FIONA_KERNEL_AUTO);
     *out = p;
     return FIONA_OK;
 }

@@ -46,6 +46,7 @@ struct fiona_ctx {
     uint64_t q_max = 0;
     LimbConst *d_limbs = nullptr;   // device copy of limbs
     int *d_flag = nullptr;          // scratch flag for fiona_check_residues
+    int *d_kerr = nullptr;          // set by a kernel whose bounded wait gave up
     int sm_count = 0;
     size_t smem_optin = 0;
 };
@@ -69,7 +70,7 @@ struct fiona_plan {
     fiona_plan_stats_t stats{};
     uint32_t mac_budget = 0;     // products a 128-bit accumulator may take before a reduction
     uint32_t signed_budget = 0;  // residues a 64-bit signed accumulator may take
-    int kernel = 0;              // 0 = direct, 1 = tiled
+    int kernel = 0;              // 0 = direct, 1 = tiled (what evaluations use)
     // direct schedule (device pointers into sched.blob)
     DeviceSchedule sched;
     const DirOut *d_dir_out = nullptr;

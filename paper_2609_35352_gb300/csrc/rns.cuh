@@ -96,5 +96,63 @@ __device__ __forceinline__ uint64_t sub_mod(uint64_t a, uint64_t b, uint64_t q)
     return a >= b ? a - b : a + (q - b);
 }
 
+// ---------------------------------------------------------------------------
+// Narrow residues (q < 2^52): radix-2^26 split form.
+//
+// A residue a < 2^52 is kept as one 64-bit word whose low 32-bit half holds
+// a0 = a mod 2^26 and whose high half holds a1 = floor(a / 2^26).  Then
+//   a * b = a1*b1 * 2^52 + (a1*b0 + a0*b1) * 2^26 + a0*b0,
+// every partial product is below 2^52, and a product-accumulate is four
+// 32x32 -> 64-bit multiply-adds into three 64-bit accumulators (lo, mid, hi).
+// mid grows by less than 2^53 per product, so the three words hold at least
+// 2047 products before any of them can wrap.
+//
+// Split words can also be summed as plain 64-bit integers: 64 of them keep
+// each half below 2^32 (64 * (2^26 - 1) < 2^32), so a packed sum of at most
+// 64 split words still reads back as (sum of a0) + (sum of a1) * 2^26.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kNarrowMacBudget = 2047;
+constexpr uint32_t kNarrowSumBudget = 64;
+
+__device__ __forceinline__ uint64_t split26(uint64_t a)
+{
+    const uint32_t lo = (uint32_t)a & 0x3FFFFFFu;
+    const uint32_t hi = (uint32_t)(a >> 26);
+    return ((uint64_t)hi << 32) | lo;
+}
+
+// value of a packed sum of at most kNarrowSumBudget split words (< 2^59)
+__device__ __forceinline__ uint64_t unsplit_sum(uint64_t w)
+{
+    return (w & 0xFFFFFFFFull) + ((w >> 32) << 26);
+}
+
+__device__ __forceinline__ void mac26(uint64_t &lo, uint64_t &mid, uint64_t &hi, uint64_t as,
+                                      uint64_t bs)
+{
+    const uint32_t a0 = (uint32_t)as, a1 = (uint32_t)(as >> 32);
+    const uint32_t b0 = (uint32_t)bs, b1 = (uint32_t)(bs >> 32);
+    asm("mad.wide.u32 %0, %3, %4, %0;\n\t"
+        "mad.wide.u32 %1, %3, %6, %1;\n\t"
+        "mad.wide.u32 %1, %5, %4, %1;\n\t"
+        "mad.wide.u32 %2, %5, %6, %2;"
+        : "+l"(lo), "+l"(mid), "+l"(hi)
+        : "r"(a0), "r"(b0), "r"(a1), "r"(b1));
+}
+
+// lo + mid * 2^26 + hi * 2^52 mod q (the sum is below 2^117)
+__device__ __forceinline__ uint64_t reduce26(uint64_t lo, uint64_t mid, uint64_t hi,
+                                             const LimbConst &m)
+{
+    uint64_t x0 = lo, x1 = 0;
+    asm("add.cc.u64 %0, %0, %2;\n\t"
+        "addc.u64   %1, %1, %3;\n\t"
+        "add.cc.u64 %0, %0, %4;\n\t"
+        "addc.u64   %1, %1, %5;"
+        : "+l"(x0), "+l"(x1)
+        : "l"(mid << 26), "l"(mid >> 38), "l"(hi << 52), "l"(hi >> 12));
+    return reduce128(x0, x1, m);
+}
+
 }  // namespace rns
 #endif  // __CUDACC__

@@ -26,11 +26,17 @@ FIONA_ERR_NOMEM = -4
 FIONA_ERR_CUDA = -5
 FIONA_ERR_RANGE = -6
 FIONA_ERR_NODEVICE = -7
+FIONA_ERR_TIMEOUT = -8
 FIONA_DEVICE_NONE = -1
+FIONA_KERNEL_AUTO = 0
+FIONA_KERNEL_DIRECT = 1
+FIONA_KERNEL_TILED = 2
+KERNELS = {"auto": FIONA_KERNEL_AUTO, "direct": FIONA_KERNEL_DIRECT, "tiled": FIONA_KERNEL_TILED}
 
 EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona_plan_destroy",
             "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host",
-            "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version")
+            "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version",
+            "fiona_plan_select_kernel", "fiona_device_check")
 
 
 class FionaError(RuntimeError):
@@ -47,7 +53,7 @@ class PlanStats(ctypes.Structure):
         "n_inputs_used", "n_plaintexts_used", "bytes_min", "wide_products")] + \
         [(n, ctypes.c_uint32) for n in (
             "N", "L", "n_in", "n_out", "n_pt", "n_groups", "tile_coeffs", "warps_per_cta",
-            "smem_bytes", "ctas_per_sm")] + [("reserved", ctypes.c_uint32 * 6)]
+            "smem_bytes", "ctas_per_sm", "kernel")] + [("reserved", ctypes.c_uint32 * 5)]
 
     def as_dict(self) -> Dict[str, int]:
         return {n: int(getattr(self, n)) for n, _ in self._fields_ if n != "reserved"}
@@ -87,6 +93,10 @@ def lib() -> ctypes.CDLL:
         L.fiona_last_error.restype = ctypes.c_char_p
         L.fiona_abi_version.argtypes = []
         L.fiona_abi_version.restype = i32
+        L.fiona_plan_select_kernel.argtypes = [p, i32]
+        L.fiona_plan_select_kernel.restype = i32
+        L.fiona_device_check.argtypes = [p, p]
+        L.fiona_device_check.restype = i32
         _lib = L
     return _lib
 
@@ -144,6 +154,14 @@ class Context:
             _check(rc, "fiona_check_residues")
         return rc
 
+    def device_check(self, stream=None) -> int:
+        """fiona_device_check: FIONA_OK, or FIONA_ERR_TIMEOUT if a kernel gave
+        up a bounded wait since the last check (raises on other errors)."""
+        rc = lib().fiona_device_check(self.handle, stream_handle(stream))
+        if rc not in (FIONA_OK, FIONA_ERR_TIMEOUT):
+            _check(rc, "fiona_device_check")
+        return rc
+
     def close(self) -> None:
         if getattr(self, "handle", None):
             lib().fiona_ctx_destroy(self.handle)
@@ -195,6 +213,11 @@ class Plan:
         s = PlanStats()
         _check(lib().fiona_plan_stats(self.handle, ctypes.byref(s)), "fiona_plan_stats")
         return s.as_dict()
+
+    def select_kernel(self, kernel) -> None:
+        """Use kernel variant "auto", "direct" or "tiled" (or its FIONA_KERNEL_* value)."""
+        k = KERNELS[kernel] if isinstance(kernel, str) else int(kernel)
+        _check(lib().fiona_plan_select_kernel(self.handle, k), "fiona_plan_select_kernel")
 
     def eval(self, inputs, plaintexts, outputs, stream=None) -> None:
         """Enqueue fiona_linear_eval on `stream` (device buffers)."""

@@ -429,7 +429,7 @@ SEED_BASE = 0xF10A0000
 
 # Shapes of the configurations (Sec. 6 layers; Sec. 3.1 weighted sum)
 WORKLOADS = ("tiny", "tiny-dag", "worked-example", "wsum-pmult", "wsum-ternary",
-             "wsum-hybrid", "vgg", "vit", "bert", "overflow60")
+             "wsum-hybrid", "vgg", "vit", "bert", "overflow60", "overflow50")
 
 
 def make_workload(name: str, N: Optional[int] = None, L: Optional[int] = None,
@@ -482,13 +482,15 @@ def make_workload(name: str, N: Optional[int] = None, L: Optional[int] = None,
         n, qs = primes(1 << 16, 12, 50)
         plan = dense_hybrid_plan(PlanRng(seed), 96, 96, 2198, 2198, 488, dag_share=0.30)
         return Workload(name, n, qs, plan, seed)
-    if name == "overflow60":
-        # worst case for lazy reduction: 60-bit primes, every residue q-1,
-        # many terms per output (one output with 300 raw + 300 signed terms,
-        # one all-signed output, one all-raw output)
+    if name in ("overflow60", "overflow50"):
+        # worst case for lazy reduction: every residue q-1 and more terms per
+        # output than the accumulators hold without a fold (60-bit primes:
+        # 256 products of 128 bits, 16 signed residues of 64 bits; 50-bit
+        # primes on the radix-2^26 path: 2047 products, 64 packed residues)
         seed = SEED_BASE + 5
-        n, qs = primes(1 << 10, 3, 60)
-        plan = _overflow_plan(PlanRng(seed))
+        bits_ = 60 if name == "overflow60" else 50
+        n, qs = primes(1 << 10, 3, bits_)
+        plan = _overflow_plan(PlanRng(seed), 400 if bits_ == 60 else 2100)
         return Workload(name, n, qs, plan, seed, fill="max")
     raise KeyError(name)
 
@@ -556,26 +558,30 @@ def _tiny_dag_plan(rng: PlanRng) -> Plan:
                        [0, 1, 2, 3], nodes, uses)
 
 
-def _overflow_plan(rng: PlanRng) -> Plan:
+def _overflow_plan(rng: PlanRng, n_raw_long: int) -> Plan:
+    """Worst case for lazy reduction on 60-bit primes: more products per output
+    than a 128-bit accumulator holds (256 for q near 2^60), and long signed
+    sums.  Inputs repeat (duplicate pairs sum), so 100 inputs suffice."""
     R, T = TERM_RAW, TERM_TERNARY
-    n_in = 600
+    n_in = 100
     per_output = []
     pt = 0
-    # output 0: alternating raw and signed terms (300 raw products + 1 scale)
+    # output 0: 300 raw products interleaved with 300 signed terms (1 scale)
     row = []
-    for i in range(n_in):
-        if i % 2 == 0:
+    for e in range(600):
+        i = (e // 2) % n_in
+        if e % 2 == 0:
             row.append((i, R, 0, pt, 0))
             pt += 1
         else:
-            row.append((i, T, 1 if (i // 2) % 3 else -1, 0, 0))
+            row.append((i, T, 1 if (e // 2) % 3 else -1, 0, 0))
     per_output.append(row)
-    # output 1: all signed, all +1 (the signed accumulator's worst case)
-    per_output.append([(i, T, 1, 0, 1) for i in range(n_in)])
-    # output 2: all raw on the first 400 inputs (400 products > 256)
+    # output 1: 600 signed terms, all +1 (the signed accumulator's worst case)
+    per_output.append([(e % n_in, T, 1, 0, 1) for e in range(600)])
+    # output 2: n_raw_long raw products
     row = []
-    for i in range(400):
-        row.append((i, R, 0, pt, 0))
+    for e in range(n_raw_long):
+        row.append((e % n_in, R, 0, pt, 0))
         pt += 1
     per_output.append(row)
     n_raw = pt

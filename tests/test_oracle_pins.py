@@ -187,10 +187,11 @@ def test_closed_form_zero_and_identity():
     np.testing.assert_array_equal(y[4], (q - X[1]) % q)
 
 
-def test_closed_form_all_max_residues_sixty_bit():
+@pytest.mark.parametrize("name", ["overflow60", "overflow50"])
+def test_closed_form_all_max_residues(name):
     """Every residue q-1 = -1: a raw product is (+1), a signed term t*(-1)
     scaled by gamma = -1 is (+t); so y = #raw + sum(t) (mod q)."""
-    wl = W.make_workload("overflow60")
+    wl = W.make_workload(name)
     X, P = small_inputs(wl, 4)
     y = oracle.linear_eval(wl.plan, wl.moduli, X, P)
     t = wl.plan.terms

@@ -36,13 +36,17 @@ SMALL = [
     ("vit", 2048, 2),
     ("bert", 1024, 1),
     ("overflow60", None, None),
+    ("overflow50", None, None),
 ]
 
 
+@pytest.mark.parametrize("kernel", ["direct", "tiled"])
 @pytest.mark.parametrize("name,N,L", SMALL)
-def test_elementwise_parity_small(name, N, L):
+def test_elementwise_parity_small(name, N, L, kernel):
     wl = W.make_workload(name, N=N, L=L)
     dl = DeviceLayer(wl)
+    dl.plan.select_kernel(kernel)
+    assert dl.plan.stats()["kernel"] == F.KERNELS[kernel]
     dl.run()
     got = dl.outputs()
     want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
@@ -51,6 +55,7 @@ def test_elementwise_parity_small(name, N, L):
     # a second launch on a dirty output buffer gives the same result
     dl.run()
     assert np.array_equal(dl.outputs(), want)
+    assert dl.ctx.device_check() == F.FIONA_OK
 
 
 def test_edge_plans():
@@ -68,10 +73,12 @@ def test_edge_plans():
     for i, p in enumerate(plans):
         wl = W.Workload("edge%d" % i, 1024, qs, p, 1000 + i)
         dl = DeviceLayer(wl)
-        dl.run()
-        want = oracle.linear_eval(p, qs, dl.X if dl.X.size else np.zeros((0, 2, 3, 1024), np.uint64),
-                                  dl.P if dl.P.size else np.zeros((0, 3, 1024), np.uint64))
-        assert np.array_equal(dl.outputs(), want), i
+        want = oracle.linear_eval(p, qs, dl.X, dl.P)
+        for kernel in ("direct", "tiled"):
+            dl.plan.select_kernel(kernel)
+            dl.d_out.fill_(-1)
+            dl.run()
+            assert np.array_equal(dl.outputs(), want), (i, kernel)
 
 
 def test_boundary_residues():
@@ -89,8 +96,11 @@ def test_boundary_residues():
     P[..., 64:72] = 0
     dl.d_in.copy_(to_device(X))
     dl.d_pt.copy_(to_device(P))
-    dl.run()
-    assert np.array_equal(dl.outputs(), oracle.linear_eval(wl.plan, qs, X, P))
+    want = oracle.linear_eval(wl.plan, qs, X, P)
+    for kernel in ("direct", "tiled"):
+        dl.plan.select_kernel(kernel)
+        dl.run()
+        assert np.array_equal(dl.outputs(), want), kernel
 
 
 FULL = ["wsum-pmult", "wsum-ternary", "wsum-hybrid", "vgg", "vit", "bert"]
@@ -98,8 +108,10 @@ FULL = ["wsum-pmult", "wsum-ternary", "wsum-hybrid", "vgg", "vit", "bert"]
 
 @pytest.mark.parametrize("name", FULL)
 def test_full_size_sampled_parity(name):
-    """Full N = 2^16 layer, inputs filled on the device; outputs compared with
-    the oracle at sampled (limb, coefficient) coordinates, every output."""
+    """Full N = 2^16 layer, inputs filled on the device, evaluated with the
+    kernel the plan selects by default (the launch the benchmark times);
+    outputs compared with the oracle at sampled (limb, coefficient)
+    coordinates, every output."""
     wl = W.make_workload(name)
     dl = DeviceLayer(wl, host_inputs=False)
     dl.run()
@@ -115,6 +127,15 @@ def test_full_size_sampled_parity(name):
     assert np.array_equal(got.reshape(want.shape), want)
     # every residue canonical
     assert dl.ctx.check_residues(dl.d_out, wl.plan.n_out * 2) == F.FIONA_OK
+    assert dl.ctx.device_check() == F.FIONA_OK
+    # the other kernel variant agrees on every residue
+    other = "direct" if dl.plan.stats()["kernel"] == F.FIONA_KERNEL_TILED else "tiled"
+    first = dl.d_out.clone()
+    dl.plan.select_kernel(other)
+    dl.d_out.fill_(-1)
+    dl.run()
+    torch.cuda.synchronize()
+    assert torch.equal(first, dl.d_out)
 
 
 def test_device_fill_matches_host_generator():
