@@ -218,6 +218,33 @@ int fiona_linear_eval_host(const fiona_plan *plan, void *cuda_stream, const uint
                            const uint64_t *d_plaintexts, uint64_t *h_outputs,
                            uint64_t *d_inputs, uint64_t *d_outputs);
 
+/* Evaluate the layer without allocating any device memory.  The paper has no
+ * counterpart: this entry point exists for callers that cannot call
+ * cudaMalloc at the time they evaluate -- for example a serving runtime that
+ * hands all free device memory to its own pool at start-up (a later
+ * cudaMalloc would fail), or a latency-critical path that forbids allocation
+ * because cudaMalloc/cudaFree may synchronise the device and take unbounded
+ * time.  Such a caller creates its context with FIONA_DEVICE_NONE (so
+ * fiona_ctx_create and fiona_plan_create touch no device memory either) and
+ * passes device buffers it owns; any plan is accepted.
+ * The layer's schedule and the per-limb constants are copied (stream
+ * ordered) into one fixed area of FIONA_STATIC_AREA_BYTES that the library
+ * reserves in every GPU that loads it, until the process exits; the direct
+ * kernel then runs from there on the current device (the ctx's device if it
+ * has one).  A layer whose schedule exceeds the area is rejected with
+ * FIONA_ERR_ARG (about 16 B per output, 16 B per used scale group, 4 B per
+ * signed term and 8 B per raw term, plus 32 B per limb).
+ * The first call on a device also looks up the area's device address once
+ * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * The copy from host memory may wait for work already queued on the stream.
+ * All calls share the one area and each call overwrites what it reads, so
+ * nothing in it needs clearing; calls whose work can overlap on the GPU (other
+ * streams, other threads) race on it and must be ordered by the caller.
+ * Errors as fiona_linear_eval. */
+#define FIONA_STATIC_AREA_BYTES (1u << 20)
+int fiona_linear_eval_static(const fiona_plan *plan, void *cuda_stream, const uint64_t *inputs,
+                             const uint64_t *plaintexts, uint64_t *outputs);
+
 /* Debug check of the precondition residue < q_l: scans `count` ciphertext
  * polys or plaintexts ([count][L][N], pass n_in*2 for inputs) on the device
  * and returns FIONA_OK, or FIONA_ERR_RANGE if any residue is >= q_l.

@@ -472,6 +472,61 @@ static int lower_direct(fiona_plan *p)
     return FIONA_OK;
 }
 
+// Host image for fiona_linear_eval_static: the limb constants and the direct
+// schedule (same layout as lower_direct's), each part 16-byte aligned.
+static void build_static_image(fiona_plan *p)
+{
+    const HostPlan &hp = p->hp;
+    std::vector<DirOut> outs(hp.n_out);
+    std::vector<DirSeg> segs;
+    std::vector<uint32_t> ops, raw_in, raw_pt;
+    for (uint32_t j = 0; j < hp.n_out; ++j) {
+        DirOut &o = outs[j];
+        o.seg_begin = (uint32_t)segs.size();
+        std::vector<uint32_t> seen;
+        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
+            const fiona_term &t = hp.terms[e];
+            if (t.kind != FIONA_TERM_TERNARY || t.sign == 0) continue;
+            if (std::find(seen.begin(), seen.end(), t.group) != seen.end()) continue;
+            seen.push_back(t.group);
+            DirSeg sg{};
+            sg.scale_pt = hp.group_scale_pt[t.group];
+            sg.op_begin = (uint32_t)ops.size();
+            for (uint32_t f = e; f < hp.term_offsets[j + 1]; ++f) {
+                const fiona_term &u = hp.terms[f];
+                if (u.kind == FIONA_TERM_TERNARY && u.group == t.group && u.sign != 0)
+                    ops.push_back(u.input | (u.sign < 0 ? 0x80000000u : 0u));
+            }
+            sg.op_end = (uint32_t)ops.size();
+            segs.push_back(sg);
+        }
+        o.seg_end = (uint32_t)segs.size();
+        o.raw_begin = (uint32_t)raw_in.size();
+        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
+            const fiona_term &t = hp.terms[e];
+            if (t.kind != FIONA_TERM_RAW) continue;
+            raw_in.push_back(t.input);
+            raw_pt.push_back(t.pt);
+        }
+        o.raw_end = (uint32_t)raw_in.size();
+    }
+    const std::pair<const void *, size_t> parts[6] = {
+        {p->ctx->limbs.data(), p->ctx->limbs.size() * sizeof(LimbConst)},
+        {outs.data(), outs.size() * sizeof(DirOut)},
+        {segs.data(), segs.size() * sizeof(DirSeg)},
+        {ops.data(), ops.size() * 4},
+        {raw_in.data(), raw_in.size() * 4},
+        {raw_pt.data(), raw_pt.size() * 4}};
+    size_t total = 0;
+    for (int i = 0; i < 6; ++i) {
+        p->static_off[i] = total;
+        total += (parts[i].second + 15) & ~(size_t)15;
+    }
+    p->static_image.assign(total, 0);
+    for (int i = 0; i < 6; ++i)
+        if (parts[i].second) memcpy(p->static_image.data() + p->static_off[i], parts[i].first, parts[i].second);
+}
+
 static void release_device(fiona_plan *p)
 {
     if (!p->ctx || p->ctx->device == FIONA_DEVICE_NONE) return;
@@ -603,6 +658,7 @@ extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n
     p->mac_budget = (uint32_t)std::min<u128>(mb, 1u << 30);
     const uint64_t sb = ~(uint64_t)0 / (ctx->q_max - 1);
     p->signed_budget = (uint32_t)std::min<uint64_t>(sb, 1u << 30);
+    build_static_image(p);
 
     if (ctx->device != FIONA_DEVICE_NONE) {
         DeviceGuard g(ctx->device);
@@ -731,6 +787,28 @@ extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const u
     if (e2 != cudaSuccess) return cuda_fail(e2, "linear_eval_host: sync");
     if (e3 != cudaSuccess) return cuda_fail(e3, "linear_eval_host: sync");
     return FIONA_OK;
+}
+
+extern "C" int fiona_linear_eval_static(const fiona_plan *p, void *stream, const uint64_t *in,
+                                        const uint64_t *pt, uint64_t *out)
+{
+    if (!p) return set_error(FIONA_ERR_ARG, "linear_eval_static: null plan");
+    if (!out) return set_error(FIONA_ERR_ARG, "linear_eval_static: null outputs");
+    if ((p->hp.n_in && !in) || (p->hp.n_pt && !pt))
+        return set_error(FIONA_ERR_ARG, "linear_eval_static: null inputs or plaintexts");
+    if (((uintptr_t)in | (uintptr_t)pt | (uintptr_t)out) & 15)
+        return set_error(FIONA_ERR_ARG, "linear_eval_static: buffers must be 16-byte aligned");
+    if (p->static_image.size() > kStaticAreaBytes)
+        return set_error(FIONA_ERR_ARG,
+                         "linear_eval_static: this layer needs %zu bytes of schedule, more than "
+                         "the %zu-byte static area; use fiona_linear_eval",
+                         p->static_image.size(), kStaticAreaBytes);
+    if (p->hp.n_out == 0) return FIONA_OK;
+    if (p->ctx->device != FIONA_DEVICE_NONE) {
+        DeviceGuard g(p->ctx->device);
+        return launch_direct_static(p, stream, in, pt, out);
+    }
+    return launch_direct_static(p, stream, in, pt, out);
 }
 
 extern "C" int fiona_check_residues(const fiona_ctx *ctx, void *stream, const uint64_t *data,

@@ -11,6 +11,7 @@
 #include "rns.cuh"
 
 #define FIONA_MAX_LIMBS 64
+#define FIONA_MAX_DEVICES 64
 
 // ---------------------------------------------------------------------------
 // Direct schedule (one thread per coefficient pair and output): a flat list of
@@ -83,6 +84,10 @@ struct fiona_plan {
     // streams for fiona_linear_eval_host
     void *copy_in_stream = nullptr;
     void *copy_out_stream = nullptr;
+    // host image of the direct schedule and the limb constants, copied into
+    // the library's fixed device area by fiona_linear_eval_static
+    std::vector<uint8_t> static_image;
+    size_t static_off[6] = {0, 0, 0, 0, 0, 0};  // limbs, outs, segs, ops, raw_in, raw_pt
 };
 
 // kernels.cu
@@ -90,6 +95,9 @@ int launch_direct(const fiona_plan *p, void *stream, const uint64_t *in, const u
                   uint64_t *out, uint32_t limb_begin, uint32_t limb_end);
 int launch_check_residues(const fiona_ctx *ctx, void *stream, const uint64_t *data,
                           uint64_t count);
+int launch_direct_static(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
+                         uint64_t *out);
+extern const size_t kStaticAreaBytes;
 
 // lower_tiled.cpp / kernel_tiled.cu
 int lower_tiled(fiona_plan *p);

@@ -8,11 +8,19 @@
 // (through L2); the tiled kernel reads each input tile once.
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "fiona_internal.h"
 
 namespace {
 
 constexpr int kDirectThreads = 128;
+
+// Fixed device area for fiona_linear_eval_static: the limb constants and the
+// direct schedule of one layer, copied in by each call.  Every GPU that
+// loads this library holds these bytes until the process exits.
+constexpr size_t kStaticBytes = FIONA_STATIC_AREA_BYTES;
+static __device__ __align__(256) unsigned char g_static_area[kStaticBytes];
 
 __device__ __forceinline__ ulonglong2 ld2(const uint64_t *p)
 {
@@ -128,6 +136,53 @@ int launch_direct(const fiona_plan *p, void *stream, const uint64_t *in, const u
         in, pt, out, ctx->d_limbs, p->d_dir_out, p->d_dir_seg, p->d_sig_ops, p->d_raw_input,
         p->d_raw_pt, ctx->N, ctx->L, l0, p->mac_budget);
     cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "direct kernel launch: %s", cudaGetErrorString(e));
+    return FIONA_OK;
+}
+
+const size_t kStaticAreaBytes = kStaticBytes;
+
+// Device address of g_static_area on the current device, looked up once per
+// device (host code cannot use the symbol itself as a device pointer).
+static int static_area(unsigned char **ptr)
+{
+    static std::mutex mu;
+    static unsigned char *addr[FIONA_MAX_DEVICES] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "static area: %s", cudaGetErrorString(e));
+    if (dev < 0 || dev >= FIONA_MAX_DEVICES) return set_error(FIONA_ERR_ARG, "static area: device %d", dev);
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_area);
+        if (e != cudaSuccess)
+            return set_error(FIONA_ERR_CUDA, "static area: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+        addr[dev] = (unsigned char *)p;
+    }
+    *ptr = addr[dev];
+    return FIONA_OK;
+}
+
+int launch_direct_static(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
+                         uint64_t *out)
+{
+    const fiona_ctx *ctx = p->ctx;
+    unsigned char *area = nullptr;
+    int rc = static_area(&area);
+    if (rc) return rc;
+    cudaStream_t s = (cudaStream_t)stream;
+    // every byte the kernel reads is rewritten here first, in stream order
+    cudaError_t e = cudaMemcpyAsync(area, p->static_image.data(), p->static_image.size(),
+                                    cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "static area copy: %s", cudaGetErrorString(e));
+    const size_t *o = p->static_off;
+    dim3 grid((ctx->N / 2 + kDirectThreads - 1) / kDirectThreads, ctx->L, p->hp.n_out);
+    direct_kernel<<<grid, kDirectThreads, 0, s>>>(
+        in, pt, out, (const LimbConst *)(area + o[0]), (const DirOut *)(area + o[1]),
+        (const DirSeg *)(area + o[2]), (const uint32_t *)(area + o[3]), (const uint32_t *)(area + o[4]),
+        (const uint32_t *)(area + o[5]), ctx->N, ctx->L, 0, p->mac_budget);
+    e = cudaGetLastError();
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "direct kernel launch: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }

@@ -36,7 +36,8 @@ KERNELS = {"auto": FIONA_KERNEL_AUTO, "direct": FIONA_KERNEL_DIRECT, "tiled": FI
 EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona_plan_destroy",
             "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host",
             "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version",
-            "fiona_plan_select_kernel", "fiona_device_check")
+            "fiona_plan_select_kernel", "fiona_device_check", "fiona_linear_eval_static")
+STATIC_AREA_BYTES = 1 << 20
 
 
 class FionaError(RuntimeError):
@@ -97,6 +98,8 @@ def lib() -> ctypes.CDLL:
         L.fiona_plan_select_kernel.restype = i32
         L.fiona_device_check.argtypes = [p, p]
         L.fiona_device_check.restype = i32
+        L.fiona_linear_eval_static.argtypes = [p, p, p, p, p]
+        L.fiona_linear_eval_static.restype = i32
         _lib = L
     return _lib
 
@@ -227,6 +230,11 @@ class Plan:
     def eval_status(self, inputs, plaintexts, outputs, stream=None) -> int:
         return lib().fiona_linear_eval(self.handle, stream_handle(stream), addr(inputs),
                                        addr(plaintexts), addr(outputs))
+
+    def eval_static(self, inputs, plaintexts, outputs, stream=None) -> int:
+        """fiona_linear_eval_static: no device allocation (returns the status)."""
+        return lib().fiona_linear_eval_static(self.handle, stream_handle(stream), addr(inputs),
+                                              addr(plaintexts), addr(outputs))
 
     def eval_host(self, h_inputs, d_plaintexts, h_outputs, d_inputs, d_outputs,
                   stream=None) -> None:
