@@ -7,7 +7,7 @@
 #include <string>
 #include <vector>
 
-#include "../../include/fiona.h"
+#include "fiona.h"
 #include "rns.cuh"
 
 #define FIONA_MAX_LIMBS 64

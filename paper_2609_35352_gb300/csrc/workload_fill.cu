@@ -3,7 +3,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/fiona_workload.h"
+#include "fiona_workload.h"
 
 namespace {
 
