@@ -12,10 +12,14 @@
 // * Outputs are assigned to warps by longest-processing-time first on an
 //   estimated cost; with fewer outputs than warps, each output is split into
 //   parts whose reduced partial sums are added at the end (exact in Z_q).
-// * Shape: 2 or 1 coefficients per lane and 8 or 16 warps per CTA, and two
-//   source buffers (the next tile staged during this one) when they fit;
-//   chosen to keep the most bytes in flight per SM.  Plans whose moduli are
-//   all below 2^52 use the radix-2^26 arithmetic.
+// * Each warp gets a program (its jobs' words) and a fetch list (the
+//   plaintext tiles it consumes, in order); the whole schedule is one word
+//   array the kernel copies into shared memory.
+// * Shape: 2 or 1 coefficients per lane, 8 or 16 warps per CTA, 16 or 8
+//   plaintext tiles in flight per warp, and two source buffers (the next
+//   tile staged during this one) when they fit; chosen to keep enough bytes
+//   in flight per SM.  Plans whose moduli are all below 2^52 use the
+//   radix-2^26 arithmetic.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -43,47 +47,24 @@ struct OutWork {
     }
 };
 
-struct JobSet {
-    std::vector<uint32_t> warp_job_off, ops;
-    std::vector<uint2> raws;
-    std::vector<TiledJob> jobs;
-    std::vector<TiledSeg> segs;
-    std::vector<uint32_t> comb_off, comb_out, comb_parts;
-    uint32_t n_part = 0;
-};
-
-// Segments of one scale group: the group's plus and minus runs as op words,
-// each run at most `budget` words long.
-void put_segments(JobSet &js, const OutWork::Seg &sg, uint32_t L, uint32_t budget,
-                  uint32_t pair_bytes)
-{
-    size_t pb = 0, mb = 0;
-    do {
-        const size_t pe = std::min(sg.plus.size(), pb + budget);
-        const size_t me = std::min(sg.minus.size(), mb + budget);
-        TiledSeg s{};
-        s.gamma_ptl = sg.scale_pt * L;
-        s.op_begin = (uint32_t)js.ops.size();
-        for (size_t i = pb; i < pe; ++i) js.ops.push_back(sg.plus[i] * pair_bytes);
-        for (size_t i = mb; i < me; ++i) js.ops.push_back(sg.minus[i] * pair_bytes);
-        s.n_plus = (uint16_t)(pe - pb);
-        s.n_minus = (uint16_t)(me - mb);
-        js.segs.push_back(s);
-        pb = pe;
-        mb = me;
-    } while (pb < sg.plus.size() || mb < sg.minus.size());
-}
-
-JobSet build_jobs(const std::vector<OutWork> &work, uint32_t n_out, uint32_t W, uint32_t L,
-                  uint32_t pair_bytes, uint32_t budget)
-{
+// Jobs for W warps: whole outputs assigned largest first to the least-loaded
+// warp; with fewer outputs than warps each output is cut into parts of about
+// equal cost whose reduced partial sums are added at the end.
+struct JobPlan {
     struct Job {
         uint32_t target;
         OutWork w;
     };
-    JobSet js;
-    std::vector<Job> jobs;
-    js.comb_off.assign(1, 0);
+    std::vector<std::vector<Job>> per_warp;
+    std::vector<uint32_t> comb_off, comb_out, comb_parts;
+    uint32_t n_part = 0;
+};
+
+JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t n_out, uint32_t W)
+{
+    JobPlan jp;
+    std::vector<JobPlan::Job> jobs;
+    jp.comb_off.assign(1, 0);
     const uint32_t parts = n_out >= W ? 1 : W / std::max<uint32_t>(n_out, 1);
     for (uint32_t j = 0; j < n_out; ++j) {
         const OutWork &w = work[j];
@@ -93,7 +74,6 @@ JobSet build_jobs(const std::vector<OutWork> &work, uint32_t n_out, uint32_t W, 
             jobs.push_back({j, w});
             continue;
         }
-        // cut the output's items into P contiguous chunks of about equal cost
         std::vector<OutWork> chunk(P);
         const uint64_t per = (c + P - 1) / P;
         uint32_t cur = 0;
@@ -123,42 +103,116 @@ JobSet build_jobs(const std::vector<OutWork> &work, uint32_t n_out, uint32_t W, 
             advance(4);
             chunk[cur].raws.push_back(r);
         }
-        js.comb_out.push_back(j);
+        jp.comb_out.push_back(j);
         for (uint32_t q = 0; q < P; ++q) {
             if (chunk[q].segs.empty() && chunk[q].raws.empty()) continue;
-            jobs.push_back({kPartBit | js.n_part, chunk[q]});
-            js.comb_parts.push_back(js.n_part++);
+            jobs.push_back({kPartBit | jp.n_part, chunk[q]});
+            jp.comb_parts.push_back(jp.n_part++);
         }
-        js.comb_off.push_back((uint32_t)js.comb_parts.size());
+        jp.comb_off.push_back((uint32_t)jp.comb_parts.size());
     }
     std::vector<uint32_t> order(jobs.size());
     std::iota(order.begin(), order.end(), 0);
     std::stable_sort(order.begin(), order.end(),
                      [&](uint32_t a, uint32_t b) { return jobs[a].w.cost() > jobs[b].w.cost(); });
     std::vector<uint64_t> load(W, 0);
-    std::vector<std::vector<uint32_t>> per_warp(W);
+    jp.per_warp.assign(W, {});
     for (uint32_t o : order) {
         const uint32_t wi = (uint32_t)(std::min_element(load.begin(), load.end()) - load.begin());
-        per_warp[wi].push_back(o);
+        jp.per_warp[wi].push_back(jobs[o]);
         load[wi] += jobs[o].w.cost() + 1;
     }
-    js.warp_job_off.assign(W + 1, 0);
-    for (uint32_t wi = 0; wi < W; ++wi) {
-        for (uint32_t o : per_warp[wi]) {
-            const Job &jb = jobs[o];
-            TiledJob t{};
-            t.target = jb.target;
-            t.seg_begin = (uint32_t)js.segs.size();
-            for (auto &sg : jb.w.segs) put_segments(js, sg, L, budget, pair_bytes);
-            t.seg_end = (uint32_t)js.segs.size();
-            t.raw_begin = (uint32_t)js.raws.size();
-            for (auto &r : jb.w.raws) js.raws.push_back(make_uint2(r.second * L, r.first * pair_bytes));
-            t.raw_end = (uint32_t)js.raws.size();
-            js.jobs.push_back(t);
-        }
-        js.warp_job_off[wi + 1] = (uint32_t)js.jobs.size();
+    return jp;
+}
+
+// Append one scale group's segments (runs of at most `budget` words) to a
+// warp program and its gamma fetches to the fetch list.
+void put_group(std::vector<uint32_t> &prog, std::vector<uint32_t> &fetch, const OutWork::Seg &sg,
+               uint32_t L, uint32_t budget, uint32_t pair_bytes, uint32_t &n_seg)
+{
+    size_t pb = 0, mb = 0;
+    do {
+        const size_t pe = std::min(sg.plus.size(), pb + budget);
+        const size_t me = std::min(sg.minus.size(), mb + budget);
+        prog.push_back((uint32_t)(pe - pb) | ((uint32_t)(me - mb) << 16));
+        for (size_t i = pb; i < pe; ++i) prog.push_back(sg.plus[i] * pair_bytes);
+        for (size_t i = mb; i < me; ++i) prog.push_back(sg.minus[i] * pair_bytes);
+        fetch.push_back(sg.scale_pt * L);
+        ++n_seg;
+        pb = pe;
+        mb = me;
+    } while (pb < sg.plus.size() || mb < sg.minus.size());
+}
+
+// The whole schedule as one word array (see tiled.h).
+struct Sched {
+    std::vector<uint32_t> w;
+    uint32_t o_level, o_node_slot, o_node_prog_off, o_prog_off, o_fetch_off, o_comb_off, o_comb_out,
+        o_comb_parts;
+};
+
+Sched encode(const JobPlan &jp, const std::vector<uint32_t> &node_level_off,
+             const std::vector<uint32_t> &node_slots, const std::vector<OutWork::Seg> &node_seg,
+             uint32_t W, uint32_t L, uint32_t budget, uint32_t pair_bytes)
+{
+    Sched sc;
+    auto &w = sc.w;
+    auto put = [&](const std::vector<uint32_t> &v) { w.insert(w.end(), v.begin(), v.end()); };
+    sc.o_level = (uint32_t)w.size();
+    put(node_level_off);
+    sc.o_node_slot = (uint32_t)w.size();
+    put(node_slots);
+    // node programs: offsets table then programs
+    sc.o_node_prog_off = (uint32_t)w.size();
+    const size_t n_nodes = node_seg.size();
+    w.resize(w.size() + n_nodes + 1);
+    for (size_t k = 0; k < n_nodes; ++k) {
+        w[sc.o_node_prog_off + k] = (uint32_t)w.size();
+        const OutWork::Seg &sg = node_seg[k];
+        w.push_back((uint32_t)sg.plus.size() | ((uint32_t)sg.minus.size() << 16));
+        for (uint32_t s : sg.plus) w.push_back(s * pair_bytes);
+        for (uint32_t s : sg.minus) w.push_back(s * pair_bytes);
     }
-    return js;
+    w[sc.o_node_prog_off + n_nodes] = (uint32_t)w.size();
+    // warp programs and fetch lists
+    std::vector<std::vector<uint32_t>> progs(W), fetches(W);
+    for (uint32_t wi = 0; wi < W; ++wi) {
+        for (const auto &jb : jp.per_warp[wi]) {
+            auto &prog = progs[wi];
+            prog.push_back(jb.target);
+            const size_t hdr = prog.size();
+            prog.push_back(0);
+            uint32_t n_seg = 0;
+            for (const auto &sg : jb.w.segs) put_group(prog, fetches[wi], sg, L, budget, pair_bytes, n_seg);
+            for (const auto &r : jb.w.raws) {
+                prog.push_back(r.first * pair_bytes);
+                fetches[wi].push_back(r.second * L);
+            }
+            prog[hdr] = n_seg | ((uint32_t)jb.w.raws.size() << 16);
+        }
+    }
+    sc.o_prog_off = (uint32_t)w.size();
+    w.resize(w.size() + W + 1);
+    for (uint32_t wi = 0; wi < W; ++wi) {
+        w[sc.o_prog_off + wi] = (uint32_t)w.size();
+        put(progs[wi]);
+    }
+    w[sc.o_prog_off + W] = (uint32_t)w.size();
+    sc.o_fetch_off = (uint32_t)w.size();
+    w.resize(w.size() + W + 1);
+    for (uint32_t wi = 0; wi < W; ++wi) {
+        w[sc.o_fetch_off + wi] = (uint32_t)w.size();
+        put(fetches[wi]);
+    }
+    w[sc.o_fetch_off + W] = (uint32_t)w.size();
+    sc.o_comb_off = (uint32_t)w.size();
+    put(jp.comb_off);
+    sc.o_comb_out = (uint32_t)w.size();
+    put(jp.comb_out);
+    sc.o_comb_parts = (uint32_t)w.size();
+    put(jp.comb_parts);
+    while (w.size() % 4) w.push_back(0);  // a multiple of 16 bytes
+    return sc;
 }
 
 int upload_blob(TiledSchedule *ts, const std::vector<std::pair<const void *, size_t>> &parts,
@@ -185,8 +239,8 @@ int upload_blob(TiledSchedule *ts, const std::vector<std::pair<const void *, siz
 }  // namespace
 
 // kernel_tiled.cu
-int tiled_configure_kernel(int C, bool narrow, size_t smem);
-int tiled_kernel_attributes(int C, bool narrow, cudaFuncAttributes *attr);
+int tiled_configure_kernel(int C, bool narrow, uint32_t depth, size_t smem);
+int tiled_kernel_attributes(int C, bool narrow, uint32_t depth, cudaFuncAttributes *attr);
 
 int lower_tiled(fiona_plan *p)
 {
@@ -263,40 +317,46 @@ int lower_tiled(fiona_plan *p)
         }
     }
 
-    // -- shape
+    // -- shape: coefficients per lane C, warps W, ring depth D, source buffers
     const size_t budget_smem = (ctx->smem_optin ? ctx->smem_optin : 227 * 1024) - 256;
     const size_t per_sm = 228 * 1024;
     const uint32_t n_src = n_in + n_slots;
     struct Shape {
         int C;
-        uint32_t W;
+        uint32_t W, D;
         bool dbl;
         uint32_t ctas;
+        size_t smem;
         uint64_t score;
     };
     std::vector<Shape> shapes;
     for (int C : {2, 1}) {
         if (ctx->N % (32u * C)) continue;
-        cudaFuncAttributes attr{};
-        if (tiled_kernel_attributes(C, narrow, &attr) != FIONA_OK) continue;
-        const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
-        const uint32_t pair_bytes = 2 * 32u * C * 8;
+        const uint32_t T = 32u * C, pair_bytes = 2 * T * 8;
         for (uint32_t W : {8u, 16u}) {
-            const uint32_t n_part_est = hp.n_out >= W ? 0 : W;
-            for (bool dbl : {true, false}) {
-                if (dbl && n_in == 0) continue;
-                const size_t smem = (size_t)n_src * pair_bytes * (dbl ? 2 : 1) +
-                                    (size_t)n_part_est * pair_bytes + 16;
-                if (smem + attr.sharedSizeBytes > budget_smem) continue;
-                const uint32_t by_smem = (uint32_t)(per_sm / (smem + attr.sharedSizeBytes + 1024));
-                const uint32_t by_threads = 2048 / (W * 32);
-                const uint32_t by_regs = 65536 / (W * 32 * regs);
-                const uint32_t ctas = std::min({by_smem, by_threads, by_regs});
-                if (!ctas) continue;
-                // resident warps x bytes per load (ties: the first listed,
-                // double-buffered before single, 8 warps before 16)
-                const uint64_t score = (uint64_t)ctas * W * C;
-                shapes.push_back({C, W, dbl, ctas, score});
+            const JobPlan jp = build_jobs(work, hp.n_out, W);
+            const Sched sc = encode(jp, node_level_off, node_slots, node_seg, W, ctx->L, budget, pair_bytes);
+            const size_t sched_bytes = sc.w.size() * 4;
+            for (uint32_t D : {16u, 8u}) {
+                cudaFuncAttributes attr{};
+                if (tiled_kernel_attributes(C, narrow, D, &attr) != FIONA_OK) continue;
+                const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
+                for (bool dbl : {true, false}) {
+                    if (dbl && n_in == 0) continue;
+                    const size_t smem = sched_bytes + (size_t)n_src * pair_bytes * (dbl ? 2 : 1) +
+                                        (size_t)jp.n_part * pair_bytes + (size_t)W * D * T * 8 + 32;
+                    if (smem + attr.sharedSizeBytes > budget_smem) continue;
+                    const uint32_t by_smem = (uint32_t)(per_sm / (smem + attr.sharedSizeBytes + 1024));
+                    const uint32_t by_threads = 2048 / (W * 32);
+                    const uint32_t by_regs = 65536 / (W * 32 * regs);
+                    const uint32_t ctas = std::min({by_smem, by_threads, by_regs});
+                    if (!ctas) continue;
+                    // plaintext bytes in flight per SM (enough at about 96 KB),
+                    // then resident warps, then wider loads
+                    const uint64_t inflight = std::min<uint64_t>((uint64_t)ctas * W * D * T * 8, 96 * 1024);
+                    const uint64_t score = (inflight << 16) | ((uint64_t)ctas * W << 4) | (uint64_t)(C * 2 + dbl);
+                    shapes.push_back({C, W, D, dbl, ctas, smem, score});
+                }
             }
         }
     }
@@ -304,72 +364,45 @@ int lower_tiled(fiona_plan *p)
         return set_error(FIONA_ERR_ARG, "tiled kernel: %u source tiles do not fit in shared memory", n_src);
     Shape best = *std::max_element(shapes.begin(), shapes.end(),
                                    [](const Shape &a, const Shape &b) { return a.score < b.score; });
-    // tuning override "C,W,double": every shape computes the same residues
+    // tuning override "C,W,D,double": every shape computes the same residues
     if (const char *env = getenv("FIONA_TILED_SHAPE")) {
-        int c = 0, w = 0, d = 0;
-        if (sscanf(env, "%d,%d,%d", &c, &w, &d) == 3)
+        int c = 0, w = 0, dd = 0, d = 0;
+        if (sscanf(env, "%d,%d,%d,%d", &c, &w, &dd, &d) == 4)
             for (auto &s : shapes)
-                if (s.C == c && s.W == (uint32_t)w && s.dbl == (d != 0)) best = s;
+                if (s.C == c && s.W == (uint32_t)w && s.D == (uint32_t)dd && s.dbl == (d != 0)) best = s;
     }
     const uint32_t T = 32u * best.C, pair_bytes = 2 * T * 8;
-    JobSet js = build_jobs(work, hp.n_out, best.W, ctx->L, pair_bytes, budget);
-    // shared sums' runs go into the same op array, after the jobs' runs
-    std::vector<TiledSeg> node_segs(n_slots);
-    for (uint32_t s = 0; s < n_slots; ++s) {
-        const size_t before = js.segs.size();
-        put_segments(js, node_seg[s], ctx->L, budget, pair_bytes);
-        node_segs[s] = js.segs[before];
-        js.segs.resize(before);
-    }
-    // the kernel reads schedule words ahead of use: pad the ends so those
-    // reads stay inside the arrays
-    js.ops.insert(js.ops.end(), kSchedPad, 0u);
-    js.raws.insert(js.raws.end(), kSchedPad, make_uint2(0, 0));
-    const size_t smem =
-        (size_t)n_src * pair_bytes * (best.dbl ? 2 : 1) + (size_t)js.n_part * pair_bytes + 16;
-    if (smem > budget_smem) return set_error(FIONA_ERR_ARG, "tiled kernel: shared memory estimate exceeded");
+    const JobPlan jp = build_jobs(work, hp.n_out, best.W);
+    const Sched sc = encode(jp, node_level_off, node_slots, node_seg, best.W, ctx->L, budget, pair_bytes);
 
     TiledSchedule *ts = new (std::nothrow) TiledSchedule;
     if (!ts) return set_error(FIONA_ERR_NOMEM, "tiled schedule: host allocation");
     ts->C = best.C;
     ts->narrow = narrow;
     ts->warps = best.W;
+    ts->depth = best.D;
     ts->tile = T;
-    ts->smem = smem;
+    ts->smem = best.smem;
     ts->ctas_per_sm = best.ctas;
-    int rc = tiled_configure_kernel(best.C, narrow, smem);
+    int rc = tiled_configure_kernel(best.C, narrow, best.D, ts->smem);
     std::vector<size_t> off;
-    if (rc == FIONA_OK)
-        rc = upload_blob(ts, {{node_level_off.data(), node_level_off.size() * 4},
-                              {node_slots.data(), node_slots.size() * 4},
-                              {node_segs.data(), node_segs.size() * sizeof(TiledSeg)},
-                              {js.warp_job_off.data(), js.warp_job_off.size() * 4},
-                              {js.jobs.data(), js.jobs.size() * sizeof(TiledJob)},
-                              {js.segs.data(), js.segs.size() * sizeof(TiledSeg)},
-                              {js.ops.data(), js.ops.size() * 4},
-                              {js.raws.data(), js.raws.size() * sizeof(uint2)},
-                              {js.comb_off.data(), js.comb_off.size() * 4},
-                              {js.comb_out.data(), js.comb_out.size() * 4},
-                              {js.comb_parts.data(), js.comb_parts.size() * 4}},
-                         off);
+    if (rc == FIONA_OK) rc = upload_blob(ts, {{sc.w.data(), sc.w.size() * 4}}, off);
     if (rc != FIONA_OK) {
         cudaFree(ts->sched.blob);
         delete ts;
         return rc;
     }
-    uint8_t *b = (uint8_t *)ts->sched.blob;
     TiledArgs &a = ts->args;
-    a.node_level_off = (const uint32_t *)(b + off[0]);
-    a.node_slots = (const uint32_t *)(b + off[1]);
-    a.node_segs = (const TiledSeg *)(b + off[2]);
-    a.warp_job_off = (const uint32_t *)(b + off[3]);
-    a.jobs = (const TiledJob *)(b + off[4]);
-    a.segs = (const TiledSeg *)(b + off[5]);
-    a.ops = (const uint32_t *)(b + off[6]);
-    a.raws = (const uint2 *)(b + off[7]);
-    a.comb_off = (const uint32_t *)(b + off[8]);
-    a.comb_out = (const uint32_t *)(b + off[9]);
-    a.comb_parts = (const uint32_t *)(b + off[10]);
+    a.sched = (const uint32_t *)ts->sched.blob;
+    a.o_level = sc.o_level;
+    a.o_node_slot = sc.o_node_slot;
+    a.o_node_prog_off = sc.o_node_prog_off;
+    a.o_prog_off = sc.o_prog_off;
+    a.o_fetch_off = sc.o_fetch_off;
+    a.o_comb_off = sc.o_comb_off;
+    a.o_comb_out = sc.o_comb_out;
+    a.o_comb_parts = sc.o_comb_parts;
+    a.sched_bytes = (uint32_t)(sc.w.size() * 4);
     a.limbs = ctx->d_limbs;
     a.err = ctx->d_kerr;
     a.N = ctx->N;
@@ -380,11 +413,11 @@ int lower_tiled(fiona_plan *p)
     a.n_in = n_in;
     a.n_nodes = n_slots;
     a.n_levels = n_levels;
-    a.n_part = js.n_part;
-    a.n_comb = (uint32_t)js.comb_out.size();
+    a.n_part = jp.n_part;
+    a.n_comb = (uint32_t)jp.comb_out.size();
     a.src_bytes = n_src * pair_bytes;
     a.double_buffer = best.dbl ? 1 : 0;
-    a.mac_budget = narrow ? 64u : p->mac_budget;  // rns.cuh: kNarrowMacBudget
+    a.mac_budget = narrow ? 1023u : p->mac_budget;  // rns.cuh: kNarrowMacBudget
     p->tiled = ts;
     return FIONA_OK;
 }

@@ -97,22 +97,23 @@ __device__ __forceinline__ uint64_t sub_mod(uint64_t a, uint64_t b, uint64_t q)
 }
 
 // ---------------------------------------------------------------------------
-// Narrow residues (q < 2^52): one operand in radix-2^26 split form.
+// Narrow residues (q < 2^52): radix-2^26 split form and Karatsuba products.
 //
 // A residue a < 2^52 is kept as one 64-bit word whose low 32-bit half holds
-// a0 = a mod 2^26 and whose high half holds a1 = floor(a / 2^26).  The other
-// factor b is any 64-bit value below 2^59, taken as b = b1 * 2^32 + b0.  Then
-//   a * b = a0*b0 + a1*b0 * 2^26 + a0*b1 * 2^32 + a1*b1 * 2^58,
-// four 32x32 -> 64-bit multiply-adds into four 64-bit accumulators.  The
-// first two grow by less than 2^58 per product and the last two by less
-// than 2^53, so the accumulators hold any 64 products without wrapping
-// (kNarrowMacBudget), and their weighted sum stays below 2^118.
+// a0 = a mod 2^26 and whose high half holds a1 = floor(a / 2^26).  For two
+// such residues,
+//   a * b = a0*b0 + ((a0+a1)*(b0+b1) - a0*b0 - a1*b1) * 2^26 + a1*b1 * 2^52
+// (Karatsuba), so a product-accumulate is three 32x32 -> 64-bit
+// multiply-adds into accumulators lo, x, hi; the middle term is recovered
+// once, at the reduction.  (a0+a1)*(b0+b1) < 2^54, so the accumulators hold
+// any 1023 products without wrapping (kNarrowMacBudget), and the weighted sum
+// stays below 2^116.
 //
 // Split words can also be summed as plain 64-bit integers: 64 of them keep
 // each half below 2^32 (64 * (2^26 - 1) < 2^32), so a packed sum of at most
 // 64 split words reads back as (sum of a0) + (sum of a1) * 2^26 < 2^59.
 // ---------------------------------------------------------------------------
-constexpr uint32_t kNarrowMacBudget = 64;
+constexpr uint32_t kNarrowMacBudget = 1023;
 constexpr uint32_t kNarrowSumBudget = 64;
 
 __device__ __forceinline__ uint64_t split26(uint64_t a)
@@ -128,34 +129,29 @@ __device__ __forceinline__ uint64_t unsplit_sum(uint64_t w)
     return (w & 0xFFFFFFFFull) + ((w >> 32) << 26);
 }
 
-// (a00, a10, a01, a11) += split a times b (b < 2^59)
-__device__ __forceinline__ void mac26(uint64_t &a00, uint64_t &a10, uint64_t &a01, uint64_t &a11,
-                                      uint64_t as, uint64_t b)
+// (lo, x, hi) += split a times split b, Karatsuba
+__device__ __forceinline__ void mac26(uint64_t &lo, uint64_t &x, uint64_t &hi, uint64_t as, uint64_t bs)
 {
-    const uint32_t x0 = (uint32_t)as, x1 = (uint32_t)(as >> 32);
-    const uint32_t y0 = (uint32_t)b, y1 = (uint32_t)(b >> 32);
-    asm("mad.wide.u32 %0, %4, %6, %0;\n\t"
+    const uint32_t a0 = (uint32_t)as, a1 = (uint32_t)(as >> 32);
+    const uint32_t b0 = (uint32_t)bs, b1 = (uint32_t)(bs >> 32);
+    asm("mad.wide.u32 %0, %3, %4, %0;\n\t"
         "mad.wide.u32 %1, %5, %6, %1;\n\t"
-        "mad.wide.u32 %2, %4, %7, %2;\n\t"
-        "mad.wide.u32 %3, %5, %7, %3;"
-        : "+l"(a00), "+l"(a10), "+l"(a01), "+l"(a11)
-        : "r"(x0), "r"(x1), "r"(y0), "r"(y1));
+        "mad.wide.u32 %2, %7, %8, %2;"
+        : "+l"(lo), "+l"(x), "+l"(hi)
+        : "r"(a0), "r"(b0), "r"(a0 + a1), "r"(b0 + b1), "r"(a1), "r"(b1));
 }
 
-// a00 + a10 * 2^26 + a01 * 2^32 + a11 * 2^58 mod q (the sum is below 2^118)
-__device__ __forceinline__ uint64_t reduce26(uint64_t a00, uint64_t a10, uint64_t a01, uint64_t a11,
-                                             const LimbConst &m)
+// lo + (x - lo - hi) * 2^26 + hi * 2^52 mod q (below 2^116)
+__device__ __forceinline__ uint64_t reduce26(uint64_t lo, uint64_t x, uint64_t hi, const LimbConst &m)
 {
-    uint64_t x0 = a00, x1 = 0;
+    const uint64_t mid = x - lo - hi;
+    uint64_t x0 = lo, x1 = 0;
     asm("add.cc.u64 %0, %0, %2;\n\t"
         "addc.u64   %1, %1, %3;\n\t"
         "add.cc.u64 %0, %0, %4;\n\t"
-        "addc.u64   %1, %1, %5;\n\t"
-        "add.cc.u64 %0, %0, %6;\n\t"
-        "addc.u64   %1, %1, %7;"
+        "addc.u64   %1, %1, %5;"
         : "+l"(x0), "+l"(x1)
-        : "l"(a10 << 26), "l"(a10 >> 38), "l"(a01 << 32), "l"(a01 >> 32), "l"(a11 << 58),
-          "l"(a11 >> 6));
+        : "l"(mid << 26), "l"(mid >> 38), "l"(hi << 52), "l"(hi >> 12));
     return reduce128(x0, x1, m);
 }
 
