@@ -62,7 +62,8 @@ typedef enum fiona_status {
     FIONA_ERR_CUDA = -5,    /* a CUDA runtime call failed (launch, copy, device) */
     FIONA_ERR_RANGE = -6,   /* fiona_check_residues found a residue >= q_l */
     FIONA_ERR_NODEVICE = -7,/* evaluation requested on a validation-only context */
-    FIONA_ERR_TIMEOUT = -8  /* a kernel gave up waiting for its own copies (see fiona_device_check) */
+    FIONA_ERR_TIMEOUT = -8, /* a kernel gave up waiting for its own copies (see fiona_device_check) */
+    FIONA_ERR_INTERNAL = -9 /* a lowered schedule failed its own consistency check (a library bug) */
 } fiona_status;
 
 /* Kernel variants (fiona_plan_select_kernel).  DIRECT: one thread per output
@@ -144,7 +145,9 @@ typedef struct fiona_plan_stats_t {
     uint32_t smem_bytes;          /* dynamic shared memory per CTA                          */
     uint32_t ctas_per_sm;         /* occupancy the lowering planned for                     */
     uint32_t kernel;              /* variant in use: FIONA_KERNEL_DIRECT or FIONA_KERNEL_TILED */
-    uint32_t reserved[5];
+    uint32_t nodes_materialized;  /* TILED: shared sums formed once per tile (the others are
+                                     expanded into their uses: same residues, more Add/Sub) */
+    uint32_t reserved[4];
 } fiona_plan_stats_t;
 
 /* Create a context for ring dimension N (a power of two, 2^10 <= N <= 2^17)

@@ -49,6 +49,7 @@ extern "C" const char *fiona_status_str(int status)
     case FIONA_ERR_RANGE: return "residue out of range";
     case FIONA_ERR_NODEVICE: return "context has no device";
     case FIONA_ERR_TIMEOUT: return "kernel wait timed out";
+    case FIONA_ERR_INTERNAL: return "internal consistency check failed";
     default: return "unknown status";
     }
 }
@@ -529,7 +530,10 @@ static void build_static_image(fiona_plan *p)
 
 static void release_device(fiona_plan *p)
 {
-    if (!p->ctx || p->ctx->device == FIONA_DEVICE_NONE) return;
+    if (!p->ctx || p->ctx->device == FIONA_DEVICE_NONE) {
+        if (p->tiled) free_tiled(p);  // host-only schedule: nothing on a device
+        return;
+    }
     DeviceGuard g(p->ctx->device);
     if (p->tiled) free_tiled(p);
     cudaFree(p->sched.blob);
@@ -537,6 +541,18 @@ static void release_device(fiona_plan *p)
     if (p->copy_in_stream) cudaStreamDestroy((cudaStream_t)p->copy_in_stream);
     if (p->copy_out_stream) cudaStreamDestroy((cudaStream_t)p->copy_out_stream);
     p->copy_in_stream = p->copy_out_stream = nullptr;
+}
+
+// The tiled schedule is optional: a plan whose tile does not fit in shared
+// memory runs on the direct kernel.  A schedule that fails its own check is
+// a library bug and is reported.
+static int lower_tiled_optional(fiona_plan *p)
+{
+    const int rc = lower_tiled(p);
+    if (rc == FIONA_ERR_INTERNAL) return rc;
+    if (rc != FIONA_OK) p->tiled = nullptr;
+    set_error(FIONA_OK, "");
+    return FIONA_OK;
 }
 
 // Kernel choice: TILED for layers with more than one output whose tile fits
@@ -563,12 +579,14 @@ static int select_kernel(fiona_plan *p, int which)
         s.warps_per_cta = p->tiled->warps;
         s.smem_bytes = (uint32_t)p->tiled->smem;
         s.ctas_per_sm = p->tiled->ctas_per_sm;
+        s.nodes_materialized = p->tiled->nodes_kept;
     } else {
         s.kernel = FIONA_KERNEL_DIRECT;
         s.tile_coeffs = 256;
         s.warps_per_cta = 4;
         s.smem_bytes = 0;
         s.ctas_per_sm = 0;
+        s.nodes_materialized = 0;
     }
     return FIONA_OK;
 }
@@ -667,12 +685,7 @@ extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n
             return set_error(FIONA_ERR_CUDA, "plan_create: cannot select device %d", ctx->device);
         }
         rc = lower_direct(p);
-        if (rc == FIONA_OK && hp.n_out > 0) {
-            // the tiled schedule is optional: a plan whose tile does not fit
-            // in shared memory runs on the direct kernel
-            if (lower_tiled(p) != FIONA_OK) p->tiled = nullptr;
-            set_error(FIONA_OK, "");
-        }
+        if (rc == FIONA_OK && hp.n_out > 0) rc = lower_tiled_optional(p);
         if (rc == FIONA_OK) {
             cudaError_t e = cudaStreamCreateWithFlags((cudaStream_t *)&p->copy_in_stream,
                                                       cudaStreamNonBlocking);
@@ -683,6 +696,15 @@ extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n
         }
         if (rc) {
             release_device(p);
+            delete p;
+            return rc;
+        }
+    }
+    if (ctx->device == FIONA_DEVICE_NONE && hp.n_out > 0) {
+        // the tiled lowering (and its schedule check) also runs without a
+        // GPU, so a validation-only context reports the shape it would use
+        rc = lower_tiled_optional(p);
+        if (rc) {
             delete p;
             return rc;
         }

@@ -2,29 +2,31 @@
 //
 // A persistent CTA walks (limb l, coefficient tile) pairs, T = 32*C
 // coefficients per tile, all outputs per tile.  Shared memory holds the
-// schedule (copied once), the source region(s), partial sums, and one
-// plaintext ring per warp.
-//  1. Thread 0 copies the (c0, c1) tile of every input into a source region
-//     with bulk asynchronous copies (cp.async.bulk, completion counted on an
-//     mbarrier), so each input residue leaves HBM once.  With two source
-//     regions the next tile's copies run during this tile; otherwise warp 0
-//     prefetches the next tile's inputs into L2.  Narrow plans (every
-//     q < 2^52) rewrite the tiles in radix-2^26 split form (rns.cuh).
-//  2. The shared signed sums U (Sec. 4.2 "Sharing Signed Sums") are formed
-//     once per tile, level by level, into the same region.
-//  3. Each warp runs its program: per scale group a signed sum over sources,
-//     then one product by gamma (Sec. 4.2 "Grouping Reconstruction
-//     Operations"); per raw term a PMult-MAC of a plaintext tile and a
-//     source.  Plaintext tiles arrive through the warp's ring: each lane
-//     copies its own C words of each tile D fetches ahead (cp.async, tracked
-//     per thread with commit/wait groups), across job and tile boundaries,
-//     and reads back only what it copied.  Signed sums are lazy; products
-//     accumulate lazily; the signed and raw routes are added before the
-//     single final reduction (Sec. 4.2 "Combining the Signed and Raw Routes").
+// schedule (bulk-copied once, completion counted on an mbarrier), the
+// source region(s) and the partial sums.
+//  1. Every thread copies its share of the (c0, c1) tile of every input into
+//     a source region with 16-byte asynchronous copies (cp.async, one commit
+//     group per tile), so each input residue leaves HBM once.  With two
+//     source regions the next tile's copies run during this tile; otherwise
+//     warp 0 prefetches the next tile's inputs into L2.  Narrow plans (every
+//     q < 2^52) rewrite the tiles in radix-2^26 split form (rns.cuh), each
+//     thread the words it copied.
+//  2. The materialised shared signed sums (Sec. 4.2 "Sharing Signed Sums")
+//     are formed once per tile, level by level, into the same region.
+//  3. Each warp runs its operation stream (tiled.h): per scale group a
+//     signed sum over sources, its additions spread over the operations
+//     before the group's product, then one product by gamma (Sec. 4.2
+//     "Grouping Reconstruction Operations"); per raw term a PMult-MAC of a
+//     plaintext tile and a source.  Plaintext tiles go from HBM straight to
+//     registers: each warp keeps the next kTiledPrefetch of its stream in
+//     flight, across job and tile boundaries, in a register queue indexed at
+//     compile time (the stream is processed in batches of that many
+//     operations).  Signed sums are lazy; products accumulate lazily; the
+//     signed and raw routes are added before the single final reduction
+//     (Sec. 4.2 "Combining the Signed and Raw Routes").
 //  4. Outputs split across warps add their reduced partial sums.
-// The only spin-waits are thread 0's bounded mbarrier waits; if one gives up,
-// the CTA raises the context's error flag, drains its own copies (bounded),
-// and stops.
+// The only spin-wait is thread 0's bounded wait for the schedule copy; if it
+// gives up, the CTA raises the context's error flag and stops.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -36,6 +38,7 @@ namespace {
 constexpr uint32_t kMaxThreads = kTiledMaxWarps * 32;
 constexpr uint32_t kWaitLimit = 2000;
 constexpr uint32_t kWaitHintNs = 1000000;
+constexpr uint32_t P = kTiledPrefetch;
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p)
 {
@@ -88,30 +91,92 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity)
     return false;
 }
 
-// Per-thread asynchronous copy of one lane's C words into shared memory.
-template <int C>
-__device__ __forceinline__ void cp_async(uint32_t dst, const uint64_t *src)
+// Per-thread asynchronous 16-byte copy global -> shared, tracked with
+// commit groups (both addresses 16-byte aligned).
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src)
 {
-    if constexpr (C == 2)
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
-    else
-        asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(dst), "l"(src) : "memory");
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
 
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 
 template <uint32_t N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
-
-// A zero that the compiler cannot see through, computed from `v`: adding it
-// to an address makes the address wait for the load that produced `v`.
-__device__ __forceinline__ uint32_t opaque_zero(uint64_t v)
+__device__ __forceinline__ void cp_async_wait()
 {
-    uint32_t z;
-    asm volatile("and.b32 %0, %1, 0;" : "=r"(z) : "r"((uint32_t)v));
-    return z;
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// L2 policy for plaintexts: each is read once, so they go first when L2
+// needs room (the staged input tiles and the schedule stay).
+__device__ __forceinline__ uint64_t evict_first_policy()
+{
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+// The limb's constants, read from shared memory where they are needed
+// (kept out of registers between uses).
+__device__ __forceinline__ LimbConst load_limb(uint32_t addr)
+{
+    LimbConst m;
+    asm volatile("ld.shared.v2.u64 {%0, %1}, [%2];" : "=l"(m.q), "=l"(m.mu_hi) : "r"(addr));
+    asm volatile("ld.shared.v2.u64 {%0, %1}, [%2+16];" : "=l"(m.mu_lo), "=l"(m.mu64) : "r"(addr));
+    return m;
+}
+
+template <int C>
+struct V {
+    uint64_t x[C];
+};
+
+// one lane's C plaintext words, not cached in L1
+template <int C>
+__device__ __forceinline__ V<C> ldg_stream(const uint64_t *p, uint64_t pol)
+{
+    V<C> v;
+    if constexpr (C == 2)
+        asm("ld.global.nc.L1::no_allocate.L2::cache_hint.v2.u64 {%0, %1}, [%2], %3;"
+            : "=l"(v.x[0]), "=l"(v.x[1])
+            : "l"(p), "l"(pol));
+    else
+        asm("ld.global.nc.L1::no_allocate.L2::cache_hint.u64 %0, [%1], %2;"
+            : "=l"(v.x[0])
+            : "l"(p), "l"(pol));
+    return v;
+}
+
+// shared memory through byte offsets from the dynamic shared array
+template <int C>
+__device__ __forceinline__ V<C> lds(const char *sm, uint32_t off)
+{
+    V<C> v;
+    if constexpr (C == 2) {
+        const ulonglong2 t = *reinterpret_cast<const ulonglong2 *>(sm + off);
+        v.x[0] = t.x;
+        v.x[1] = t.y;
+    } else {
+        v.x[0] = *reinterpret_cast<const uint64_t *>(sm + off);
+    }
+    return v;
+}
+
+template <int C>
+__device__ __forceinline__ void sts(char *sm, uint32_t off, const V<C> &v)
+{
+    if constexpr (C == 2)
+        *reinterpret_cast<ulonglong2 *>(sm + off) = make_ulonglong2(v.x[0], v.x[1]);
+    else
+        *reinterpret_cast<uint64_t *>(sm + off) = v.x[0];
+}
+
+template <int C>
+__device__ __forceinline__ void stg(uint64_t *p, const V<C> &v)
+{
+    if constexpr (C == 2)
+        *reinterpret_cast<ulonglong2 *>(p) = make_ulonglong2(v.x[0], v.x[1]);
+    else
+        *p = v.x[0];
 }
 
 // ---------------------------------------------------------------------------
@@ -136,6 +201,11 @@ struct Arith<false> {
         a.lo = reduce(a, m);
         a.hi = 0;
     }
+    // canonical residue of P - M, each a plain sum within the lazy-sum bound
+    __device__ static uint64_t signed_value(uint64_t p, uint64_t mm, const LimbConst &m)
+    {
+        return rns::sub_mod(rns::reduce64(p, m), rns::reduce64(mm, m), m.q);
+    }
 };
 
 // q < 2^52: every factor in split form (sources in shared memory, the other
@@ -157,364 +227,313 @@ struct Arith<true> {
         a.x = a.lo;  // the middle term x - lo - hi stays 0
         a.hi = 0;
     }
+    // P - M + 64q is below 2^59 (each packed sum reads back below 2^58)
+    __device__ static uint64_t signed_value(uint64_t p, uint64_t mm, const LimbConst &m)
+    {
+        const uint64_t k = (uint64_t)rns::kNarrowSumBudget * m.q;
+        return rns::reduce64(rns::unsplit_sum(p) + k - rns::unsplit_sum(mm), m);
+    }
 };
 
-template <int C>
-struct V {
-    uint64_t x[C];
-};
-
-// shared-memory access through 32-bit addresses
-template <int C>
-__device__ __forceinline__ V<C> lds(uint32_t addr)
-{
-    V<C> v;
-    if constexpr (C == 2)
-        asm volatile("ld.shared.v2.u64 {%0, %1}, [%2];" : "=l"(v.x[0]), "=l"(v.x[1]) : "r"(addr));
-    else
-        asm volatile("ld.shared.u64 %0, [%1];" : "=l"(v.x[0]) : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ uint32_t lds_u32(uint32_t addr)
-{
-    uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
-    return v;
-}
-
-template <int C>
-__device__ __forceinline__ void sts(uint32_t addr, const V<C> &v)
-{
-    if constexpr (C == 2)
-        asm volatile("st.shared.v2.u64 [%0], {%1, %2};" ::"r"(addr), "l"(v.x[0]), "l"(v.x[1]) : "memory");
-    else
-        asm volatile("st.shared.u64 [%0], %1;" ::"r"(addr), "l"(v.x[0]) : "memory");
-}
-
-template <int C>
-__device__ __forceinline__ void stg(uint64_t *p, const V<C> &v)
-{
-    if constexpr (C == 2)
-        *reinterpret_cast<ulonglong2 *>(p) = make_ulonglong2(v.x[0], v.x[1]);
-    else
-        *p = v.x[0];
-}
-
-// Sum of n source tiles (both polys) whose words start at shared address
-// `words`; `src` = this lane's address in the source region.
+// Sum of the n source tiles of one poly named by the 16-bit indices packed
+// two per word from schedule byte offset `wp`; `src` = this lane's offset in
+// the source region plus the poly's offset.  Four tiles per step, their
+// loads independent.  Returns the offset just past the run's words.
 template <int C, uint32_t TB>
-__device__ __forceinline__ void run_sum(uint32_t src, uint32_t words, uint32_t n, V<C> &s0, V<C> &s1)
+__device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32_t wp, uint32_t n, V<C> &s)
 {
+    constexpr uint32_t PB = 2 * TB;
     uint32_t k = 0;
-    for (; k + 2 <= n; k += 2) {
-        const uint32_t o0 = lds_u32(words + 4 * k), o1 = lds_u32(words + 4 * k + 4);
-        const V<C> a0 = lds<C>(src + o0), b0 = lds<C>(src + o1);
-        const V<C> a1 = lds<C>(src + o0 + TB), b1 = lds<C>(src + o1 + TB);
+    for (; k + 4 <= n; k += 4, wp += 8) {
+        const uint32_t w0 = *reinterpret_cast<const uint32_t *>(sm + wp);
+        const uint32_t w1 = *reinterpret_cast<const uint32_t *>(sm + wp + 4);
+        const V<C> a = lds<C>(sm, src + (w0 & 0xffffu) * PB), b = lds<C>(sm, src + (w0 >> 16) * PB);
+        const V<C> c = lds<C>(sm, src + (w1 & 0xffffu) * PB), d = lds<C>(sm, src + (w1 >> 16) * PB);
 #pragma unroll
-        for (int x = 0; x < C; ++x) {
-            s0.x[x] += a0.x[x] + b0.x[x];
-            s1.x[x] += a1.x[x] + b1.x[x];
-        }
+        for (int x = 0; x < C; ++x) s.x[x] += (a.x[x] + b.x[x]) + (c.x[x] + d.x[x]);
+    }
+    for (; k + 2 <= n; k += 2, wp += 4) {
+        const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp);
+        const V<C> a = lds<C>(sm, src + (w & 0xffffu) * PB), b = lds<C>(sm, src + (w >> 16) * PB);
+#pragma unroll
+        for (int x = 0; x < C; ++x) s.x[x] += a.x[x] + b.x[x];
     }
     if (k < n) {
-        const uint32_t o0 = lds_u32(words + 4 * k);
-        const V<C> a0 = lds<C>(src + o0), a1 = lds<C>(src + o0 + TB);
+        const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp);
+        const V<C> a = lds<C>(sm, src + (w & 0xffffu) * PB);
 #pragma unroll
-        for (int x = 0; x < C; ++x) {
-            s0.x[x] += a0.x[x];
-            s1.x[x] += a1.x[x];
-        }
+        for (int x = 0; x < C; ++x) s.x[x] += a.x[x];
+        wp += 4;
     }
+    return wp;
 }
 
-// Signed sum of the segment whose header word is at `hdr` (n_plus | n_minus
-// << 16, then the words), both polys, reduced once to the canonical residue
-// (narrow: from P - M + 64q, below 2^59 since each packed sum is below
-// 2^58).  Returns the shared address just past the segment.
+// Signed sum of the program at byte offset `hdr` (n_plus | n_minus << 16,
+// then the plus run, then the minus run), both polys (one after the other,
+// to keep few values live), as canonical residues.  Returns the offset just
+// past the program.
 template <bool NARROW, int C, uint32_t TB>
-__device__ __forceinline__ uint32_t signed_sum(uint32_t src, uint32_t hdr, const LimbConst &m,
+__device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uint32_t hdr, uint32_t lim,
                                                V<C> &o0, V<C> &o1)
 {
-    const uint32_t h = lds_u32(hdr);
-    const uint32_t np = h & 0xffffu, nm = h >> 16;
-    V<C> p0{}, p1{}, m0{}, m1{};
-    run_sum<C, TB>(src, hdr + 4, np, p0, p1);
-    run_sum<C, TB>(src, hdr + 4 + 4 * np, nm, m0, m1);
+    using A = Arith<NARROW>;
+    const uint32_t h = *reinterpret_cast<const uint32_t *>(sm + hdr);
+    uint32_t wp = 0;
 #pragma unroll
-    for (int x = 0; x < C; ++x) {
-        if constexpr (NARROW) {
-            const uint64_t k = (uint64_t)rns::kNarrowSumBudget * m.q;
-            o0.x[x] = rns::reduce64(rns::unsplit_sum(p0.x[x]) + k - rns::unsplit_sum(m0.x[x]), m);
-            o1.x[x] = rns::reduce64(rns::unsplit_sum(p1.x[x]) + k - rns::unsplit_sum(m1.x[x]), m);
-        } else {
-            o0.x[x] = rns::sub_mod(rns::reduce64(p0.x[x], m), rns::reduce64(m0.x[x], m), m.q);
-            o1.x[x] = rns::sub_mod(rns::reduce64(p1.x[x], m), rns::reduce64(m1.x[x], m), m.q);
-        }
+    for (int c = 0; c < 2; ++c) {
+        V<C> p{}, mm{};
+        wp = run_sum<C, TB>(sm, src + c * TB, hdr + 4, h & 0xffffu, p);
+        wp = run_sum<C, TB>(sm, src + c * TB, wp, h >> 16, mm);
+        const LimbConst m = load_limb(lim);
+        V<C> &o = c ? o1 : o0;
+#pragma unroll
+        for (int x = 0; x < C; ++x) o.x[x] = A::signed_value(p.x[x], mm.x[x], m);
     }
-    return hdr + 4 * (1 + np + nm);
+    return wp;
 }
 
-template <int C, bool NARROW, uint32_t D>
+template <int C, bool NARROW>
 __global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
 {
     using A = Arith<NARROW>;
     using Acc = typename A::Acc;
     constexpr uint32_t T = 32 * C;
     constexpr uint32_t TB = T * 8;  // bytes of one poly's tile
+    constexpr uint32_t PB = 2 * TB; // bytes of one source (c0, c1)
     constexpr uint32_t VB = C * 8;  // bytes of one lane's words in a tile
-    extern __shared__ __align__(16) uint64_t smem[];
+    extern __shared__ __align__(16) char sm[];
     __shared__ int s_abort;
+    __shared__ __align__(16) LimbConst s_limb;
+    const uint32_t lim = smem_addr(&s_limb);
     const uint32_t n_warps = blockDim.x >> 5;
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const uint32_t sch = smem_addr(smem);  // schedule words
     const uint32_t n_buf = a.double_buffer ? 2 : 1;
-    const uint32_t src0 = sch + a.sched_bytes;
+    const uint32_t src0 = a.sched_bytes;  // byte offsets in `sm`
     const uint32_t part_base = src0 + n_buf * a.src_bytes;
-    const uint32_t ring_base = part_base + a.n_part * 2 * TB;
-    const uint32_t bar0 = ring_base + n_warps * D * TB;  // regions 0, 1; schedule
+    const uint32_t bar_off = part_base + a.n_part * PB;  // the schedule copy's mbarrier
+    const uint32_t bar0 = smem_addr(sm) + bar_off;
     const uint32_t total = a.n_limbs * a.tiles_per_limb;
     const uint32_t lane_off = lane * VB;
-    auto sw = [&](uint32_t k) -> uint32_t { return lds_u32(sch + 4 * k); };
+    const uint32_t *sw = reinterpret_cast<const uint32_t *>(sm);
 
     // the schedule, once per CTA
     if (threadIdx.x == 0) {
         mbar_init(bar0, 1);
-        mbar_init(bar0 + 8, 1);
-        mbar_init(bar0 + 16, 1);
-        mbar_expect_tx(bar0 + 16, a.sched_bytes);
+        mbar_expect_tx(bar0, a.sched_bytes);
         for (uint32_t o = 0; o < a.sched_bytes; o += 32768)
-            bulk_g2s(sch + o, reinterpret_cast<const char *>(a.sched) + o, min(32768u, a.sched_bytes - o),
-                     bar0 + 16);
-        s_abort = mbar_wait(bar0 + 16, 0) ? 0 : 1;
+            bulk_g2s(smem_addr(sm) + o, reinterpret_cast<const char *>(a.sched) + o,
+                     min(32768u, a.sched_bytes - o), bar0);
+        s_abort = mbar_wait(bar0, 0) ? 0 : 1;
         if (s_abort) atomicExch(a.err, 1);
     }
     __syncthreads();
     if (s_abort) return;
-    mbar_wait(bar0 + 16, 0);
+    mbar_wait(bar0, 0);  // completed: orders the copied schedule before this thread's reads
+    // the zero tile of each source region (read by NOP operations); published
+    // by the first tile's barrier
+    for (uint32_t i = threadIdx.x; i < n_buf * (PB / 16); i += blockDim.x) {
+        const uint32_t reg = i / (PB / 16), o = i % (PB / 16);
+        *reinterpret_cast<ulonglong2 *>(sm + src0 + reg * a.src_bytes + a.src_bytes - PB + o * 16) =
+            make_ulonglong2(0, 0);
+    }
 
-    // ---- this warp's plaintext ring
-    const uint32_t f_begin = sw(a.o_fetch_off + warp);
-    const uint32_t F = sw(a.o_fetch_off + warp + 1) - f_begin;
-    const uint32_t my_tiles = blockIdx.x < total ? (total - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
-    const uint32_t total_f = F * my_tiles;
-    const uint32_t ring = ring_base + warp * D * TB + lane_off;
-    auto tile_ptl = [&](uint32_t t) -> const uint64_t * {
+    // ---- this warp's operation stream and its plaintext queue
+    const uint32_t wt = a.o_warp + warp * kWarpTableWords;
+    const uint32_t op0 = sw[wt] * 4, n_batches = sw[wt + 1] / P;
+    const uint32_t seg0 = sw[wt + 2] * 4, tg0 = sw[wt + 3];
+    const uint64_t pol = evict_first_policy();
+    const size_t stride_bytes = (size_t)a.pt_stride * 8;
+    auto tile_ptl = [&](uint32_t t) -> const char * {
+        if (t >= total || !a.has_pt) return nullptr;
         const uint32_t l = a.limb0 + t / a.tiles_per_limb, k0 = (t % a.tiles_per_limb) * T;
-        return a.pt + (size_t)l * a.N + k0 + lane * C;
+        return reinterpret_cast<const char *>(a.pt + (size_t)l * a.N + k0 + lane * C);
     };
-    uint32_t p_next = 0, p_k = 0, p_tile = blockIdx.x;
-    const uint64_t *p_ptl = tile_ptl(p_tile);
-    // fetch p_next into its slot (or commit an empty group past the end)
-    auto issue = [&](uint32_t dep) {
-        if (p_next < total_f) {
-            const uint32_t w = sw(f_begin + p_k);
-            cp_async<C>(ring + (p_next % D) * TB + dep, p_ptl + ((uint64_t)w << a.log2N));
-            if (++p_k == F) {
-                p_k = 0;
-                p_tile += gridDim.x;
-                if (p_tile < total) p_ptl = tile_ptl(p_tile);
-            }
-        }
-        cp_async_commit();
-        ++p_next;
+    auto op_word = [&](uint32_t off) -> uint32_t {
+        uint32_t w;
+        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(w) : "r"(smem_addr(sm) + off));
+        return w;
     };
-    for (uint32_t i = 0; i < D; ++i) issue(0);
-    uint32_t c_next = 0;
-    // the next plaintext words of this lane; its slot is refilled D ahead,
-    // after the read has landed (the refill address depends on it)
-    auto consume = [&]() -> V<C> {
-        cp_async_wait<D - 1>();
-        const V<C> v = lds<C>(ring + (c_next % D) * TB);
-        ++c_next;
-        issue(opaque_zero(v.x[0]));
-        return v;
+    // the plaintext words of operation word `w` in the tile at `base` (with
+    // stride 0 and the schedule's own address when there is no next tile: a
+    // harmless valid load)
+    auto fetch = [&](const char *base, size_t stride, uint32_t w) -> V<C> {
+        return ldg_stream<C>(reinterpret_cast<const uint64_t *>(base + (size_t)(w >> kOpPtShift) * stride), pol);
     };
-    // the next two, with one wait
-    auto consume2 = [&](V<C> &v0, V<C> &v1) {
-        cp_async_wait<D - 2>();
-        v0 = lds<C>(ring + (c_next % D) * TB);
-        v1 = lds<C>(ring + ((c_next + 1) % D) * TB);
-        c_next += 2;
-        issue(opaque_zero(v0.x[0]));
-        issue(opaque_zero(v1.x[0]));
-    };
-
-    // thread 0: start the copies of tile `t` into region `r`
-    auto stage = [&](uint32_t t, uint32_t r) {
-        const uint32_t l = a.limb0 + t / a.tiles_per_limb, k0 = (t % a.tiles_per_limb) * T;
-        const uint32_t bar = bar0 + 8 * r;
-        mbar_expect_tx(bar, a.n_in * 2 * TB);
-        const uint32_t dst = src0 + r * a.src_bytes;
-        for (uint32_t s = 0; s < 2 * a.n_in; ++s)
-            bulk_g2s(dst + s * TB, a.in + ((size_t)s * a.L + l) * a.N + k0, TB, bar);
-    };
-
-    uint32_t phase0 = 0, phase1 = 0, buf = 0;
+    V<C> r[P];
     uint32_t tile = blockIdx.x;
-    if (a.n_in && threadIdx.x == 0 && tile < total) stage(tile, 0);
+    const char *cur_ptl = tile_ptl(tile);
+    if (n_batches && tile < total) {
+        const char *b0 = cur_ptl ? cur_ptl : reinterpret_cast<const char *>(a.sched);
+        const size_t s0 = cur_ptl ? stride_bytes : 0;
+#pragma unroll
+        for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, s0, op_word(op0 + 4 * i));
+    }
+
+    // every thread: start its 16-byte asynchronous copies of tile `t`'s
+    // inputs into region `reg` (one commit group per tile)
+    constexpr uint32_t kChunks = TB / 16;  // per source poly
+    const uint32_t n_chunks = 2 * a.n_in * kChunks;
+    auto stage = [&](uint32_t t, uint32_t reg) {
+        const uint32_t l = a.limb0 + t / a.tiles_per_limb, k0 = (t % a.tiles_per_limb) * T;
+        const uint32_t dst = smem_addr(sm) + src0 + reg * a.src_bytes;
+        const char *base = reinterpret_cast<const char *>(a.in + (size_t)l * a.N + k0);
+        const size_t LN8 = (size_t)a.L * a.N * 8;
+        for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x)
+            cp_async16(dst + i * 16, base + (size_t)(i / kChunks) * LN8 + (i % kChunks) * 16);
+        cp_async_commit();
+    };
+
+    uint32_t buf = 0;
+    if (a.n_in && tile < total) stage(tile, 0);
     for (; tile < total; tile += gridDim.x) {
         const uint32_t next = tile + gridDim.x;
+        const char *next_ptl = tile_ptl(next);
         const uint32_t l = a.limb0 + tile / a.tiles_per_limb;
         const uint32_t k0 = (tile % a.tiles_per_limb) * T;
-        const LimbConst m = a.limbs[l];
+        if (threadIdx.x == 0) s_limb = a.limbs[l];  // read after the barrier below
         const uint32_t sb = src0 + buf * a.src_bytes;  // this tile's source region
         const uint32_t src = sb + lane_off;
 
-        // 1. inputs of this tile
+        // 1. inputs of this tile: this thread's copies have landed (the next
+        //    tile's, when started here, may still be in flight); narrow plans
+        //    rewrite them in split form; the barrier publishes them
         if (a.n_in) {
-            if (threadIdx.x == 0) {
-                if (a.double_buffer && next < total) stage(next, buf ^ 1);
-                s_abort = mbar_wait(bar0 + 8 * buf, buf ? phase1 : phase0) ? 0 : 1;
-                if (s_abort) {
-                    atomicExch(a.err, 1);
-                    if (a.double_buffer && next < total) mbar_wait(bar0 + 8 * (buf ^ 1), buf ? phase0 : phase1);
+            if (a.double_buffer && next < total) {
+                stage(next, buf ^ 1);
+                cp_async_wait<1>();
+            } else {
+                cp_async_wait<0>();
+            }
+            if (NARROW) {
+                for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x) {
+                    ulonglong2 *p = reinterpret_cast<ulonglong2 *>(sm + sb + i * 16);
+                    const ulonglong2 x = *p;
+                    *p = make_ulonglong2(A::operand(x.x), A::operand(x.y));
                 }
             }
-            __syncthreads();
-            if (s_abort) {
-                cp_async_wait_all();
-                return;
-            }
-            // the phase has completed: this returns at once and orders the
-            // bulk-copied tiles before this thread's reads
-            mbar_wait(bar0 + 8 * buf, buf ? phase1 : phase0);
-            if (buf) phase1 ^= 1; else phase0 ^= 1;
             if (!a.double_buffer && next < total && warp == 0) {
                 const uint32_t ln = a.limb0 + next / a.tiles_per_limb;
                 const uint32_t kn = (next % a.tiles_per_limb) * T;
                 for (uint32_t s = lane; s < 2 * a.n_in; s += 32)
                     prefetch_l2(a.in + ((size_t)s * a.L + ln) * a.N + kn, TB);
             }
-            if (NARROW) {
-                for (uint32_t i = threadIdx.x; i < a.n_in * 2 * T; i += blockDim.x) {
-                    const uint32_t ad = sb + i * 8;
-                    sts<1>(ad, V<1>{{A::operand(lds<1>(ad).x[0])}});
-                }
-                __syncthreads();
-            }
         }
+        __syncthreads();
 
-        // 2. shared signed sums, children first
+        // 2. materialised shared sums, children first
         for (uint32_t lev = 0; lev < a.n_levels; ++lev) {
-            for (uint32_t x = sw(a.o_level + lev) + warp; x < sw(a.o_level + lev + 1); x += n_warps) {
-                const uint32_t nd = sw(a.o_node_slot + x);
+            for (uint32_t x = sw[a.o_level + lev] + warp; x < sw[a.o_level + lev + 1]; x += n_warps) {
                 V<C> u0, u1;
-                signed_sum<NARROW, C, TB>(src, sch + 4 * sw(a.o_node_prog_off + nd), m, u0, u1);
+                signed_sum<NARROW, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, u0, u1);
 #pragma unroll
                 for (int x2 = 0; x2 < C; ++x2) {
                     u0.x[x2] = A::operand(u0.x[x2]);
                     u1.x[x2] = A::operand(u1.x[x2]);
                 }
-                const uint32_t dst = src + (a.n_in + nd) * 2 * TB;
-                sts<C>(dst, u0);
-                sts<C>(dst + TB, u1);
+                const uint32_t dst = src + (a.n_in + x) * PB;
+                sts<C>(sm, dst, u0);
+                sts<C>(sm, dst + TB, u1);
             }
             __syncthreads();
         }
 
-        // 3. this warp's program
-        uint32_t jp = sch + 4 * sw(a.o_prog_off + warp);
-        const uint32_t jend = sch + 4 * sw(a.o_prog_off + warp + 1);
-        while (jp < jend) {
-            const uint32_t target = lds_u32(jp), hdr = lds_u32(jp + 4);
-            jp += 8;
-            const uint32_t n_seg = hdr & 0xffffu, n_raw = hdr >> 16;
-            Acc acc[2][C];
+        // 3. this warp's operations, in batches of P; the plaintexts of the
+        //    next batch are requested as these are consumed.  SEG and FOLD
+        //    only open a batch and LAST only closes one, so the unrolled body
+        //    has no branch: load, product-accumulate, request.
+        Acc acc[2][C];
 #pragma unroll
-            for (int c = 0; c < 2; ++c)
+        for (int c = 0; c < 2; ++c)
 #pragma unroll
-                for (int x = 0; x < C; ++x) A::zero(acc[c][x]);
-            uint32_t nprod = 0;
-            auto fold = [&]() {
+            for (int x = 0; x < C; ++x) A::zero(acc[c][x]);
+        uint32_t sp = seg0, tp = tg0;
+        for (uint32_t b = 0; b < n_batches; ++b) {
+            const bool wrap = b + 1 == n_batches;
+            const char *nb = wrap ? next_ptl : cur_ptl;
+            size_t ns = stride_bytes;
+            if (!nb) {  // no next tile: a harmless valid load
+                nb = reinterpret_cast<const char *>(a.sched);
+                ns = 0;
+            }
+            const uint32_t cur_off = op0 + b * P * 4, next_off = wrap ? op0 : cur_off + P * 4;
+            const uint32_t first = op_word(cur_off);
+            if (first & kOpFold) {
+                const LimbConst m = load_limb(lim);
 #pragma unroll
                 for (int c = 0; c < 2; ++c)
 #pragma unroll
                     for (int x = 0; x < C; ++x) A::fold(acc[c][x], m);
-                nprod = 1;
-            };
-
-            for (uint32_t sgi = 0; sgi < n_seg; ++sgi) {
+            }
+            V<C> g0, g1;  // the signed sum of this batch's SEG (operand form)
+            const bool seg = first & kOpSeg;
+            if (seg) {
+                sp = signed_sum<NARROW, C, TB>(sm, src, sp, lim, g0, g1);
+#pragma unroll
+                for (int x = 0; x < C; ++x) {
+                    g0.x[x] = A::operand(g0.x[x]);
+                    g1.x[x] = A::operand(g1.x[x]);
+                }
+            }
+#pragma unroll
+            for (uint32_t i = 0; i < P; ++i) {
+                const uint32_t op = i == 0 ? first : op_word(cur_off + 4 * i);
                 V<C> s0, s1;
-                jp = signed_sum<NARROW, C, TB>(src, jp, m, s0, s1);
-                const V<C> g = consume();
-                if (nprod + 1 > a.mac_budget) fold();
+                if (i == 0 && seg) {
+                    s0 = g0;
+                    s1 = g1;
+                } else {
+                    const uint32_t so = src + (op & (kOpMaxSources - 1)) * PB;
+                    s0 = lds<C>(sm, so);
+                    s1 = lds<C>(sm, so + TB);
+                }
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
-                    const uint64_t gx = A::operand(g.x[x]);
-                    A::mac(acc[0][x], gx, A::operand(s0.x[x]));
-                    A::mac(acc[1][x], gx, A::operand(s1.x[x]));
+                    const uint64_t g = A::operand(r[i].x[x]);
+                    A::mac(acc[0][x], g, s0.x[x]);
+                    A::mac(acc[1][x], g, s1.x[x]);
                 }
-                ++nprod;
+                r[i] = fetch(nb, ns, op_word(next_off + 4 * i));
             }
-            // at most mac_budget products may sit in an accumulator: jobs
-            // within the bound (all but extreme ones) skip the per-term checks
-            const bool check = nprod + n_raw > a.mac_budget;
-            uint32_t r = 0;
-            for (; r + 2 <= n_raw; r += 2) {
-                const uint32_t off0 = lds_u32(jp + 4 * r), off1 = lds_u32(jp + 4 * r + 4);
-                V<C> p0, p1;
-                consume2(p0, p1);
-                const V<C> v00 = lds<C>(src + off0), v01 = lds<C>(src + off0 + TB);
-                const V<C> v10 = lds<C>(src + off1), v11 = lds<C>(src + off1 + TB);
-                if (check && nprod + 2 > a.mac_budget) fold();
+            if (op_word(cur_off + 4 * (P - 1)) & kOpLast) {
+                const LimbConst m = load_limb(lim);
+                V<C> y0, y1;
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
-                    const uint64_t q0 = A::operand(p0.x[x]), q1 = A::operand(p1.x[x]);
-                    A::mac(acc[0][x], v00.x[x], q0);
-                    A::mac(acc[1][x], v01.x[x], q0);
-                    A::mac(acc[0][x], v10.x[x], q1);
-                    A::mac(acc[1][x], v11.x[x], q1);
+                    y0.x[x] = A::reduce(acc[0][x], m);
+                    y1.x[x] = A::reduce(acc[1][x], m);
+                    A::zero(acc[0][x]);
+                    A::zero(acc[1][x]);
                 }
-                nprod += 2;
-            }
-            if (r < n_raw) {
-                const uint32_t off = lds_u32(jp + 4 * r);
-                const V<C> pv = consume();
-                const V<C> v0 = lds<C>(src + off), v1 = lds<C>(src + off + TB);
-                if (check && nprod + 1 > a.mac_budget) fold();
-#pragma unroll
-                for (int x = 0; x < C; ++x) {
-                    const uint64_t q = A::operand(pv.x[x]);
-                    A::mac(acc[0][x], v0.x[x], q);
-                    A::mac(acc[1][x], v1.x[x], q);
+                const uint32_t target = sw[tp++];
+                if (target & kPartBit) {
+                    const uint32_t dst = part_base + (target & ~kPartBit) * PB + lane_off;
+                    sts<C>(sm, dst, y0);
+                    sts<C>(sm, dst + TB, y1);
+                } else {
+                    uint64_t *dst = a.out + ((size_t)target * 2 * a.L + l) * a.N + k0 + lane * C;
+                    stg<C>(dst, y0);
+                    stg<C>(dst + (size_t)a.L * a.N, y1);
                 }
-                ++nprod;
-            }
-            jp += 4 * n_raw;
-
-            V<C> y0, y1;
-#pragma unroll
-            for (int x = 0; x < C; ++x) {
-                y0.x[x] = A::reduce(acc[0][x], m);
-                y1.x[x] = A::reduce(acc[1][x], m);
-            }
-            if (target & kPartBit) {
-                const uint32_t dst = part_base + (target & ~kPartBit) * 2 * TB + lane_off;
-                sts<C>(dst, y0);
-                sts<C>(dst + TB, y1);
-            } else {
-                uint64_t *dst = a.out + ((size_t)target * 2 * a.L + l) * a.N + k0 + lane * C;
-                stg<C>(dst, y0);
-                stg<C>(dst + (size_t)a.L * a.N, y1);
             }
         }
+        cur_ptl = next_ptl;
 
         // 4. outputs split across warps: add the partial sums
         if (a.n_comb) {
             __syncthreads();
-            for (uint32_t r = warp; r < a.n_comb; r += n_warps) {
+            const uint64_t q = load_limb(lim).q;
+            for (uint32_t rr = warp; rr < a.n_comb; rr += n_warps) {
                 V<C> y0{}, y1{};
-                for (uint32_t q = sw(a.o_comb_off + r); q < sw(a.o_comb_off + r + 1); ++q) {
-                    const uint32_t ps = part_base + sw(a.o_comb_parts + q) * 2 * TB + lane_off;
-                    const V<C> v0 = lds<C>(ps), v1 = lds<C>(ps + TB);
+                for (uint32_t pi = sw[a.o_comb_off + rr]; pi < sw[a.o_comb_off + rr + 1]; ++pi) {
+                    const uint32_t ps = part_base + sw[a.o_comb_parts + pi] * PB + lane_off;
+                    const V<C> v0 = lds<C>(sm, ps), v1 = lds<C>(sm, ps + TB);
 #pragma unroll
                     for (int x = 0; x < C; ++x) {
-                        y0.x[x] = rns::add_mod(y0.x[x], v0.x[x], m.q);
-                        y1.x[x] = rns::add_mod(y1.x[x], v1.x[x], m.q);
+                        y0.x[x] = rns::add_mod(y0.x[x], v0.x[x], q);
+                        y1.x[x] = rns::add_mod(y1.x[x], v1.x[x], q);
                     }
                 }
-                uint64_t *dst = a.out + ((size_t)sw(a.o_comb_out + r) * 2 * a.L + l) * a.N + k0 + lane * C;
+                uint64_t *dst = a.out + ((size_t)sw[a.o_comb_out + rr] * 2 * a.L + l) * a.N + k0 + lane * C;
                 stg<C>(dst, y0);
                 stg<C>(dst + (size_t)a.L * a.N, y1);
             }
@@ -524,38 +543,33 @@ __global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
         // bulk copies that will overwrite the region
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncthreads();
-        if (a.n_in && !a.double_buffer && next < total && threadIdx.x == 0) stage(next, 0);
+        if (a.n_in && !a.double_buffer && next < total) stage(next, 0);
         buf ^= a.double_buffer;
     }
-    cp_async_wait_all();
 }
 
-template <int C, bool NARROW>
-void *select_depth(uint32_t depth)
+void *select_ptr(int C, bool narrow)
 {
-    return depth == 16 ? reinterpret_cast<void *>(&tiled_kernel<C, NARROW, 16>)
-                       : reinterpret_cast<void *>(&tiled_kernel<C, NARROW, 8>);
-}
-
-void *select_ptr(int C, bool narrow, uint32_t depth)
-{
-    if (C == 2) return narrow ? select_depth<2, true>(depth) : select_depth<2, false>(depth);
-    return narrow ? select_depth<1, true>(depth) : select_depth<1, false>(depth);
+    if (C == 2)
+        return narrow ? reinterpret_cast<void *>(&tiled_kernel<2, true>)
+                      : reinterpret_cast<void *>(&tiled_kernel<2, false>);
+    return narrow ? reinterpret_cast<void *>(&tiled_kernel<1, true>)
+                  : reinterpret_cast<void *>(&tiled_kernel<1, false>);
 }
 
 }  // namespace
 
-int tiled_kernel_attributes(int C, bool narrow, uint32_t depth, cudaFuncAttributes *attr)
+int tiled_kernel_attributes(int C, bool narrow, cudaFuncAttributes *attr)
 {
-    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, depth));
+    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow));
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attributes: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
 
-int tiled_configure_kernel(int C, bool narrow, uint32_t depth, size_t smem)
+int tiled_configure_kernel(int C, bool narrow, size_t smem)
 {
-    cudaError_t e = cudaFuncSetAttribute(select_ptr(C, narrow, depth),
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(select_ptr(C, narrow), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attribute: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
@@ -577,7 +591,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     dim3 grid(std::min(tiles, resident));
     dim3 block(ts->warps * 32);
     cudaStream_t s = (cudaStream_t)stream;
-    void *fn = select_ptr(ts->C, ts->narrow, ts->depth);
+    void *fn = select_ptr(ts->C, ts->narrow);
     void *args[] = {&a};
     cudaError_t e = cudaLaunchKernel(fn, grid, block, args, ts->smem, s);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel launch: %s", cudaGetErrorString(e));

@@ -1,28 +1,30 @@
 // lower_tiled.cpp -- lowering of a validated plan to the tiled kernel's
 // schedule (host side, once per layer).
 //
-// * Shared signed sums (Sec. 4.2 "Sharing Signed Sums") become sources
-//   computed once per tile, in topological levels (children first).  Only
-//   sums reachable from a use are kept.
-// * Each output's used scale groups become segments: the group's signed terms
-//   not covered by a use, plus one source per use (sign sigma), summed and
-//   then multiplied once by gamma (Sec. 4.2 "Grouping Reconstruction
-//   Operations").  Plus and minus operands form two runs, cut so that a run
-//   never exceeds the lazy-sum bound (a cut repeats gamma, which is exact).
+// * Shared signed sums (Sec. 4.2 "Sharing Signed Sums") reachable from a use
+//   are materialised once per tile as extra sources, in topological levels
+//   (children first), as many as shared memory holds: the sums are ranked by
+//   the additions they save, and a sum left out is expanded into its
+//   children wherever it is used (the same residues, a few more additions).
+// * Each output's used scale groups become SEG operations: the group's
+//   signed terms not covered by a use, plus one operand per use (sign
+//   sigma), summed and then multiplied once by gamma (Sec. 4.2 "Grouping
+//   Reconstruction Operations").  Plus and minus runs longer than the
+//   lazy-sum bound are cut into several operations with the same gamma
+//   (gamma*S1 + gamma*S2 = gamma*(S1+S2) mod q).  Each raw term is a RAW
+//   operation.
 // * Outputs are assigned to warps by longest-processing-time first on an
-//   estimated cost; with fewer outputs than warps, each output is split into
+//   estimated cost; an output larger than a warp's fair share is split into
 //   parts whose reduced partial sums are added at the end (exact in Z_q).
-// * Each warp gets a program (its jobs' words) and a fetch list (the
-//   plaintext tiles it consumes, in order); the whole schedule is one word
-//   array the kernel copies into shared memory.
-// * Shape: 2 or 1 coefficients per lane, 8 or 16 warps per CTA, 16 or 8
-//   plaintext tiles in flight per warp, and two source buffers (the next
-//   tile staged during this one) when they fit; chosen to keep enough bytes
-//   in flight per SM.  Plans whose moduli are all below 2^52 use the
-//   radix-2^26 arithmetic.
+// * Shape: 2 or 1 coefficients per lane, 4 to 16 warps per CTA, one or two
+//   source regions; the lowering estimates each shape's time per tile from
+//   its instruction, multiplier, shared-memory and HBM demand and keeps the
+//   fastest.  Plans whose moduli are all below 2^52 use the radix-2^26
+//   arithmetic.
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -32,226 +34,553 @@
 
 namespace {
 
-struct OutWork {
-    struct Seg {
-        uint32_t scale_pt;
-        std::vector<uint32_t> plus, minus;  // source indices
-    };
-    std::vector<Seg> segs;
-    std::vector<std::pair<uint32_t, uint32_t>> raws;  // (input, pt)
-    uint64_t cost() const
-    {
-        uint64_t c = 4 * raws.size();
-        for (auto &s : segs) c += s.plus.size() + s.minus.size() + 6;
-        return c;
-    }
+constexpr uint32_t kNodeTag = 0x80000000u;  // operand naming a shared sum
+
+// One SEG operation (after cuts) or the unresolved operand list of a group.
+struct Seg {
+    uint32_t scale_pt;
+    std::vector<uint32_t> plus, minus;  // source indices
 };
 
-// Jobs for W warps: whole outputs assigned largest first to the least-loaded
-// warp; with fewer outputs than warps each output is cut into parts of about
-// equal cost whose reduced partial sums are added at the end.
+struct OutWork {
+    std::vector<Seg> segs;
+    std::vector<std::pair<uint32_t, uint32_t>> raws;  // (source, pt)
+};
+
+// Estimated issue cost of operations, in warp instructions, and of the
+// resources they draw on (see the shape search).
+struct Costs {
+    double raw, seg, operand, last, nop;
+    double imad_op;          // wide multiplies (quarter rate) per product operation
+    double smem_operand;     // shared-memory bytes per source read (both polys)
+};
+
+Costs costs_for(int C, bool narrow)
+{
+    Costs c{};
+    if (narrow) {
+        c = C == 2 ? Costs{34, 70, 8.5, 90, 6, 12, 1024} : Costs{22, 40, 6, 50, 5, 6, 512};
+    } else {
+        c = C == 2 ? Costs{60, 80, 8.5, 110, 6, 32, 1024} : Costs{35, 45, 6, 60, 5, 16, 512};
+    }
+    return c;
+}
+
+double work_cost(const OutWork &w, const Costs &k)
+{
+    double c = k.last + k.raw * (double)w.raws.size();
+    for (auto &s : w.segs) c += k.seg + k.operand * (double)(s.plus.size() + s.minus.size());
+    // NOP padding: each SEG opens a batch, the job fills its last one
+    const size_t ops = w.segs.size() + w.raws.size();
+    const size_t P = kTiledPrefetch;
+    size_t slots = 0;
+    if (w.segs.empty()) {
+        slots = (w.raws.size() + P - 1) / P * P;
+    } else {
+        slots = (w.segs.size() - 1) * P + (1 + w.raws.size() + P - 1) / P * P;
+    }
+    c += k.nop * (double)(std::max(slots, std::max<size_t>(ops, 1)) - ops);
+    return c;
+}
+
+struct Job {
+    uint32_t target;
+    OutWork w;
+};
+
 struct JobPlan {
-    struct Job {
-        uint32_t target;
-        OutWork w;
-    };
     std::vector<std::vector<Job>> per_warp;
     std::vector<uint32_t> comb_off, comb_out, comb_parts;
     uint32_t n_part = 0;
 };
 
-JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t n_out, uint32_t W)
+// Cut `w` into P parts of about equal cost (segments are cut between
+// operands; each piece keeps its gamma).
+std::vector<OutWork> split_work(const OutWork &w, uint32_t P, const Costs &k)
+{
+    std::vector<OutWork> chunk(P);
+    const double per = work_cost(w, k) / P;
+    uint32_t cur = 0;
+    double acc = 0;
+    auto advance = [&](double add) {
+        if (acc + add > per && acc > 0 && cur + 1 < P) {
+            ++cur;
+            acc = 0;
+        }
+        acc += add;
+    };
+    for (auto &sg : w.segs) {
+        advance(k.seg);
+        int open = -1;
+        auto add = [&](uint32_t src, bool minus) {
+            advance(k.operand);
+            if (open != (int)cur) {
+                chunk[cur].segs.push_back({sg.scale_pt, {}, {}});
+                open = (int)cur;
+            }
+            (minus ? chunk[cur].segs.back().minus : chunk[cur].segs.back().plus).push_back(src);
+        };
+        for (uint32_t s : sg.plus) add(s, false);
+        for (uint32_t s : sg.minus) add(s, true);
+    }
+    for (auto &r : w.raws) {
+        advance(k.raw);
+        chunk[cur].raws.push_back(r);
+    }
+    return chunk;
+}
+
+// Jobs for W warps: every output worth splitting is cut into `split` parts
+// (more if it costs more than a fair share, total / W), then all jobs are
+// assigned largest first to the least-loaded warp.  `makespan` receives the
+// largest warp load.
+JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Costs &k, uint32_t split,
+                         double &makespan)
 {
     JobPlan jp;
-    std::vector<JobPlan::Job> jobs;
+    std::vector<Job> jobs;
     jp.comb_off.assign(1, 0);
-    const uint32_t parts = n_out >= W ? 1 : W / std::max<uint32_t>(n_out, 1);
-    for (uint32_t j = 0; j < n_out; ++j) {
-        const OutWork &w = work[j];
-        const uint64_t c = w.cost();
-        const uint32_t P = (uint32_t)std::max<uint64_t>(1, std::min<uint64_t>(parts, c / 16));
-        if (P == 1) {
-            jobs.push_back({j, w});
+    double total = 0;
+    for (auto &w : work) total += work_cost(w, k);
+    const double share = total / W;
+    for (uint32_t j = 0; j < work.size(); ++j) {
+        const double c = work_cost(work[j], k);
+        uint32_t P = (uint32_t)std::max(1.0, std::round(c / std::max(share, 1.0)));
+        P = std::min(W, std::max(P, split));
+        // a part must be worth its partial slot and final addition
+        if (P <= 1 || c < 4 * k.last) {
+            jobs.push_back({j, work[j]});
             continue;
         }
-        std::vector<OutWork> chunk(P);
-        const uint64_t per = (c + P - 1) / P;
-        uint32_t cur = 0;
-        uint64_t acc = 0;
-        auto advance = [&](uint64_t add) {
-            if (acc + add > per && acc > 0 && cur + 1 < P) {
-                ++cur;
-                acc = 0;
-            }
-            acc += add;
-        };
-        for (auto &sg : w.segs) {
-            advance(6);
-            int open = -1;
-            auto add = [&](uint32_t src, bool minus) {
-                advance(1);
-                if (open != (int)cur) {
-                    chunk[cur].segs.push_back({sg.scale_pt, {}, {}});
-                    open = (int)cur;
-                }
-                (minus ? chunk[cur].segs.back().minus : chunk[cur].segs.back().plus).push_back(src);
-            };
-            for (uint32_t s : sg.plus) add(s, false);
-            for (uint32_t s : sg.minus) add(s, true);
-        }
-        for (auto &r : w.raws) {
-            advance(4);
-            chunk[cur].raws.push_back(r);
-        }
+        std::vector<OutWork> chunk = split_work(work[j], P, k);
         jp.comb_out.push_back(j);
-        for (uint32_t q = 0; q < P; ++q) {
-            if (chunk[q].segs.empty() && chunk[q].raws.empty()) continue;
-            jobs.push_back({kPartBit | jp.n_part, chunk[q]});
+        for (auto &ch : chunk) {
+            if (ch.segs.empty() && ch.raws.empty()) continue;
+            jobs.push_back({kPartBit | jp.n_part, std::move(ch)});
             jp.comb_parts.push_back(jp.n_part++);
         }
         jp.comb_off.push_back((uint32_t)jp.comb_parts.size());
     }
     std::vector<uint32_t> order(jobs.size());
     std::iota(order.begin(), order.end(), 0);
-    std::stable_sort(order.begin(), order.end(),
-                     [&](uint32_t a, uint32_t b) { return jobs[a].w.cost() > jobs[b].w.cost(); });
-    std::vector<uint64_t> load(W, 0);
+    std::vector<double> jc(jobs.size());
+    for (size_t i = 0; i < jobs.size(); ++i) jc[i] = work_cost(jobs[i].w, k);
+    std::stable_sort(order.begin(), order.end(), [&](uint32_t a, uint32_t b) { return jc[a] > jc[b]; });
+    std::vector<double> load(W, 0);
     jp.per_warp.assign(W, {});
     for (uint32_t o : order) {
         const uint32_t wi = (uint32_t)(std::min_element(load.begin(), load.end()) - load.begin());
-        jp.per_warp[wi].push_back(jobs[o]);
-        load[wi] += jobs[o].w.cost() + 1;
+        jp.per_warp[wi].push_back(std::move(jobs[o]));
+        load[wi] += jc[o];
     }
+    makespan = *std::max_element(load.begin(), load.end());
     return jp;
 }
 
-// Append one scale group's segments (runs of at most `budget` words) to a
-// warp program and its gamma fetches to the fetch list.
-void put_group(std::vector<uint32_t> &prog, std::vector<uint32_t> &fetch, const OutWork::Seg &sg,
-               uint32_t L, uint32_t budget, uint32_t pair_bytes, uint32_t &n_seg)
+// The split (1 to 4 parts per output) with the smallest largest warp load;
+// a finer split must gain at least 3% to be taken.
+JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t W, const Costs &k)
 {
-    size_t pb = 0, mb = 0;
-    do {
-        const size_t pe = std::min(sg.plus.size(), pb + budget);
-        const size_t me = std::min(sg.minus.size(), mb + budget);
-        prog.push_back((uint32_t)(pe - pb) | ((uint32_t)(me - mb) << 16));
-        for (size_t i = pb; i < pe; ++i) prog.push_back(sg.plus[i] * pair_bytes);
-        for (size_t i = mb; i < me; ++i) prog.push_back(sg.minus[i] * pair_bytes);
-        fetch.push_back(sg.scale_pt * L);
-        ++n_seg;
-        pb = pe;
-        mb = me;
-    } while (pb < sg.plus.size() || mb < sg.minus.size());
+    double best_ms = 0;
+    JobPlan best = build_jobs_split(work, W, k, 1, best_ms);
+    for (uint32_t split = 2; split <= 4; ++split) {
+        double ms = 0;
+        JobPlan jp = build_jobs_split(work, W, k, split, ms);
+        if (ms < 0.97 * best_ms) {
+            best_ms = ms;
+            best = std::move(jp);
+        }
+    }
+    return best;
 }
 
-// The whole schedule as one word array (see tiled.h).
+// Program words of a signed sum: n_plus | n_minus << 16, then each run as
+// 16-bit indices, two per word.
+void put_program(std::vector<uint32_t> &w, const std::vector<uint32_t> &plus, const std::vector<uint32_t> &minus)
+{
+    w.push_back((uint32_t)plus.size() | ((uint32_t)minus.size() << 16));
+    for (const auto *run : {&plus, &minus})
+        for (size_t i = 0; i < run->size(); i += 2)
+            w.push_back((*run)[i] | (i + 1 < run->size() ? (*run)[i + 1] << 16 : 0u));
+}
+
+// The whole schedule (see tiled.h).
 struct Sched {
     std::vector<uint32_t> w;
-    uint32_t o_level, o_node_slot, o_node_prog_off, o_prog_off, o_fetch_off, o_comb_off, o_comb_out,
-        o_comb_parts;
+    uint32_t o_level = 0, o_node_off = 0, o_warp = 0, o_comb_off = 0, o_comb_out = 0, o_comb_parts = 0;
+    uint64_t pt_ops = 0;  // plaintext tiles fetched per tile
 };
 
-Sched encode(const JobPlan &jp, const std::vector<uint32_t> &node_level_off,
-             const std::vector<uint32_t> &node_slots, const std::vector<OutWork::Seg> &node_seg,
-             uint32_t W, uint32_t L, uint32_t budget, uint32_t pair_bytes)
+void pad4(std::vector<uint32_t> &w)
+{
+    while (w.size() % 4) w.push_back(0);
+}
+
+Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const std::vector<Seg> &nodes, uint32_t W,
+             uint32_t mac_budget, uint32_t zero_index)
 {
     Sched sc;
     auto &w = sc.w;
-    auto put = [&](const std::vector<uint32_t> &v) { w.insert(w.end(), v.begin(), v.end()); };
-    sc.o_level = (uint32_t)w.size();
-    put(node_level_off);
-    sc.o_node_slot = (uint32_t)w.size();
-    put(node_slots);
-    // node programs: offsets table then programs
-    sc.o_node_prog_off = (uint32_t)w.size();
-    const size_t n_nodes = node_seg.size();
-    w.resize(w.size() + n_nodes + 1);
-    for (size_t k = 0; k < n_nodes; ++k) {
-        w[sc.o_node_prog_off + k] = (uint32_t)w.size();
-        const OutWork::Seg &sg = node_seg[k];
-        w.push_back((uint32_t)sg.plus.size() | ((uint32_t)sg.minus.size() << 16));
-        for (uint32_t s : sg.plus) w.push_back(s * pair_bytes);
-        for (uint32_t s : sg.minus) w.push_back(s * pair_bytes);
+    sc.o_level = 0;
+    w.insert(w.end(), level_off.begin(), level_off.end());
+    sc.o_node_off = (uint32_t)w.size();
+    w.resize(w.size() + nodes.size());
+    for (size_t k = 0; k < nodes.size(); ++k) {
+        w[sc.o_node_off + k] = (uint32_t)w.size();
+        put_program(w, nodes[k].plus, nodes[k].minus);
     }
-    w[sc.o_node_prog_off + n_nodes] = (uint32_t)w.size();
-    // warp programs and fetch lists
-    std::vector<std::vector<uint32_t>> progs(W), fetches(W);
+    pad4(w);
+    sc.o_warp = (uint32_t)w.size();
+    w.resize(w.size() + (size_t)W * kWarpTableWords);
+    std::vector<std::vector<uint32_t>> ops(W), segw(W), tgt(W);
+    constexpr uint32_t P = kTiledPrefetch;
+    const uint32_t zero_src = zero_index;
     for (uint32_t wi = 0; wi < W; ++wi) {
-        for (const auto &jb : jp.per_warp[wi]) {
-            auto &prog = progs[wi];
-            prog.push_back(jb.target);
-            const size_t hdr = prog.size();
-            prog.push_back(0);
-            uint32_t n_seg = 0;
-            for (const auto &sg : jb.w.segs) put_group(prog, fetches[wi], sg, L, budget, pair_bytes, n_seg);
-            for (const auto &r : jb.w.raws) {
-                prog.push_back(r.first * pair_bytes);
-                fetches[wi].push_back(r.second * L);
+        auto &o = ops[wi];
+        for (const Job &jb : jp.per_warp[wi]) {
+            const size_t first = o.size();
+            const auto &raws = jb.w.raws;
+            size_t r = 0;
+            auto raw_op = [&]() { return (raws[r].second << kOpPtShift) | raws[r].first; };
+            // each SEG opens a batch; the batch before it is filled with raw
+            // terms where there are any left
+            for (const Seg &sg : jb.w.segs) {
+                while ((o.size() - first) % P) o.push_back(r < raws.size() ? raw_op() : (kOpNop | zero_src)), r += r < raws.size();
+                put_program(segw[wi], sg.plus, sg.minus);
+                o.push_back((sg.scale_pt << kOpPtShift) | kOpSeg);
             }
-            prog[hdr] = n_seg | ((uint32_t)jb.w.raws.size() << 16);
+            for (; r < raws.size(); ++r) o.push_back(raw_op());
+            if (o.size() == first) o.push_back(kOpNop | zero_src);  // an output with no terms
+            while ((o.size() - first) % P) o.push_back(kOpNop | zero_src);
+            o.back() |= kOpLast;
+            // at most mac_budget products in an accumulator between reductions
+            uint32_t nprod = 0;
+            for (size_t b = first; b < o.size(); b += P) {
+                uint32_t cnt = 0;
+                for (size_t i = b; i < b + P; ++i) cnt += (o[i] & kOpNop) ? 0 : 1;
+                if (nprod + cnt > mac_budget) {
+                    o[b] |= kOpFold;
+                    nprod = 1;
+                }
+                nprod += cnt;
+                sc.pt_ops += cnt;
+            }
+            tgt[wi].push_back(jb.target);
+        }
+        // a NOP loads a plaintext tile that another operation of its batch (or
+        // the nearest earlier one) loads too
+        uint32_t last_pt = 0;
+        for (size_t b = 0; b < o.size(); b += P) {
+            for (size_t i = b; i < b + P; ++i)
+                if (!(o[i] & kOpNop)) {
+                    last_pt = o[i] >> kOpPtShift;
+                    break;
+                }
+            for (size_t i = b; i < b + P; ++i)
+                if (o[i] & kOpNop) o[i] = (o[i] & ((1u << kOpPtShift) - 1)) | (last_pt << kOpPtShift);
         }
     }
-    sc.o_prog_off = (uint32_t)w.size();
-    w.resize(w.size() + W + 1);
     for (uint32_t wi = 0; wi < W; ++wi) {
-        w[sc.o_prog_off + wi] = (uint32_t)w.size();
-        put(progs[wi]);
+        pad4(w);
+        w[sc.o_warp + wi * kWarpTableWords + 0] = (uint32_t)w.size();
+        w[sc.o_warp + wi * kWarpTableWords + 1] = (uint32_t)ops[wi].size();
+        w.insert(w.end(), ops[wi].begin(), ops[wi].end());
     }
-    w[sc.o_prog_off + W] = (uint32_t)w.size();
-    sc.o_fetch_off = (uint32_t)w.size();
-    w.resize(w.size() + W + 1);
     for (uint32_t wi = 0; wi < W; ++wi) {
-        w[sc.o_fetch_off + wi] = (uint32_t)w.size();
-        put(fetches[wi]);
+        w[sc.o_warp + wi * kWarpTableWords + 2] = (uint32_t)w.size();
+        w.insert(w.end(), segw[wi].begin(), segw[wi].end());
     }
-    w[sc.o_fetch_off + W] = (uint32_t)w.size();
+    for (uint32_t wi = 0; wi < W; ++wi) {
+        w[sc.o_warp + wi * kWarpTableWords + 3] = (uint32_t)w.size();
+        w.insert(w.end(), tgt[wi].begin(), tgt[wi].end());
+    }
     sc.o_comb_off = (uint32_t)w.size();
-    put(jp.comb_off);
+    w.insert(w.end(), jp.comb_off.begin(), jp.comb_off.end());
     sc.o_comb_out = (uint32_t)w.size();
-    put(jp.comb_out);
+    w.insert(w.end(), jp.comb_out.begin(), jp.comb_out.end());
     sc.o_comb_parts = (uint32_t)w.size();
-    put(jp.comb_parts);
-    while (w.size() % 4) w.push_back(0);  // a multiple of 16 bytes
+    w.insert(w.end(), jp.comb_parts.begin(), jp.comb_parts.end());
+    pad4(w);  // a multiple of 16 bytes
     return sc;
 }
 
-int upload_blob(TiledSchedule *ts, const std::vector<std::pair<const void *, size_t>> &parts,
-                std::vector<size_t> &off)
-{
-    size_t total = 0;
-    off.clear();
-    for (auto &pr : parts) {
-        off.push_back(total);
-        total += (pr.second + 255) & ~(size_t)255;
+// Shared sums of the plan (those reachable from a use), their unresolved
+// operand lists, and what keeping each one saves.
+struct NodeInfo {
+    std::vector<uint32_t> ids;                                  // plan node ids in index order
+    std::vector<std::vector<std::pair<uint32_t, int>>> kids;    // per plan node: (operand, sign)
+    std::vector<double> benefit;                                // per plan node
+};
+
+// Resolution of operands against a set of kept shared sums.
+struct Resolver {
+    const NodeInfo &ni;
+    const std::vector<int32_t> &slot;  // per plan node: source index if kept, else -1
+    void add(uint32_t opnd, int sign, std::vector<uint32_t> &plus, std::vector<uint32_t> &minus) const
+    {
+        if (!(opnd & kNodeTag)) {
+            (sign < 0 ? minus : plus).push_back(opnd);
+            return;
+        }
+        const uint32_t k = opnd & ~kNodeTag;
+        if (slot[k] >= 0) {
+            (sign < 0 ? minus : plus).push_back((uint32_t)slot[k]);
+            return;
+        }
+        for (auto &c : ni.kids[k]) add(c.first, sign * c.second, plus, minus);
     }
-    if (!total) total = 256;
-    std::vector<uint8_t> host(total, 0);
-    for (size_t i = 0; i < parts.size(); ++i)
-        if (parts[i].second) memcpy(host.data() + off[i], parts[i].first, parts[i].second);
-    cudaError_t e = cudaMalloc(&ts->sched.blob, total);
+};
+
+struct Lowered {
+    std::vector<OutWork> work;      // resolved, runs cut to the lazy-sum bound
+    std::vector<Seg> nodes;         // kept sums in slot order
+    std::vector<uint32_t> level_off;
+    uint32_t n_levels = 0;
+};
+
+// Resolve every operand list against the `keep` set (plan node ids, at most
+// `keep_n` of them taken from `rank` order); a kept sum whose own runs would
+// exceed `budget` is dropped, since it must be one lazy sum.  Scale groups
+// are cut into pieces whose plus and minus runs are at most `budget` long.
+Lowered resolve(const HostPlan &hp, const NodeInfo &ni, const std::vector<OutWork> &groups,
+                const std::vector<uint32_t> &rank, uint32_t keep_n, uint32_t budget)
+{
+    const uint32_t n_in = hp.n_in;
+    std::vector<uint8_t> kept(hp.n_nodes, 0);
+    for (uint32_t i = 0; i < keep_n && i < rank.size(); ++i) kept[rank[i]] = 1;
+    std::vector<int32_t> slot(hp.n_nodes, -1);
+    std::vector<uint32_t> level(hp.n_nodes, 0);
+    Lowered lw;
+    for (bool changed = true; changed;) {
+        changed = false;
+        // slots in index order (children first: a child's index is lower)
+        std::fill(slot.begin(), slot.end(), -1);
+        uint32_t n = 0;
+        for (uint32_t k : ni.ids)
+            if (kept[k]) slot[k] = (int32_t)(n_in + n++);
+        Resolver rv{ni, slot};
+        for (uint32_t k : ni.ids) {
+            if (!kept[k]) continue;
+            Seg s;
+            for (auto &c : ni.kids[k]) rv.add(c.first, c.second, s.plus, s.minus);
+            if (s.plus.size() > budget || s.minus.size() > budget) {
+                kept[k] = 0;
+                changed = true;
+                break;
+            }
+        }
+    }
+    Resolver rv{ni, slot};
+    // kept sums ordered by level, then index
+    std::vector<uint32_t> order;
+    for (uint32_t k : ni.ids) {
+        if (!kept[k]) continue;
+        uint32_t lev = 0;
+        std::vector<uint32_t> stack;
+        for (auto &c : ni.kids[k]) stack.push_back(c.first);
+        while (!stack.empty()) {  // kept descendants reached through dropped sums
+            const uint32_t o = stack.back();
+            stack.pop_back();
+            if (!(o & kNodeTag)) continue;
+            const uint32_t c = o & ~kNodeTag;
+            if (kept[c]) lev = std::max(lev, level[c] + 1);
+            else for (auto &g : ni.kids[c]) stack.push_back(g.first);
+        }
+        level[k] = lev;
+        lw.n_levels = std::max(lw.n_levels, lev + 1);
+        order.push_back(k);
+    }
+    std::stable_sort(order.begin(), order.end(), [&](uint32_t a, uint32_t b) { return level[a] < level[b]; });
+    // renumber slots in level order
+    std::vector<int32_t> slot2(hp.n_nodes, -1);
+    for (uint32_t i = 0; i < order.size(); ++i) slot2[order[i]] = (int32_t)(n_in + i);
+    Resolver rv2{ni, slot2};
+    lw.level_off.assign(lw.n_levels + 1, 0);
+    for (uint32_t k : order) {
+        Seg s;
+        for (auto &c : ni.kids[k]) rv2.add(c.first, c.second, s.plus, s.minus);
+        lw.nodes.push_back(std::move(s));
+        ++lw.level_off[level[k] + 1];
+    }
+    for (uint32_t l = 0; l < lw.n_levels; ++l) lw.level_off[l + 1] += lw.level_off[l];
+    (void)rv;
+    lw.work.resize(groups.size());
+    for (size_t j = 0; j < groups.size(); ++j) {
+        OutWork &o = lw.work[j];
+        o.raws = groups[j].raws;
+        for (const Seg &g : groups[j].segs) {
+            // g.plus holds tagged operands with their signs folded in: plus and minus lists
+            Seg s;
+            s.scale_pt = g.scale_pt;
+            for (uint32_t op : g.plus) rv2.add(op, +1, s.plus, s.minus);
+            for (uint32_t op : g.minus) rv2.add(op, -1, s.plus, s.minus);
+            if (s.plus.empty() && s.minus.empty()) continue;
+            size_t pb = 0, mb = 0;
+            do {  // runs of at most `budget` words
+                const size_t pe = std::min(s.plus.size(), pb + budget);
+                const size_t me = std::min(s.minus.size(), mb + budget);
+                Seg piece;
+                piece.scale_pt = s.scale_pt;
+                piece.plus.assign(s.plus.begin() + pb, s.plus.begin() + pe);
+                piece.minus.assign(s.minus.begin() + mb, s.minus.begin() + me);
+                o.segs.push_back(std::move(piece));
+                pb = pe;
+                mb = me;
+            } while (pb < s.plus.size() || mb < s.minus.size());
+        }
+    }
+    return lw;
+}
+
+int upload_blob(TiledSchedule *ts, const std::vector<uint32_t> &words)
+{
+    const size_t bytes = std::max<size_t>(words.size() * 4, 256);
+    cudaError_t e = cudaMalloc(&ts->sched.blob, bytes);
     if (e != cudaSuccess) return set_error(FIONA_ERR_NOMEM, "tiled schedule: %s", cudaGetErrorString(e));
-    ts->sched.bytes = total;
-    e = cudaMemcpy(ts->sched.blob, host.data(), total, cudaMemcpyHostToDevice);
+    ts->sched.bytes = bytes;
+    e = cudaMemcpy(ts->sched.blob, words.data(), words.size() * 4, cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled schedule: %s", cudaGetErrorString(e));
     return FIONA_OK;
+}
+
+// Walk the schedule words exactly as the kernel does and check every index
+// and offset it will use: plaintexts, sources, partial slots, outputs, the
+// ends of each stream, alignment, and the shared-memory layout.  Returns an
+// explanation of the first violation, or null.
+const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, uint32_t W, uint32_t n_out,
+                           uint32_t n_pt, size_t smem, uint32_t PB)
+{
+    const size_t nw = w.size();
+    if (a.sched_bytes != nw * 4 || a.sched_bytes % 16) return "schedule size";
+    const uint32_t n_src = a.n_in + a.n_nodes, zero = n_src;  // the zero tile follows the sources
+    if (n_src + 1 > kOpMaxSources) return "too many sources";
+    if ((size_t)a.sched_bytes + (size_t)(a.double_buffer ? 2 : 1) * a.src_bytes + (size_t)a.n_part * PB + 24 >
+        smem)
+        return "shared-memory layout";
+    if (a.src_bytes != (n_src + 1) * PB) return "source region size";
+    auto at = [&](size_t i, uint32_t &v) {
+        if (i >= nw) return false;
+        v = w[i];
+        return true;
+    };
+    // a signed-sum program at word `o` whose indices must be below `lim`
+    auto program = [&](size_t o, uint32_t lim, size_t end, size_t &next) -> bool {
+        uint32_t h;
+        if (o >= end || !at(o, h)) return false;
+        const uint32_t np = h & 0xffffu, nm = h >> 16;
+        size_t p = o + 1;
+        for (uint32_t n : {np, nm}) {
+            for (uint32_t i = 0; i < n; i += 2) {
+                uint32_t x;
+                if (p >= end || !at(p, x)) return false;
+                if ((x & 0xffffu) >= lim) return false;
+                if (i + 1 < n && (x >> 16) >= lim) return false;
+                ++p;
+            }
+        }
+        next = p;
+        return true;
+    };
+    // levels and node programs
+    for (uint32_t l = 0; l <= a.n_levels; ++l) {
+        uint32_t v;
+        if (!at(a.o_level + l, v) || v > a.n_nodes) return "level table";
+        if (l > 0 && v < w[a.o_level + l - 1]) return "level order";
+    }
+    if (a.n_levels && w[a.o_level + a.n_levels] != a.n_nodes) return "level table end";
+    for (uint32_t l = 0; l < a.n_levels; ++l)
+        for (uint32_t x = w[a.o_level + l]; x < w[a.o_level + l + 1]; ++x) {
+            uint32_t off;
+            size_t next;
+            // a node reads inputs and nodes of lower levels only
+            if (!at(a.o_node_off + x, off) || !program(off, a.n_in + w[a.o_level + l], a.o_warp, next))
+                return "node program";
+        }
+    // warp streams
+    for (uint32_t wi = 0; wi < W; ++wi) {
+        const size_t t = a.o_warp + (size_t)wi * kWarpTableWords;
+        if (t + kWarpTableWords > nw) return "warp table";
+        const uint32_t op0 = w[t], n_ops = w[t + 1], seg0 = w[t + 2], tg0 = w[t + 3];
+        if (op0 % 4 || n_ops % kTiledPrefetch || (size_t)op0 + n_ops > nw) return "op stream";
+        size_t sp = seg0, tp = tg0;
+        const size_t seg_end = wi + 1 < W ? w[t + kWarpTableWords + 2] : w[a.o_warp + 3];
+        const size_t tg_end = wi + 1 < W ? w[t + kWarpTableWords + 3] : a.o_comb_off;
+        bool open = false;
+        for (uint32_t f = 0; f < n_ops; ++f) {
+            const uint32_t op = w[op0 + f];
+            const uint32_t pos = f % kTiledPrefetch;
+            if ((op & (kOpSeg | kOpFold)) && pos != 0) return "SEG or FOLD inside a batch";
+            if ((op & kOpLast) && pos != kTiledPrefetch - 1) return "LAST inside a batch";
+            // every operation loads a plaintext tile, NOPs included
+            if ((op >> kOpPtShift) >= std::max<uint32_t>(n_pt, 1)) return "plaintext index";
+            if (op & kOpNop) {
+                if (op & kOpSeg) return "SEG marked NOP";
+                if ((op & (kOpMaxSources - 1)) != zero) return "NOP source";
+            } else if (op & kOpSeg) {
+                size_t next;
+                if (!program(sp, n_src, seg_end, next)) return "segment program";
+                sp = next;
+                open = true;
+            } else {
+                if ((op & (kOpMaxSources - 1)) >= n_src) return "source index";
+                open = true;
+            }
+            if (op & kOpLast) {
+                uint32_t tg;
+                if (tp >= tg_end || !at(tp, tg)) return "target stream";
+                ++tp;
+                if (tg & kPartBit) {
+                    if ((tg & ~kPartBit) >= a.n_part) return "partial slot";
+                } else if (tg >= n_out) {
+                    return "output index";
+                }
+                open = false;
+            }
+        }
+        if (open) return "job without LAST";
+        if (sp != seg_end) return "segment stream length";
+        if (tp != tg_end) return "target stream length";
+    }
+    // combine lists
+    for (uint32_t r = 0; r <= a.n_comb; ++r) {
+        uint32_t v;
+        if (!at(a.o_comb_off + r, v)) return "combine table";
+    }
+    for (uint32_t r = 0; r < a.n_comb; ++r) {
+        uint32_t o;
+        if (!at(a.o_comb_out + r, o) || o >= n_out) return "combine output";
+        for (uint32_t q = w[a.o_comb_off + r]; q < w[a.o_comb_off + r + 1]; ++q) {
+            uint32_t ps;
+            if (!at(a.o_comb_parts + q, ps) || ps >= a.n_part) return "combine part";
+        }
+    }
+    return nullptr;
 }
 
 }  // namespace
 
 // kernel_tiled.cu
-int tiled_configure_kernel(int C, bool narrow, uint32_t depth, size_t smem);
-int tiled_kernel_attributes(int C, bool narrow, uint32_t depth, cudaFuncAttributes *attr);
+int tiled_configure_kernel(int C, bool narrow, size_t smem);
+int tiled_kernel_attributes(int C, bool narrow, cudaFuncAttributes *attr);
 
 int lower_tiled(fiona_plan *p)
 {
     const HostPlan &hp = p->hp;
     const fiona_ctx *ctx = p->ctx;
     const bool narrow = ctx->q_max < (1ull << 52);
+    const bool device = ctx->device != FIONA_DEVICE_NONE;
     // lazy-sum bound in words: 64 split words (rns.cuh), or
     // floor((2^64-1)/(q-1)) canonical residues
     const uint32_t budget = narrow ? 64u : std::min<uint32_t>(p->signed_budget, 1u << 14);
+    const uint32_t mac_budget = narrow ? 1023u : p->mac_budget;  // rns.cuh: kNarrowMacBudget
 
-    // -- shared sums reachable from a use, numbered in index order (children first)
+    if (hp.n_pt >= kOpMaxPlaintexts)
+        return set_error(FIONA_ERR_ARG, "tiled kernel: more than %u plaintexts", kOpMaxPlaintexts - 1);
+    if (hp.n_in >= kOpMaxSources)
+        return set_error(FIONA_ERR_ARG, "tiled kernel: more than %u inputs", kOpMaxSources - 1);
+
+    // -- shared sums reachable from a use
+    NodeInfo ni;
     std::vector<uint8_t> need(hp.n_nodes, 0);
     for (uint32_t u = 0; u < hp.n_uses; ++u) need[hp.uses[u].node] = 1;
     for (int k = (int)hp.n_nodes - 1; k >= 0; --k) {
@@ -259,50 +588,39 @@ int lower_tiled(fiona_plan *p)
         for (uint32_t c = hp.node_offsets[k]; c < hp.node_offsets[k + 1]; ++c)
             if (hp.children[c].is_node) need[hp.children[c].ref] = 1;
     }
-    std::vector<int32_t> slot(hp.n_nodes, -1);
-    uint32_t n_slots = 0;
-    for (uint32_t k = 0; k < hp.n_nodes; ++k)
-        if (need[k]) slot[k] = (int32_t)n_slots++;
-    const uint32_t n_in = hp.n_in;
-    std::vector<uint32_t> level(hp.n_nodes, 0);
-    uint32_t n_levels = 0;
-    std::vector<OutWork::Seg> node_seg(n_slots);
+    ni.kids.resize(hp.n_nodes);
+    ni.benefit.assign(hp.n_nodes, 0);
+    std::vector<uint32_t> refs(hp.n_nodes, 0);
+    for (uint32_t u = 0; u < hp.n_uses; ++u) ++refs[hp.uses[u].node];
     for (uint32_t k = 0; k < hp.n_nodes; ++k) {
         if (!need[k]) continue;
-        uint32_t lev = 0;
-        OutWork::Seg &sg = node_seg[(uint32_t)slot[k]];
+        ni.ids.push_back(k);
         for (uint32_t c = hp.node_offsets[k]; c < hp.node_offsets[k + 1]; ++c) {
             const fiona_sum_child &ch = hp.children[c];
-            const uint32_t src = ch.is_node ? n_in + (uint32_t)slot[ch.ref] : ch.ref;
-            if (ch.is_node) lev = std::max(lev, level[ch.ref] + 1);
-            (ch.sign < 0 ? sg.minus : sg.plus).push_back(src);
+            ni.kids[k].push_back({ch.is_node ? (kNodeTag | ch.ref) : ch.ref, ch.sign < 0 ? -1 : 1});
+            if (ch.is_node) ++refs[ch.ref];
         }
-        level[k] = lev;
-        n_levels = std::max(n_levels, lev + 1);
     }
-    for (auto &sg : node_seg)
-        if (sg.plus.size() > budget || sg.minus.size() > budget)
-            return set_error(FIONA_ERR_ARG, "tiled kernel: a shared sum has more than %u children", budget);
-    std::vector<uint32_t> node_level_off(n_levels + 1, 0), node_slots;
-    for (uint32_t lev = 0; lev < n_levels; ++lev) {
-        for (uint32_t k = 0; k < hp.n_nodes; ++k)
-            if (need[k] && level[k] == lev) node_slots.push_back((uint32_t)slot[k]);
-        node_level_off[lev + 1] = (uint32_t)node_slots.size();
-    }
+    // a kept sum of m operands referenced r times saves about (r - 1) * (m - 1) additions
+    for (uint32_t k : ni.ids)
+        ni.benefit[k] = ((double)refs[k] - 1.0) * ((double)ni.kids[k].size() - 1.0);
+    std::vector<uint32_t> rank = ni.ids;
+    std::stable_sort(rank.begin(), rank.end(), [&](uint32_t a, uint32_t b) { return ni.benefit[a] > ni.benefit[b]; });
+    while (!rank.empty() && ni.benefit[rank.back()] <= 0) rank.pop_back();
 
-    // -- per-output work
-    std::vector<OutWork> work(hp.n_out);
+    // -- per-output operand lists (unresolved: tagged shared sums), raw terms
+    std::vector<OutWork> groups(hp.n_out);
     for (uint32_t j = 0; j < hp.n_out; ++j) {
-        std::vector<uint32_t> groups;
+        std::vector<uint32_t> gl;
         for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
             const fiona_term &t = hp.terms[e];
             if (t.kind == FIONA_TERM_RAW)
-                work[j].raws.push_back({t.input, t.pt});
-            else if (t.sign != 0 && std::find(groups.begin(), groups.end(), t.group) == groups.end())
-                groups.push_back(t.group);
+                groups[j].raws.push_back({t.input, t.pt});
+            else if (t.sign != 0 && std::find(gl.begin(), gl.end(), t.group) == gl.end())
+                gl.push_back(t.group);
         }
-        for (uint32_t g : groups) {
-            OutWork::Seg sg;
+        for (uint32_t g : gl) {
+            Seg sg;
             sg.scale_pt = hp.group_scale_pt[g];
             for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
                 const fiona_term &t = hp.terms[e];
@@ -311,94 +629,146 @@ int lower_tiled(fiona_plan *p)
             }
             for (uint32_t u = 0; u < hp.n_uses; ++u)
                 if (hp.uses[u].output == j && hp.uses[u].group == g)
-                    (hp.uses[u].sign < 0 ? sg.minus : sg.plus)
-                        .push_back(n_in + (uint32_t)slot[hp.uses[u].node]);
-            work[j].segs.push_back(sg);
+                    (hp.uses[u].sign < 0 ? sg.minus : sg.plus).push_back(kNodeTag | hp.uses[u].node);
+            groups[j].segs.push_back(std::move(sg));
         }
     }
 
-    // -- shape: coefficients per lane C, warps W, ring depth D, source buffers
-    const size_t budget_smem = (ctx->smem_optin ? ctx->smem_optin : 227 * 1024) - 256;
+    // -- shape search
+    const size_t smem_cap = (ctx->smem_optin ? ctx->smem_optin : 227 * 1024) - 256;
     const size_t per_sm = 228 * 1024;
-    const uint32_t n_src = n_in + n_slots;
+    const uint32_t sms = ctx->sm_count > 0 ? (uint32_t)ctx->sm_count : 152;
     struct Shape {
-        int C;
-        uint32_t W, D;
-        bool dbl;
-        uint32_t ctas;
-        size_t smem;
-        uint64_t score;
+        int C = 0;
+        uint32_t W = 0;
+        bool dbl = false;
+        uint32_t keep = 0, ctas = 0;  // shared sums requested (top of the ranking)
+        size_t smem = 0;
+        double est = 0;
     };
     std::vector<Shape> shapes;
     for (int C : {2, 1}) {
         if (ctx->N % (32u * C)) continue;
-        const uint32_t T = 32u * C, pair_bytes = 2 * T * 8;
-        for (uint32_t W : {8u, 16u}) {
-            const JobPlan jp = build_jobs(work, hp.n_out, W);
-            const Sched sc = encode(jp, node_level_off, node_slots, node_seg, W, ctx->L, budget, pair_bytes);
-            const size_t sched_bytes = sc.w.size() * 4;
-            for (uint32_t D : {16u, 8u}) {
-                cudaFuncAttributes attr{};
-                if (tiled_kernel_attributes(C, narrow, D, &attr) != FIONA_OK) continue;
-                const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
-                for (bool dbl : {true, false}) {
-                    if (dbl && n_in == 0) continue;
-                    const size_t smem = sched_bytes + (size_t)n_src * pair_bytes * (dbl ? 2 : 1) +
-                                        (size_t)jp.n_part * pair_bytes + (size_t)W * D * T * 8 + 32;
-                    if (smem + attr.sharedSizeBytes > budget_smem) continue;
-                    const uint32_t by_smem = (uint32_t)(per_sm / (smem + attr.sharedSizeBytes + 1024));
-                    const uint32_t by_threads = 2048 / (W * 32);
-                    const uint32_t by_regs = 65536 / (W * 32 * regs);
-                    const uint32_t ctas = std::min({by_smem, by_threads, by_regs});
-                    if (!ctas) continue;
-                    // plaintext bytes in flight per SM (enough at about 96 KB),
-                    // then resident warps, then wider loads
-                    const uint64_t inflight = std::min<uint64_t>((uint64_t)ctas * W * D * T * 8, 96 * 1024);
-                    const uint64_t score = (inflight << 16) | ((uint64_t)ctas * W << 4) | (uint64_t)(C * 2 + dbl);
-                    shapes.push_back({C, W, D, dbl, ctas, smem, score});
+        const uint32_t T = 32u * C, PB = 2 * T * 8;
+        const Costs k = costs_for(C, narrow);
+        cudaFuncAttributes attr{};
+        if (!device) {  // lowering without a GPU: the build's usual figures
+            attr.numRegs = 128;
+            attr.sharedSizeBytes = 64;
+        } else if (tiled_kernel_attributes(C, narrow, &attr) != FIONA_OK) {
+            continue;
+        }
+        const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
+        for (uint32_t W : {16u, 12u, 8u, 4u}) {
+            for (bool dbl : {true, false}) {
+                if (dbl && hp.n_in == 0) continue;
+                const uint32_t nbuf = dbl ? 2 : 1;
+                // most shared sums that fit: smem grows with each kept sum
+                auto smem_for = [&](uint32_t keep, Lowered &lw, JobPlan &jp, Sched &sc) {
+                    lw = resolve(hp, ni, groups, rank, keep, budget);
+                    jp = build_jobs(lw.work, W, k);
+                    sc = encode(jp, lw.level_off, lw.nodes, W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size());
+                    const uint32_t n_src = hp.n_in + (uint32_t)lw.nodes.size() + 1;  // + the zero tile
+                    if (n_src > kOpMaxSources) return (size_t)-1;
+                    return sc.w.size() * 4 + (size_t)n_src * PB * nbuf + (size_t)jp.n_part * PB + 32 +
+                           attr.sharedSizeBytes;
+                };
+                Lowered lw;
+                JobPlan jp;
+                Sched sc;
+                uint32_t lo = 0, hi = (uint32_t)rank.size();
+                if (smem_for(0, lw, jp, sc) > smem_cap) continue;
+                if (smem_for(hi, lw, jp, sc) > smem_cap) {
+                    while (lo + 1 < hi) {  // smem_for(lo) fits, smem_for(hi) does not
+                        const uint32_t mid = (lo + hi) / 2;
+                        if (smem_for(mid, lw, jp, sc) <= smem_cap) lo = mid;
+                        else hi = mid;
+                    }
+                    hi = lo;
                 }
+                const size_t smem = smem_for(hi, lw, jp, sc);
+                const uint32_t by_smem = (uint32_t)(per_sm / (smem + 1024));
+                const uint32_t by_threads = 2048 / (W * 32);
+                const uint32_t by_regs = 65536 / (W * 32 * regs);
+                const uint32_t ctas = std::min({by_smem, by_threads, by_regs, 32u});
+                if (!ctas) continue;
+                // per-tile demand of one CTA (cycles of the resource it uses)
+                double issue = 0, imad = 0, lds = 0, slowest = 0;
+                for (uint32_t wi = 0; wi < W; ++wi) {
+                    double c = 0;
+                    for (const Job &jb : jp.per_warp[wi]) {
+                        c += work_cost(jb.w, k);
+                        const double prods = (double)(jb.w.raws.size() + jb.w.segs.size());
+                        imad += prods * k.imad_op;
+                        double opnds = (double)jb.w.raws.size();
+                        for (auto &s : jb.w.segs) opnds += (double)(s.plus.size() + s.minus.size());
+                        lds += opnds * k.smem_operand / 128.0;
+                    }
+                    issue += c;
+                    slowest = std::max(slowest, c);
+                }
+                double node_ops = 0;
+                for (auto &s : lw.nodes) node_ops += k.seg + k.operand * (double)(s.plus.size() + s.minus.size());
+                const double hbm_bytes = (double)(sc.pt_ops + 2ull * hp.n_in + 2ull * hp.n_out) * T * 8;
+                const double hbm = hbm_bytes / 22.0;  // about 22 bytes per SM cycle at the measured copy rate
+                const double shared = std::max({issue / 4.0, imad, lds, hbm});
+                const double serial = slowest * 2.5 + node_ops / W * 2.5 + 150.0 * (lw.n_levels + 2) +
+                                      (dbl ? 0.0 : 1500.0 + (double)hp.n_in * PB / 64.0);
+                const double tiles = (double)ctx->N / T * ctx->L;
+                const double rounds = std::ceil(tiles / ((double)sms * ctas));
+                const double per_round = std::max(ctas * shared, serial + (ctas == 1 ? 0.25 * shared : 0.0));
+                Shape s;
+                s.C = C;
+                s.W = W;
+                s.dbl = dbl;
+                s.keep = hi;
+                s.ctas = ctas;
+                s.smem = smem - attr.sharedSizeBytes;
+                s.est = rounds * per_round;
+                shapes.push_back(s);
+                if (getenv("FIONA_TILED_DEBUG"))
+                    fprintf(stderr, "C=%d W=%u dbl=%d keep=%u sched=%zu parts=%u smem=%zu ctas=%u est=%.0f (issue %.0f imad %.0f lds %.0f hbm %.0f serial %.0f)\n",
+                            C, W, (int)dbl, s.keep, sc.w.size() * 4, jp.n_part, smem, ctas, s.est, issue / 4, imad, lds, hbm, serial);
             }
         }
     }
-    if (shapes.empty())
-        return set_error(FIONA_ERR_ARG, "tiled kernel: %u source tiles do not fit in shared memory", n_src);
-    Shape best = *std::max_element(shapes.begin(), shapes.end(),
-                                   [](const Shape &a, const Shape &b) { return a.score < b.score; });
-    // tuning override "C,W,D,double": every shape computes the same residues
+    if (shapes.empty()) return set_error(FIONA_ERR_ARG, "tiled kernel: the input tiles do not fit in shared memory");
+    Shape best = *std::min_element(shapes.begin(), shapes.end(),
+                                   [](const Shape &a, const Shape &b) { return a.est < b.est; });
+    // tuning override "C,W,double[,most shared sums kept]": every shape
+    // computes the same residues
     if (const char *env = getenv("FIONA_TILED_SHAPE")) {
-        int c = 0, w = 0, dd = 0, d = 0;
-        if (sscanf(env, "%d,%d,%d,%d", &c, &w, &dd, &d) == 4)
+        int c = 0, w = 0, d = 0, keep = 0;
+        const int n = sscanf(env, "%d,%d,%d,%d", &c, &w, &d, &keep);
+        if (n >= 3)
             for (auto &s : shapes)
-                if (s.C == c && s.W == (uint32_t)w && s.D == (uint32_t)dd && s.dbl == (d != 0)) best = s;
+                if (s.C == c && s.W == (uint32_t)w && s.dbl == (d != 0)) {
+                    best = s;
+                    if (n == 4 && keep >= 0) best.keep = std::min(best.keep, (uint32_t)keep);
+                }
     }
-    const uint32_t T = 32u * best.C, pair_bytes = 2 * T * 8;
-    const JobPlan jp = build_jobs(work, hp.n_out, best.W);
-    const Sched sc = encode(jp, node_level_off, node_slots, node_seg, best.W, ctx->L, budget, pair_bytes);
+    const uint32_t T = 32u * best.C, PB = 2 * T * 8;
+    const Costs k = costs_for(best.C, narrow);
+    const Lowered lw = resolve(hp, ni, groups, rank, best.keep, budget);
+    const JobPlan jp = build_jobs(lw.work, best.W, k);
+    const Sched sc = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size());
+    best.smem = sc.w.size() * 4 + (size_t)(hp.n_in + lw.nodes.size() + 1) * PB * (best.dbl ? 2 : 1) +
+                (size_t)jp.n_part * PB + 32;
 
     TiledSchedule *ts = new (std::nothrow) TiledSchedule;
     if (!ts) return set_error(FIONA_ERR_NOMEM, "tiled schedule: host allocation");
     ts->C = best.C;
     ts->narrow = narrow;
     ts->warps = best.W;
-    ts->depth = best.D;
     ts->tile = T;
     ts->smem = best.smem;
     ts->ctas_per_sm = best.ctas;
-    int rc = tiled_configure_kernel(best.C, narrow, best.D, ts->smem);
-    std::vector<size_t> off;
-    if (rc == FIONA_OK) rc = upload_blob(ts, {{sc.w.data(), sc.w.size() * 4}}, off);
-    if (rc != FIONA_OK) {
-        cudaFree(ts->sched.blob);
-        delete ts;
-        return rc;
-    }
+    ts->nodes_kept = (uint32_t)lw.nodes.size();
+    ts->nodes_expanded = (uint32_t)ni.ids.size() - ts->nodes_kept;
     TiledArgs &a = ts->args;
-    a.sched = (const uint32_t *)ts->sched.blob;
     a.o_level = sc.o_level;
-    a.o_node_slot = sc.o_node_slot;
-    a.o_node_prog_off = sc.o_node_prog_off;
-    a.o_prog_off = sc.o_prog_off;
-    a.o_fetch_off = sc.o_fetch_off;
+    a.o_node_off = sc.o_node_off;
+    a.o_warp = sc.o_warp;
     a.o_comb_off = sc.o_comb_off;
     a.o_comb_out = sc.o_comb_out;
     a.o_comb_parts = sc.o_comb_parts;
@@ -407,17 +777,30 @@ int lower_tiled(fiona_plan *p)
     a.err = ctx->d_kerr;
     a.N = ctx->N;
     a.L = ctx->L;
-    a.log2N = 0;
-    while ((1u << a.log2N) < ctx->N) ++a.log2N;
+    a.pt_stride = ctx->L * ctx->N;
     a.tiles_per_limb = ctx->N / T;
-    a.n_in = n_in;
-    a.n_nodes = n_slots;
-    a.n_levels = n_levels;
+    a.n_in = hp.n_in;
+    a.n_nodes = (uint32_t)lw.nodes.size();
+    a.n_levels = lw.n_levels;
     a.n_part = jp.n_part;
     a.n_comb = (uint32_t)jp.comb_out.size();
-    a.src_bytes = n_src * pair_bytes;
+    a.src_bytes = (hp.n_in + a.n_nodes + 1) * PB;  // + the zero tile
     a.double_buffer = best.dbl ? 1 : 0;
-    a.mac_budget = narrow ? 1023u : p->mac_budget;  // rns.cuh: kNarrowMacBudget
+    a.has_pt = hp.n_pt ? 1 : 0;
+    if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB)) {
+        delete ts;
+        return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
+    }
+    if (device) {
+        int rc = tiled_configure_kernel(best.C, narrow, ts->smem);
+        if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
+        if (rc != FIONA_OK) {
+            cudaFree(ts->sched.blob);
+            delete ts;
+            return rc;
+        }
+        a.sched = (const uint32_t *)ts->sched.blob;
+    }
     p->tiled = ts;
     return FIONA_OK;
 }
@@ -425,7 +808,7 @@ int lower_tiled(fiona_plan *p)
 void free_tiled(fiona_plan *p)
 {
     if (!p->tiled) return;
-    cudaFree(p->tiled->sched.blob);
+    if (p->tiled->sched.blob) cudaFree(p->tiled->sched.blob);
     delete p->tiled;
     p->tiled = nullptr;
 }

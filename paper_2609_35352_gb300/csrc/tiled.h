@@ -2,33 +2,62 @@
 // kernel_tiled.cu).
 //
 // A persistent CTA walks the (limb, coefficient tile) pairs.  For each it
-// holds, in shared memory, the tile of every input and of every shared
-// signed sum ("sources").  Each warp runs a fixed program of jobs for every
-// tile; a job is one output (or one part of an output split across warps),
-// made of scale-group segments (a signed sum over sources, then one product
-// by gamma) and raw terms (PMult-MAC).  The whole schedule is one array of
-// 32-bit words, copied once per CTA into shared memory:
+// holds, in shared memory, the tile of every input and of every materialised
+// shared signed sum ("sources"), plus one tile of zeros.  Each warp runs a
+// fixed stream of operations for every tile; each operation consumes one
+// plaintext tile:
 //
-//   node program   per shared sum: n_plus | n_minus << 16, then the words
-//   warp program   per job: target, n_seg | n_raw << 16; per segment
-//                  n_plus | n_minus << 16 and the words; then one word per
-//                  raw term (the input's tile offset)
-//   fetch list     per warp, the plaintext tiles its program consumes, in
-//                  order (gamma of each segment, then each raw term), as
-//                  plaintext index * L
-//   combine lists  outputs split across warps: partial slots to add
+//   RAW  acc += pt * source                     (PMult-MAC of a raw term)
+//   SEG  acc += gamma * (sum of +sources - sum of -sources)
+//        (one scale group, or a piece of it: Sec. 4.2 "Grouping
+//        Reconstruction Operations")
+//   NOP  padding: acc += pt * 0, with pt a tile another operation of the
+//        batch also reads, so the loop body has no branch and no extra HBM
+//        traffic
+// with flags FOLD (reduce the accumulator before this batch) and LAST (this
+// job's result is complete after this batch: reduce, store, clear).  The
+// stream is processed in batches of kTiledPrefetch operations: every job
+// starts a batch and is padded to whole batches; SEG and FOLD only open a
+// batch (a SEG's signed sum is formed before its batch) and LAST only closes
+// one.  A job is one output, or one part of an output split across warps
+// whose reduced partial sums are added at the end of the tile.
 //
-// A "word" naming a source is the byte offset of its tile pair (c0, c1)
-// inside the source region.  Sign runs are at most the lazy-sum bound long
-// (longer sums are cut into several segments with the same gamma: exact,
-// since gamma*S1 + gamma*S2 = gamma*(S1+S2) mod q).
+// The schedule is one array of 32-bit words, copied once per CTA into shared
+// memory:
+//   level offsets   shared sums of level l are nodes [lev[l], lev[l+1])
+//   node offsets    word offset of each node's program
+//   node programs   n_plus | n_minus << 16, then the plus then the minus
+//                   source indices, two 16-bit indices per word (each run
+//                   starts on a new word)
+//   warp table      per warp: op stream offset, op count (a multiple of the
+//                   prefetch depth), segment stream offset, target offset
+//   op streams      one word per operation (layout below)
+//   segment streams per SEG operation, in order: a program as above
+//   target streams  per job: output index, or kPartBit | partial slot
+//   combine lists   per split output: its partial slots
+// Source index s names the tile pair (c0, c1) at s * 2T words of the source
+// region: inputs first, then the materialised shared sums in level order,
+// then the zero tile.
 #pragma once
 #include <stdint.h>
 
 #include "fiona_internal.h"
 
 constexpr uint32_t kTiledMaxWarps = 16;
+constexpr uint32_t kTiledPrefetch = 8;  // plaintext tiles in flight per warp
 constexpr uint32_t kPartBit = 0x80000000u;  // job target: partial slot
+
+// operation word: [31:13] plaintext index, [12:9] flags, [8:0] source index
+constexpr uint32_t kOpSrcBits = 9;
+constexpr uint32_t kOpMaxSources = 1u << kOpSrcBits;
+constexpr uint32_t kOpSeg = 1u << 9;
+constexpr uint32_t kOpLast = 1u << 10;
+constexpr uint32_t kOpFold = 1u << 11;
+constexpr uint32_t kOpNop = 1u << 12;
+constexpr uint32_t kOpPtShift = 13;
+constexpr uint32_t kOpMaxPlaintexts = 1u << (32 - kOpPtShift);
+
+constexpr uint32_t kWarpTableWords = 4;  // op offset, op count, seg offset, target offset
 
 struct TiledArgs {
     const uint64_t *in;
@@ -38,26 +67,27 @@ struct TiledArgs {
     const uint32_t *sched;   // schedule words (global), copied to shared memory
     int *err;                // set to 1 when a bounded wait gives up
     // word offsets of the schedule's sections
-    uint32_t o_level, o_node_slot, o_node_prog_off, o_prog_off, o_fetch_off, o_comb_off,
-        o_comb_out, o_comb_parts;
+    uint32_t o_level, o_node_off, o_warp, o_comb_off, o_comb_out, o_comb_parts;
     uint32_t sched_bytes;    // multiple of 16
-    uint32_t N, L, log2N;
+    uint32_t N, L;
+    uint32_t pt_stride;      // L * N: elements between plaintexts
     uint32_t limb0, n_limbs;
     uint32_t tiles_per_limb;
     uint32_t n_in, n_nodes, n_levels, n_part, n_comb;
-    uint32_t src_bytes;      // one source region (inputs, then shared sums)
+    uint32_t src_bytes;      // one source region (inputs, shared sums, zero tile)
     uint32_t double_buffer;  // 1: two source regions, next tile staged early
-    uint32_t mac_budget;     // products per accumulator between folds
+    uint32_t has_pt;         // 0: the plan has no plaintexts (every load reads the schedule)
 };
 
 struct TiledSchedule {
     int C = 2;                 // coefficients per lane
     bool narrow = false;       // every modulus < 2^52: radix-2^26 arithmetic
     uint32_t warps = 8;        // warps per CTA
-    uint32_t depth = 8;        // plaintext tiles in flight per warp
     uint32_t tile = 64;        // coefficients per CTA tile
     size_t smem = 0;           // dynamic shared memory per CTA
     uint32_t ctas_per_sm = 0;  // occupancy the lowering planned for
+    uint32_t nodes_kept = 0;   // shared sums materialised per tile
+    uint32_t nodes_expanded = 0;  // shared sums expanded into their uses
     DeviceSchedule sched;
     TiledArgs args{};          // device pointers (data pointers unset)
 };

@@ -27,6 +27,7 @@ FIONA_ERR_CUDA = -5
 FIONA_ERR_RANGE = -6
 FIONA_ERR_NODEVICE = -7
 FIONA_ERR_TIMEOUT = -8
+FIONA_ERR_INTERNAL = -9
 FIONA_DEVICE_NONE = -1
 FIONA_KERNEL_AUTO = 0
 FIONA_KERNEL_DIRECT = 1
@@ -54,7 +55,7 @@ class PlanStats(ctypes.Structure):
         "n_inputs_used", "n_plaintexts_used", "bytes_min", "wide_products")] + \
         [(n, ctypes.c_uint32) for n in (
             "N", "L", "n_in", "n_out", "n_pt", "n_groups", "tile_coeffs", "warps_per_cta",
-            "smem_bytes", "ctas_per_sm", "kernel")] + [("reserved", ctypes.c_uint32 * 5)]
+            "smem_bytes", "ctas_per_sm", "kernel", "nodes_materialized")] + [("reserved", ctypes.c_uint32 * 4)]
 
     def as_dict(self) -> Dict[str, int]:
         return {n: int(getattr(self, n)) for n, _ in self._fields_ if n != "reserved"}

@@ -58,6 +58,36 @@ def test_elementwise_parity_small(name, N, L, kernel):
     assert dl.ctx.device_check() == F.FIONA_OK
 
 
+# Tiled shapes (coefficients per lane, warps, source regions[, most shared
+# sums kept]) chosen through the lowering's override; every shape must give
+# the same residues.  The last two force shared sums to be expanded into
+# their uses.
+SHAPES = ["2,16,0", "2,8,1", "1,16,1", "1,4,0", "2,12,1,0", "1,8,0,3"]
+SHAPE_CASES = [("tiny-dag", None, None), ("vit", 2048, 2), ("bert", 1024, 1), ("vgg", 1024, 2),
+               ("overflow60", None, None), ("overflow50", None, None)]
+
+
+@pytest.mark.parametrize("shape", SHAPES)
+@pytest.mark.parametrize("name,N,L", SHAPE_CASES)
+def test_tiled_shapes(name, N, L, shape, monkeypatch):
+    monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+    wl = W.make_workload(name, N=N, L=L)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel("tiled")
+    st = dl.plan.stats()
+    f = [int(v) for v in shape.split(",")]
+    if (st["tile_coeffs"], st["warps_per_cta"]) != (32 * f[0], f[1]):
+        pytest.skip("shape %s does not fit this layer in shared memory" % shape)
+    if len(f) == 4:
+        assert st["nodes_materialized"] <= f[3]
+    dl.run()
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    got = dl.outputs()
+    mism = np.argwhere(got != want)
+    assert mism.shape[0] == 0, "first mismatches (j, c, l, k): %s" % mism[:5].tolist()
+    assert dl.ctx.device_check() == F.FIONA_OK
+
+
 def test_edge_plans():
     R, T = W.TERM_RAW, W.TERM_TERNARY
     qs = W.ntt_primes(1024, 50, 3)
