@@ -235,59 +235,85 @@ struct Arith<true> {
     }
 };
 
-// Sum of the n source tiles of one poly named by the 16-bit indices packed
+// Sum of the n source tiles (both polys) named by the 16-bit indices packed
 // two per word from schedule byte offset `wp`; `src` = this lane's offset in
-// the source region plus the poly's offset.  Four tiles per step, their
-// loads independent.  Returns the offset just past the run's words.
+// the source region.  K indices per step (each index decoded once, its two
+// polys read at offsets 0 and TB), their loads independent.  Returns the
+// offset just past the run's words.
 template <int C, uint32_t TB>
-__device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32_t wp, uint32_t n, V<C> &s)
+__device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32_t wp, uint32_t n, V<C> &s0,
+                                            V<C> &s1)
 {
     constexpr uint32_t PB = 2 * TB;
+    constexpr uint32_t K = C == 1 ? 4 : 2;  // 4 independent loads of C words in flight per poly pair
     uint32_t k = 0;
-    for (; k + 4 <= n; k += 4, wp += 8) {
-        const uint32_t w0 = *reinterpret_cast<const uint32_t *>(sm + wp);
-        const uint32_t w1 = *reinterpret_cast<const uint32_t *>(sm + wp + 4);
-        const V<C> a = lds<C>(sm, src + (w0 & 0xffffu) * PB), b = lds<C>(sm, src + (w0 >> 16) * PB);
-        const V<C> c = lds<C>(sm, src + (w1 & 0xffffu) * PB), d = lds<C>(sm, src + (w1 >> 16) * PB);
+    for (; k + K <= n; k += K, wp += 2 * K) {
+        uint32_t o[K];
 #pragma unroll
-        for (int x = 0; x < C; ++x) s.x[x] += (a.x[x] + b.x[x]) + (c.x[x] + d.x[x]);
+        for (uint32_t j = 0; j < K; j += 2) {
+            const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp + 2 * j);
+            o[j] = src + (w & 0xffffu) * PB;
+            o[j + 1] = src + (w >> 16) * PB;
+        }
+        V<C> a[K], b[K];
+#pragma unroll
+        for (uint32_t j = 0; j < K; ++j) {
+            a[j] = lds<C>(sm, o[j]);
+            b[j] = lds<C>(sm, o[j] + TB);
+        }
+#pragma unroll
+        for (int x = 0; x < C; ++x) {
+            uint64_t t0 = a[0].x[x] + a[1].x[x], t1 = b[0].x[x] + b[1].x[x];
+#pragma unroll
+            for (uint32_t j = 2; j < K; ++j) {
+                t0 += a[j].x[x];
+                t1 += b[j].x[x];
+            }
+            s0.x[x] += t0;
+            s1.x[x] += t1;
+        }
     }
     for (; k + 2 <= n; k += 2, wp += 4) {
         const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp);
-        const V<C> a = lds<C>(sm, src + (w & 0xffffu) * PB), b = lds<C>(sm, src + (w >> 16) * PB);
+        const uint32_t o0 = src + (w & 0xffffu) * PB, o1 = src + (w >> 16) * PB;
+        const V<C> a0 = lds<C>(sm, o0), a1 = lds<C>(sm, o1), b0 = lds<C>(sm, o0 + TB), b1 = lds<C>(sm, o1 + TB);
 #pragma unroll
-        for (int x = 0; x < C; ++x) s.x[x] += a.x[x] + b.x[x];
+        for (int x = 0; x < C; ++x) {
+            s0.x[x] += a0.x[x] + a1.x[x];
+            s1.x[x] += b0.x[x] + b1.x[x];
+        }
     }
     if (k < n) {
         const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp);
-        const V<C> a = lds<C>(sm, src + (w & 0xffffu) * PB);
+        const uint32_t o0 = src + (w & 0xffffu) * PB;
+        const V<C> a0 = lds<C>(sm, o0), b0 = lds<C>(sm, o0 + TB);
 #pragma unroll
-        for (int x = 0; x < C; ++x) s.x[x] += a.x[x];
+        for (int x = 0; x < C; ++x) {
+            s0.x[x] += a0.x[x];
+            s1.x[x] += b0.x[x];
+        }
         wp += 4;
     }
     return wp;
 }
 
 // Signed sum of the program at byte offset `hdr` (n_plus | n_minus << 16,
-// then the plus run, then the minus run), both polys (one after the other,
-// to keep few values live), as canonical residues.  Returns the offset just
-// past the program.
+// then the plus run, then the minus run), both polys, as canonical residues.
+// Returns the offset just past the program.
 template <bool NARROW, int C, uint32_t TB>
 __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uint32_t hdr, uint32_t lim,
                                                V<C> &o0, V<C> &o1)
 {
     using A = Arith<NARROW>;
     const uint32_t h = *reinterpret_cast<const uint32_t *>(sm + hdr);
-    uint32_t wp = 0;
+    V<C> p0{}, p1{}, m0{}, m1{};
+    uint32_t wp = run_sum<C, TB>(sm, src, hdr + 4, h & 0xffffu, p0, p1);
+    wp = run_sum<C, TB>(sm, src, wp, h >> 16, m0, m1);
+    const LimbConst m = load_limb(lim);
 #pragma unroll
-    for (int c = 0; c < 2; ++c) {
-        V<C> p{}, mm{};
-        wp = run_sum<C, TB>(sm, src + c * TB, hdr + 4, h & 0xffffu, p);
-        wp = run_sum<C, TB>(sm, src + c * TB, wp, h >> 16, mm);
-        const LimbConst m = load_limb(lim);
-        V<C> &o = c ? o1 : o0;
-#pragma unroll
-        for (int x = 0; x < C; ++x) o.x[x] = A::signed_value(p.x[x], mm.x[x], m);
+    for (int x = 0; x < C; ++x) {
+        o0.x[x] = A::signed_value(p0.x[x], m0.x[x], m);
+        o1.x[x] = A::signed_value(p1.x[x], m1.x[x], m);
     }
     return wp;
 }

@@ -17,10 +17,8 @@
 //   estimated cost; an output larger than a warp's fair share is split into
 //   parts whose reduced partial sums are added at the end (exact in Z_q).
 // * Shape: 2 or 1 coefficients per lane, 4 to 16 warps per CTA, one or two
-//   source regions; the lowering estimates each shape's time per tile from
-//   its instruction, multiplier, shared-memory and HBM demand and keeps the
-//   fastest.  Plans whose moduli are all below 2^52 use the radix-2^26
-//   arithmetic.
+//   source regions, ranked as described at the choice below.  Plans whose
+//   moduli are all below 2^52 use the radix-2^26 arithmetic.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -29,6 +27,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <numeric>
+#include <tuple>
 
 #include "tiled.h"
 
@@ -240,16 +239,41 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
         for (const Job &jb : jp.per_warp[wi]) {
             const size_t first = o.size();
             const auto &raws = jb.w.raws;
+            const auto &segs = jb.w.segs;
             size_t r = 0;
-            auto raw_op = [&]() { return (raws[r].second << kOpPtShift) | raws[r].first; };
-            // each SEG opens a batch; the batch before it is filled with raw
-            // terms where there are any left
-            for (const Seg &sg : jb.w.segs) {
-                while ((o.size() - first) % P) o.push_back(r < raws.size() ? raw_op() : (kOpNop | zero_src)), r += r < raws.size();
-                put_program(segw[wi], sg.plus, sg.minus);
-                o.push_back((sg.scale_pt << kOpPtShift) | kOpSeg);
+            auto raw_or_nop = [&]() {
+                if (r < raws.size()) {
+                    const auto &t = raws[r++];
+                    return (t.second << kOpPtShift) | t.first;
+                }
+                return kOpNop | zero_src;
+            };
+            // Each SEG opens a batch.  The batches holding them are staggered
+            // across warps and jobs, so that the signed sums (shared-memory
+            // reads, formed before their batch) of different warps fall at
+            // different times of the tile instead of all at its start.
+            const size_t nb = std::max(segs.size(), (segs.size() + raws.size() + P - 1) / P);
+            std::vector<uint8_t> seg_at(nb, 0);
+            if (!segs.empty()) {
+                const size_t step = nb / segs.size(), phase = (wi * 5 + tgt[wi].size() * 3) % nb;
+                for (size_t k = 0; k < segs.size(); ++k) {
+                    size_t b = (phase + k * step) % nb;
+                    while (seg_at[b]) b = (b + 1) % nb;
+                    seg_at[b] = 1;
+                }
             }
-            for (; r < raws.size(); ++r) o.push_back(raw_op());
+            size_t k = 0;
+            for (size_t b = 0; b < nb; ++b) {
+                size_t fill = P;
+                if (seg_at[b]) {
+                    const Seg &sg = segs[k++];
+                    put_program(segw[wi], sg.plus, sg.minus);
+                    o.push_back((sg.scale_pt << kOpPtShift) | kOpSeg);
+                    fill = P - 1;
+                }
+                for (size_t i = 0; i < fill; ++i) o.push_back(raw_or_nop());
+            }
+            while (r < raws.size()) o.push_back(raw_or_nop());
             if (o.size() == first) o.push_back(kOpNop | zero_src);  // an output with no terms
             while ((o.size() - first) % P) o.push_back(kOpNop | zero_src);
             o.back() |= kOpLast;
@@ -733,8 +757,16 @@ int lower_tiled(fiona_plan *p)
         }
     }
     if (shapes.empty()) return set_error(FIONA_ERR_ARG, "tiled kernel: the input tiles do not fit in shared memory");
-    Shape best = *std::min_element(shapes.begin(), shapes.end(),
-                                   [](const Shape &a, const Shape &b) { return a.est < b.est; });
+    // Ranking (from shape sweeps of the layer workloads): a second source
+    // region first (the next tile's inputs arrive during this one), then
+    // resident warps up to 16 per SM, then 2 coefficients per lane (half the
+    // per-operation overhead per coefficient), then more CTAs per SM (their
+    // per-tile phases overlap), then the cost estimate.
+    auto key = [](const Shape &s) {
+        return std::make_tuple(s.dbl ? 1 : 0, std::min<uint32_t>(s.ctas * s.W, 16), s.C, s.ctas, -s.est);
+    };
+    Shape best = *std::max_element(shapes.begin(), shapes.end(),
+                                   [&](const Shape &a, const Shape &b) { return key(a) < key(b); });
     // tuning override "C,W,double[,most shared sums kept]": every shape
     // computes the same residues
     if (const char *env = getenv("FIONA_TILED_SHAPE")) {
