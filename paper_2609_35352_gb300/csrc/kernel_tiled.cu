@@ -368,29 +368,27 @@ __global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
     const uint32_t op0 = sw[wt] * 4, n_batches = sw[wt + 1] / P;
     const uint32_t seg0 = sw[wt + 2] * 4, tg0 = sw[wt + 3];
     const uint64_t pol = evict_first_policy();
-    const size_t stride_bytes = (size_t)a.pt_stride * 8;
+    const uint32_t stride_bytes = a.pt_stride * 8;  // L * N * 8 < 2^32 (lowering)
     auto tile_ptl = [&](uint32_t t) -> const char * {
         if (t >= total || !a.has_pt) return nullptr;
         const uint32_t l = a.limb0 + t / a.tiles_per_limb, k0 = (t % a.tiles_per_limb) * T;
         return reinterpret_cast<const char *>(a.pt + (size_t)l * a.N + k0 + lane * C);
     };
-    auto op_word = [&](uint32_t off) -> uint32_t {
-        uint32_t w;
-        asm volatile("ld.shared.u32 %0, [%1];" : "=r"(w) : "r"(smem_addr(sm) + off));
-        return w;
-    };
+    // operation words (read-only while the kernel runs: plain loads the
+    // compiler may schedule early)
+    auto op_word = [&](uint32_t off) -> uint32_t { return *reinterpret_cast<const uint32_t *>(sm + off); };
     // the plaintext words of operation word `w` in the tile at `base` (with
     // stride 0 and the schedule's own address when there is no next tile: a
     // harmless valid load)
-    auto fetch = [&](const char *base, size_t stride, uint32_t w) -> V<C> {
-        return ldg_stream<C>(reinterpret_cast<const uint64_t *>(base + (size_t)(w >> kOpPtShift) * stride), pol);
+    auto fetch = [&](const char *base, uint32_t stride, uint32_t w) -> V<C> {
+        return ldg_stream<C>(reinterpret_cast<const uint64_t *>(base + (uint64_t)(w >> kOpPtShift) * stride), pol);
     };
     V<C> r[P];
     uint32_t tile = blockIdx.x;
     const char *cur_ptl = tile_ptl(tile);
     if (n_batches && tile < total) {
         const char *b0 = cur_ptl ? cur_ptl : reinterpret_cast<const char *>(a.sched);
-        const size_t s0 = cur_ptl ? stride_bytes : 0;
+        const uint32_t s0 = cur_ptl ? stride_bytes : 0;
 #pragma unroll
         for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, s0, op_word(op0 + 4 * i));
     }
@@ -476,7 +474,7 @@ __global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
         for (uint32_t b = 0; b < n_batches; ++b) {
             const bool wrap = b + 1 == n_batches;
             const char *nb = wrap ? next_ptl : cur_ptl;
-            size_t ns = stride_bytes;
+            uint32_t ns = stride_bytes;
             if (!nb) {  // no next tile: a harmless valid load
                 nb = reinterpret_cast<const char *>(a.sched);
                 ns = 0;
