@@ -196,7 +196,7 @@ def measured_peak():
 
 
 KERNEL_FILES = {"direct": ["kernel_direct.cu", "rns.cuh"],
-                "tiled": ["kernel_tiled.cu", "rns.cuh"]}
+                "tiled": ["kernel_tiled.cu", "tiled.h", "lower_tiled.cpp", "rns.cuh"]}
 
 
 def kernel_source_hash(kernel: str) -> str:
@@ -295,12 +295,12 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     torch.cuda.set_device(local_rank)
     dev = local_rank
     name = args.workload
-    wl = W.make_workload(name)
+    wl = W.make_workload(name, L=args.limbs)
     p = wl.plan
 
     # CPU baseline first (rank 0, N = 1): spawned workers, before heavy GPU use
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu:
+    if rank == 0 and world == 1 and not args.no_cpu and args.limbs is None:
         cores = host_cores()
         smp = OracleSampler(name, cores, args.cpu_budget)
         w, pos = smp.step()
@@ -360,7 +360,8 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     achieved = stats["bytes_min"] / avg_kernel_s / 1e9
     kernel = "tiled" if stats["kernel"] == 2 else "direct"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": profiled_traffic(name, kernel),
+                "frac": achieved / peak,
+                "traffic": profiled_traffic(name, kernel) if args.limbs is None else None,
                 "kernel": kernel,
                 "peak_kind": peak_kind,
                 "algorithmic_bytes_per_launch": stats["bytes_min"],
@@ -423,6 +424,8 @@ def main():
                     help="seconds of oracle work per host core for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--limbs", type=int, default=None,
+                    help="profiling aid: the same layer with this many RNS limbs (no cpu_baseline)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
