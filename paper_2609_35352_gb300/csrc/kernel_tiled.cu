@@ -263,14 +263,13 @@ __device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32
         }
 #pragma unroll
         for (int x = 0; x < C; ++x) {
-            uint64_t t0 = a[0].x[x] + a[1].x[x], t1 = b[0].x[x] + b[1].x[x];
-#pragma unroll
-            for (uint32_t j = 2; j < K; ++j) {
-                t0 += a[j].x[x];
-                t1 += b[j].x[x];
+            if constexpr (K == 4) {  // two three-input additions per poly
+                s0.x[x] = s0.x[x] + (a[0].x[x] + a[1].x[x] + a[2].x[x]) + a[3].x[x];
+                s1.x[x] = s1.x[x] + (b[0].x[x] + b[1].x[x] + b[2].x[x]) + b[3].x[x];
+            } else {
+                s0.x[x] = s0.x[x] + a[0].x[x] + a[1].x[x];
+                s1.x[x] = s1.x[x] + b[0].x[x] + b[1].x[x];
             }
-            s0.x[x] += t0;
-            s1.x[x] += t1;
         }
     }
     for (; k + 2 <= n; k += 2, wp += 4) {
@@ -471,6 +470,28 @@ __global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
 #pragma unroll
             for (int x = 0; x < C; ++x) A::zero(acc[c][x]);
         uint32_t sp = seg0, tp = tg0;
+        // the job's result: reduce, store (output or partial slot), clear
+        auto finish = [&]() {
+            const LimbConst m = load_limb(lim);
+            V<C> y0, y1;
+#pragma unroll
+            for (int x = 0; x < C; ++x) {
+                y0.x[x] = A::reduce(acc[0][x], m);
+                y1.x[x] = A::reduce(acc[1][x], m);
+                A::zero(acc[0][x]);
+                A::zero(acc[1][x]);
+            }
+            const uint32_t target = sw[tp++];
+            if (target & kPartBit) {
+                const uint32_t dst = part_base + (target & ~kPartBit) * PB + lane_off;
+                sts<C>(sm, dst, y0);
+                sts<C>(sm, dst + TB, y1);
+            } else {
+                uint64_t *dst = a.out + ((size_t)target * 2 * a.L + l) * a.N + k0 + lane * C;
+                stg<C>(dst, y0);
+                stg<C>(dst + (size_t)a.L * a.N, y1);
+            }
+        };
         for (uint32_t b = 0; b < n_batches; ++b) {
             const bool wrap = b + 1 == n_batches;
             const char *nb = wrap ? next_ptl : cur_ptl;
@@ -518,27 +539,7 @@ __global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
                 }
                 r[i] = fetch(nb, ns, op_word(next_off + 4 * i));
             }
-            if (op_word(cur_off + 4 * (P - 1)) & kOpLast) {
-                const LimbConst m = load_limb(lim);
-                V<C> y0, y1;
-#pragma unroll
-                for (int x = 0; x < C; ++x) {
-                    y0.x[x] = A::reduce(acc[0][x], m);
-                    y1.x[x] = A::reduce(acc[1][x], m);
-                    A::zero(acc[0][x]);
-                    A::zero(acc[1][x]);
-                }
-                const uint32_t target = sw[tp++];
-                if (target & kPartBit) {
-                    const uint32_t dst = part_base + (target & ~kPartBit) * PB + lane_off;
-                    sts<C>(sm, dst, y0);
-                    sts<C>(sm, dst + TB, y1);
-                } else {
-                    uint64_t *dst = a.out + ((size_t)target * 2 * a.L + l) * a.N + k0 + lane * C;
-                    stg<C>(dst, y0);
-                    stg<C>(dst + (size_t)a.L * a.N, y1);
-                }
-            }
+            if (op_word(cur_off + 4 * (P - 1)) & kOpLast) finish();
         }
         cur_ptl = next_ptl;
 

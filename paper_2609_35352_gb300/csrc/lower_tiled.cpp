@@ -3,9 +3,10 @@
 //
 // * Shared signed sums (Sec. 4.2 "Sharing Signed Sums") reachable from a use
 //   are materialised once per tile as extra sources, in topological levels
-//   (children first), as many as shared memory holds: the sums are ranked by
-//   the additions they save, and a sum left out is expanded into its
-//   children wherever it is used (the same residues, a few more additions).
+//   (children first), when they save enough additions to pay for that phase
+//   and as many as shared memory holds: the sums are ranked by the additions
+//   they save, and a sum left out is expanded into its children wherever it
+//   is used (the same residues, a few more additions).
 // * Each output's used scale groups become SEG operations: the group's
 //   signed terms not covered by a use, plus one operand per use (sign
 //   sigma), summed and then multiplied once by gamma (Sec. 4.2 "Grouping
@@ -251,37 +252,46 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
             // Each SEG opens a batch.  The batches holding them are staggered
             // across warps and jobs, so that the signed sums (shared-memory
             // reads, formed before their batch) of different warps fall at
-            // different times of the tile instead of all at its start.
-            const size_t nb = std::max(segs.size(), (segs.size() + raws.size() + P - 1) / P);
-            std::vector<uint8_t> seg_at(nb, 0);
+            // different times of the tile instead of all at its start.  A job
+            // starts a batch (`first`) and is padded to whole batches.
+            constexpr size_t H = P;
+            const size_t len = segs.size() + raws.size();
+            const size_t b0 = (first + P - 1) / P * P;  // first batch start in the job
+            const size_t nbs = std::max(segs.size(), first + len > b0 ? (first + len - b0 + P - 1) / P : 0);
+            std::vector<uint8_t> seg_at(nbs, 0);
             if (!segs.empty()) {
-                const size_t step = nb / segs.size(), phase = (wi * 5 + tgt[wi].size() * 3) % nb;
+                const size_t step = nbs / segs.size(), phase = (wi * 5 + tgt[wi].size() * 3) % nbs;
                 for (size_t k = 0; k < segs.size(); ++k) {
-                    size_t b = (phase + k * step) % nb;
-                    while (seg_at[b]) b = (b + 1) % nb;
+                    size_t b = (phase + k * step) % nbs;
+                    while (seg_at[b]) b = (b + 1) % nbs;
                     seg_at[b] = 1;
                 }
             }
             size_t k = 0;
-            for (size_t b = 0; b < nb; ++b) {
-                size_t fill = P;
-                if (seg_at[b]) {
+            for (size_t p = first; k < segs.size() || r < raws.size(); ++p) {
+                if (p % P == 0 && k < segs.size() && seg_at[(p - b0) / P]) {
                     const Seg &sg = segs[k++];
                     put_program(segw[wi], sg.plus, sg.minus);
                     o.push_back((sg.scale_pt << kOpPtShift) | kOpSeg);
-                    fill = P - 1;
+                } else {
+                    o.push_back(raw_or_nop());  // a NOP while a SEG waits for its batch
                 }
-                for (size_t i = 0; i < fill; ++i) o.push_back(raw_or_nop());
             }
-            while (r < raws.size()) o.push_back(raw_or_nop());
             if (o.size() == first) o.push_back(kOpNop | zero_src);  // an output with no terms
-            while ((o.size() - first) % P) o.push_back(kOpNop | zero_src);
+            while (o.size() % H) o.push_back(kOpNop | zero_src);
             o.back() |= kOpLast;
             // at most mac_budget products in an accumulator between reductions
-            uint32_t nprod = 0;
-            for (size_t b = first; b < o.size(); b += P) {
+            // (a FOLD opens a batch inside the job)
+            auto products = [&](size_t from, size_t to) {
                 uint32_t cnt = 0;
-                for (size_t i = b; i < b + P; ++i) cnt += (o[i] & kOpNop) ? 0 : 1;
+                for (size_t i = from; i < to; ++i) cnt += (o[i] & kOpNop) ? 0 : 1;
+                return cnt;
+            };
+            const size_t end = o.size();
+            uint32_t nprod = products(first, std::min(b0, end));
+            sc.pt_ops += nprod;
+            for (size_t b = b0; b < end; b += P) {
+                const uint32_t cnt = products(b, std::min(b + P, end));
                 if (nprod + cnt > mac_budget) {
                     o[b] |= kOpFold;
                     nprod = 1;
@@ -291,6 +301,7 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
             }
             tgt[wi].push_back(jb.target);
         }
+        while (o.size() % P) o.push_back(kOpNop | zero_src);
         // a NOP loads a plaintext tile that another operation of its batch (or
         // the nearest earlier one) loads too
         uint32_t last_pt = 0;
@@ -656,6 +667,26 @@ int lower_tiled(fiona_plan *p)
                     (hp.uses[u].sign < 0 ? sg.minus : sg.plus).push_back(kNodeTag | hp.uses[u].node);
             groups[j].segs.push_back(std::move(sg));
         }
+    }
+
+    // -- forming shared sums once per tile is a phase of its own (a barrier per
+    //    DAG level, no plaintext traffic issued meanwhile): measured on the ViT
+    //    and BERT layers it costs more than the additions it saves (about 9% of
+    //    the signed operands there), so sums are formed only when they save at
+    //    least 15%; otherwise every use is expanded (the same residues).  A
+    //    tuning override with a fourth field keeps the sums in play.
+    bool force_keep = false;
+    if (const char *env = getenv("FIONA_TILED_SHAPE")) {
+        int c = 0, w = 0, d = 0, keep = 0;
+        force_keep = sscanf(env, "%d,%d,%d,%d", &c, &w, &d, &keep) == 4;
+    }
+    if (!rank.empty() && !force_keep) {
+        const Lowered flat = resolve(hp, ni, groups, rank, 0, budget);
+        double opnds = 0, save = 0;
+        for (auto &w : flat.work)
+            for (auto &sg : w.segs) opnds += (double)(sg.plus.size() + sg.minus.size());
+        for (uint32_t k : rank) save += ni.benefit[k];
+        if (save < 0.15 * opnds) rank.clear();
     }
 
     // -- shape search

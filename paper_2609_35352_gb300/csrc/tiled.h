@@ -19,8 +19,10 @@
 // stream is processed in batches of kTiledPrefetch operations: every job
 // starts a batch and is padded to whole batches; SEG and FOLD only open a
 // batch (a SEG's signed sum is formed before its batch) and LAST only closes
-// one.  A job is one output, or one part of an output split across warps
-// whose reduced partial sums are added at the end of the tile.
+// one.  (Measured: letting jobs end mid-batch, to pad less, costs more in the
+// loop than the padding it saves.)  A job is one output, or one part of an
+// output split across warps whose reduced partial sums are added at the end
+// of the tile.
 //
 // The schedule is one array of 32-bit words, copied once per CTA into shared
 // memory:
