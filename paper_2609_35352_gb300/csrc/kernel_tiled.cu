@@ -18,7 +18,7 @@
 //     before the group's product, then one product by gamma (Sec. 4.2
 //     "Grouping Reconstruction Operations"); per raw term a PMult-MAC of a
 //     plaintext tile and a source.  Plaintext tiles go from HBM straight to
-//     registers: each warp keeps the next kTiledPrefetch of its stream in
+//     registers: each warp keeps the next P (8 or 4) of its stream in
 //     flight, across job and tile boundaries, in a register queue indexed at
 //     compile time (the stream is processed in batches of that many
 //     operations).  Signed sums are lazy; products accumulate lazily; the
@@ -35,10 +35,8 @@
 
 namespace {
 
-constexpr uint32_t kMaxThreads = kTiledMaxWarps * 32;
 constexpr uint32_t kWaitLimit = 2000;
 constexpr uint32_t kWaitHintNs = 1000000;
-constexpr uint32_t P = kTiledPrefetch;
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p)
 {
@@ -317,8 +315,8 @@ __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uin
     return wp;
 }
 
-template <int C, bool NARROW>
-__global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
+template <int C, bool NARROW, uint32_t P>
+__global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledArgs a)
 {
     using A = Arith<NARROW>;
     using Acc = typename A::Acc;
@@ -573,28 +571,31 @@ __global__ void __launch_bounds__(kMaxThreads) tiled_kernel(const TiledArgs a)
     }
 }
 
-void *select_ptr(int C, bool narrow)
+template <uint32_t P>
+void *select_ptr_p(int C, bool narrow)
 {
     if (C == 2)
-        return narrow ? reinterpret_cast<void *>(&tiled_kernel<2, true>)
-                      : reinterpret_cast<void *>(&tiled_kernel<2, false>);
-    return narrow ? reinterpret_cast<void *>(&tiled_kernel<1, true>)
-                  : reinterpret_cast<void *>(&tiled_kernel<1, false>);
+        return narrow ? reinterpret_cast<void *>(&tiled_kernel<2, true, P>)
+                      : reinterpret_cast<void *>(&tiled_kernel<2, false, P>);
+    return narrow ? reinterpret_cast<void *>(&tiled_kernel<1, true, P>)
+                  : reinterpret_cast<void *>(&tiled_kernel<1, false, P>);
 }
+
+void *select_ptr(int C, bool narrow, uint32_t P) { return P == 4 ? select_ptr_p<4>(C, narrow) : select_ptr_p<8>(C, narrow); }
 
 }  // namespace
 
-int tiled_kernel_attributes(int C, bool narrow, cudaFuncAttributes *attr)
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, cudaFuncAttributes *attr)
 {
-    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow));
+    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P));
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attributes: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
 
-int tiled_configure_kernel(int C, bool narrow, size_t smem)
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, size_t smem)
 {
     cudaError_t e =
-        cudaFuncSetAttribute(select_ptr(C, narrow), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(select_ptr(C, narrow, P), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attribute: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
@@ -616,7 +617,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     dim3 grid(std::min(tiles, resident));
     dim3 block(ts->warps * 32);
     cudaStream_t s = (cudaStream_t)stream;
-    void *fn = select_ptr(ts->C, ts->narrow);
+    void *fn = select_ptr(ts->C, ts->narrow, ts->batch);
     void *args[] = {&a};
     cudaError_t e = cudaLaunchKernel(fn, grid, block, args, ts->smem, s);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel launch: %s", cudaGetErrorString(e));

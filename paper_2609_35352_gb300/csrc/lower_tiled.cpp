@@ -66,13 +66,12 @@ Costs costs_for(int C, bool narrow)
     return c;
 }
 
-double work_cost(const OutWork &w, const Costs &k)
-{
+double work_cost(const OutWork &w, const Costs &k, size_t P)
+{  // P: operations per batch
     double c = k.last + k.raw * (double)w.raws.size();
     for (auto &s : w.segs) c += k.seg + k.operand * (double)(s.plus.size() + s.minus.size());
     // NOP padding: each SEG opens a batch, the job fills its last one
     const size_t ops = w.segs.size() + w.raws.size();
-    const size_t P = kTiledPrefetch;
     size_t slots = 0;
     if (w.segs.empty()) {
         slots = (w.raws.size() + P - 1) / P * P;
@@ -96,10 +95,10 @@ struct JobPlan {
 
 // Cut `w` into P parts of about equal cost (segments are cut between
 // operands; each piece keeps its gamma).
-std::vector<OutWork> split_work(const OutWork &w, uint32_t P, const Costs &k)
+std::vector<OutWork> split_work(const OutWork &w, uint32_t P, const Costs &k, size_t batch)
 {
     std::vector<OutWork> chunk(P);
-    const double per = work_cost(w, k) / P;
+    const double per = work_cost(w, k, batch) / P;
     uint32_t cur = 0;
     double acc = 0;
     auto advance = [&](double add) {
@@ -135,16 +134,16 @@ std::vector<OutWork> split_work(const OutWork &w, uint32_t P, const Costs &k)
 // assigned largest first to the least-loaded warp.  `makespan` receives the
 // largest warp load.
 JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Costs &k, uint32_t split,
-                         double &makespan)
+                         double &makespan, size_t batch)
 {
     JobPlan jp;
     std::vector<Job> jobs;
     jp.comb_off.assign(1, 0);
     double total = 0;
-    for (auto &w : work) total += work_cost(w, k);
+    for (auto &w : work) total += work_cost(w, k, batch);
     const double share = total / W;
     for (uint32_t j = 0; j < work.size(); ++j) {
-        const double c = work_cost(work[j], k);
+        const double c = work_cost(work[j], k, batch);
         uint32_t P = (uint32_t)std::max(1.0, std::round(c / std::max(share, 1.0)));
         P = std::min(W, std::max(P, split));
         // a part must be worth its partial slot and final addition
@@ -152,7 +151,7 @@ JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Cos
             jobs.push_back({j, work[j]});
             continue;
         }
-        std::vector<OutWork> chunk = split_work(work[j], P, k);
+        std::vector<OutWork> chunk = split_work(work[j], P, k, batch);
         jp.comb_out.push_back(j);
         for (auto &ch : chunk) {
             if (ch.segs.empty() && ch.raws.empty()) continue;
@@ -164,7 +163,7 @@ JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Cos
     std::vector<uint32_t> order(jobs.size());
     std::iota(order.begin(), order.end(), 0);
     std::vector<double> jc(jobs.size());
-    for (size_t i = 0; i < jobs.size(); ++i) jc[i] = work_cost(jobs[i].w, k);
+    for (size_t i = 0; i < jobs.size(); ++i) jc[i] = work_cost(jobs[i].w, k, batch);
     std::stable_sort(order.begin(), order.end(), [&](uint32_t a, uint32_t b) { return jc[a] > jc[b]; });
     std::vector<double> load(W, 0);
     jp.per_warp.assign(W, {});
@@ -179,13 +178,13 @@ JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Cos
 
 // The split (1 to 4 parts per output) with the smallest largest warp load;
 // a finer split must gain at least 3% to be taken.
-JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t W, const Costs &k)
+JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t W, const Costs &k, size_t batch)
 {
     double best_ms = 0;
-    JobPlan best = build_jobs_split(work, W, k, 1, best_ms);
+    JobPlan best = build_jobs_split(work, W, k, 1, best_ms, batch);
     for (uint32_t split = 2; split <= 4; ++split) {
         double ms = 0;
-        JobPlan jp = build_jobs_split(work, W, k, split, ms);
+        JobPlan jp = build_jobs_split(work, W, k, split, ms, batch);
         if (ms < 0.97 * best_ms) {
             best_ms = ms;
             best = std::move(jp);
@@ -217,7 +216,7 @@ void pad4(std::vector<uint32_t> &w)
 }
 
 Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const std::vector<Seg> &nodes, uint32_t W,
-             uint32_t mac_budget, uint32_t zero_index)
+             uint32_t mac_budget, uint32_t zero_index, uint32_t P)
 {
     Sched sc;
     auto &w = sc.w;
@@ -233,7 +232,6 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
     sc.o_warp = (uint32_t)w.size();
     w.resize(w.size() + (size_t)W * kWarpTableWords);
     std::vector<std::vector<uint32_t>> ops(W), segw(W), tgt(W);
-    constexpr uint32_t P = kTiledPrefetch;
     const uint32_t zero_src = zero_index;
     for (uint32_t wi = 0; wi < W; ++wi) {
         auto &o = ops[wi];
@@ -254,7 +252,7 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
             // reads, formed before their batch) of different warps fall at
             // different times of the tile instead of all at its start.  A job
             // starts a batch (`first`) and is padded to whole batches.
-            constexpr size_t H = P;
+            const size_t H = P;
             const size_t len = segs.size() + raws.size();
             const size_t b0 = (first + P - 1) / P * P;  // first batch start in the job
             const size_t nbs = std::max(segs.size(), first + len > b0 ? (first + len - b0 + P - 1) / P : 0);
@@ -483,7 +481,7 @@ int upload_blob(TiledSchedule *ts, const std::vector<uint32_t> &words)
 // ends of each stream, alignment, and the shared-memory layout.  Returns an
 // explanation of the first violation, or null.
 const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, uint32_t W, uint32_t n_out,
-                           uint32_t n_pt, size_t smem, uint32_t PB)
+                           uint32_t n_pt, size_t smem, uint32_t PB, uint32_t P)
 {
     const size_t nw = w.size();
     if (a.sched_bytes != nw * 4 || a.sched_bytes % 16) return "schedule size";
@@ -536,16 +534,16 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
         const size_t t = a.o_warp + (size_t)wi * kWarpTableWords;
         if (t + kWarpTableWords > nw) return "warp table";
         const uint32_t op0 = w[t], n_ops = w[t + 1], seg0 = w[t + 2], tg0 = w[t + 3];
-        if (op0 % 4 || n_ops % kTiledPrefetch || (size_t)op0 + n_ops > nw) return "op stream";
+        if (op0 % 4 || n_ops % P || (size_t)op0 + n_ops > nw) return "op stream";
         size_t sp = seg0, tp = tg0;
         const size_t seg_end = wi + 1 < W ? w[t + kWarpTableWords + 2] : w[a.o_warp + 3];
         const size_t tg_end = wi + 1 < W ? w[t + kWarpTableWords + 3] : a.o_comb_off;
         bool open = false;
         for (uint32_t f = 0; f < n_ops; ++f) {
             const uint32_t op = w[op0 + f];
-            const uint32_t pos = f % kTiledPrefetch;
+            const uint32_t pos = f % P;
             if ((op & (kOpSeg | kOpFold)) && pos != 0) return "SEG or FOLD inside a batch";
-            if ((op & kOpLast) && pos != kTiledPrefetch - 1) return "LAST inside a batch";
+            if ((op & kOpLast) && pos != P - 1) return "LAST inside a batch";
             // every operation loads a plaintext tile, NOPs included
             if ((op >> kOpPtShift) >= std::max<uint32_t>(n_pt, 1)) return "plaintext index";
             if (op & kOpNop) {
@@ -595,8 +593,8 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
 }  // namespace
 
 // kernel_tiled.cu
-int tiled_configure_kernel(int C, bool narrow, size_t smem);
-int tiled_kernel_attributes(int C, bool narrow, cudaFuncAttributes *attr);
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, size_t smem);
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, cudaFuncAttributes *attr);
 
 int lower_tiled(fiona_plan *p)
 {
@@ -677,8 +675,8 @@ int lower_tiled(fiona_plan *p)
     //    tuning override with a fourth field keeps the sums in play.
     bool force_keep = false;
     if (const char *env = getenv("FIONA_TILED_SHAPE")) {
-        int c = 0, w = 0, d = 0, keep = 0;
-        force_keep = sscanf(env, "%d,%d,%d,%d", &c, &w, &d, &keep) == 4;
+        int c = 0, w = 0, d = 0, keep = -1;
+        force_keep = sscanf(env, "%d,%d,%d,%d", &c, &w, &d, &keep) == 4 && keep >= 0;
     }
     if (!rank.empty() && !force_keep) {
         const Lowered flat = resolve(hp, ni, groups, rank, 0, budget);
@@ -695,14 +693,16 @@ int lower_tiled(fiona_plan *p)
     const uint32_t sms = ctx->sm_count > 0 ? (uint32_t)ctx->sm_count : 152;
     struct Shape {
         int C = 0;
-        uint32_t W = 0;
+        uint32_t W = 0, P = 8;
+        double pad = 0;               // share of padding operations
         bool dbl = false;
         uint32_t keep = 0, ctas = 0;  // shared sums requested (top of the ranking)
         size_t smem = 0;
         double est = 0;
     };
     std::vector<Shape> shapes;
-    for (int C : {2, 1}) {
+    for (int C : {2, 1})
+    for (uint32_t batch : {8u, 4u}) {
         if (ctx->N % (32u * C)) continue;
         const uint32_t T = 32u * C, PB = 2 * T * 8;
         const Costs k = costs_for(C, narrow);
@@ -710,7 +710,7 @@ int lower_tiled(fiona_plan *p)
         if (!device) {  // lowering without a GPU: the build's usual figures
             attr.numRegs = 128;
             attr.sharedSizeBytes = 64;
-        } else if (tiled_kernel_attributes(C, narrow, &attr) != FIONA_OK) {
+        } else if (tiled_kernel_attributes(C, narrow, batch, &attr) != FIONA_OK) {
             continue;
         }
         const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
@@ -721,8 +721,9 @@ int lower_tiled(fiona_plan *p)
                 // most shared sums that fit: smem grows with each kept sum
                 auto smem_for = [&](uint32_t keep, Lowered &lw, JobPlan &jp, Sched &sc) {
                     lw = resolve(hp, ni, groups, rank, keep, budget);
-                    jp = build_jobs(lw.work, W, k);
-                    sc = encode(jp, lw.level_off, lw.nodes, W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size());
+                    jp = build_jobs(lw.work, W, k, batch);
+                    sc = encode(jp, lw.level_off, lw.nodes, W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(),
+                                batch);
                     const uint32_t n_src = hp.n_in + (uint32_t)lw.nodes.size() + 1;  // + the zero tile
                     if (n_src > kOpMaxSources) return (size_t)-1;
                     return sc.w.size() * 4 + (size_t)n_src * PB * nbuf + (size_t)jp.n_part * PB + 32 +
@@ -752,7 +753,7 @@ int lower_tiled(fiona_plan *p)
                 for (uint32_t wi = 0; wi < W; ++wi) {
                     double c = 0;
                     for (const Job &jb : jp.per_warp[wi]) {
-                        c += work_cost(jb.w, k);
+                        c += work_cost(jb.w, k, batch);
                         const double prods = (double)(jb.w.raws.size() + jb.w.segs.size());
                         imad += prods * k.imad_op;
                         double opnds = (double)jb.w.raws.size();
@@ -775,6 +776,10 @@ int lower_tiled(fiona_plan *p)
                 Shape s;
                 s.C = C;
                 s.W = W;
+                s.P = batch;
+                size_t n_ops = 0;
+                for (uint32_t wi = 0; wi < W; ++wi) n_ops += sc.w[sc.o_warp + wi * kWarpTableWords + 1];
+                s.pad = n_ops ? 1.0 - (double)sc.pt_ops / (double)n_ops : 0.0;
                 s.dbl = dbl;
                 s.keep = hi;
                 s.ctas = ctas;
@@ -782,8 +787,8 @@ int lower_tiled(fiona_plan *p)
                 s.est = rounds * per_round;
                 shapes.push_back(s);
                 if (getenv("FIONA_TILED_DEBUG"))
-                    fprintf(stderr, "C=%d W=%u dbl=%d keep=%u sched=%zu parts=%u smem=%zu ctas=%u est=%.0f (issue %.0f imad %.0f lds %.0f hbm %.0f serial %.0f)\n",
-                            C, W, (int)dbl, s.keep, sc.w.size() * 4, jp.n_part, smem, ctas, s.est, issue / 4, imad, lds, hbm, serial);
+                    fprintf(stderr, "C=%d P=%u W=%u dbl=%d keep=%u sched=%zu parts=%u smem=%zu ctas=%u pad=%.2f est=%.0f\n",
+                            C, batch, W, (int)dbl, s.keep, sc.w.size() * 4, jp.n_part, smem, ctas, s.pad, s.est);
             }
         }
     }
@@ -792,29 +797,33 @@ int lower_tiled(fiona_plan *p)
     // region first (the next tile's inputs arrive during this one), then
     // resident warps up to 16 per SM, then 2 coefficients per lane (half the
     // per-operation overhead per coefficient), then more CTAs per SM (their
-    // per-tile phases overlap), then the cost estimate.
+    // per-tile phases overlap), then batches of 4 with 2 coefficients per
+    // lane and of 8 with one (BERT and ViT ran faster with 4, VGG with 8),
+    // then the cost estimate.
     auto key = [](const Shape &s) {
-        return std::make_tuple(s.dbl ? 1 : 0, std::min<uint32_t>(s.ctas * s.W, 16), s.C, s.ctas, -s.est);
+        return std::make_tuple(s.dbl ? 1 : 0, std::min<uint32_t>(s.ctas * s.W, 16), s.C, s.ctas,
+                               (s.C == 2) == (s.P == 4) ? 1 : 0, -s.est);
     };
     Shape best = *std::max_element(shapes.begin(), shapes.end(),
                                    [&](const Shape &a, const Shape &b) { return key(a) < key(b); });
-    // tuning override "C,W,double[,most shared sums kept]": every shape
+    // tuning override "C,W,double[,most shared sums kept[,P]]": every shape
     // computes the same residues
     if (const char *env = getenv("FIONA_TILED_SHAPE")) {
-        int c = 0, w = 0, d = 0, keep = 0;
-        const int n = sscanf(env, "%d,%d,%d,%d", &c, &w, &d, &keep);
+        int c = 0, w = 0, d = 0, keep = -1, pb = 8;
+        const int n = sscanf(env, "%d,%d,%d,%d,%d", &c, &w, &d, &keep, &pb);
         if (n >= 3)
             for (auto &s : shapes)
-                if (s.C == c && s.W == (uint32_t)w && s.dbl == (d != 0)) {
+                if (s.C == c && s.W == (uint32_t)w && s.dbl == (d != 0) && s.P == (uint32_t)pb) {
                     best = s;
-                    if (n == 4 && keep >= 0) best.keep = std::min(best.keep, (uint32_t)keep);
+                    if (n >= 4 && keep >= 0) best.keep = std::min(best.keep, (uint32_t)keep);
                 }
     }
     const uint32_t T = 32u * best.C, PB = 2 * T * 8;
     const Costs k = costs_for(best.C, narrow);
     const Lowered lw = resolve(hp, ni, groups, rank, best.keep, budget);
-    const JobPlan jp = build_jobs(lw.work, best.W, k);
-    const Sched sc = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size());
+    const JobPlan jp = build_jobs(lw.work, best.W, k, best.P);
+    const Sched sc =
+        encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(), best.P);
     best.smem = sc.w.size() * 4 + (size_t)(hp.n_in + lw.nodes.size() + 1) * PB * (best.dbl ? 2 : 1) +
                 (size_t)jp.n_part * PB + 32;
 
@@ -824,6 +833,7 @@ int lower_tiled(fiona_plan *p)
     ts->narrow = narrow;
     ts->warps = best.W;
     ts->tile = T;
+    ts->batch = best.P;
     ts->smem = best.smem;
     ts->ctas_per_sm = best.ctas;
     ts->nodes_kept = (uint32_t)lw.nodes.size();
@@ -850,12 +860,12 @@ int lower_tiled(fiona_plan *p)
     a.src_bytes = (hp.n_in + a.n_nodes + 1) * PB;  // + the zero tile
     a.double_buffer = best.dbl ? 1 : 0;
     a.has_pt = hp.n_pt ? 1 : 0;
-    if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB)) {
+    if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB, best.P)) {
         delete ts;
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
     }
     if (device) {
-        int rc = tiled_configure_kernel(best.C, narrow, ts->smem);
+        int rc = tiled_configure_kernel(best.C, narrow, best.P, ts->smem);
         if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
         if (rc != FIONA_OK) {
             cudaFree(ts->sched.blob);

@@ -16,7 +16,8 @@
 //        traffic
 // with flags FOLD (reduce the accumulator before this batch) and LAST (this
 // job's result is complete after this batch: reduce, store, clear).  The
-// stream is processed in batches of kTiledPrefetch operations: every job
+// stream is processed in batches of P operations (P = 8 or 4, the number of
+// plaintext tiles each warp keeps in flight): every job
 // starts a batch and is padded to whole batches; SEG and FOLD only open a
 // batch (a SEG's signed sum is formed before its batch) and LAST only closes
 // one.  (Measured: letting jobs end mid-batch, to pad less, costs more in the
@@ -45,8 +46,9 @@
 
 #include "fiona_internal.h"
 
+// most warps per CTA (the kernels are built for it: at most 128 registers a
+// thread; a bound of 20 warps measured slower, its register cap spills)
 constexpr uint32_t kTiledMaxWarps = 16;
-constexpr uint32_t kTiledPrefetch = 8;  // plaintext tiles in flight per warp
 constexpr uint32_t kPartBit = 0x80000000u;  // job target: partial slot
 
 // operation word: [31:13] plaintext index, [12:9] flags, [8:0] source index
@@ -86,6 +88,7 @@ struct TiledSchedule {
     bool narrow = false;       // every modulus < 2^52: radix-2^26 arithmetic
     uint32_t warps = 8;        // warps per CTA
     uint32_t tile = 64;        // coefficients per CTA tile
+    uint32_t batch = 8;        // P: operations per batch, plaintext tiles in flight per warp
     size_t smem = 0;           // dynamic shared memory per CTA
     uint32_t ctas_per_sm = 0;  // occupancy the lowering planned for
     uint32_t nodes_kept = 0;   // shared sums materialised per tile

@@ -59,10 +59,11 @@ def test_elementwise_parity_small(name, N, L, kernel):
 
 
 # Tiled shapes (coefficients per lane, warps, source regions[, most shared
-# sums kept]) chosen through the lowering's override; every shape must give
-# the same residues.  The last two force shared sums to be expanded into
-# their uses.
-SHAPES = ["2,16,0", "2,8,1", "1,16,1", "1,4,0", "2,12,1,0", "1,8,0,3"]
+# sums kept (-1: the lowering's choice)[, operations per batch]]) chosen
+# through the lowering's override; every shape must give the same residues.
+# A fourth field forces the shared sums in play (0: all expanded), a fifth
+# selects batches of 4.
+SHAPES = ["2,16,0", "2,8,1", "1,16,1", "1,4,0", "2,12,1,0", "1,8,0,3", "2,8,1,-1,4", "1,16,0,2,4"]
 SHAPE_CASES = [("tiny-dag", None, None), ("vit", 2048, 2), ("bert", 1024, 1), ("vgg", 1024, 2),
                ("overflow60", None, None), ("overflow50", None, None)]
 
@@ -78,7 +79,7 @@ def test_tiled_shapes(name, N, L, shape, monkeypatch):
     f = [int(v) for v in shape.split(",")]
     if (st["tile_coeffs"], st["warps_per_cta"]) != (32 * f[0], f[1]):
         pytest.skip("shape %s does not fit this layer in shared memory" % shape)
-    if len(f) == 4:
+    if len(f) >= 4 and f[3] >= 0:
         assert st["nodes_materialized"] <= f[3]
     dl.run()
     want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
