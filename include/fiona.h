@@ -190,6 +190,51 @@ int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out, uint3
                       uint32_t n_uses, const fiona_sum_use *uses, fiona_plan **out);
 void fiona_plan_destroy(fiona_plan *plan); /* NULL is a no-op */
 
+/* Route of the weights of output j on input i, for the plan compiler.
+ * 8 bytes. */
+typedef struct fiona_route {
+    int8_t kind;      /* FIONA_TERM_RAW or FIONA_TERM_TERNARY                         */
+    int8_t sign;      /* TERNARY: h_g in {-1, 0, +1}; RAW: 0                           */
+    uint16_t reserved;/* must be 0                                                     */
+    uint32_t pt;      /* RAW: the group's plaintext; TERNARY: the output's reconstruction-
+                         factor plaintext gamma (terms with one gamma share one PMult)  */
+} fiona_route;
+
+enum {
+    FIONA_COMPILE_SHARE = 1,       /* search shared signed sums                        */
+    FIONA_COMPILE_SHARE_EXACT = 2  /* with SHARE: accept a sum of m inputs used by k
+                                      outputs when (k-1)(m-1) > 0 (the Add/Sub it saves
+                                      under the n-1 rule) instead of km-m-k > 0        */
+};
+
+/* Host plan compiler (Sec. 4.2): from the dense route matrix
+ * routes[j * n_in + i] of a layer to the arrays fiona_plan_create takes.
+ *   Terms: one per (output, input) pair, in input order (term_offsets[j] =
+ *   j * n_in).  Grouping Reconstruction Operations: the TERNARY terms of one
+ *   output with the same gamma form one scale group (groups numbered in
+ *   order of first appearance).  Sharing Signed Sums (with
+ *   FIONA_COMPILE_SHARE): every pair of scale groups of different outputs
+ *   proposes the signed terms they have in common (the same inputs with the
+ *   same signs, or with all signs reversed) as a sum; a sum of m inputs that
+ *   k groups can take is estimated to save km - m - k Add/Sub (the paper's
+ *   conservative count; (k-1)(m-1) with FIONA_COMPILE_SHARE_EXACT), and the
+ *   sums are accepted largest estimate first while the estimate over the
+ *   groups still free to take them is positive.  A group takes at most one of
+ *   any two overlapping sums, so a term is covered at most once.  Nodes are
+ *   sums of inputs (one level).
+ * Caller-allocated outputs, each with room for n_out * n_in entries
+ * (term_offsets and node_offsets: one more): terms, group_scale_pt,
+ * group_output, node_offsets, children, uses; counts in *n_groups,
+ * *n_nodes, *n_uses.  Pure host code: no context, no device.
+ * Errors: FIONA_ERR_ARG (null argument, unknown flag, more than 2^24 pairs),
+ * FIONA_ERR_PLAN (a route with an unknown kind, a sign outside its range,
+ * a plaintext >= n_pt, or a nonzero reserved field). */
+int fiona_plan_compile(uint32_t n_in, uint32_t n_out, uint32_t n_pt, const fiona_route *routes,
+                       uint32_t flags, uint32_t *term_offsets, fiona_term *terms, uint32_t *n_groups,
+                       uint32_t *group_scale_pt, uint32_t *group_output, uint32_t *n_nodes,
+                       uint32_t *node_offsets, fiona_sum_child *children, uint32_t *n_uses,
+                       fiona_sum_use *uses);
+
 int fiona_plan_stats(const fiona_plan *plan, fiona_plan_stats_t *out);
 
 /* Choose the kernel variant used by later evaluations of `plan`
@@ -208,6 +253,18 @@ int fiona_plan_select_kernel(fiona_plan *plan, int kernel);
  * FIONA_ERR_CUDA (launch failure, reported from cudaGetLastError). */
 int fiona_linear_eval(const fiona_plan *plan, void *cuda_stream, const uint64_t *inputs,
                       const uint64_t *plaintexts, uint64_t *outputs);
+
+/* Evaluate the layer at a lower level: the ciphertexts and plaintexts hold
+ * only the first `L_eval` RNS limbs (moduli q_0 .. q_{L_eval-1}; CKKS drops
+ * the last limbs as a ciphertext goes down in level, Sec. 2.2), laid out
+ * [n_in][2][L_eval][N], [n_pt][L_eval][N] and [n_out][2][L_eval][N].  One
+ * plan serves every level: the layer's routes, groups and shared sums do
+ * not depend on the limb count, and every limb is computed independently.
+ * Asynchronous like fiona_linear_eval.  Errors: FIONA_ERR_ARG (L_eval
+ * outside [1, L], null or misaligned pointer), FIONA_ERR_NODEVICE,
+ * FIONA_ERR_CUDA. */
+int fiona_linear_eval_level(const fiona_plan *plan, void *cuda_stream, uint32_t L_eval,
+                            const uint64_t *inputs, const uint64_t *plaintexts, uint64_t *outputs);
 
 /* End-to-end evaluation from host memory: copies `h_inputs` (host, layout
  * [n_in][2][L][N], pinned for overlap) to the caller's device buffer

@@ -25,7 +25,8 @@ FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", 
          "--expt-relaxed-constexpr", "-I" + INCLUDE]
 
 LIBRARIES = {
-    "libfiona.so": ["fiona_host.cpp", "lower_tiled.cpp", "kernel_direct.cu", "kernel_tiled.cu"],
+    "libfiona.so": ["fiona_host.cpp", "lower_tiled.cpp", "plan_compile.cpp", "kernel_direct.cu",
+                    "kernel_tiled.cu"],
     "libfiona_workload.so": ["workload_fill.cu"],
 }
 

@@ -745,10 +745,10 @@ static int check_eval_args(const fiona_plan *p, const void *in, const void *pt, 
 }
 
 static int launch_range(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
-                        uint64_t *out, uint32_t l0, uint32_t l1)
+                        uint64_t *out, uint32_t l0, uint32_t l1, uint32_t layout_L)
 {
-    if (p->kernel == 1) return launch_tiled(p, stream, in, pt, out, l0, l1);
-    return launch_direct(p, stream, in, pt, out, l0, l1);
+    if (p->kernel == 1) return launch_tiled(p, stream, in, pt, out, l0, l1, layout_L);
+    return launch_direct(p, stream, in, pt, out, l0, l1, layout_L);
 }
 
 extern "C" int fiona_linear_eval(const fiona_plan *p, void *stream, const uint64_t *in,
@@ -758,7 +758,20 @@ extern "C" int fiona_linear_eval(const fiona_plan *p, void *stream, const uint64
     if (rc) return rc;
     if (p->hp.n_out == 0) return FIONA_OK;
     DeviceGuard g(p->ctx->device);
-    return launch_range(p, stream, in, pt, out, 0, p->ctx->L);
+    return launch_range(p, stream, in, pt, out, 0, p->ctx->L, p->ctx->L);
+}
+
+extern "C" int fiona_linear_eval_level(const fiona_plan *p, void *stream, uint32_t L_eval,
+                                       const uint64_t *in, const uint64_t *pt, uint64_t *out)
+{
+    if (!p) return set_error(FIONA_ERR_ARG, "linear_eval_level: null plan");
+    if (L_eval < 1 || L_eval > p->ctx->L)
+        return set_error(FIONA_ERR_ARG, "linear_eval_level: level %u outside [1, %u]", L_eval, p->ctx->L);
+    int rc = check_eval_args(p, in, pt, out);
+    if (rc) return rc;
+    if (p->hp.n_out == 0) return FIONA_OK;
+    DeviceGuard g(p->ctx->device);
+    return launch_range(p, stream, in, pt, out, 0, L_eval, L_eval);
 }
 
 extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const uint64_t *h_in,
@@ -794,7 +807,7 @@ extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const u
         }
         if ((e = cudaEventRecord(ev[2 * c], sin)) != cudaSuccess) break;
         if ((e = cudaStreamWaitEvent(s, ev[2 * c], 0)) != cudaSuccess) break;
-        rc = launch_range(p, s, d_in, d_pt, d_out, l0, l1);
+        rc = launch_range(p, s, d_in, d_pt, d_out, l0, l1, L);
         if (rc) break;
         if ((e = cudaEventRecord(ev[2 * c + 1], s)) != cudaSuccess) break;
         if ((e = cudaStreamWaitEvent(sout, ev[2 * c + 1], 0)) != cudaSuccess) break;

@@ -90,9 +90,11 @@ struct fiona_plan {
     size_t static_off[6] = {0, 0, 0, 0, 0, 0};  // limbs, outs, segs, ops, raw_in, raw_pt
 };
 
-// kernels.cu
+// kernel_direct.cu.  Launches evaluate limbs [limb_begin, limb_end) of
+// buffers laid out with `layout_L` limbs per poly (the ctx's L, or fewer for
+// an evaluation at a lower level).
 int launch_direct(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
-                  uint64_t *out, uint32_t limb_begin, uint32_t limb_end);
+                  uint64_t *out, uint32_t limb_begin, uint32_t limb_end, uint32_t layout_L);
 int launch_check_residues(const fiona_ctx *ctx, void *stream, const uint64_t *data,
                           uint64_t count);
 int launch_direct_static(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
@@ -103,7 +105,7 @@ extern const size_t kStaticAreaBytes;
 int lower_tiled(fiona_plan *p);
 void free_tiled(fiona_plan *p);
 int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
-                 uint64_t *out, uint32_t limb_begin, uint32_t limb_end);
+                 uint64_t *out, uint32_t limb_begin, uint32_t limb_end, uint32_t layout_L);
 
 // fiona_host.cpp
 int set_error(int code, const char *fmt, ...);

@@ -127,14 +127,14 @@ __global__ void check_residues_kernel(const uint64_t *__restrict__ data, uint64_
 }  // namespace
 
 int launch_direct(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
-                  uint64_t *out, uint32_t l0, uint32_t l1)
+                  uint64_t *out, uint32_t l0, uint32_t l1, uint32_t layout_L)
 {
     const fiona_ctx *ctx = p->ctx;
     if (l1 <= l0) return FIONA_OK;
     dim3 grid((ctx->N / 2 + kDirectThreads - 1) / kDirectThreads, l1 - l0, p->hp.n_out);
     direct_kernel<<<grid, kDirectThreads, 0, (cudaStream_t)stream>>>(
         in, pt, out, ctx->d_limbs, p->d_dir_out, p->d_dir_seg, p->d_sig_ops, p->d_raw_input,
-        p->d_raw_pt, ctx->N, ctx->L, l0, p->mac_budget);
+        p->d_raw_pt, ctx->N, layout_L, l0, p->mac_budget);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "direct kernel launch: %s", cudaGetErrorString(e));
     return FIONA_OK;

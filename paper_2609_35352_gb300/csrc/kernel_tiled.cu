@@ -235,38 +235,41 @@ struct Arith<true> {
 
 // Sum of the n source tiles (both polys) named by the 16-bit indices packed
 // two per word from schedule byte offset `wp`; `src` = this lane's offset in
-// the source region.  K indices per step (each index decoded once, its two
-// polys read at offsets 0 and TB), their loads independent.  Returns the
-// offset just past the run's words.
+// the source region.  K indices per step (each decoded once, its two polys
+// read at offsets 0 and TB), their loads independent, and the next step's
+// index words requested before this step's additions (the last request may
+// read words past the run: they lie inside the dynamic shared memory, which
+// continues with the source region, and are not used).  Returns the offset
+// just past the run's words.
 template <int C, uint32_t TB>
 __device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32_t wp, uint32_t n, V<C> &s0,
                                             V<C> &s1)
 {
     constexpr uint32_t PB = 2 * TB;
-    constexpr uint32_t K = C == 1 ? 4 : 2;  // 4 independent loads of C words in flight per poly pair
+    constexpr uint32_t K = C == 1 ? 8 : 2;  // 2K loads of C words in flight
+    constexpr uint32_t NW = K / 2;          // index words per step
     uint32_t k = 0;
-    for (; k + K <= n; k += K, wp += 2 * K) {
-        uint32_t o[K];
+    if (n >= K) {
+        uint32_t w[NW];
 #pragma unroll
-        for (uint32_t j = 0; j < K; j += 2) {
-            const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp + 2 * j);
-            o[j] = src + (w & 0xffffu) * PB;
-            o[j + 1] = src + (w >> 16) * PB;
-        }
-        V<C> a[K], b[K];
+        for (uint32_t j = 0; j < NW; ++j) w[j] = *reinterpret_cast<const uint32_t *>(sm + wp + 4 * j);
+        for (; k + K <= n; k += K, wp += 4 * NW) {
+            V<C> a[K], b[K];
 #pragma unroll
-        for (uint32_t j = 0; j < K; ++j) {
-            a[j] = lds<C>(sm, o[j]);
-            b[j] = lds<C>(sm, o[j] + TB);
-        }
+            for (uint32_t j = 0; j < K; ++j) {
+                const uint32_t o = src + ((j & 1) ? (w[j / 2] >> 16) : (w[j / 2] & 0xffffu)) * PB;
+                a[j] = lds<C>(sm, o);
+                b[j] = lds<C>(sm, o + TB);
+            }
 #pragma unroll
-        for (int x = 0; x < C; ++x) {
-            if constexpr (K == 4) {  // two three-input additions per poly
-                s0.x[x] = s0.x[x] + (a[0].x[x] + a[1].x[x] + a[2].x[x]) + a[3].x[x];
-                s1.x[x] = s1.x[x] + (b[0].x[x] + b[1].x[x] + b[2].x[x]) + b[3].x[x];
-            } else {
-                s0.x[x] = s0.x[x] + a[0].x[x] + a[1].x[x];
-                s1.x[x] = s1.x[x] + b[0].x[x] + b[1].x[x];
+            for (uint32_t j = 0; j < NW; ++j) w[j] = *reinterpret_cast<const uint32_t *>(sm + wp + 4 * NW + 4 * j);
+#pragma unroll
+            for (int x = 0; x < C; ++x) {
+#pragma unroll
+                for (uint32_t j = 0; j + 1 < K; j += 2) {  // three-input additions
+                    s0.x[x] = s0.x[x] + a[j].x[x] + a[j + 1].x[x];
+                    s1.x[x] = s1.x[x] + b[j].x[x] + b[j + 1].x[x];
+                }
             }
         }
     }
@@ -601,7 +604,7 @@ int tiled_configure_kernel(int C, bool narrow, uint32_t P, size_t smem)
 }
 
 int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
-                 uint64_t *out, uint32_t l0, uint32_t l1)
+                 uint64_t *out, uint32_t l0, uint32_t l1, uint32_t layout_L)
 {
     const TiledSchedule *ts = p->tiled;
     if (!ts) return set_error(FIONA_ERR_ARG, "tiled kernel not available for this plan");
@@ -612,6 +615,8 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     a.out = out;
     a.limb0 = l0;
     a.n_limbs = l1 - l0;
+    a.L = layout_L;
+    a.pt_stride = layout_L * a.N;
     const uint32_t tiles = a.n_limbs * a.tiles_per_limb;
     const uint32_t resident = ts->ctas_per_sm * (uint32_t)std::max(p->ctx->sm_count, 1);
     dim3 grid(std::min(tiles, resident));

@@ -669,10 +669,12 @@ int lower_tiled(fiona_plan *p)
 
     // -- forming shared sums once per tile is a phase of its own (a barrier per
     //    DAG level, no plaintext traffic issued meanwhile): measured on the ViT
-    //    and BERT layers it costs more than the additions it saves (about 9% of
-    //    the signed operands there), so sums are formed only when they save at
-    //    least 15%; otherwise every use is expanded (the same residues).  A
-    //    tuning override with a fourth field keeps the sums in play.
+    //    and BERT layers it costs more than the additions it saves (9% of the
+    //    signed operands with the generated sums, 12-17% with the compiled
+    //    ones; VGG's compiled sums, 27%, gain under 1%), so sums are formed
+    //    only when they save at least 30%; otherwise every use is expanded
+    //    (the same residues).  A tuning override with a fourth field keeps
+    //    the sums in play.
     bool force_keep = false;
     if (const char *env = getenv("FIONA_TILED_SHAPE")) {
         int c = 0, w = 0, d = 0, keep = -1;
@@ -684,7 +686,7 @@ int lower_tiled(fiona_plan *p)
         for (auto &w : flat.work)
             for (auto &sg : w.segs) opnds += (double)(sg.plus.size() + sg.minus.size());
         for (uint32_t k : rank) save += ni.benefit[k];
-        if (save < 0.15 * opnds) rank.clear();
+        if (save < 0.30 * opnds) rank.clear();
     }
 
     // -- shape search

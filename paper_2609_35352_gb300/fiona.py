@@ -37,8 +37,15 @@ KERNELS = {"auto": FIONA_KERNEL_AUTO, "direct": FIONA_KERNEL_DIRECT, "tiled": FI
 EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona_plan_destroy",
             "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host",
             "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version",
-            "fiona_plan_select_kernel", "fiona_device_check", "fiona_linear_eval_static")
+            "fiona_plan_select_kernel", "fiona_device_check", "fiona_linear_eval_static",
+            "fiona_linear_eval_level", "fiona_plan_compile")
 STATIC_AREA_BYTES = 1 << 20
+
+
+FIONA_COMPILE_SHARE = 1
+FIONA_COMPILE_SHARE_EXACT = 2
+ROUTE_DTYPE = np.dtype([("kind", "i1"), ("sign", "i1"), ("reserved", "<u2"), ("pt", "<u4")])
+assert ROUTE_DTYPE.itemsize == 8
 
 
 class FionaError(RuntimeError):
@@ -100,6 +107,10 @@ def lib() -> ctypes.CDLL:
         L.fiona_device_check.argtypes = [p, p]
         L.fiona_device_check.restype = i32
         L.fiona_linear_eval_static.argtypes = [p, p, p, p, p]
+        L.fiona_linear_eval_level.argtypes = [p, p, u32, p, p, p]
+        L.fiona_linear_eval_level.restype = i32
+        L.fiona_plan_compile.argtypes = [u32, u32, u32, p, u32, p, p, p, p, p, p, p, p, p, p]
+        L.fiona_plan_compile.restype = i32
         L.fiona_linear_eval_static.restype = i32
         _lib = L
     return _lib
@@ -232,6 +243,15 @@ class Plan:
         return lib().fiona_linear_eval(self.handle, stream_handle(stream), addr(inputs),
                                        addr(plaintexts), addr(outputs))
 
+    def eval_level(self, L_eval, inputs, plaintexts, outputs, stream=None) -> None:
+        """fiona_linear_eval_level: buffers holding the first L_eval limbs."""
+        _check(lib().fiona_linear_eval_level(self.handle, stream_handle(stream), int(L_eval), addr(inputs),
+                                             addr(plaintexts), addr(outputs)), "fiona_linear_eval_level")
+
+    def eval_level_status(self, L_eval, inputs, plaintexts, outputs, stream=None) -> int:
+        return lib().fiona_linear_eval_level(self.handle, stream_handle(stream), int(L_eval), addr(inputs),
+                                             addr(plaintexts), addr(outputs))
+
     def eval_static(self, inputs, plaintexts, outputs, stream=None) -> int:
         """fiona_linear_eval_static: no device allocation (returns the status)."""
         return lib().fiona_linear_eval_static(self.handle, stream_handle(stream), addr(inputs),
@@ -281,3 +301,35 @@ def device_fill(dst, outer: int, L: int, N: int, moduli, key: int, mode: int = 0
                                             q.ctypes.data, key, mode)
     if rc != 0:
         raise RuntimeError("fiona_workload_fill failed (%d)" % rc)
+
+
+# -- host plan compiler -------------------------------------------------------
+def compile_plan(n_in: int, n_out: int, n_pt: int, routes: np.ndarray, share: bool = True,
+                 exact: bool = False):
+    """fiona_plan_compile: the dense route matrix ``routes`` (ROUTE_DTYPE,
+    shape [n_out][n_in]) to a plan description (workloads.Plan) for
+    ``Plan(ctx, desc)``: terms, scale groups and, with ``share``, shared
+    signed sums (``exact``: accept by the exact Add/Sub saving)."""
+    from . import workloads as W
+    r = np.ascontiguousarray(routes, dtype=ROUTE_DTYPE).reshape(-1)
+    if r.shape[0] != n_in * n_out:
+        raise ValueError("routes must hold n_out * n_in entries")
+    cap = max(n_in * n_out, 1)
+    offs = np.zeros(n_out + 1, np.uint32)
+    terms = np.zeros(cap, W.TERM_DTYPE)
+    gsp = np.zeros(cap, np.uint32)
+    gout = np.zeros(cap, np.uint32)
+    noffs = np.zeros(cap + 1, np.uint32)
+    ch = np.zeros(cap, W.CHILD_DTYPE)
+    us = np.zeros(cap, W.USE_DTYPE)
+    ng, nn, nu = ctypes.c_uint32(), ctypes.c_uint32(), ctypes.c_uint32()
+    flags = (FIONA_COMPILE_SHARE if share else 0) | (FIONA_COMPILE_SHARE_EXACT if share and exact else 0)
+    _check(lib().fiona_plan_compile(n_in, n_out, n_pt, r.ctypes.data if r.size else None, flags,
+                                    offs.ctypes.data, terms.ctypes.data, ctypes.byref(ng), gsp.ctypes.data,
+                                    gout.ctypes.data, ctypes.byref(nn), noffs.ctypes.data, ch.ctypes.data,
+                                    ctypes.byref(nu), us.ctypes.data), "fiona_plan_compile")
+    n_terms = int(offs[n_out])
+    return W.Plan(n_in=n_in, n_out=n_out, n_pt=n_pt, term_offsets=offs, terms=terms[:n_terms].copy(),
+                  group_scale_pt=gsp[:ng.value].copy(), group_output=gout[:ng.value].copy(),
+                  node_offsets=noffs[:nn.value + 1].copy(), children=ch[:int(noffs[nn.value])].copy(),
+                  uses=us[:nu.value].copy())

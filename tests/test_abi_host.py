@@ -226,3 +226,15 @@ def test_edge_plans_accepted():
     s = F.Plan(ctx_none(), p).stats()
     assert s["n_skipped_terms"] == 2 and s["n_scale_groups_used"] == 0
     assert s["n_plaintexts_used"] == 1 and s["n_inputs_used"] == 1
+
+
+def test_lower_level_arguments():
+    """fiona_linear_eval_level checks the level before anything else; a
+    validation-only context then refuses to evaluate."""
+    wl = W.make_workload("tiny")
+    ctx = F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE)
+    plan = F.Plan(ctx, wl.plan)
+    buf = np.zeros(16, dtype=np.uint64)
+    for bad in (0, wl.L + 1):
+        assert plan.eval_level_status(bad, buf, buf, buf) == F.FIONA_ERR_ARG
+    assert plan.eval_level_status(1, buf, buf, buf) == F.FIONA_ERR_NODEVICE

@@ -89,6 +89,65 @@ def test_tiled_shapes(name, N, L, shape, monkeypatch):
     assert dl.ctx.device_check() == F.FIONA_OK
 
 
+@pytest.mark.parametrize("kernel", ["direct", "tiled"])
+@pytest.mark.parametrize("name,N,L,levels", [("tiny", None, None, [1, 2]), ("vit", 2048, 3, [1, 2]),
+                                              ("overflow50", None, None, [1])])
+def test_lower_level_parity(name, N, L, levels, kernel):
+    """fiona_linear_eval_level: buffers holding the first L_eval limbs, the
+    same plan; the oracle on the first L_eval moduli."""
+    wl = W.make_workload(name, N=N, L=L)
+    ctx = F.Context(wl.N, wl.moduli, device=0)
+    plan = F.Plan(ctx, wl.plan)
+    plan.select_kernel(kernel)
+    X, P = wl.host_inputs(), wl.host_plaintexts()
+    p = wl.plan
+    for Le in levels:
+        Xl = np.ascontiguousarray(X[:, :, :Le, :])
+        Pl = np.ascontiguousarray(P[:, :Le, :])
+        d_out = torch.full((p.n_out * 2 * Le * wl.N,), -1, dtype=torch.int64, device="cuda")
+        plan.eval_level(Le, to_device(Xl), to_device(Pl), d_out)
+        torch.cuda.synchronize()
+        got = to_host(d_out).reshape(p.n_out, 2, Le, wl.N)
+        want = oracle.linear_eval(p, wl.moduli[:Le], Xl, Pl)
+        mism = np.argwhere(got != want)
+        assert mism.shape[0] == 0, (Le, mism[:5].tolist())
+    assert plan.eval_level_status(0, to_device(X), to_device(P), d_out) == F.FIONA_ERR_ARG
+    assert plan.eval_level_status(wl.L + 1, to_device(X), to_device(P), d_out) == F.FIONA_ERR_ARG
+
+
+@pytest.mark.parametrize("shape", [None, "2,8,1,64", "1,4,0,64,4"])
+def test_compiled_plan_parity(shape, monkeypatch):
+    """A dense layer through the host plan compiler (shared sums found by the
+    Sec. 4.2 search), evaluated by both kernels (the shapes keep the sums in
+    play, so the kernel forms them per tile), against the oracle's flat form."""
+    if shape:
+        monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+    rng = np.random.default_rng(7)
+    n_in, n_out = 24, 12
+    r = np.zeros((n_out, n_in), F.ROUTE_DTYPE)
+    n_raw = 0
+    for j in range(n_out):
+        for i in range(n_in):
+            u = rng.random()
+            if u < 0.3:
+                r[j, i] = (W.TERM_RAW, 0, 0, n_out + n_raw)
+                n_raw += 1
+            else:
+                r[j, i] = (W.TERM_TERNARY, 0 if u < 0.35 else int(rng.choice([-1, 1])), 0, j)
+    d = F.compile_plan(n_in, n_out, n_out + n_raw, r, share=True, exact=True)
+    assert d.node_offsets.shape[0] > 1
+    wl = W.Workload("compiled", 2048, W.ntt_primes(2048, 50, 2), d, 99)
+    dl = DeviceLayer(wl)
+    want = oracle.linear_eval(d, wl.moduli, dl.X, dl.P)
+    for kernel in ("direct", "tiled"):
+        dl.plan.select_kernel(kernel)
+        dl.d_out.fill_(-1)
+        dl.run()
+        assert np.array_equal(dl.outputs(), want), kernel
+    if shape:
+        assert dl.plan.stats()["nodes_materialized"] > 0
+
+
 def test_edge_plans():
     R, T = W.TERM_RAW, W.TERM_TERNARY
     qs = W.ntt_primes(1024, 50, 3)
