@@ -6,6 +6,8 @@ CPU-baseline leg of ``bench.py`` are the only callers.  The product path
 
 Contents
   oracle.c       schoolbook modular evaluation of the layer (flat and DAG form)
+  rescale.c      negacyclic NTT (by definition and radix-2) and the rescale by
+                 the last prime that follows the layer
   crt.py         brute-force evaluation over Z_Q with Python integers (pin P2)
   ckks_tiny.py   tiny-N CKKS encode/encrypt/decrypt round trip (pin P3)
 
@@ -16,3 +18,4 @@ full modulus Q, a CKKS round trip against a float64 slot-wise mat-vec,
 special cases with closed forms, and a planted-mistake check.
 """
 from .liboracle import build, linear_eval, linear_eval_dag, load, load_variant  # noqa: F401
+from .liboracle import intt, min_root, ntt, rescale  # noqa: F401

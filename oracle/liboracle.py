@@ -10,6 +10,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
+_SRCS = [_SRC, os.path.join(_HERE, "rescale.c")]
 _OUT_DIR = os.path.join(_HERE, "_build")
 _LIB = os.path.join(_OUT_DIR, "liboracle.so")
 _handle: Optional[ctypes.CDLL] = None
@@ -18,10 +19,9 @@ _handle: Optional[ctypes.CDLL] = None
 def build(force: bool = False) -> str:
     """Compile oracle.c with the host C compiler (plain -O2, no tuning)."""
     os.makedirs(_OUT_DIR, exist_ok=True)
-    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+    if force or not os.path.exists(_LIB) or any(os.path.getmtime(_LIB) < os.path.getmtime(f) for f in _SRCS):
         tmp = _LIB + ".tmp%d" % os.getpid()
-        subprocess.run(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-o", tmp, _SRC],
-                       check=True)
+        subprocess.run(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-o", tmp] + _SRCS, check=True)
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -36,6 +36,17 @@ def _setup(lib: ctypes.CDLL) -> ctypes.CDLL:
                                            u32, p, u32, p, p, p, p, u32, p, p, p, p,
                                            p, p, p]
     lib.oracle_linear_eval_dag.restype = ctypes.c_int
+    if hasattr(lib, "oracle_rescale"):
+        lib.oracle_min_root.argtypes = [u64, u32]
+        lib.oracle_min_root.restype = u64
+        for f in ("oracle_ntt_direct", "oracle_intt_direct"):
+            getattr(lib, f).argtypes = [p, p, u32, u64, u64]
+            getattr(lib, f).restype = None
+        for f in ("oracle_ntt_fast", "oracle_intt_fast"):
+            getattr(lib, f).argtypes = [p, u32, u64, u64]
+            getattr(lib, f).restype = None
+        lib.oracle_rescale.argtypes = [u64, u32, u32, p, p, p, ctypes.c_int]
+        lib.oracle_rescale.restype = ctypes.c_int
     return lib
 
 
@@ -117,4 +128,49 @@ def linear_eval_dag(plan, moduli, inputs: np.ndarray, plaintexts: np.ndarray,
                                     _ptr(inputs), _ptr(plaintexts), _ptr(out))
     if rc != 0:
         raise ValueError("oracle rejected the plan or its DAG")
+    return out
+
+
+# -- rescale (rescale.c) --------------------------------------------------------
+def min_root(q: int, N: int) -> int:
+    """The least primitive 2N-th root of unity mod q."""
+    return int(load().oracle_min_root(q, N))
+
+
+def ntt(a: np.ndarray, q: int, fast: bool = True) -> np.ndarray:
+    """Forward NTT of one length-N residue vector (bit-reversed order)."""
+    a = _c(a, np.uint64)
+    N = a.shape[0]
+    psi = min_root(q, N)
+    if fast:
+        out = a.copy()
+        load().oracle_ntt_fast(_ptr(out), N, q, psi)
+    else:
+        out = np.zeros_like(a)
+        load().oracle_ntt_direct(_ptr(a), _ptr(out), N, q, psi)
+    return out
+
+
+def intt(A: np.ndarray, q: int, fast: bool = True) -> np.ndarray:
+    A = _c(A, np.uint64)
+    N = A.shape[0]
+    psi = min_root(q, N)
+    if fast:
+        out = A.copy()
+        load().oracle_intt_fast(_ptr(out), N, q, psi)
+    else:
+        out = np.zeros_like(A)
+        load().oracle_intt_direct(_ptr(A), _ptr(out), N, q, psi)
+    return out
+
+
+def rescale(moduli, polys: np.ndarray, fast: bool = True) -> np.ndarray:
+    """Rescale polys [count][L][N] (NTT form) by the last modulus -> [count][L-1][N]."""
+    y = _c(polys, np.uint64)
+    count, L, N = y.shape
+    out = np.zeros((count, L - 1, N), np.uint64)
+    qs = _c(list(moduli)[:L], np.uint64)
+    rc = load().oracle_rescale(count, N, L, _ptr(qs), _ptr(y), _ptr(out), 1 if fast else 0)
+    if rc != 0:
+        raise ValueError("oracle_rescale: arguments it cannot evaluate")
     return out
