@@ -204,6 +204,7 @@ extern "C" void fiona_ctx_destroy(fiona_ctx *ctx)
         cudaFree(ctx->d_limbs);
         cudaFree(ctx->d_flag);
         cudaFree(ctx->d_kerr);
+        free_rescale_tables(ctx);
     }
     delete ctx;
 }
@@ -844,6 +845,58 @@ extern "C" int fiona_linear_eval_static(const fiona_plan *p, void *stream, const
         return launch_direct_static(p, stream, in, pt, out);
     }
     return launch_direct_static(p, stream, in, pt, out);
+}
+
+static bool overlaps(const void *a, uint64_t a_bytes, const void *b, uint64_t b_bytes)
+{
+    const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+    return a_bytes && b_bytes && x < y + b_bytes && y < x + a_bytes;
+}
+
+static int check_rescale_args(const fiona_ctx *ctx, uint32_t L_cur, uint64_t count, const uint64_t *polys,
+                              const uint64_t *out, const char *who)
+{
+    if (!ctx) return set_error(FIONA_ERR_ARG, "%s: null ctx", who);
+    if (ctx->device == FIONA_DEVICE_NONE) return set_error(FIONA_ERR_NODEVICE, "%s: validation-only context", who);
+    if (L_cur < 2 || L_cur > ctx->L)
+        return set_error(FIONA_ERR_ARG, "%s: level %u outside [2, %u]", who, L_cur, ctx->L);
+    if (count > (1ull << 40) / ((uint64_t)L_cur * ctx->N))
+        return set_error(FIONA_ERR_ARG, "%s: %llu polys", who, (unsigned long long)count);
+    if (count == 0) return FIONA_OK;
+    if (!polys || !out) return set_error(FIONA_ERR_ARG, "%s: null buffer", who);
+    if (((uintptr_t)polys | (uintptr_t)out) & 15)
+        return set_error(FIONA_ERR_ARG, "%s: buffers must be 16-byte aligned", who);
+    const uint64_t poly_bytes = (uint64_t)ctx->N * 8;
+    if (overlaps(polys, count * L_cur * poly_bytes, out, count * (L_cur - 1) * poly_bytes))
+        return set_error(FIONA_ERR_ARG, "%s: output overlaps the input", who);
+    return FIONA_OK;
+}
+
+extern "C" int fiona_rescale(const fiona_ctx *ctx, void *stream, uint32_t L_cur, uint64_t count, uint64_t *polys,
+                             uint64_t *out)
+{
+    int rc = check_rescale_args(ctx, L_cur, count, polys, out, "rescale");
+    if (rc) return rc;
+    DeviceGuard g(ctx->device);
+    return launch_rescale(ctx, stream, L_cur, count, polys, out);
+}
+
+extern "C" int fiona_linear_eval_rescale(const fiona_plan *p, void *stream, uint32_t L_eval, const uint64_t *in,
+                                         const uint64_t *pt, uint64_t *work, uint64_t *out)
+{
+    int rc = check_eval_args(p, in, pt, work);
+    if (rc) return rc;
+    const uint64_t count = 2ull * p->hp.n_out;
+    rc = check_rescale_args(p->ctx, L_eval, count, work, out, "linear_eval_rescale");
+    if (rc) return rc;
+    const uint64_t poly_bytes = (uint64_t)p->ctx->N * 8;
+    if (overlaps(out, count * (L_eval - 1) * poly_bytes, in, 2ull * p->hp.n_in * L_eval * poly_bytes))
+        return set_error(FIONA_ERR_ARG, "linear_eval_rescale: output overlaps the inputs");
+    if (p->hp.n_out == 0) return FIONA_OK;
+    DeviceGuard g(p->ctx->device);
+    rc = launch_range(p, stream, in, pt, work, 0, L_eval, L_eval);
+    if (rc) return rc;
+    return launch_rescale(p->ctx, stream, L_eval, count, work, out);
 }
 
 extern "C" int fiona_check_residues(const fiona_ctx *ctx, void *stream, const uint64_t *data,

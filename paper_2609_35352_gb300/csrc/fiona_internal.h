@@ -50,6 +50,7 @@ struct fiona_ctx {
     int *d_kerr = nullptr;          // set by a kernel whose bounded wait gave up
     int sm_count = 0;
     size_t smem_optin = 0;
+    mutable void *d_ntt = nullptr;  // rescale tables, built on the first rescale (rescale.cu)
 };
 
 struct HostPlan {
@@ -106,6 +107,12 @@ int lower_tiled(fiona_plan *p);
 void free_tiled(fiona_plan *p);
 int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
                  uint64_t *out, uint32_t limb_begin, uint32_t limb_end, uint32_t layout_L);
+
+// rescale.cu.  Rescales `count` polys [count][Lc][N] (the last limb of each
+// is overwritten with its coefficients) into out [count][Lc-1][N].
+int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t count, uint64_t *polys,
+                   uint64_t *out);
+void free_rescale_tables(const fiona_ctx *ctx);
 
 // fiona_host.cpp
 int set_error(int code, const char *fmt, ...);

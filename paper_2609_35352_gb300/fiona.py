@@ -38,7 +38,8 @@ EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona
             "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host",
             "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version",
             "fiona_plan_select_kernel", "fiona_device_check", "fiona_linear_eval_static",
-            "fiona_linear_eval_level", "fiona_plan_compile")
+            "fiona_linear_eval_level", "fiona_plan_compile", "fiona_rescale",
+            "fiona_linear_eval_rescale")
 STATIC_AREA_BYTES = 1 << 20
 
 
@@ -109,6 +110,10 @@ def lib() -> ctypes.CDLL:
         L.fiona_linear_eval_static.argtypes = [p, p, p, p, p]
         L.fiona_linear_eval_level.argtypes = [p, p, u32, p, p, p]
         L.fiona_linear_eval_level.restype = i32
+        L.fiona_rescale.argtypes = [p, p, u32, ctypes.c_uint64, p, p]
+        L.fiona_rescale.restype = i32
+        L.fiona_linear_eval_rescale.argtypes = [p, p, u32, p, p, p, p]
+        L.fiona_linear_eval_rescale.restype = i32
         L.fiona_plan_compile.argtypes = [u32, u32, u32, p, u32, p, p, p, p, p, p, p, p, p, p]
         L.fiona_plan_compile.restype = i32
         L.fiona_linear_eval_static.restype = i32
@@ -176,6 +181,16 @@ class Context:
         if rc not in (FIONA_OK, FIONA_ERR_TIMEOUT):
             _check(rc, "fiona_device_check")
         return rc
+
+    def rescale(self, L_cur, count, polys, out, stream=None) -> None:
+        """fiona_rescale: divide `count` polys ([count][L_cur][N], NTT form)
+        by q_{L_cur-1} into out ([count][L_cur-1][N]); the last limb of each
+        input poly is overwritten."""
+        _check(self.rescale_status(L_cur, count, polys, out, stream), "fiona_rescale")
+
+    def rescale_status(self, L_cur, count, polys, out, stream=None) -> int:
+        return lib().fiona_rescale(self.handle, stream_handle(stream), int(L_cur), int(count), addr(polys),
+                                   addr(out))
 
     def close(self) -> None:
         if getattr(self, "handle", None):
@@ -251,6 +266,16 @@ class Plan:
     def eval_level_status(self, L_eval, inputs, plaintexts, outputs, stream=None) -> int:
         return lib().fiona_linear_eval_level(self.handle, stream_handle(stream), int(L_eval), addr(inputs),
                                              addr(plaintexts), addr(outputs))
+
+    def eval_rescale(self, L_eval, inputs, plaintexts, work, outputs, stream=None) -> None:
+        """fiona_linear_eval_rescale: the layer at level L_eval into `work`,
+        then its rescale into `outputs` ([n_out][2][L_eval-1][N])."""
+        _check(self.eval_rescale_status(L_eval, inputs, plaintexts, work, outputs, stream),
+               "fiona_linear_eval_rescale")
+
+    def eval_rescale_status(self, L_eval, inputs, plaintexts, work, outputs, stream=None) -> int:
+        return lib().fiona_linear_eval_rescale(self.handle, stream_handle(stream), int(L_eval), addr(inputs),
+                                               addr(plaintexts), addr(work), addr(outputs))
 
     def eval_static(self, inputs, plaintexts, outputs, stream=None) -> int:
         """fiona_linear_eval_static: no device allocation (returns the status)."""

@@ -238,3 +238,16 @@ def test_lower_level_arguments():
     for bad in (0, wl.L + 1):
         assert plan.eval_level_status(bad, buf, buf, buf) == F.FIONA_ERR_ARG
     assert plan.eval_level_status(1, buf, buf, buf) == F.FIONA_ERR_NODEVICE
+
+
+def test_rescale_arguments_on_the_host():
+    """fiona_rescale and fiona_linear_eval_rescale refuse a null ctx or plan
+    and a validation-only context before touching any buffer."""
+    buf = np.zeros(16, dtype=np.uint64)
+    assert F.lib().fiona_rescale(None, None, 2, 1, F.addr(buf), F.addr(buf)) == F.FIONA_ERR_ARG
+    ctx = ctx_none()
+    assert ctx.rescale_status(2, 1, buf, buf) == F.FIONA_ERR_NODEVICE
+    wl = W.make_workload("tiny")
+    plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
+    assert plan.eval_rescale_status(2, buf, buf, buf, buf) == F.FIONA_ERR_NODEVICE
+    assert F.lib().fiona_linear_eval_rescale(None, None, 2, 0, 0, 0, 0) == F.FIONA_ERR_ARG
