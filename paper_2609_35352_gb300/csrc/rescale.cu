@@ -8,20 +8,43 @@
 // NTT form: A[k] = a(psi^(2 brv(k) + 1)) mod q, psi the least primitive
 // 2N-th root of unity mod q, brv reversing the log2(N) bits of k.
 //
-// A transform of N = 2^n points is two passes over memory, each a set of
-// independent sub-transforms held in shared memory (N = R1 * R2,
-// R1 = 2^floor(n/2)):
-//   high pass  the radix-2 stages whose butterfly distance is a multiple of
-//              R2: for a fixed low index lo, the R1 elements hi * R2 + lo
-//              form one sub-transform (a CTA takes tile / R1 of them, loaded
-//              as rows of consecutive elements);
-//   low pass   the remaining stages, inside blocks of R2 consecutive
-//              elements (a CTA takes tile / R2 blocks).
-// Forward stages run high then low (Cooley-Tukey: at the stage with m blocks,
-// block i uses psi^brv(m + i)); inverse stages low then high
-// (Gentleman-Sande with psi^-brv(m + i), then N^-1).  Products by table
-// constants use Shoup's method: with w' = floor(w * 2^64 / q), w < q < 2^63,
-// x*w - floor(x*w' / 2^64)*q lies in [0, 2q) for any 64-bit x.
+// Transform structure.  The radix-2 stages of an N = 2^n point transform
+// (Cooley-Tukey forward: at the stage with m blocks, block i pairs elements
+// at distance N / 2m with twiddle psi^brv(m + i); Gentleman-Sande inverse
+// with psi^-brv(m + i), then N^-1) are split between two passes over memory
+// (N = R1 * R2, R1 = 2^floor(n/2)):
+//   high pass  the first log2(R1) stages: for a fixed low index, the R1
+//              elements hi * R2 + lo form one sub-transform; a CTA takes
+//              tile / R1 of them (adjacent columns, so accesses coalesce);
+//   low pass   the other stages, inside blocks of R2 consecutive elements;
+//              a CTA takes tile / R2 blocks.
+// A pass runs its stages in rounds of up to 4: in a round each thread holds
+// the 2^K elements of one group in registers, spaced by the round's smallest
+// distance, and applies the round's K stages to them (a group needs 2^K - 1
+// twiddles).  Rounds hand over through shared memory ([sub-transform]
+// [position], one word of padding per row against bank conflicts); the first
+// and last rounds of a pass read and write global memory directly wherever
+// their access pattern coalesces.  The CTA's twiddles are copied to shared
+// memory (cp.async) while its data loads are in flight.  The forward stages
+// run high pass then low pass; the inverse stages low then high.  Kernels
+// are instantiated per log2 N, so all index arithmetic is constant-folded.
+//
+// Arithmetic.  Residues are 64-bit words and every modulus is below 2^60.
+// A product by a table constant w uses Shoup's precomputed w' = floor(w 2^64
+// / q): r = x w - floor(x w' / 2^64) q lies in [0, 2q) for any 64-bit x.  The
+// quotient is taken from three of the four 32-bit partial products of x w'
+// (the low-by-low one and the carries below bit 64 are dropped), which
+// underestimates it by at most 2, so r lies in [0, 4q).  Values are kept
+// lazily between stages:
+//   forward, general   in [0, 8q): x is brought below 4q before each
+//                      butterfly (x + t, x - t + 4q with t in [0, 4q));
+//   forward, q < 2^56  (and q_{Lc-1} < 4 q_l) no reduction at all: each stage
+//                      adds less than 4q to the bound, so after at most 17
+//                      stages values stay below 72q < 2^63;
+//   inverse            in [0, 4q): x + y is brought below 4q, and
+//                      x - y + 4q is only multiplied.
+// A pass makes its values canonical where it writes its final result.
+//
 // The rescale is four launches on the caller's stream: the two inverse passes
 // on the last limb of every poly (in place: it becomes the coefficients r),
 // then the two forward passes of every other limb; the first reads r and
@@ -41,8 +64,9 @@ namespace {
 
 typedef unsigned __int128 u128;
 
-constexpr uint32_t kTile = 4096;  // elements of one CTA's sub-transforms (32 KB)
+constexpr int kLogTileMax = 12;  // at most 4096 elements per CTA
 constexpr uint32_t kThreads = 256;
+constexpr int kLogNMin = 10, kLogNMax = 17;  // the ring dimensions a context accepts
 
 // per limb, in device memory (the tables follow the array of these)
 struct NttLimb {
@@ -54,178 +78,384 @@ struct NttLimb {
     ulonglong2 ninv;         // N^-1 mod q (Shoup)
 };
 
-struct Geo {
-    uint32_t N, n, n1;       // N = 2^n, R1 = 2^n1, R2 = 2^(n - n1)
-    uint32_t lt;             // log2(tile), tile = min(kTile, N)
-    uint32_t ltiles;         // log2(N / tile): tiles per transform
-    uint32_t Lc;             // limbs per poly: the level being rescaled
-};
-
-__device__ __forceinline__ uint64_t mul_shoup(uint64_t x, ulonglong2 w, uint64_t q)
+// x w mod q up to 3q: in [0, 4q) (see the file comment)
+__device__ __forceinline__ uint64_t mul_shoup_lazy(uint64_t x, ulonglong2 w, uint64_t q)
 {
-    const uint64_t qh = __umul64hi(x, w.y);
-    const uint64_t r = x * w.x - qh * q;
-    return r >= q ? r - q : r;
+    const uint32_t xl = (uint32_t)x, xh = (uint32_t)(x >> 32);
+    const uint32_t wl = (uint32_t)w.y, wh = (uint32_t)(w.y >> 32);
+    const uint64_t qh = (uint64_t)xh * wh + __umulhi(xh, wl) + __umulhi(xl, wh);
+    return x * w.x + qh * (0 - q);
 }
 
-__device__ __forceinline__ uint64_t addq(uint64_t a, uint64_t b, uint64_t q)
-{
-    const uint64_t s = a + b;
-    return s >= q ? s - q : s;
-}
+__device__ __forceinline__ uint64_t csub(uint64_t x, uint64_t c) { return x >= c ? x - c : x; }
 
-__device__ __forceinline__ uint64_t subq(uint64_t a, uint64_t b, uint64_t q) { return a >= b ? a - b : a + (q - b); }
+// x in [0, 4q) -> canonical
+__device__ __forceinline__ uint64_t canon4(uint64_t x, uint64_t q) { return csub(csub(x, 2 * q), q); }
 
 // x mod q for any 64-bit x: floor(x * mu64 / 2^64) is floor(x / q) or one less
 __device__ __forceinline__ uint64_t reduce_any(uint64_t x, uint64_t q, uint64_t mu64)
 {
-    const uint64_t r = x - __umul64hi(x, mu64) * q;
-    return r >= q ? r - q : r;
+    return csub(x - __umul64hi(x, mu64) * q, q);
+}
+
+// Cooley-Tukey butterfly (x + w y, x - w y); see the file comment for ranges
+template <bool FAST>
+__device__ __forceinline__ void ct_bfly(uint64_t &x, uint64_t &y, ulonglong2 w, uint64_t q)
+{
+    const uint64_t a = FAST ? x : csub(x, 4 * q);
+    const uint64_t t = mul_shoup_lazy(y, w, q);  // [0, 4q)
+    x = a + t;
+    y = a + 4 * q - t;
+}
+
+// Gentleman-Sande butterfly on [0, 4q): (x + y, w (x - y))
+__device__ __forceinline__ void gs_bfly(uint64_t &x, uint64_t &y, ulonglong2 w, uint64_t q)
+{
+    const uint64_t a = x, b = y;
+    x = csub(a + b, 4 * q);
+    y = mul_shoup_lazy(a + 4 * q - b, w, q);
 }
 
 // ---------------------------------------------------------------------------
-// High pass: columns [col0, col0 + C) with C = tile / R1, rows hi < R1; the
-// shared layout is s[hi * C + c].  Global stage st (0 <= st < n1) has
-// butterfly distance R1 >> (st + 1) rows.
+// Compile-time geometry
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void high_stages(uint64_t *s, const Geo &G, const NttLimb &T, bool inverse)
-{
-    const uint32_t lC = G.lt - G.n1, half = 1u << (G.lt - 1);
-    for (uint32_t i = 0; i < G.n1; ++i) {
-        const uint32_t st = inverse ? G.n1 - 1 - i : i;
-        const uint32_t lth = G.n1 - 1 - st;  // log2 of the distance in rows
-        const uint32_t m = 1u << st;
-        __syncthreads();
-        for (uint32_t b = threadIdx.x; b < half; b += kThreads) {
-            const uint32_t c = b & ((1u << lC) - 1), k = b >> lC;
-            const uint32_t hi = ((k >> lth) << (lth + 1)) | (k & ((1u << lth) - 1));
-            uint64_t *u = &s[(hi << lC) + c], *v = &s[((hi + (1u << lth)) << lC) + c];
-            const uint64_t x = *u;
-            if (!inverse) {
-                const uint64_t y = mul_shoup(*v, __ldg(&T.fwd[m + (k >> lth)]), T.q);
-                *u = addq(x, y, T.q);
-                *v = subq(x, y, T.q);
-            } else {
-                const uint64_t y = *v;
-                *u = addq(x, y, T.q);
-                *v = mul_shoup(subq(x, y, T.q), __ldg(&T.inv[m + (k >> lth)]), T.q);
-            }
+template <int LOGN>
+struct Shape {
+    static constexpr int n1 = LOGN / 2;
+    static constexpr int lt = LOGN < kLogTileMax ? LOGN : kLogTileMax;  // log2(tile)
+    static constexpr int ltiles = LOGN - lt;                            // log2(tiles per transform)
+};
+
+// A pass over a tile: 2^LSUBS sub-transforms of 2^S positions, in rounds.
+template <int S, int LSUBS, bool HIGH>
+struct PassShape {
+    static constexpr int s = S, lsubs = LSUBS, subs = 1 << LSUBS;
+    static constexpr int tile = 1 << (S + LSUBS);
+    static constexpr int pitch = (1 << S) + 1;
+    static constexpr int nr = (S + 3) / 4;
+    __host__ __device__ static constexpr int K(int r) { return S / nr + (r < S % nr ? 1 : 0); }
+    __host__ __device__ static constexpr int J0(int r) { return r == 0 ? 0 : J0(r - 1) + K(r - 1); }
+    static constexpr bool high = HIGH;
+    // shared memory: the staged twiddles (2^s entries for the high pass, at
+    // most one per tile element for the low pass), then the padded tile
+    static constexpr int tw_entries = HIGH ? 1 << S : 1 << (S + LSUBS);
+    static constexpr size_t smem_bytes = sizeof(ulonglong2) * tw_entries + sizeof(uint64_t) * subs * pitch;
+};
+
+template <int LOGN>
+using HighPass = PassShape<Shape<LOGN>::n1, Shape<LOGN>::lt - Shape<LOGN>::n1, true>;
+template <int LOGN>
+using LowPass = PassShape<LOGN - Shape<LOGN>::n1, Shape<LOGN>::lt - (LOGN - Shape<LOGN>::n1), false>;
+
+// Group g of round R: sub-transform `sub`, and the element positions
+// (hi << (lD + K)) + (i << lD) + lo, i < 2^K.  High pass: sub-transforms
+// fastest (adjacent columns); low pass: lo fastest (adjacent elements).
+template <class PS, int R>
+struct Group {
+    static constexpr int K = PS::K(R), J0 = PS::J0(R), LD = PS::s - J0 - K;
+    static constexpr int groups = PS::tile >> K;
+    static constexpr int per_thread = (groups + (int)kThreads - 1) / (int)kThreads;
+    uint32_t sub, hi, lo;
+    __device__ __forceinline__ explicit Group(uint32_t g)
+    {
+        if (PS::high) {
+            sub = g & (PS::subs - 1);
+            const uint32_t rest = g >> PS::lsubs;
+            lo = rest & ((1u << LD) - 1);
+            hi = rest >> LD;
+        } else {
+            lo = g & ((1u << LD) - 1);
+            const uint32_t rest = g >> LD;
+            sub = rest & (PS::subs - 1);
+            hi = rest >> PS::lsubs;
         }
     }
+    __device__ __forceinline__ uint32_t pos(int i) const { return (hi << (LD + K)) + ((uint32_t)i << LD) + lo; }
+    // twiddle of local stage J0 + k, block b of the group, in the staged layout
+    __device__ __forceinline__ uint32_t tw(int k, int b) const
+    {
+        const int j = J0 + k;
+        if (PS::high) return (1u << j) + (hi << k) + b;
+        return ((PS::subs << j) - PS::subs) + (((hi << k) + b) << PS::lsubs) + sub;
+    }
+};
+
+template <class PS, int R, int k, bool INV, bool FAST>
+__device__ __forceinline__ void group_stage(uint64_t (&x)[1 << PS::K(R)], const Group<PS, R> &G,
+                                            const ulonglong2 *stw, uint64_t q)
+{
+    constexpr int K = PS::K(R), h = 1 << (K - 1 - k);
+#pragma unroll
+    for (int b = 0; b < (1 << k); ++b) {
+        const ulonglong2 w = stw[G.tw(k, b)];
+#pragma unroll
+        for (int a = 0; a < h; ++a) {
+            if (INV)
+                gs_bfly(x[b * 2 * h + a], x[b * 2 * h + a + h], w, q);
+            else
+                ct_bfly<FAST>(x[b * 2 * h + a], x[b * 2 * h + a + h], w, q);
+        }
+    }
+}
+
+template <class PS, int R, bool INV, bool FAST>
+__device__ __forceinline__ void group_stages(uint64_t (&x)[1 << PS::K(R)], const Group<PS, R> &G,
+                                             const ulonglong2 *stw, uint64_t q)
+{
+    constexpr int K = PS::K(R);
+    if constexpr (!INV) {
+        group_stage<PS, R, 0, false, FAST>(x, G, stw, q);
+        if constexpr (K > 1) group_stage<PS, R, 1, false, FAST>(x, G, stw, q);
+        if constexpr (K > 2) group_stage<PS, R, 2, false, FAST>(x, G, stw, q);
+        if constexpr (K > 3) group_stage<PS, R, 3, false, FAST>(x, G, stw, q);
+    } else {
+        if constexpr (K > 3) group_stage<PS, R, 3, true, FAST>(x, G, stw, q);
+        if constexpr (K > 2) group_stage<PS, R, 2, true, FAST>(x, G, stw, q);
+        if constexpr (K > 1) group_stage<PS, R, 1, true, FAST>(x, G, stw, q);
+        group_stage<PS, R, 0, true, FAST>(x, G, stw, q);
+    }
+}
+
+// One round: every group of this thread is loaded (ld(sub, pos)), then
+// `between()` runs (once, on every thread), then the groups are transformed
+// and stored (st(sub, pos, value)).
+template <class PS, int R, bool INV, bool FAST, class Ld, class Between, class St>
+__device__ __forceinline__ void round(const ulonglong2 *stw, uint64_t q, Ld ld, Between between, St st)
+{
+    using Gr = Group<PS, R>;
+    constexpr int P = Gr::per_thread, E = 1 << Gr::K;
+    uint64_t x[P][E];
+#pragma unroll
+    for (int gi = 0; gi < P; ++gi) {
+        const uint32_t g = threadIdx.x + gi * kThreads;
+        if (Gr::groups % kThreads == 0 || g < Gr::groups) {
+            const Gr G(g);
+#pragma unroll
+            for (int i = 0; i < E; ++i) x[gi][i] = ld(G.sub, G.pos(i));
+        }
+    }
+    between();
+#pragma unroll
+    for (int gi = 0; gi < P; ++gi) {
+        const uint32_t g = threadIdx.x + gi * kThreads;
+        if (Gr::groups % kThreads == 0 || g < Gr::groups) {
+            const Gr G(g);
+            group_stages<PS, R, INV, FAST>(x[gi], G, stw, q);
+#pragma unroll
+            for (int i = 0; i < E; ++i) st(G.sub, G.pos(i), x[gi][i]);
+        }
+    }
+}
+
+// the rounds strictly between the first and the last, through shared memory
+template <class PS, int R, int REND, bool INV, bool FAST>
+__device__ __forceinline__ void middle_rounds(uint64_t *sm, const ulonglong2 *stw, uint64_t q)
+{
+    if constexpr (R != REND) {
+        round<PS, R, INV, FAST>(
+            stw, q, [&](uint32_t sub, uint32_t pos) { return sm[sub * PS::pitch + pos]; }, [] {},
+            [&](uint32_t sub, uint32_t pos, uint64_t v) { sm[sub * PS::pitch + pos] = v; });
+        __syncthreads();
+        middle_rounds<PS, (INV ? R - 1 : R + 1), REND, INV, FAST>(sm, stw, q);
+    }
+}
+
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem)
+{
+    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sa), "l"(gmem) : "memory");
+}
+
+// Stage the pass's twiddles (cp.async; waited by wait_twiddles).
+//   high pass  the entry of local stage j for position pos is 2^j + (pos >>
+//              (s - j)) for every sub-transform: entries [0, 2^s) are copied;
+//   low pass   sub-transform `sub` is poly row first + sub and its entry is
+//              ((R1 + first + sub) << j) + t, t < 2^j; stage j's entries
+//              are stored from (subs << j) - subs, t-major ([t][sub]), so
+//              that adjacent sub-transforms read adjacent words.
+template <int LOGN, class PS>
+__device__ __forceinline__ void stage_twiddles(ulonglong2 *stw, const ulonglong2 *tab, uint32_t first)
+{
+    if constexpr (PS::high) {
+        for (uint32_t e = threadIdx.x; e < (1u << PS::s); e += kThreads) cp_async16(&stw[e], &tab[e]);
+    } else {
+        const uint32_t u = (1u << Shape<LOGN>::n1) + first;
+#pragma unroll 1
+        for (int j = 0; j < PS::s; ++j) {
+            const uint32_t cnt = PS::subs << j, off = cnt - PS::subs;
+            for (uint32_t e = threadIdx.x; e < cnt; e += kThreads)
+                cp_async16(&stw[off + ((e & ((1u << j) - 1)) << PS::lsubs) + (e >> j)], &tab[(u << j) + e]);
+        }
+    }
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+
+__device__ __forceinline__ void wait_twiddles()
+{
+    asm volatile("cp.async.wait_all;\n" ::: "memory");
     __syncthreads();
 }
 
-// ---------------------------------------------------------------------------
-// Low pass: blocks [row0, row0 + B) with B = tile / R2, lo < R2; the shared
-// layout is s[r * R2 + lo].  Global stage st (n1 <= st < n) has butterfly
-// distance N >> (st + 1) < R2.
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ void low_stages(uint64_t *s, const Geo &G, uint32_t row0, const NttLimb &T,
-                                           bool inverse)
+// A coalesced sweep over the tile's elements e (tile / kThreads per thread):
+// every load first, then every store.
+template <class PS, class Ld, class St>
+__device__ __forceinline__ void sweep(Ld ld, St st)
 {
-    const uint32_t lR2 = G.n - G.n1, half = 1u << (G.lt - 1);
-    for (uint32_t i = 0; i < G.n - G.n1; ++i) {
-        const uint32_t st = inverse ? G.n - 1 - i : G.n1 + i;
-        const uint32_t ld = G.n - 1 - st;  // log2 of the distance
-        const uint32_t m = 1u << st;
-        __syncthreads();
-        for (uint32_t b = threadIdx.x; b < half; b += kThreads) {
-            const uint32_t r = b >> (lR2 - 1), k = b & ((1u << (lR2 - 1)) - 1);
-            const uint32_t lo = ((k >> ld) << (ld + 1)) | (k & ((1u << ld) - 1));
-            const uint32_t blk = (((row0 + r) << lR2) | lo) >> (ld + 1);
-            uint64_t *u = &s[(r << lR2) + lo], *v = u + (1u << ld);
-            const uint64_t x = *u;
-            if (!inverse) {
-                const uint64_t y = mul_shoup(*v, __ldg(&T.fwd[m + blk]), T.q);
-                *u = addq(x, y, T.q);
-                *v = subq(x, y, T.q);
-            } else {
-                const uint64_t y = *v;
-                *u = addq(x, y, T.q);
-                *v = mul_shoup(subq(x, y, T.q), __ldg(&T.inv[m + blk]), T.q);
-            }
-        }
+    constexpr int P = (PS::tile + (int)kThreads - 1) / (int)kThreads;
+    uint64_t v[P];
+#pragma unroll
+    for (int i = 0; i < P; ++i) {
+        const uint32_t e = threadIdx.x + i * kThreads;
+        if (PS::tile % kThreads == 0 || e < PS::tile) v[i] = ld(e);
     }
-    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < P; ++i) {
+        const uint32_t e = threadIdx.x + i * kThreads;
+        if (PS::tile % kThreads == 0 || e < PS::tile) st(e, v[i]);
+    }
 }
 
-// element e of a high-pass tile -> its index in the poly
-__device__ __forceinline__ size_t col_index(uint32_t e, const Geo &G, uint32_t col0)
-{
-    const uint32_t lC = G.lt - G.n1;
-    return ((size_t)(e >> lC) << (G.n - G.n1)) + col0 + (e & ((1u << lC) - 1));
-}
+#define FIONA_SMEM(PS)                                          \
+    extern __shared__ __align__(16) uint8_t smem_raw[];         \
+    ulonglong2 *stw = reinterpret_cast<ulonglong2 *>(smem_raw); \
+    uint64_t *sm = reinterpret_cast<uint64_t *>(stw + PS::tw_entries)
+
+struct Args {
+    uint64_t *polys;   // [count][Lc][N]
+    uint64_t *out;     // [count][Lc-1][N]
+    const NttLimb *T;
+    uint32_t Lc;
+};
 
 // ---------------------------------------------------------------------------
 // The four launches.  blockIdx.x = transform * tiles + tile; the transforms
 // are the polys (inverse passes) or poly * (Lc - 1) + limb (forward passes).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) k_inv_low(uint64_t *polys, Geo G, const NttLimb *T)
+
+// inverse, low stages, on the last limb in place: coalesced sweep in (the
+// first round's groups are runs of adjacent elements), rounds, the last
+// round (lo fastest) stores directly
+template <int LOGN>
+__global__ void __launch_bounds__(kThreads, 2) k_inv_low(Args A)
 {
-    __shared__ uint64_t s[kTile];
-    const uint32_t tile = blockIdx.x & ((1u << G.ltiles) - 1);
-    const uint64_t p = blockIdx.x >> G.ltiles;
-    const uint32_t row0 = tile << (G.lt - (G.n - G.n1));
-    uint64_t *g = polys + (p * G.Lc + (G.Lc - 1)) * G.N + ((size_t)tile << G.lt);
-    const NttLimb &Tl = T[G.Lc - 1];
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads) s[e] = g[e];
-    low_stages(s, G, row0, Tl, true);
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads) g[e] = s[e];
+    using SH = Shape<LOGN>;
+    using PS = LowPass<LOGN>;
+    FIONA_SMEM(PS);
+    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
+    const uint32_t first = tile << PS::lsubs;
+    uint64_t *g = A.polys + ((size_t)p * A.Lc + (A.Lc - 1)) * (1u << LOGN) + ((size_t)first << PS::s);
+    const NttLimb &Tl = A.T[A.Lc - 1];
+    const uint64_t q = Tl.q;
+    stage_twiddles<LOGN, PS>(stw, Tl.inv, first);
+    sweep<PS>([&](uint32_t e) { return g[e]; },
+              [&](uint32_t e, uint64_t v) { sm[(e >> PS::s) * PS::pitch + (e & ((1u << PS::s) - 1))] = v; });
+    wait_twiddles();
+    middle_rounds<PS, PS::nr - 1, 0, true, false>(sm, stw, q);
+    round<PS, 0, true, false>(
+        stw, q, [&](uint32_t sub, uint32_t pos) { return sm[sub * PS::pitch + pos]; }, [] {},
+        [&](uint32_t sub, uint32_t pos, uint64_t v) { g[(sub << PS::s) + pos] = v; });
 }
 
-__global__ void __launch_bounds__(kThreads) k_inv_high(uint64_t *polys, Geo G, const NttLimb *T)
+// inverse, high stages: the first round (sub-transforms fastest) loads
+// directly, the last stores r = N^-1 x, canonical
+template <int LOGN>
+__global__ void __launch_bounds__(kThreads, 3) k_inv_high(Args A)
 {
-    __shared__ uint64_t s[kTile];
-    const uint32_t tile = blockIdx.x & ((1u << G.ltiles) - 1);
-    const uint64_t p = blockIdx.x >> G.ltiles;
-    const uint32_t col0 = tile << (G.lt - G.n1);
-    uint64_t *g = polys + (p * G.Lc + (G.Lc - 1)) * G.N;
-    const NttLimb &Tl = T[G.Lc - 1];
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads) s[e] = g[col_index(e, G, col0)];
-    high_stages(s, G, Tl, true);
+    using SH = Shape<LOGN>;
+    using PS = HighPass<LOGN>;
+    constexpr uint32_t R2 = 1u << (LOGN - SH::n1);
+    FIONA_SMEM(PS);
+    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
+    const uint32_t first = tile << PS::lsubs;
+    uint64_t *g = A.polys + ((size_t)p * A.Lc + (A.Lc - 1)) * (1u << LOGN) + first;
+    const NttLimb &Tl = A.T[A.Lc - 1];
+    const uint64_t q = Tl.q;
     const ulonglong2 ninv = Tl.ninv;
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads)
-        g[col_index(e, G, col0)] = mul_shoup(s[e], ninv, Tl.q);
+    stage_twiddles<LOGN, PS>(stw, Tl.inv, first);
+    auto gload = [&](uint32_t sub, uint32_t pos) { return g[(size_t)pos * R2 + sub]; };
+    auto sload = [&](uint32_t sub, uint32_t pos) { return sm[sub * PS::pitch + pos]; };
+    auto sstore = [&](uint32_t sub, uint32_t pos, uint64_t v) { sm[sub * PS::pitch + pos] = v; };
+    auto gstore = [&](uint32_t sub, uint32_t pos, uint64_t v) {
+        g[(size_t)pos * R2 + sub] = canon4(mul_shoup_lazy(v, ninv, q), q);
+    };
+    if constexpr (PS::nr == 1) {
+        round<PS, 0, true, false>(stw, q, gload, wait_twiddles, gstore);
+    } else {
+        round<PS, PS::nr - 1, true, false>(stw, q, gload, wait_twiddles, sstore);
+        __syncthreads();
+        middle_rounds<PS, PS::nr - 2, 0, true, false>(sm, stw, q);
+        round<PS, 0, true, false>(stw, q, sload, [] {}, gstore);
+    }
 }
 
-// r (the last limb's coefficients) mod q_l, then the high forward stages, into out
-__global__ void __launch_bounds__(kThreads) k_fwd_high(const uint64_t *polys, uint64_t *out, Geo G,
-                                                       const NttLimb *T)
+// forward, high stages: r (the last limb's coefficients), reduced mod q_l
+// unless FAST, loaded directly by the first round; the last round stores
+// directly into out
+template <int LOGN, bool FAST>
+__global__ void __launch_bounds__(kThreads, 3) k_fwd_high(Args A)
 {
-    __shared__ uint64_t s[kTile];
-    const uint32_t tile = blockIdx.x & ((1u << G.ltiles) - 1);
-    const uint64_t t = blockIdx.x >> G.ltiles;
-    const uint64_t p = t / (G.Lc - 1);
-    const uint32_t l = (uint32_t)(t % (G.Lc - 1));
-    const uint32_t col0 = tile << (G.lt - G.n1);
-    const uint64_t *g = polys + (p * G.Lc + (G.Lc - 1)) * G.N;
-    const NttLimb &Tl = T[l];
+    using SH = Shape<LOGN>;
+    using PS = HighPass<LOGN>;
+    constexpr uint32_t R2 = 1u << (LOGN - SH::n1);
+    FIONA_SMEM(PS);
+    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), tr = blockIdx.x >> SH::ltiles;
+    const uint32_t p = tr / (A.Lc - 1), l = tr % (A.Lc - 1);
+    const uint32_t first = tile << PS::lsubs;
+    const uint64_t *g = A.polys + ((size_t)p * A.Lc + (A.Lc - 1)) * (1u << LOGN) + first;
+    uint64_t *o = A.out + (size_t)tr * (1u << LOGN) + first;
+    const NttLimb &Tl = A.T[l];
     const uint64_t q = Tl.q, mu = Tl.mu64;
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads)
-        s[e] = reduce_any(g[col_index(e, G, col0)], q, mu);
-    high_stages(s, G, Tl, false);
-    uint64_t *o = out + t * G.N;
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads) o[col_index(e, G, col0)] = s[e];
+    stage_twiddles<LOGN, PS>(stw, Tl.fwd, first);
+    auto gload = [&](uint32_t sub, uint32_t pos) {
+        const uint64_t v = g[(size_t)pos * R2 + sub];
+        return FAST ? v : reduce_any(v, q, mu);
+    };
+    auto sload = [&](uint32_t sub, uint32_t pos) { return sm[sub * PS::pitch + pos]; };
+    auto sstore = [&](uint32_t sub, uint32_t pos, uint64_t v) { sm[sub * PS::pitch + pos] = v; };
+    auto gstore = [&](uint32_t sub, uint32_t pos, uint64_t v) { o[(size_t)pos * R2 + sub] = v; };
+    if constexpr (PS::nr == 1) {
+        round<PS, 0, false, FAST>(stw, q, gload, wait_twiddles, gstore);
+    } else {
+        round<PS, 0, false, FAST>(stw, q, gload, wait_twiddles, sstore);
+        __syncthreads();
+        middle_rounds<PS, 1, PS::nr - 1, false, FAST>(sm, stw, q);
+        round<PS, PS::nr - 1, false, FAST>(stw, q, sload, [] {}, gstore);
+    }
 }
 
-// the low forward stages, then y' = (y_l - t) * q_{Lc-1}^-1
-__global__ void __launch_bounds__(kThreads) k_fwd_low(const uint64_t *polys, uint64_t *out, Geo G,
-                                                      const NttLimb *T)
+// forward, low stages: the first round (lo fastest) loads directly; the last
+// round goes through shared memory to a coalesced sweep that writes
+// y' = (y_l - t) * q_{Lc-1}^-1
+template <int LOGN, bool FAST>
+__global__ void __launch_bounds__(kThreads, 2) k_fwd_low(Args A)
 {
-    __shared__ uint64_t s[kTile];
-    const uint32_t tile = blockIdx.x & ((1u << G.ltiles) - 1);
-    const uint64_t t = blockIdx.x >> G.ltiles;
-    const uint64_t p = t / (G.Lc - 1);
-    const uint32_t l = (uint32_t)(t % (G.Lc - 1));
-    const uint32_t row0 = tile << (G.lt - (G.n - G.n1));
-    uint64_t *o = out + t * G.N + ((size_t)tile << G.lt);
-    const uint64_t *y = polys + (p * G.Lc + l) * G.N + ((size_t)tile << G.lt);
-    const NttLimb &Tl = T[l];
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads) s[e] = o[e];
-    low_stages(s, G, row0, Tl, false);
-    const ulonglong2 qi = Tl.qinv[G.Lc - 1];
-    for (uint32_t e = threadIdx.x; e < (1u << G.lt); e += kThreads)
-        o[e] = mul_shoup(subq(y[e], s[e], Tl.q), qi, Tl.q);
+    using SH = Shape<LOGN>;
+    using PS = LowPass<LOGN>;
+    FIONA_SMEM(PS);
+    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), tr = blockIdx.x >> SH::ltiles;
+    const uint32_t p = tr / (A.Lc - 1), l = tr % (A.Lc - 1);
+    const uint32_t first = tile << PS::lsubs;
+    uint64_t *o = A.out + (size_t)tr * (1u << LOGN) + ((size_t)first << PS::s);
+    const uint64_t *y = A.polys + ((size_t)p * A.Lc + l) * (1u << LOGN) + ((size_t)first << PS::s);
+    const NttLimb &Tl = A.T[l];
+    const uint64_t q = Tl.q;
+    const ulonglong2 qi = Tl.qinv[A.Lc - 1];
+    stage_twiddles<LOGN, PS>(stw, Tl.fwd, first);
+    // y is read only by the epilogue: start bringing it into L2 now
+    for (uint32_t e = threadIdx.x * 16; e < PS::tile; e += kThreads * 16)
+        asm volatile("prefetch.global.L2 [%0];\n" ::"l"(y + e));
+    auto sstore = [&](uint32_t sub, uint32_t pos, uint64_t v) { sm[sub * PS::pitch + pos] = v; };
+    round<PS, 0, false, FAST>(
+        stw, q, [&](uint32_t sub, uint32_t pos) { return o[(sub << PS::s) + pos]; }, wait_twiddles, sstore);
+    __syncthreads();
+    middle_rounds<PS, 1, PS::nr, false, FAST>(sm, stw, q);
+    // transform values: below 72q (FAST) or 8q; M = 128q or 8q bounds them
+    const uint64_t M = (FAST ? 128 : 8) * q;
+    sweep<PS>([&](uint32_t e) { return y[e]; },
+              [&](uint32_t e, uint64_t v) {
+                  const uint64_t t = sm[(e >> PS::s) * PS::pitch + (e & ((1u << PS::s) - 1))];
+                  o[e] = canon4(mul_shoup_lazy(v + M - t, qi, q), q);
+              });
 }
 
 // ---------------------------------------------------------------------------
@@ -341,29 +571,73 @@ int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t cou
     const int rc = ensure_tables(ctx);
     if (rc) return rc;
     if (count == 0) return FIONA_OK;
-    Geo G;
-    G.N = ctx->N;
-    G.n = 0;
-    while ((1u << G.n) < G.N) ++G.n;
-    G.n1 = G.n / 2;
-    G.lt = std::min<uint32_t>(G.n, 12);
-    G.ltiles = G.n - G.lt;
-    G.Lc = Lc;
+    uint32_t n = 0;
+    while ((1u << n) < ctx->N) ++n;
+    if (n < (uint32_t)kLogNMin || n > (uint32_t)kLogNMax)
+        return set_error(FIONA_ERR_ARG, "rescale: N = %u outside [2^%d, 2^%d]", ctx->N, kLogNMin, kLogNMax);
+    // the reduction-free forward butterflies need q < 2^56 and r < 4 q_l
+    bool fast = true;
+    const uint64_t qlast = ctx->moduli[Lc - 1];
+    for (uint32_t l = 0; l + 1 < Lc; ++l)
+        if (ctx->moduli[l] >= (1ull << 56) || qlast >= 4 * ctx->moduli[l]) fast = false;
+    const uint32_t lt = std::min<uint32_t>(n, kLogTileMax), ltiles = n - lt;
+    const int ix = (int)n - kLogNMin;
+    typedef void (*Kern)(Args);
+    static const Kern inv_low[] = {k_inv_low<10>, k_inv_low<11>, k_inv_low<12>, k_inv_low<13>,
+                                   k_inv_low<14>, k_inv_low<15>, k_inv_low<16>, k_inv_low<17>};
+    static const Kern inv_high[] = {k_inv_high<10>, k_inv_high<11>, k_inv_high<12>, k_inv_high<13>,
+                                    k_inv_high<14>, k_inv_high<15>, k_inv_high<16>, k_inv_high<17>};
+    static const Kern fwd_high[2][8] = {
+        {k_fwd_high<10, false>, k_fwd_high<11, false>, k_fwd_high<12, false>, k_fwd_high<13, false>,
+         k_fwd_high<14, false>, k_fwd_high<15, false>, k_fwd_high<16, false>, k_fwd_high<17, false>},
+        {k_fwd_high<10, true>, k_fwd_high<11, true>, k_fwd_high<12, true>, k_fwd_high<13, true>,
+         k_fwd_high<14, true>, k_fwd_high<15, true>, k_fwd_high<16, true>, k_fwd_high<17, true>}};
+    static const Kern fwd_low[2][8] = {
+        {k_fwd_low<10, false>, k_fwd_low<11, false>, k_fwd_low<12, false>, k_fwd_low<13, false>,
+         k_fwd_low<14, false>, k_fwd_low<15, false>, k_fwd_low<16, false>, k_fwd_low<17, false>},
+        {k_fwd_low<10, true>, k_fwd_low<11, true>, k_fwd_low<12, true>, k_fwd_low<13, true>,
+         k_fwd_low<14, true>, k_fwd_low<15, true>, k_fwd_low<16, true>, k_fwd_low<17, true>}};
+    const Kern ks[4] = {inv_low[ix], inv_high[ix], fwd_high[fast][ix], fwd_low[fast][ix]};
+    static const size_t low_smem[] = {LowPass<10>::smem_bytes, LowPass<11>::smem_bytes, LowPass<12>::smem_bytes,
+                                      LowPass<13>::smem_bytes, LowPass<14>::smem_bytes, LowPass<15>::smem_bytes,
+                                      LowPass<16>::smem_bytes, LowPass<17>::smem_bytes};
+    static const size_t high_smem[] = {HighPass<10>::smem_bytes, HighPass<11>::smem_bytes, HighPass<12>::smem_bytes,
+                                       HighPass<13>::smem_bytes, HighPass<14>::smem_bytes, HighPass<15>::smem_bytes,
+                                       HighPass<16>::smem_bytes, HighPass<17>::smem_bytes};
+    const size_t smem[4] = {low_smem[ix], high_smem[ix], high_smem[ix], low_smem[ix]};
+    cudaError_t e = cudaSuccess;
+    {
+        // the dynamic shared memory limit, once per device and kernel
+        static bool configured[FIONA_MAX_DEVICES][kLogNMax - kLogNMin + 1][2] = {};
+        std::lock_guard<std::mutex> lock(g_ntt_mu);
+        if (ctx->device < 0 || ctx->device >= FIONA_MAX_DEVICES)
+            return set_error(FIONA_ERR_ARG, "rescale: device %d", ctx->device);
+        if (!configured[ctx->device][ix][fast]) {
+            for (int i = 0; i < 4 && e == cudaSuccess; ++i)
+                e = cudaFuncSetAttribute((const void *)ks[i], cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem[i]);
+            if (e != cudaSuccess)
+                return set_error(FIONA_ERR_CUDA, "rescale: kernel attributes: %s", cudaGetErrorString(e));
+            configured[ctx->device][ix][fast] = true;
+        }
+    }
     // grid.x < 2^31: transforms * tiles, in chunks of whole polys
-    const uint64_t max_polys = ((1ull << 31) - 1) / ((uint64_t)(Lc - 1) << G.ltiles);
+    const uint64_t max_polys = ((1ull << 31) - 1) / ((uint64_t)(Lc - 1) << ltiles);
     const NttLimb *T = reinterpret_cast<const NttLimb *>(ctx->d_ntt);
     cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e = cudaSuccess;
     for (uint64_t p0 = 0; p0 < count && e == cudaSuccess; p0 += max_polys) {
         const uint64_t np = std::min<uint64_t>(count - p0, max_polys);
-        uint64_t *pp = polys + p0 * Lc * (uint64_t)G.N;
-        uint64_t *op = out + p0 * (Lc - 1) * (uint64_t)G.N;
-        const uint32_t inv_blocks = (uint32_t)(np << G.ltiles);
-        const uint32_t fwd_blocks = (uint32_t)((np * (Lc - 1)) << G.ltiles);
-        k_inv_low<<<inv_blocks, kThreads, 0, s>>>(pp, G, T);
-        k_inv_high<<<inv_blocks, kThreads, 0, s>>>(pp, G, T);
-        k_fwd_high<<<fwd_blocks, kThreads, 0, s>>>(pp, op, G, T);
-        k_fwd_low<<<fwd_blocks, kThreads, 0, s>>>(pp, op, G, T);
+        Args a;
+        a.polys = polys + p0 * Lc * (uint64_t)ctx->N;
+        a.out = out + p0 * (Lc - 1) * (uint64_t)ctx->N;
+        a.T = T;
+        a.Lc = Lc;
+        const uint32_t inv_blocks = (uint32_t)(np << ltiles);
+        const uint32_t fwd_blocks = (uint32_t)((np * (Lc - 1)) << ltiles);
+        ks[0]<<<inv_blocks, kThreads, smem[0], s>>>(a);
+        ks[1]<<<inv_blocks, kThreads, smem[1], s>>>(a);
+        ks[2]<<<fwd_blocks, kThreads, smem[2], s>>>(a);
+        ks[3]<<<fwd_blocks, kThreads, smem[3], s>>>(a);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "rescale launch: %s", cudaGetErrorString(e));
