@@ -15,6 +15,11 @@ sum, scale PMult, raw PMult-MAC and the final reduction) through the C ABI
   cpu_baseline the CPU oracle on a bounded sample of the same layer, on every
                host core (one spawn process per core)
 
+--op rescale times the rescale that follows the layer instead (fiona_rescale
+on the layer's 2 n_out output polys, N and L of the workload): value is
+polys rescaled per second and the roofline is the integer-multiply pipe
+(the NTT butterflies), not HBM.
+
 --impl reference times the CPU oracle as the reference arm.
 Multi-GPU (torchrun): every rank evaluates its own replica of the layer
 (independent queries, weak scaling, no data-path collective).
@@ -412,6 +417,150 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     ctx.close()
 
 
+# ----------------------------------------------------------------------------
+# --op rescale
+# ----------------------------------------------------------------------------
+# Integer multiplies (IMAD on the FMA-heavy pipe, 64 per clock per SM) that
+# one forward butterfly needs at least: the quotient estimate (a wide
+# product and two high halves) and the two 64-bit low products (a wide
+# product and two plain multiplies each); a wide product takes two issue
+# slots.  See the design doc for the derivation of the peak.
+IMAD_SLOTS_PER_BUTTERFLY = 12
+IMAD_PER_CLK_PER_SM = 64
+SM_COUNT = 152
+SM_MAX_MHZ = 2070.0
+
+
+def rescale_butterflies(N: int, L: int) -> int:
+    """Radix-2 butterflies of one poly's rescale: one inverse transform of
+    the last limb and L - 1 forward transforms."""
+    return L * (N // 2) * (N.bit_length() - 1)
+
+
+def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
+    import torch
+
+    from paper_2609_35352_gb300 import build as B
+    from paper_2609_35352_gb300 import fiona as F
+
+    if rank == 0:
+        B.build()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.set_device(local_rank)
+    dev = local_rank
+    name = args.workload
+    wl = W.make_workload(name, L=args.limbs)
+    N, L = wl.N, wl.L
+    count = 2 * wl.plan.n_out
+    unit = "polys/s"
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        import oracle
+        oracle.build()
+        flat = np.arange(L * N, dtype=np.uint64).reshape(1, L, N)
+        y0 = W.residues_np(wl.key(W.STREAM_INPUTS), flat, wl.moduli_np.reshape(1, L, 1))
+        dt, done = 0.0, 0
+        while done < count and (done == 0 or dt < args.cpu_budget):
+            t0 = time.perf_counter()
+            oracle.rescale(wl.moduli, y0)
+            dt += time.perf_counter() - t0
+            done += 1
+        cpu = {"value": done / dt, "unit": unit, "cores": 1, "kind": "oracle",
+               "sample": "%d rescales of the first of the %d polys (radix-2 NTT oracle, one thread)"
+                         % (done, count)}
+
+    ctx = F.Context(N, wl.moduli, device=dev)
+    n_y, n_o = count * L * N, count * (L - 1) * N
+    d_y = torch.empty(n_y, dtype=torch.int64, device="cuda")
+    d_o = torch.empty(n_o, dtype=torch.int64, device="cuda")
+    stream = torch.cuda.Stream()
+    F.device_fill(d_y, count, L, N, wl.moduli, wl.key(W.STREAM_INPUTS), 0, stream)
+    stream.synchronize()
+    for _ in range(args.warmup):
+        ctx.rescale(L, count, d_y, d_o, stream=stream)
+    stream.synchronize()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = ClockSampler(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    for s in range(args.steps):
+        starts[s].record(stream)
+        ctx.rescale(L, count, d_y, d_o, stream=stream)
+        stops[s].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    step_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
+    elapsed_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    value = world * count * args.steps / (elapsed_ms / 1e3)
+    avg_s = statistics.mean(step_ms) / 1e3
+    bfly = count * rescale_butterflies(N, L)
+    peak_bfly = SM_COUNT * IMAD_PER_CLK_PER_SM * SM_MAX_MHZ * 1e6 / IMAD_SLOTS_PER_BUTTERFLY
+    achieved = bfly / avg_s
+    hbm_bytes = count * (2 * L - 1) * N * 8
+    hbm_peak, hbm_kind = measured_peak()
+    roofline = {"bound": "alu", "achieved": achieved / 1e9, "peak": peak_bfly / 1e9, "unit": "Gbutterfly/s",
+                "frac": achieved / peak_bfly, "traffic": None,
+                "kernel": "rescale (k_inv_low, k_inv_high, k_fwd_high, k_fwd_low)",
+                "peak_kind": "derived: %d SMs x %d IMAD/clk x %.0f MHz / %d IMAD slots per butterfly"
+                             % (SM_COUNT, IMAD_PER_CLK_PER_SM, SM_MAX_MHZ, IMAD_SLOTS_PER_BUTTERFLY),
+                "butterflies_per_launch": bfly,
+                "hbm_gbs_algorithmic": hbm_bytes / avg_s / 1e9,
+                "hbm_frac": hbm_bytes / avg_s / 1e9 / hbm_peak, "hbm_peak_kind": hbm_kind,
+                "step_ms_median": statistics.median(step_ms)}
+
+    e2e = None
+    if not args.no_e2e:
+        h_y = torch.empty(n_y, dtype=torch.int64, pin_memory=True)
+        h_o = torch.empty(n_o, dtype=torch.int64, pin_memory=True)
+        h_y.copy_(d_y.cpu())
+        e2e_steps = max(3, min(args.steps, args.e2e_steps))
+
+        def one():
+            with torch.cuda.stream(stream):
+                d_y.copy_(h_y, non_blocking=True)
+                ctx.rescale(L, count, d_y, d_o, stream=stream)
+                h_o.copy_(d_o, non_blocking=True)
+            stream.synchronize()
+
+        one()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            one()
+        dt = time.perf_counter() - t0
+        e2e = {"value": world * count * e2e_steps / dt, "unit": unit, "h2d_bytes_per_step": n_y * 8,
+               "d2h_bytes_per_step": n_o * 8, "ms_per_step": 1e3 * dt / e2e_steps, "steps": e2e_steps}
+
+    if rank == 0:
+        line = {
+            "metric": "rescale of the layer's outputs: polys/s, NTT butterflies/s (%% of the integer-multiply "
+                      "pipe), N=2^%d" % (N.bit_length() - 1),
+            "value": value, "unit": unit, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u64",
+            "data": "synthetic (seeded SplitMix64 residues, filled on the device)",
+            "config": {"workload": "rescale of the %s layer's outputs: %d polys, N=2^%d, L=%d -> %d limbs of "
+                                   "%d-bit primes" % (name, count, N.bit_length() - 1, L, L - 1,
+                                                      max(wl.moduli).bit_length()),
+                       "polys": count, "N": N, "L": L,
+                       "l2": "inputs larger than L2 (%.2f GB per step, L2 129 MB)" % (hbm_bytes / 1e9)},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": 4 * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    ctx.close()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -424,6 +573,7 @@ def main():
                     help="seconds of oracle work per host core for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--op", choices=["layer", "rescale"], default="layer")
     ap.add_argument("--limbs", type=int, default=None,
                     help="profiling aid: the same layer with this many RNS limbs (no cpu_baseline)")
     args = ap.parse_args()
@@ -441,7 +591,7 @@ def main():
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
     try:
-        run_ours(args, rank, world, local_rank)
+        (run_rescale if args.op == "rescale" else run_ours)(args, rank, world, local_rank)
     finally:
         if world > 1:
             import torch
