@@ -300,6 +300,42 @@ int fiona_linear_eval_rescale(const fiona_plan *plan, void *cuda_stream, uint32_
                               const uint64_t *inputs, const uint64_t *plaintexts, uint64_t *work,
                               uint64_t *outputs);
 
+/* Plaintext encoding on the GPU (Sec. 2.2 "Ciphertexts and Slots": CKKS
+ * packs a vector of numbers into the slots of a plaintext; the layer's gamma
+ * and raw plaintexts are encodings of the model's weights).
+ *
+ * fiona_ckks_embed: `slots` holds `count` vectors of N/2 complex numbers
+ * ([count][N/2][2] doubles: re, im; real weights have im = 0).  For each,
+ * the real poly m of degree < N with m(zeta^(5^j)) = z_j and
+ * m(zeta^(-5^j)) = conj(z_j), zeta = exp(i pi / N) (slot j at the odd
+ * power 5^j mod 2N), is computed in fp64 and its coefficients
+ * round(scale * m_i) (ties away from zero) are written to `coeffs`
+ * ([count][N] int64).  `work` is scratch of count * N * 16 bytes.  The
+ * rounding is floating point: a coefficient whose exact value lies within
+ * the transform's fp64 error of a half-integer may round either way.  A
+ * coefficient that is not finite or reaches 2^62 in magnitude is written as
+ * 0 and reported by the next fiona_device_check (FIONA_ERR_RANGE).
+ *
+ * fiona_encode_coeffs: integer polys `coeffs` ([count][N] int64, any value)
+ * to RNS NTT form at level L_cur: out[p][l] = NTT_l(coeffs[p] mod q_l)
+ * ([count][L_cur][N], canonical; NTT form as for fiona_rescale).  Exact.
+ *
+ * fiona_encode: fiona_ckks_embed then fiona_encode_coeffs (`coeffs` and
+ * `work` as above).
+ *
+ * Device pointers of the ctx's device, 16-byte aligned, pairwise
+ * non-overlapping; asynchronous on `cuda_stream`, except that the first call
+ * on a ctx builds its tables (twiddles, slot order; synchronous, before any
+ * stream capture).  Errors: FIONA_ERR_ARG (scale not positive, L_cur outside
+ * [1, L], null, misaligned or overlapping buffers), FIONA_ERR_NODEVICE,
+ * FIONA_ERR_NOMEM, FIONA_ERR_CUDA. */
+int fiona_ckks_embed(const fiona_ctx *ctx, void *cuda_stream, uint64_t count, const double *slots,
+                     double scale, int64_t *coeffs, double *work);
+int fiona_encode_coeffs(const fiona_ctx *ctx, void *cuda_stream, uint32_t L_cur, uint64_t count,
+                        const int64_t *coeffs, uint64_t *out);
+int fiona_encode(const fiona_ctx *ctx, void *cuda_stream, uint32_t L_cur, uint64_t count,
+                 const double *slots, double scale, int64_t *coeffs, double *work, uint64_t *out);
+
 /* End-to-end evaluation from host memory: copies `h_inputs` (host, layout
  * [n_in][2][L][N], pinned for overlap) to the caller's device buffer
  * `d_inputs`, evaluates with the device-resident `d_plaintexts` (the model's
@@ -346,11 +382,12 @@ int fiona_linear_eval_static(const fiona_plan *plan, void *cuda_stream, const ui
 int fiona_check_residues(const fiona_ctx *ctx, void *cuda_stream, const uint64_t *data,
                          uint64_t count);
 
-/* Report kernel-side failures of earlier evaluations on this context:
- * synchronises `cuda_stream`, then returns FIONA_ERR_TIMEOUT (and clears the
- * flag) if a tiled kernel gave up waiting for its bulk copies (every such
- * wait is bounded; the CTA then leaves its tile unwritten), FIONA_ERR_CUDA on
- * a CUDA error, FIONA_OK otherwise. */
+/* Report kernel-side failures of earlier calls on this context:
+ * synchronises `cuda_stream`, then returns FIONA_ERR_TIMEOUT if a tiled
+ * kernel gave up waiting for its bulk copies (every such wait is bounded; the
+ * CTA then leaves its tile unwritten), FIONA_ERR_RANGE if an encoding met a
+ * coefficient out of range (fiona_ckks_embed), FIONA_ERR_CUDA on a CUDA
+ * error, FIONA_OK otherwise; the flags are cleared. */
 int fiona_device_check(const fiona_ctx *ctx, void *cuda_stream);
 
 const char *fiona_status_str(int status);

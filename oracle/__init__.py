@@ -8,6 +8,9 @@ Contents
   oracle.c       schoolbook modular evaluation of the layer (flat and DAG form)
   rescale.c      negacyclic NTT (by definition and radix-2) and the rescale by
                  the last prime that follows the layer
+  encode.c       plaintext encoding: slots -> integer coefficients by the
+                 inversion formula of the canonical embedding, and integer
+                 coefficients -> RNS NTT form
   crt.py         brute-force evaluation over Z_Q with Python integers (pin P2)
   ckks_tiny.py   tiny-N CKKS encode/encrypt/decrypt round trip (pin P3)
 
@@ -19,3 +22,4 @@ special cases with closed forms, and a planted-mistake check.
 """
 from .liboracle import build, linear_eval, linear_eval_dag, load, load_variant  # noqa: F401
 from .liboracle import intt, min_root, ntt, rescale  # noqa: F401
+from .liboracle import ckks_embed, encode_coeffs  # noqa: F401

@@ -10,7 +10,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
-_SRCS = [_SRC, os.path.join(_HERE, "rescale.c")]
+_SRCS = [_SRC, os.path.join(_HERE, "rescale.c"), os.path.join(_HERE, "encode.c")]
 _OUT_DIR = os.path.join(_HERE, "_build")
 _LIB = os.path.join(_OUT_DIR, "liboracle.so")
 _handle: Optional[ctypes.CDLL] = None
@@ -21,7 +21,7 @@ def build(force: bool = False) -> str:
     os.makedirs(_OUT_DIR, exist_ok=True)
     if force or not os.path.exists(_LIB) or any(os.path.getmtime(_LIB) < os.path.getmtime(f) for f in _SRCS):
         tmp = _LIB + ".tmp%d" % os.getpid()
-        subprocess.run(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-o", tmp] + _SRCS, check=True)
+        subprocess.run(["gcc", "-O2", "-std=c11", "-shared", "-fPIC", "-o", tmp] + _SRCS + ["-lm"], check=True)
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -47,6 +47,11 @@ def _setup(lib: ctypes.CDLL) -> ctypes.CDLL:
             getattr(lib, f).restype = None
         lib.oracle_rescale.argtypes = [u64, u32, u32, p, p, p, ctypes.c_int]
         lib.oracle_rescale.restype = ctypes.c_int
+    if hasattr(lib, "oracle_ckks_embed"):
+        lib.oracle_ckks_embed.argtypes = [u32, p, ctypes.c_double, p, u32, p]
+        lib.oracle_ckks_embed.restype = ctypes.c_int
+        lib.oracle_encode_coeffs.argtypes = [u32, u32, p, u64, p, p, ctypes.c_int]
+        lib.oracle_encode_coeffs.restype = ctypes.c_int
     return lib
 
 
@@ -173,4 +178,35 @@ def rescale(moduli, polys: np.ndarray, fast: bool = True) -> np.ndarray:
     rc = load().oracle_rescale(count, N, L, _ptr(qs), _ptr(y), _ptr(out), 1 if fast else 0)
     if rc != 0:
         raise ValueError("oracle_rescale: arguments it cannot evaluate")
+    return out
+
+
+# -- plaintext encoding (encode.c) ------------------------------------------------
+def ckks_embed(slots: np.ndarray, scale: float, idx=None) -> np.ndarray:
+    """Integer coefficients round(scale * m_i) of the encoding of one slot
+    vector (complex, length N/2), at the coefficient indices idx (all if
+    None)."""
+    z = np.ascontiguousarray(np.asarray(slots, dtype=np.complex128))
+    n = z.shape[0]
+    N = 2 * n
+    zz = np.ascontiguousarray(np.stack([z.real, z.imag], axis=-1), dtype=np.float64)
+    ix = _c(np.arange(N) if idx is None else idx, np.uint32)
+    out = np.zeros(ix.shape[0], dtype=np.int64)
+    rc = load().oracle_ckks_embed(N, _ptr(zz), float(scale), _ptr(ix), ix.shape[0], _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle_ckks_embed: coefficient out of range or bad argument")
+    return out
+
+
+def encode_coeffs(moduli, coeffs: np.ndarray, fast: bool = True) -> np.ndarray:
+    """Integer polys [count][N] (int64) -> NTT form [count][L][N] (uint64)."""
+    c = _c(coeffs, np.int64)
+    if c.ndim == 1:
+        c = c.reshape(1, -1)
+    count, N = c.shape
+    q = _c(list(moduli), np.uint64)
+    out = np.zeros((count, q.shape[0], N), np.uint64)
+    rc = load().oracle_encode_coeffs(N, q.shape[0], _ptr(q), count, _ptr(c), _ptr(out), 1 if fast else 0)
+    if rc != 0:
+        raise ValueError("oracle_encode_coeffs: a modulus has no primitive 2N-th root")
     return out

@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -205,6 +206,7 @@ extern "C" void fiona_ctx_destroy(fiona_ctx *ctx)
         cudaFree(ctx->d_flag);
         cudaFree(ctx->d_kerr);
         free_rescale_tables(ctx);
+        free_encode_tables(ctx);
     }
     delete ctx;
 }
@@ -610,8 +612,9 @@ extern "C" int fiona_device_check(const fiona_ctx *ctx, void *stream)
     if (e == cudaSuccess) e = cudaMemcpy(&flag, ctx->d_kerr, sizeof(int), cudaMemcpyDeviceToHost);
     if (e == cudaSuccess && flag) e = cudaMemset(ctx->d_kerr, 0, sizeof(int));
     if (e != cudaSuccess) return cuda_fail(e, "device_check");
-    return flag ? set_error(FIONA_ERR_TIMEOUT, "a kernel gave up waiting for its bulk copies")
-                : FIONA_OK;
+    if (flag & 1) return set_error(FIONA_ERR_TIMEOUT, "a kernel gave up waiting for its bulk copies");
+    if (flag & 2) return set_error(FIONA_ERR_RANGE, "an encoded coefficient was not finite or reached 2^62");
+    return FIONA_OK;
 }
 
 extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out,
@@ -897,6 +900,84 @@ extern "C" int fiona_linear_eval_rescale(const fiona_plan *p, void *stream, uint
     rc = launch_range(p, stream, in, pt, work, 0, L_eval, L_eval);
     if (rc) return rc;
     return launch_rescale(p->ctx, stream, L_eval, count, work, out);
+}
+
+static int check_encode_ctx(const fiona_ctx *ctx, const char *who)
+{
+    if (!ctx) return set_error(FIONA_ERR_ARG, "%s: null ctx", who);
+    if (ctx->device == FIONA_DEVICE_NONE) return set_error(FIONA_ERR_NODEVICE, "%s: validation-only context", who);
+    return FIONA_OK;
+}
+
+static int check_embed_args(const fiona_ctx *ctx, uint64_t count, const double *slots, double scale,
+                            const int64_t *coeffs, const double *work, const char *who)
+{
+    int rc = check_encode_ctx(ctx, who);
+    if (rc) return rc;
+    if (!(scale > 0.0) || !std::isfinite(scale)) return set_error(FIONA_ERR_ARG, "%s: scale must be positive", who);
+    if (count > (1ull << 40) / ctx->N) return set_error(FIONA_ERR_ARG, "%s: %llu polys", who, (unsigned long long)count);
+    if (count == 0) return FIONA_OK;
+    if (!slots || !coeffs || !work) return set_error(FIONA_ERR_ARG, "%s: null buffer", who);
+    if (((uintptr_t)slots | (uintptr_t)coeffs | (uintptr_t)work) & 15)
+        return set_error(FIONA_ERR_ARG, "%s: buffers must be 16-byte aligned", who);
+    const uint64_t N = ctx->N;
+    if (overlaps(work, count * N * 16, slots, count * N * 8) || overlaps(work, count * N * 16, coeffs, count * N * 8) ||
+        overlaps(coeffs, count * N * 8, slots, count * N * 8))
+        return set_error(FIONA_ERR_ARG, "%s: overlapping buffers", who);
+    return FIONA_OK;
+}
+
+static int check_encode_coeff_args(const fiona_ctx *ctx, uint32_t L_cur, uint64_t count, const int64_t *coeffs,
+                                   const uint64_t *out, const char *who)
+{
+    int rc = check_encode_ctx(ctx, who);
+    if (rc) return rc;
+    if (L_cur < 1 || L_cur > ctx->L) return set_error(FIONA_ERR_ARG, "%s: level %u outside [1, %u]", who, L_cur, ctx->L);
+    if (count > (1ull << 40) / ((uint64_t)L_cur * ctx->N))
+        return set_error(FIONA_ERR_ARG, "%s: %llu polys", who, (unsigned long long)count);
+    if (count == 0) return FIONA_OK;
+    if (!coeffs || !out) return set_error(FIONA_ERR_ARG, "%s: null buffer", who);
+    if (((uintptr_t)coeffs | (uintptr_t)out) & 15) return set_error(FIONA_ERR_ARG, "%s: buffers must be 16-byte aligned", who);
+    const uint64_t N = ctx->N;
+    if (overlaps(coeffs, count * N * 8, out, count * L_cur * N * 8))
+        return set_error(FIONA_ERR_ARG, "%s: output overlaps the coefficients", who);
+    return FIONA_OK;
+}
+
+extern "C" int fiona_ckks_embed(const fiona_ctx *ctx, void *stream, uint64_t count, const double *slots,
+                                double scale, int64_t *coeffs, double *work)
+{
+    int rc = check_embed_args(ctx, count, slots, scale, coeffs, work, "ckks_embed");
+    if (rc || count == 0) return rc;
+    DeviceGuard g(ctx->device);
+    return launch_embed(ctx, stream, count, slots, scale, coeffs, work);
+}
+
+extern "C" int fiona_encode_coeffs(const fiona_ctx *ctx, void *stream, uint32_t L_cur, uint64_t count,
+                                   const int64_t *coeffs, uint64_t *out)
+{
+    int rc = check_encode_coeff_args(ctx, L_cur, count, coeffs, out, "encode_coeffs");
+    if (rc || count == 0) return rc;
+    DeviceGuard g(ctx->device);
+    return launch_encode_coeffs(ctx, stream, L_cur, count, coeffs, out);
+}
+
+extern "C" int fiona_encode(const fiona_ctx *ctx, void *stream, uint32_t L_cur, uint64_t count, const double *slots,
+                            double scale, int64_t *coeffs, double *work, uint64_t *out)
+{
+    int rc = check_embed_args(ctx, count, slots, scale, coeffs, work, "encode");
+    if (rc == FIONA_OK) rc = check_encode_coeff_args(ctx, L_cur, count, coeffs, out, "encode");
+    if (rc == FIONA_OK && count) {
+        const uint64_t N = ctx->N;
+        if (overlaps(out, count * L_cur * N * 8, slots, count * N * 8) ||
+            overlaps(out, count * L_cur * N * 8, work, count * N * 16))
+            rc = set_error(FIONA_ERR_ARG, "encode: output overlaps the slots or the work area");
+    }
+    if (rc || count == 0) return rc;
+    DeviceGuard g(ctx->device);
+    rc = launch_embed(ctx, stream, count, slots, scale, coeffs, work);
+    if (rc) return rc;
+    return launch_encode_coeffs(ctx, stream, L_cur, count, coeffs, out);
 }
 
 extern "C" int fiona_check_residues(const fiona_ctx *ctx, void *stream, const uint64_t *data,

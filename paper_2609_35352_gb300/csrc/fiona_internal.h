@@ -50,7 +50,8 @@ struct fiona_ctx {
     int *d_kerr = nullptr;          // set by a kernel whose bounded wait gave up
     int sm_count = 0;
     size_t smem_optin = 0;
-    mutable void *d_ntt = nullptr;  // rescale tables, built on the first rescale (rescale.cu)
+    mutable void *d_ntt = nullptr;  // modular NTT tables, built on first use (rescale.cu)
+    mutable void *d_enc = nullptr;  // encoder tables, built on first use (encode.cu)
 };
 
 struct HostPlan {
@@ -113,6 +114,20 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
 int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t count, uint64_t *polys,
                    uint64_t *out);
 void free_rescale_tables(const fiona_ctx *ctx);
+namespace fiona_ntt {
+struct NttLimb;
+}
+// the modular NTT tables of every limb (built on the first call)
+int ntt_tables(const fiona_ctx *ctx, const fiona_ntt::NttLimb **limbs);
+
+// encode.cu.  Slots [count][N/2] (complex, fp64) -> integer coefficients
+// [count][N] (work: [count][N] complex); integer coefficients -> RNS NTT
+// form [count][Lc][N].
+int launch_embed(const fiona_ctx *ctx, void *stream, uint64_t count, const double *slots, double scale,
+                 int64_t *coeffs, double *work);
+int launch_encode_coeffs(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t count, const int64_t *coeffs,
+                         uint64_t *out);
+void free_encode_tables(const fiona_ctx *ctx);
 
 // fiona_host.cpp
 int set_error(int code, const char *fmt, ...);

@@ -350,7 +350,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
             bulk_g2s(smem_addr(sm) + o, reinterpret_cast<const char *>(a.sched) + o,
                      min(32768u, a.sched_bytes - o), bar0);
         s_abort = mbar_wait(bar0, 0) ? 0 : 1;
-        if (s_abort) atomicExch(a.err, 1);
+        if (s_abort) atomicOr(a.err, 1);
     }
     __syncthreads();
     if (s_abort) return;

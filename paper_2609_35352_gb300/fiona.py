@@ -39,7 +39,7 @@ EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona
             "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version",
             "fiona_plan_select_kernel", "fiona_device_check", "fiona_linear_eval_static",
             "fiona_linear_eval_level", "fiona_plan_compile", "fiona_rescale",
-            "fiona_linear_eval_rescale")
+            "fiona_linear_eval_rescale", "fiona_ckks_embed", "fiona_encode_coeffs", "fiona_encode")
 STATIC_AREA_BYTES = 1 << 20
 
 
@@ -114,6 +114,12 @@ def lib() -> ctypes.CDLL:
         L.fiona_rescale.restype = i32
         L.fiona_linear_eval_rescale.argtypes = [p, p, u32, p, p, p, p]
         L.fiona_linear_eval_rescale.restype = i32
+        L.fiona_ckks_embed.argtypes = [p, p, ctypes.c_uint64, p, ctypes.c_double, p, p]
+        L.fiona_ckks_embed.restype = i32
+        L.fiona_encode_coeffs.argtypes = [p, p, u32, ctypes.c_uint64, p, p]
+        L.fiona_encode_coeffs.restype = i32
+        L.fiona_encode.argtypes = [p, p, u32, ctypes.c_uint64, p, ctypes.c_double, p, p, p]
+        L.fiona_encode.restype = i32
         L.fiona_plan_compile.argtypes = [u32, u32, u32, p, u32, p, p, p, p, p, p, p, p, p, p]
         L.fiona_plan_compile.restype = i32
         L.fiona_linear_eval_static.restype = i32
@@ -175,10 +181,11 @@ class Context:
         return rc
 
     def device_check(self, stream=None) -> int:
-        """fiona_device_check: FIONA_OK, or FIONA_ERR_TIMEOUT if a kernel gave
-        up a bounded wait since the last check (raises on other errors)."""
+        """fiona_device_check: FIONA_OK, FIONA_ERR_TIMEOUT if a kernel gave up
+        a bounded wait, or FIONA_ERR_RANGE if an encoding met a coefficient out
+        of range, since the last check (raises on other errors)."""
         rc = lib().fiona_device_check(self.handle, stream_handle(stream))
-        if rc not in (FIONA_OK, FIONA_ERR_TIMEOUT):
+        if rc not in (FIONA_OK, FIONA_ERR_TIMEOUT, FIONA_ERR_RANGE):
             _check(rc, "fiona_device_check")
         return rc
 
@@ -191,6 +198,31 @@ class Context:
     def rescale_status(self, L_cur, count, polys, out, stream=None) -> int:
         return lib().fiona_rescale(self.handle, stream_handle(stream), int(L_cur), int(count), addr(polys),
                                    addr(out))
+
+    def ckks_embed_status(self, count, slots, scale, coeffs, work, stream=None) -> int:
+        """fiona_ckks_embed: slots [count][N/2][2] float64 -> coeffs [count][N]
+        int64 (work: count * N * 16 bytes)."""
+        return lib().fiona_ckks_embed(self.handle, stream_handle(stream), int(count), addr(slots), float(scale),
+                                      addr(coeffs), addr(work))
+
+    def ckks_embed(self, count, slots, scale, coeffs, work, stream=None) -> None:
+        _check(self.ckks_embed_status(count, slots, scale, coeffs, work, stream), "fiona_ckks_embed")
+
+    def encode_coeffs_status(self, L_cur, count, coeffs, out, stream=None) -> int:
+        """fiona_encode_coeffs: int64 coeffs [count][N] -> out [count][L_cur][N]."""
+        return lib().fiona_encode_coeffs(self.handle, stream_handle(stream), int(L_cur), int(count), addr(coeffs),
+                                         addr(out))
+
+    def encode_coeffs(self, L_cur, count, coeffs, out, stream=None) -> None:
+        _check(self.encode_coeffs_status(L_cur, count, coeffs, out, stream), "fiona_encode_coeffs")
+
+    def encode_status(self, L_cur, count, slots, scale, coeffs, work, out, stream=None) -> int:
+        return lib().fiona_encode(self.handle, stream_handle(stream), int(L_cur), int(count), addr(slots),
+                                  float(scale), addr(coeffs), addr(work), addr(out))
+
+    def encode(self, L_cur, count, slots, scale, coeffs, work, out, stream=None) -> None:
+        """fiona_encode: slots -> RNS NTT plaintexts [count][L_cur][N]."""
+        _check(self.encode_status(L_cur, count, slots, scale, coeffs, work, out, stream), "fiona_encode")
 
     def close(self) -> None:
         if getattr(self, "handle", None):
