@@ -20,6 +20,9 @@ on the layer's 2 n_out output polys, N and L of the workload): value is
 polys rescaled per second and the roofline is the integer-multiply pipe
 (the NTT butterflies), not HBM.
 
+--op encode times the plaintext encoding (fiona_encode: slot vectors ->
+integer coefficients -> RNS NTT form) of up to 256 of the layer's plaintexts.
+
 --impl reference times the CPU oracle as the reference arm.
 Multi-GPU (torchrun): every rank evaluates its own replica of the layer
 (independent queries, weak scaling, no data-path collective).
@@ -561,6 +564,138 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
     ctx.close()
 
 
+# ----------------------------------------------------------------------------
+# --op encode
+# ----------------------------------------------------------------------------
+FP64_NOMINAL_TFLOPS = 1.25   # GB300 dense fp64 (nominal)
+FLOPS_PER_COMPLEX_BUTTERFLY = 10  # one complex product (6) and a complex sum and difference (4)
+
+
+def run_encode(args, rank: int, world: int, local_rank: int) -> None:
+    import torch
+
+    from paper_2609_35352_gb300 import build as B
+    from paper_2609_35352_gb300 import fiona as F
+
+    if rank == 0:
+        B.build()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.set_device(local_rank)
+    dev = local_rank
+    name = args.workload
+    wl = W.make_workload(name, L=args.limbs)
+    N, L = wl.N, wl.L
+    count = min(wl.plan.n_pt, 256)
+    unit = "plaintexts/s"
+    scale = 2.0 ** 40
+    rng = np.random.default_rng(wl.seed)
+    h_slots = rng.uniform(-1.0, 1.0, size=(count, N // 2, 2))
+    h_slots[:, :, 1] = 0.0  # weights are real
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        import oracle
+        oracle.build()
+        # the definition sum costs N/2 terms per coefficient: time it on a
+        # sample of coefficients and scale to N; the NTT form on a whole poly
+        z = h_slots[0, :, 0] + 0j
+        n_idx = 256
+        idx = np.arange(0, N, N // n_idx, dtype=np.uint32)
+        t0 = time.perf_counter()
+        oracle.ckks_embed(z, scale, idx)
+        t_emb = (time.perf_counter() - t0) * N / n_idx
+        c = np.zeros(N, np.int64)
+        t0 = time.perf_counter()
+        oracle.encode_coeffs(wl.moduli, c)
+        t_ntt = time.perf_counter() - t0
+        cpu = {"value": 1.0 / (t_emb + t_ntt), "unit": unit, "cores": 1, "kind": "oracle",
+               "sample": "one plaintext, one thread: the embedding sum timed on %d of its %d coefficients and "
+                         "scaled by %d (%.1f s), the RNS NTT form of %d limbs timed whole (%.2f s)"
+                         % (n_idx, N, N // n_idx, t_emb, L, t_ntt)}
+
+    ctx = F.Context(N, wl.moduli, device=dev)
+    d_slots = torch.from_numpy(h_slots).to("cuda")
+    d_c = torch.empty(count * N, dtype=torch.int64, device="cuda")
+    d_w = torch.empty(count * N, dtype=torch.float64, device="cuda")
+    d_o = torch.empty(count * L * N, dtype=torch.int64, device="cuda")
+    stream = torch.cuda.Stream()
+    for _ in range(args.warmup):
+        ctx.encode(L, count, d_slots, scale, d_c, d_w, d_o, stream=stream)
+    stream.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(dev)
+    torch.cuda.synchronize()
+    clocks.start()
+    for a, b, c in ev:
+        a.record(stream)
+        ctx.ckks_embed(count, d_slots, scale, d_c, d_w, stream=stream)
+        b.record(stream)
+        ctx.encode_coeffs(L, count, d_c, d_o, stream=stream)
+        c.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if ctx.device_check(stream) != F.FIONA_OK:
+        raise RuntimeError("encoding reported a coefficient out of range")
+    step_ms = [a.elapsed_time(c) for a, b, c in ev]
+    emb_ms = [a.elapsed_time(b) for a, b, c in ev]
+    ntt_ms = [b.elapsed_time(c) for a, b, c in ev]
+    elapsed_ms = sum(step_ms)
+    value = world * count * args.steps / (elapsed_ms / 1e3)
+    logn = N.bit_length() - 1
+    # the embedding is a complex transform of size N/2
+    emb_flops = count * (N // 4) * (logn - 1) * FLOPS_PER_COMPLEX_BUTTERFLY
+    achieved = emb_flops / (statistics.mean(emb_ms) / 1e3) / 1e12
+    ntt_bfly = count * L * (N // 2) * logn
+    peak_bfly = SM_COUNT * IMAD_PER_CLK_PER_SM * SM_MAX_MHZ * 1e6 / IMAD_SLOTS_PER_BUTTERFLY
+    roofline = {"bound": "fp64", "achieved": achieved, "peak": FP64_NOMINAL_TFLOPS, "unit": "TFLOP/s",
+                "frac": achieved / FP64_NOMINAL_TFLOPS, "traffic": None,
+                "kernel": "embedding (k_embed_low, k_embed_high): complex fp64 transform",
+                "peak_kind": "nominal GB300 dense fp64", "flops_per_launch": emb_flops,
+                "embed_ms_median": statistics.median(emb_ms),
+                "rns_ntt": {"bound": "alu", "ms_median": statistics.median(ntt_ms),
+                            "achieved_gbfly_s": ntt_bfly / (statistics.mean(ntt_ms) / 1e3) / 1e9,
+                            "peak_gbfly_s": peak_bfly / 1e9,
+                            "frac": ntt_bfly / (statistics.mean(ntt_ms) / 1e3) / peak_bfly}}
+
+    e2e = None
+    if not args.no_e2e:
+        h_in = torch.from_numpy(h_slots).pin_memory()
+        h_out = torch.empty(count * L * N, dtype=torch.int64, pin_memory=True)
+        e2e_steps = max(3, min(args.steps, args.e2e_steps))
+
+        def one():
+            with torch.cuda.stream(stream):
+                d_slots.copy_(h_in, non_blocking=True)
+                ctx.encode(L, count, d_slots, scale, d_c, d_w, d_o, stream=stream)
+                h_out.copy_(d_o, non_blocking=True)
+            stream.synchronize()
+
+        one()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            one()
+        dt = time.perf_counter() - t0
+        e2e = {"value": world * count * e2e_steps / dt, "unit": unit, "h2d_bytes_per_step": h_slots.nbytes,
+               "d2h_bytes_per_step": count * L * N * 8, "ms_per_step": 1e3 * dt / e2e_steps, "steps": e2e_steps}
+
+    if rank == 0:
+        line = {
+            "metric": "plaintext encoding: plaintexts/s (slots -> RNS NTT form), N=2^%d" % logn,
+            "value": value, "unit": unit, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64+u64", "data": "synthetic (seeded uniform real weights in [-1, 1])",
+            "config": {"workload": "encoding of %d of the %s layer's plaintexts: N=2^%d, %d limbs of %d-bit primes, "
+                                   "scale 2^40" % (count, name, logn, L, max(wl.moduli).bit_length()),
+                       "plaintexts": count, "N": N, "L": L},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": 4 * args.steps,
+        }
+        print(json.dumps(line), flush=True)
+    ctx.close()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -573,7 +708,7 @@ def main():
                     help="seconds of oracle work per host core for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--op", choices=["layer", "rescale"], default="layer")
+    ap.add_argument("--op", choices=["layer", "rescale", "encode"], default="layer")
     ap.add_argument("--limbs", type=int, default=None,
                     help="profiling aid: the same layer with this many RNS limbs (no cpu_baseline)")
     args = ap.parse_args()
@@ -591,7 +726,8 @@ def main():
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
     try:
-        (run_rescale if args.op == "rescale" else run_ours)(args, rank, world, local_rank)
+        run = {"layer": run_ours, "rescale": run_rescale, "encode": run_encode}[args.op]
+        run(args, rank, world, local_rank)
     finally:
         if world > 1:
             import torch

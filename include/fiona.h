@@ -310,7 +310,7 @@ int fiona_linear_eval_rescale(const fiona_plan *plan, void *cuda_stream, uint32_
  * m(zeta^(-5^j)) = conj(z_j), zeta = exp(i pi / N) (slot j at the odd
  * power 5^j mod 2N), is computed in fp64 and its coefficients
  * round(scale * m_i) (ties away from zero) are written to `coeffs`
- * ([count][N] int64).  `work` is scratch of count * N * 16 bytes.  The
+ * ([count][N] int64).  `work` is scratch of count * N * 8 bytes.  The
  * rounding is floating point: a coefficient whose exact value lies within
  * the transform's fp64 error of a half-integer may round either way.  A
  * coefficient that is not finite or reaches 2^62 in magnitude is written as

@@ -8,11 +8,17 @@
 //      and m(zeta^(-5^j)) = conj(z_j), zeta = exp(i pi / N) (slot j sits at
 //      the odd power 5^j mod 2N; the powers +-5^j are every odd residue);
 //      the integer coefficients are c_i = round(Delta * m_i), ties away from
-//      zero.  The values of m at all odd powers of zeta, in the order
-//      A[k] = m(zeta^(2 brv(k) + 1)), are the forward negacyclic transform
-//      of m over C, so m is its inverse transform (ntt.cuh, complex fp64):
-//      the inverse low pass gathers A[k] from z, the inverse high pass
-//      rounds Delta N^-1 Re(.) to 64-bit integers.
+//      zero.  By the inversion formula over the odd powers of zeta,
+//      m_i = (2/N) Re(u_i) and m_{i+n} = (2/N) Im(u_i), n = N/2, with
+//        u_i = sum_j z_j zeta^(-5^j i) = sum_r y_r zeta^(-(4r+1) i),
+//      y_r = z_j for 5^j = 4r + 1 mod 2N (the powers of 5 are the residues
+//      1 mod 4).  With A[k] = y_brv(k) (n-bit reversal) and psi = zeta^2,
+//        u_i = zeta^i sum_k A[k] psi^(-(2 brv(k) + 1) i),
+//      which is n times the inverse negacyclic transform of A of size n
+//      (ntt.cuh over complex fp64) twisted by zeta^i.  So the inverse low
+//      pass gathers A[k] from z, and the inverse high pass multiplies by
+//      zeta^i and rounds Delta (2/N) of the real and imaginary parts to the
+//      64-bit coefficients i and i + n.
 //   2. RNS/NTT form: c_i mod q_l for every limb, then the forward NTT mod
 //      q_l (ntt.cuh, the tables the rescale uses), canonical.
 // Step 1 is floating point: it reproduces round(Delta m_i) except where
@@ -32,21 +38,21 @@ using namespace fiona_ntt;
 
 namespace {
 
-// in device memory: N complex twiddles zeta^-brv(k) = (cos, sin), then N
-// gather words (slot index | conjugate << 31) for A[k]
+// in device memory, n = N/2 entries each: the twiddles psi^-brv(k) =
+// zeta^(-2 brv(k)) as (cos, sin), the slot index of A[k], and the twists
+// zeta^i
 struct EncTables {
     const double2 *cinv;
     const uint32_t *gather;
+    const double2 *twist;
 };
-
-constexpr uint32_t kConj = 1u << 31;
 
 struct EmbArgs {
     const double2 *slots;  // [count][N/2]
-    double2 *work;         // [count][N]
+    double2 *work;         // [count][N/2]
     int64_t *coeffs;       // [count][N]
     EncTables E;
-    double factor;         // Delta / N
+    double factor;         // Delta (2 / N)
     int *err;              // bit 1: a coefficient reached 2^62 (or was not finite)
 };
 
@@ -57,53 +63,56 @@ struct EncArgs {
     uint32_t Lc;
 };
 
-// embedding, inverse low stages: A[k] gathered from the slots
-template <int LOGN>
+// round(x) as a 64-bit integer; 0 and the range flag when |x| >= 2^62 or x
+// is not finite
+__device__ __forceinline__ int64_t round_coeff(double x, int *err)
+{
+    if (fabs(x) < 0x1p62) return llround(x);
+    atomicOr(err, 2);
+    return 0;
+}
+
+// embedding, inverse low stages of the size-n transform (LN = log2 n):
+// A[k] gathered from the slots
+template <int LN>
 __global__ void __launch_bounds__(kThreads, 1) k_embed_low(EmbArgs A)
 {
-    using SH = Shape<LOGN>;
-    using PS = LowPass<LOGN>;
+    using SH = Shape<LN>;
+    using PS = LowPass<LN>;
     extern __shared__ __align__(16) uint8_t smem_raw[];
     const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
     const uint32_t first = tile << PS::lsubs;
     const size_t base = (size_t)first << PS::s;
-    const double2 *z = A.slots + ((size_t)p << (LOGN - 1));
+    const double2 *z = A.slots + ((size_t)p << LN);
     const uint32_t *gat = A.E.gather + base;
-    double2 *w = A.work + ((size_t)p << LOGN) + base;
-    inv_low_pass<LOGN>(
-        smem_raw, A.E.cinv, first, CplxArith{},
-        [&](uint32_t e) {
-            const uint32_t sel = gat[e];
-            double2 v = z[sel & ~kConj];
-            if (sel & kConj) v.y = -v.y;
-            return v;
-        },
+    double2 *w = A.work + ((size_t)p << LN) + base;
+    inv_low_pass<LN>(
+        smem_raw, A.E.cinv, first, CplxArith{}, [&](uint32_t e) { return z[gat[e]]; },
         [&](uint32_t sub, uint32_t pos, double2 v) { w[(sub << PS::s) + pos] = v; });
 }
 
-// embedding, inverse high stages: c = round(Delta N^-1 Re(x))
-template <int LOGN>
+// embedding, inverse high stages: x zeta^i, rounded Delta (2/N) Re and Im to
+// coefficients i and i + n
+template <int LN>
 __global__ void __launch_bounds__(kThreads, 2) k_embed_high(EmbArgs A)
 {
-    using SH = Shape<LOGN>;
-    using PS = HighPass<LOGN>;
-    constexpr uint32_t R2 = 1u << (LOGN - SH::n1);
+    using SH = Shape<LN>;
+    using PS = HighPass<LN>;
+    constexpr uint32_t R2 = 1u << (LN - SH::n1);
     extern __shared__ __align__(16) uint8_t smem_raw[];
     const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
     const uint32_t first = tile << PS::lsubs;
-    const double2 *g = A.work + ((size_t)p << LOGN) + first;
-    int64_t *c = A.coeffs + ((size_t)p << LOGN) + first;
+    const double2 *g = A.work + ((size_t)p << LN) + first;
+    const double2 *tw = A.E.twist + first;
+    int64_t *c = A.coeffs + ((size_t)p << (LN + 1)) + first;
     const double f = A.factor;
-    inv_high_pass<LOGN>(
+    inv_high_pass<LN>(
         smem_raw, A.E.cinv, first, CplxArith{}, [&](uint32_t sub, uint32_t pos) { return g[(size_t)pos * R2 + sub]; },
         [&](uint32_t sub, uint32_t pos, double2 v) {
-            const double x = v.x * f;
-            int64_t r = 0;
-            if (fabs(x) < 0x1p62)
-                r = llround(x);
-            else
-                atomicOr(A.err, 2);
-            c[(size_t)pos * R2 + sub] = r;
+            const size_t i = (size_t)pos * R2 + sub;
+            const double2 u = CplxArith::mul(v, tw[i]);
+            c[i] = round_coeff(u.x * f, A.err);
+            c[i + (1u << LN)] = round_coeff(u.y * f, A.err);
         });
 }
 
@@ -166,32 +175,31 @@ int build_encode_tables(const fiona_ctx *ctx)
 {
     std::lock_guard<std::mutex> lock(g_enc_mu);
     if (ctx->d_enc) return FIONA_OK;
-    const uint32_t N = ctx->N, n = log2u(N), M = 2 * N;
-    const size_t tw_bytes = sizeof(double2) * N, bytes = tw_bytes + sizeof(uint32_t) * N;
+    const uint32_t N = ctx->N, n = N / 2, ln = log2u(n), M = 2 * N;
+    const size_t tw_bytes = sizeof(double2) * n, gat_bytes = sizeof(uint32_t) * n;
+    const size_t bytes = 2 * tw_bytes + gat_bytes;
     std::vector<uint8_t> host(bytes);
     double2 *tw = reinterpret_cast<double2 *>(host.data());
-    uint32_t *gat = reinterpret_cast<uint32_t *>(host.data() + tw_bytes);
+    double2 *twist = reinterpret_cast<double2 *>(host.data() + tw_bytes);
+    uint32_t *gat = reinterpret_cast<uint32_t *>(host.data() + 2 * tw_bytes);
     const long double pi = 3.141592653589793238462643383279502884L;
-    for (uint32_t k = 0; k < N; ++k) {
-        const long double a = -pi * (long double)bit_reverse(k, n) / (long double)N;
+    for (uint32_t k = 0; k < n; ++k) {
+        // psi^-brv(k) = zeta^(-2 brv(k)) and zeta^k, zeta = exp(i pi / N)
+        const long double a = -2 * pi * (long double)bit_reverse(k, ln) / (long double)N;
         tw[k] = make_double2((double)cosl(a), (double)sinl(a));
+        const long double b = pi * (long double)k / (long double)N;
+        twist[k] = make_double2((double)cosl(b), (double)sinl(b));
     }
-    // slot j sits at the odd exponent 5^j mod 2N, its conjugate at -5^j
-    std::vector<int64_t> slot_at(M, -1);
+    // slot j sits at the exponent 5^j mod 2N, which is 4r + 1 for one r < n
+    std::vector<int64_t> slot_of_r(n, -1);
     uint64_t e5 = 1;
-    for (uint32_t j = 0; j < N / 2; ++j) {
-        slot_at[e5] = j;
+    for (uint32_t j = 0; j < n; ++j) {
+        if (e5 % 4 != 1 || slot_of_r[(e5 - 1) / 4] >= 0)
+            return set_error(FIONA_ERR_INTERNAL, "encode tables: 5^%u mod 2N = %llu", j, (unsigned long long)e5);
+        slot_of_r[(e5 - 1) / 4] = j;
         e5 = e5 * 5 % M;
     }
-    for (uint32_t k = 0; k < N; ++k) {
-        const uint32_t e = 2 * bit_reverse(k, n) + 1;
-        if (slot_at[e] >= 0)
-            gat[k] = (uint32_t)slot_at[e];
-        else if (slot_at[M - e] >= 0)
-            gat[k] = (uint32_t)slot_at[M - e] | kConj;
-        else
-            return set_error(FIONA_ERR_INTERNAL, "encode tables: exponent %u is no power of 5 up to sign", e);
-    }
+    for (uint32_t k = 0; k < n; ++k) gat[k] = (uint32_t)slot_of_r[bit_reverse(k, ln)];
     void *dev = nullptr;
     cudaError_t err = cudaMalloc(&dev, bytes);
     if (err != cudaSuccess) return set_error(FIONA_ERR_NOMEM, "encode tables: %s", cudaGetErrorString(err));
@@ -209,8 +217,8 @@ typedef void (*EncKern)(EncArgs);
 
 template <int LOGN>
 struct Inst {
-    static constexpr size_t emb_low = LowPass<LOGN>::template smem_bytes<CplxArith>();
-    static constexpr size_t emb_high = HighPass<LOGN>::template smem_bytes<CplxArith>();
+    static constexpr size_t emb_low = LowPass<LOGN - 1>::template smem_bytes<CplxArith>();
+    static constexpr size_t emb_high = HighPass<LOGN - 1>::template smem_bytes<CplxArith>();
     static constexpr size_t enc_low = LowPass<LOGN>::template smem_bytes<ModArith<false>>();
     static constexpr size_t enc_high = HighPass<LOGN>::template smem_bytes<ModArith<false>>();
 };
@@ -224,8 +232,8 @@ struct Kernels {
 template <int LOGN>
 constexpr Kernels kernels_for()
 {
-    return Kernels{k_embed_low<LOGN>,
-                   k_embed_high<LOGN>,
+    return Kernels{k_embed_low<LOGN - 1>,
+                   k_embed_high<LOGN - 1>,
                    {k_enc_high<LOGN, false>, k_enc_high<LOGN, true>},
                    {k_enc_low<LOGN, false>, k_enc_low<LOGN, true>},
                    Inst<LOGN>::emb_low,
@@ -275,12 +283,13 @@ int launch_embed(const fiona_ctx *ctx, void *stream, uint64_t count, const doubl
     if (rc) return rc;
     if (count == 0) return FIONA_OK;
     const Kernels &K = kernels(n);
-    const uint32_t ltiles = n - std::min<uint32_t>(n, kLogTileMax);
+    const uint32_t ln = n - 1, ltiles = ln - std::min<uint32_t>(ln, kLogTileMax);
+    const uint8_t *tab = static_cast<const uint8_t *>(ctx->d_enc);
     EmbArgs a;
-    a.E.cinv = reinterpret_cast<const double2 *>(ctx->d_enc);
-    a.E.gather = reinterpret_cast<const uint32_t *>(static_cast<const uint8_t *>(ctx->d_enc) +
-                                                    sizeof(double2) * ctx->N);
-    a.factor = scale / (double)ctx->N;
+    a.E.cinv = reinterpret_cast<const double2 *>(tab);
+    a.E.twist = reinterpret_cast<const double2 *>(tab + sizeof(double2) * (ctx->N / 2));
+    a.E.gather = reinterpret_cast<const uint32_t *>(tab + 2 * sizeof(double2) * (ctx->N / 2));
+    a.factor = 2.0 * scale / (double)ctx->N;
     a.err = ctx->d_kerr;
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaSuccess;
@@ -288,7 +297,7 @@ int launch_embed(const fiona_ctx *ctx, void *stream, uint64_t count, const doubl
     for (uint64_t p0 = 0; p0 < count && e == cudaSuccess; p0 += max_polys) {
         const uint64_t np = std::min<uint64_t>(count - p0, max_polys);
         a.slots = reinterpret_cast<const double2 *>(slots) + p0 * (ctx->N / 2);
-        a.work = reinterpret_cast<double2 *>(work) + p0 * ctx->N;
+        a.work = reinterpret_cast<double2 *>(work) + p0 * (ctx->N / 2);
         a.coeffs = coeffs + p0 * ctx->N;
         const uint32_t blocks = (uint32_t)(np << ltiles);
         K.emb_low<<<blocks, kThreads, K.s_emb_low, s>>>(a);

@@ -921,7 +921,7 @@ static int check_embed_args(const fiona_ctx *ctx, uint64_t count, const double *
     if (((uintptr_t)slots | (uintptr_t)coeffs | (uintptr_t)work) & 15)
         return set_error(FIONA_ERR_ARG, "%s: buffers must be 16-byte aligned", who);
     const uint64_t N = ctx->N;
-    if (overlaps(work, count * N * 16, slots, count * N * 8) || overlaps(work, count * N * 16, coeffs, count * N * 8) ||
+    if (overlaps(work, count * N * 8, slots, count * N * 8) || overlaps(work, count * N * 8, coeffs, count * N * 8) ||
         overlaps(coeffs, count * N * 8, slots, count * N * 8))
         return set_error(FIONA_ERR_ARG, "%s: overlapping buffers", who);
     return FIONA_OK;
@@ -970,7 +970,7 @@ extern "C" int fiona_encode(const fiona_ctx *ctx, void *stream, uint32_t L_cur, 
     if (rc == FIONA_OK && count) {
         const uint64_t N = ctx->N;
         if (overlaps(out, count * L_cur * N * 8, slots, count * N * 8) ||
-            overlaps(out, count * L_cur * N * 8, work, count * N * 16))
+            overlaps(out, count * L_cur * N * 8, work, count * N * 8))
             rc = set_error(FIONA_ERR_ARG, "encode: output overlaps the slots or the work area");
     }
     if (rc || count == 0) return rc;

@@ -121,7 +121,7 @@ struct NttLimb;
 int ntt_tables(const fiona_ctx *ctx, const fiona_ntt::NttLimb **limbs);
 
 // encode.cu.  Slots [count][N/2] (complex, fp64) -> integer coefficients
-// [count][N] (work: [count][N] complex); integer coefficients -> RNS NTT
+// [count][N] (work: [count][N/2] complex); integer coefficients -> RNS NTT
 // form [count][Lc][N].
 int launch_embed(const fiona_ctx *ctx, void *stream, uint64_t count, const double *slots, double scale,
                  int64_t *coeffs, double *work);

@@ -201,7 +201,7 @@ class Context:
 
     def ckks_embed_status(self, count, slots, scale, coeffs, work, stream=None) -> int:
         """fiona_ckks_embed: slots [count][N/2][2] float64 -> coeffs [count][N]
-        int64 (work: count * N * 16 bytes)."""
+        int64 (work: count * N * 8 bytes)."""
         return lib().fiona_ckks_embed(self.handle, stream_handle(stream), int(count), addr(slots), float(scale),
                                       addr(coeffs), addr(work))
 
