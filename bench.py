@@ -58,6 +58,7 @@ WORKLOAD_TEXT = {
     "vgg": "VGG11-style conv layer, 144 rotated inputs -> 16 outputs, 79% ternary",
     "vit": "ViT-B-style BSGS projection, 32 -> 24, 65% ternary, 25% shared sums",
     "bert": "BERT-base-style FFN column packing, 96 -> 96, 53% ternary, 30% shared sums",
+    "bert-const": "the bert layer with every raw weight broadcast to all slots (constant raw plaintexts)",
 }
 FALLBACK_HBM_GBS = 6800.0
 
@@ -328,6 +329,8 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     stream = torch.cuda.Stream()
     F.device_fill(d_in, 2 * p.n_in, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_INPUTS), 0, stream)
     F.device_fill(d_pt, p.n_pt, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_PLAINTEXTS), 0, stream)
+    if wl.const_pts:  # constant raw plaintexts (one residue per limb) come first
+        F.device_fill(d_pt, wl.const_pts, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_PLAINTEXTS), 2, stream)
     stream.synchronize()
 
     for _ in range(args.warmup):

@@ -81,17 +81,24 @@ enum { FIONA_KERNEL_AUTO = 0, FIONA_KERNEL_DIRECT = 1, FIONA_KERNEL_TILED = 2 };
 #define FIONA_DEVICE_NONE (-1)
 
 /* Route of one term (Sec. 4.1: a pure group takes the signed route, every
- * other group the raw route). */
-enum { FIONA_TERM_RAW = 0, FIONA_TERM_TERNARY = 1 };
+ * other group the raw route).  FIONA_TERM_RAW_CONST is a raw term whose
+ * plaintext encodes one value in every slot (column packing broadcasts a
+ * single weight to all slots, Sec. 6 "BERT"): the encoding of a constant
+ * slot vector is a constant poly, so in NTT form every coefficient of limb l
+ * holds the same residue.  The kernels read only that residue, the first of
+ * each limb (plaintexts[pt][l][0]); the plaintext keeps its [L][N] place in
+ * the plaintext buffer, and its other residues are not read. */
+enum { FIONA_TERM_RAW = 0, FIONA_TERM_TERNARY = 1, FIONA_TERM_RAW_CONST = 2 };
 
 /* One term = one execution group g_{j,i}: the weights of output j applied to
  * input A_i through one plaintext operand (Sec. 2.3 "Packing Layout and
  * Execution Groups"; Sec. 4.2 notation g_{j,i}).  16 bytes. */
 typedef struct fiona_term {
     uint32_t input;   /* i, index of the input ciphertext, < n_in                     */
-    uint32_t pt;      /* RAW: index of the raw-group plaintext, < n_pt; TERNARY: 0     */
+    uint32_t pt;      /* RAW, RAW_CONST: index of the raw-group plaintext, < n_pt;
+                         TERNARY: 0                                                   */
     uint32_t group;   /* TERNARY: scale group, < n_groups, owned by this output; RAW: 0 */
-    int8_t kind;      /* FIONA_TERM_RAW or FIONA_TERM_TERNARY                          */
+    int8_t kind;      /* FIONA_TERM_RAW, FIONA_TERM_TERNARY or FIONA_TERM_RAW_CONST     */
     int8_t sign;      /* TERNARY: h_g in {-1, 0, +1}; RAW: 0                           */
     uint16_t reserved;/* must be 0                                                      */
 } fiona_term;
@@ -135,7 +142,8 @@ typedef struct fiona_plan_stats_t {
     uint64_t rescale_combined;    /* one rescale per output with any nonzero term           */
     uint64_t n_inputs_used;       /* inputs read by at least one nonzero term               */
     uint64_t n_plaintexts_used;   /* distinct plaintexts read                               */
-    uint64_t bytes_min;           /* each used input, plaintext and each output moved once  */
+    uint64_t bytes_min;           /* each used input, plaintext and each output moved once
+                                     (a plaintext read only by RAW_CONST terms: L words)     */
     uint64_t wide_products;       /* 64x64->128-bit products per evaluation                 */
     uint32_t N;
     uint32_t L;
@@ -193,10 +201,10 @@ void fiona_plan_destroy(fiona_plan *plan); /* NULL is a no-op */
 /* Route of the weights of output j on input i, for the plan compiler.
  * 8 bytes. */
 typedef struct fiona_route {
-    int8_t kind;      /* FIONA_TERM_RAW or FIONA_TERM_TERNARY                         */
-    int8_t sign;      /* TERNARY: h_g in {-1, 0, +1}; RAW: 0                           */
+    int8_t kind;      /* FIONA_TERM_RAW, FIONA_TERM_TERNARY or FIONA_TERM_RAW_CONST     */
+    int8_t sign;      /* TERNARY: h_g in {-1, 0, +1}; RAW, RAW_CONST: 0                */
     uint16_t reserved;/* must be 0                                                     */
-    uint32_t pt;      /* RAW: the group's plaintext; TERNARY: the output's reconstruction-
+    uint32_t pt;      /* RAW, RAW_CONST: the group's plaintext; TERNARY: the output's reconstruction-
                          factor plaintext gamma (terms with one gamma share one PMult)  */
 } fiona_route;
 

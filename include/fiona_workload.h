@@ -19,7 +19,9 @@ extern "C" {
 
 /* Fill dst[outer][L][N] (device memory, 8-byte aligned) with the residues of
  * stream `key`; moduli is a HOST array of L values.  mode 0 = uniform
- * residues, mode 1 = every residue q-1.  Asynchronous on cuda_stream.
+ * residues, mode 1 = every residue q-1, mode 2 = uniform residues constant
+ * over each limb-poly (element n takes the value of element n - n mod N: a
+ * constant plaintext).  Asynchronous on cuda_stream.
  * Returns 0, or -1 on a bad argument, -5 on a CUDA error. */
 int fiona_workload_fill(void *cuda_stream, uint64_t *dst, uint64_t outer, uint32_t L, uint32_t N,
                         const uint64_t *moduli, uint64_t key, int mode);

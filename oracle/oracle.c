@@ -37,7 +37,10 @@
  *   outputs     [n_out][2][L][n_coef]
  * Terms of output j are term_*[term_offsets[j] .. term_offsets[j+1]).
  * kind 0 = raw route (uses term_pt), kind 1 = signed route (term_sign in
- * {-1,0,+1}, term_group = scale group whose plaintext is group_scale_pt[g]).
+ * {-1,0,+1}, term_group = scale group whose plaintext is group_scale_pt[g]),
+ * kind 2 = raw route whose plaintext encodes one value in every slot: the
+ * encoding of a constant slot vector is a constant poly, so every
+ * coefficient of limb l is the limb's first residue, plaintexts[pt][l][0].
  *
  * Return 0 on success, -1 on an argument the oracle cannot evaluate.
  */
@@ -123,10 +126,10 @@ static uint64_t eval_one(uint32_t j, uint32_t c, uint32_t l, uint64_t k,
 
     /* raw route: one PMult per raw group, added at the same scale */
     for (uint32_t e = e0; e < e1; ++e) {
-        if (term_kind[e] != 0)
+        if (term_kind[e] != 0 && term_kind[e] != 2)
             continue;
         uint64_t a = inputs[in_idx(term_input[e], c, l, k, L, n_coef)];
-        uint64_t p = plaintexts[pt_idx(term_pt[e], l, k, L, n_coef)];
+        uint64_t p = plaintexts[pt_idx(term_pt[e], l, term_kind[e] == 2 ? 0 : k, L, n_coef)];
         y = add_mod(y, mul_mod(p, a, q), q);
     }
     return y;
@@ -147,7 +150,7 @@ static int check_common(uint32_t L, const uint64_t *moduli, uint32_t n_in, uint3
     for (uint32_t e = 0; e < term_offsets[n_out]; ++e) {
         if (term_input[e] >= n_in)
             return -1;
-        if (term_kind[e] == 0) {
+        if (term_kind[e] == 0 || term_kind[e] == 2) {
             if (term_pt[e] >= n_pt)
                 return -1;
         } else if (term_kind[e] == 1) {

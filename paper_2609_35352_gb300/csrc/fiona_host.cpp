@@ -235,7 +235,7 @@ static int validate(const fiona_ctx *ctx, HostPlan &hp)
             if (t.input >= hp.n_in)
                 return set_error(FIONA_ERR_PLAN, "term %u: input %u >= n_in", e, t.input);
             if (t.reserved != 0) return set_error(FIONA_ERR_PLAN, "term %u: reserved != 0", e);
-            if (t.kind == FIONA_TERM_RAW) {
+            if (t.kind == FIONA_TERM_RAW || t.kind == FIONA_TERM_RAW_CONST) {
                 if (t.pt >= hp.n_pt)
                     return set_error(FIONA_ERR_PLAN, "term %u: plaintext %u >= n_pt", e, t.pt);
                 if (t.sign != 0 || t.group != 0)
@@ -351,6 +351,7 @@ static void compute_stats(const fiona_ctx *ctx, const HostPlan &hp, fiona_plan_s
     s.n_groups = hp.n_groups;
     s.n_nodes = hp.n_nodes;
     s.n_uses = hp.n_uses;
+    // pt_used: 1 = read whole (raw or scale plaintext), 2 = only residue 0 of each limb
     std::vector<uint8_t> in_used(hp.n_in, 0), pt_used(hp.n_pt, 0), grp_used(hp.n_groups, 0);
     for (uint32_t j = 0; j < hp.n_out; ++j) {
         uint64_t S = 0, R = 0, ops_direct = 0;
@@ -358,10 +359,13 @@ static void compute_stats(const fiona_ctx *ctx, const HostPlan &hp, fiona_plan_s
         for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
             const fiona_term &t = hp.terms[e];
             ++s.n_terms;
-            if (t.kind == FIONA_TERM_RAW) {
+            if (t.kind == FIONA_TERM_RAW || t.kind == FIONA_TERM_RAW_CONST) {
                 ++R;
                 in_used[t.input] = 1;
-                pt_used[t.pt] = 1;
+                if (t.kind == FIONA_TERM_RAW)
+                    pt_used[t.pt] = 1;
+                else if (!pt_used[t.pt])
+                    pt_used[t.pt] = 2;
             } else if (t.sign == 0) {
                 ++s.n_skipped_terms;
             } else {
@@ -389,12 +393,17 @@ static void compute_stats(const fiona_ctx *ctx, const HostPlan &hp, fiona_plan_s
         s.addsub_shared += hp.node_offsets[k + 1] - hp.node_offsets[k] - 1;
     for (uint32_t g = 0; g < hp.n_groups; ++g) s.n_scale_groups_used += grp_used[g];
     for (uint8_t v : in_used) s.n_inputs_used += v;
-    for (uint8_t v : pt_used) s.n_plaintexts_used += v;
+    uint64_t n_pt_whole = 0, n_pt_const = 0;
+    for (uint8_t v : pt_used) {
+        s.n_plaintexts_used += v != 0;
+        n_pt_whole += v == 1;
+        n_pt_const += v == 2;
+    }
     s.n_nonzero_terms = s.n_raw_terms + s.n_signed_terms;
     s.pmult_per_term = s.n_raw_terms + s.n_signed_terms;
     s.pmult_grouped = s.n_raw_terms + s.n_scale_groups_used;
     const uint64_t limb_poly = (uint64_t)ctx->N * ctx->L * 8;
-    s.bytes_min = limb_poly * (2 * s.n_inputs_used + s.n_plaintexts_used + 2ull * hp.n_out);
+    s.bytes_min = limb_poly * (2 * s.n_inputs_used + n_pt_whole + 2ull * hp.n_out) + n_pt_const * ctx->L * 8ull;
     s.wide_products = 2ull * ctx->L * ctx->N * s.pmult_grouped;
 }
 
@@ -453,9 +462,9 @@ static int lower_direct(fiona_plan *p)
         o.raw_begin = (uint32_t)raw_in.size();
         for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
             const fiona_term &t = hp.terms[e];
-            if (t.kind != FIONA_TERM_RAW) continue;
+            if (t.kind != FIONA_TERM_RAW && t.kind != FIONA_TERM_RAW_CONST) continue;
             raw_in.push_back(t.input);
-            raw_pt.push_back(t.pt);
+            raw_pt.push_back(t.pt | (t.kind == FIONA_TERM_RAW_CONST ? 0x80000000u : 0u));
         }
         o.raw_end = (uint32_t)raw_in.size();
     }
@@ -508,9 +517,9 @@ static void build_static_image(fiona_plan *p)
         o.raw_begin = (uint32_t)raw_in.size();
         for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
             const fiona_term &t = hp.terms[e];
-            if (t.kind != FIONA_TERM_RAW) continue;
+            if (t.kind != FIONA_TERM_RAW && t.kind != FIONA_TERM_RAW_CONST) continue;
             raw_in.push_back(t.input);
-            raw_pt.push_back(t.pt);
+            raw_pt.push_back(t.pt | (t.kind == FIONA_TERM_RAW_CONST ? 0x80000000u : 0u));
         }
         o.raw_end = (uint32_t)raw_in.size();
     }

@@ -90,7 +90,10 @@ direct_kernel(const uint64_t *__restrict__ in, const uint64_t *__restrict__ pt,
     }
     for (uint32_t r = o.raw_begin; r < o.raw_end; ++r) {
         const uint32_t i = raw_in[r];
-        const ulonglong2 p = ld2(ptl + (size_t)raw_pt[r] * LN);
+        // bit 31: a constant plaintext, its limb's residue 0 at every coefficient
+        const uint32_t wp = raw_pt[r];
+        ulonglong2 p = ld2(((wp >> 31) ? ptl - k : ptl) + (size_t)(wp & 0x7fffffffu) * LN);
+        if (wp >> 31) p.y = p.x;
         const ulonglong2 a0 = ld2(inl + (size_t)(2 * i) * LN);
         const ulonglong2 a1 = ld2(inl + (size_t)(2 * i + 1) * LN);
         rns::mac(lo[0][0], hi[0][0], p.x, a0.x);

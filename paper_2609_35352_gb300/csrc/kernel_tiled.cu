@@ -318,7 +318,7 @@ __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uin
     return wp;
 }
 
-template <int C, bool NARROW, uint32_t P>
+template <int C, bool NARROW, uint32_t P, bool KC>
 __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledArgs a)
 {
     using A = Arith<NARROW>;
@@ -377,20 +377,25 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     // operation words (read-only while the kernel runs: plain loads the
     // compiler may schedule early)
     auto op_word = [&](uint32_t off) -> uint32_t { return *reinterpret_cast<const uint32_t *>(sm + off); };
+    // byte offset of this lane's words in the limb of tile t
+    auto tile_koff = [&](uint32_t t) -> uint32_t { return ((t % a.tiles_per_limb) * T + lane * C) * 8; };
     // the plaintext words of operation word `w` in the tile at `base` (with
-    // stride 0 and the schedule's own address when there is no next tile: a
-    // harmless valid load)
-    auto fetch = [&](const char *base, uint32_t stride, uint32_t w) -> V<C> {
-        return ldg_stream<C>(reinterpret_cast<const uint64_t *>(base + (uint64_t)(w >> kOpPtShift) * stride), pol);
+    // stride 0, offset 0 and the schedule's own address when there is no next
+    // tile: a harmless valid load); a CONST operation reads the limb's first
+    // words instead (base - koff)
+    auto fetch = [&](const char *base, uint32_t koff, uint32_t stride, uint32_t w) -> V<C> {
+        const char *b = KC ? base - ((w & kOpConst) ? koff : 0u) : base;
+        return ldg_stream<C>(reinterpret_cast<const uint64_t *>(b + (uint64_t)(w >> kOpPtShift) * stride), pol);
     };
     V<C> r[P];
     uint32_t tile = blockIdx.x;
     const char *cur_ptl = tile_ptl(tile);
+    uint32_t cur_ko = cur_ptl ? tile_koff(tile) : 0;
     if (n_batches && tile < total) {
         const char *b0 = cur_ptl ? cur_ptl : reinterpret_cast<const char *>(a.sched);
         const uint32_t s0 = cur_ptl ? stride_bytes : 0;
 #pragma unroll
-        for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, s0, op_word(op0 + 4 * i));
+        for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, cur_ko, s0, op_word(op0 + 4 * i));
     }
 
     // every thread: start its 16-byte asynchronous copies of tile `t`'s
@@ -412,6 +417,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     for (; tile < total; tile += gridDim.x) {
         const uint32_t next = tile + gridDim.x;
         const char *next_ptl = tile_ptl(next);
+        const uint32_t next_ko = next_ptl ? tile_koff(next) : 0;
         const uint32_t l = a.limb0 + tile / a.tiles_per_limb;
         const uint32_t k0 = (tile % a.tiles_per_limb) * T;
         if (threadIdx.x == 0) s_limb = a.limbs[l];  // read after the barrier below
@@ -496,10 +502,11 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
         for (uint32_t b = 0; b < n_batches; ++b) {
             const bool wrap = b + 1 == n_batches;
             const char *nb = wrap ? next_ptl : cur_ptl;
-            uint32_t ns = stride_bytes;
+            uint32_t ns = stride_bytes, nko = wrap ? next_ko : cur_ko;
             if (!nb) {  // no next tile: a harmless valid load
                 nb = reinterpret_cast<const char *>(a.sched);
                 ns = 0;
+                nko = 0;
             }
             const uint32_t cur_off = op0 + b * P * 4, next_off = wrap ? op0 : cur_off + P * 4;
             const uint32_t first = op_word(cur_off);
@@ -534,15 +541,17 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
                 }
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
-                    const uint64_t g = A::operand(r[i].x[x]);
+                    // a CONST plaintext is its limb's residue 0 at every coefficient
+                    const uint64_t g = A::operand((KC && x > 0 && (op & kOpConst)) ? r[i].x[0] : r[i].x[x]);
                     A::mac(acc[0][x], g, s0.x[x]);
                     A::mac(acc[1][x], g, s1.x[x]);
                 }
-                r[i] = fetch(nb, ns, op_word(next_off + 4 * i));
+                r[i] = fetch(nb, nko, ns, op_word(next_off + 4 * i));
             }
             if (op_word(cur_off + 4 * (P - 1)) & kOpLast) finish();
         }
         cur_ptl = next_ptl;
+        cur_ko = next_ko;
 
         // 4. outputs split across warps: add the partial sums
         if (a.n_comb) {
@@ -574,31 +583,36 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     }
 }
 
-template <uint32_t P>
+template <uint32_t P, bool KC>
 void *select_ptr_p(int C, bool narrow)
 {
     if (C == 2)
-        return narrow ? reinterpret_cast<void *>(&tiled_kernel<2, true, P>)
-                      : reinterpret_cast<void *>(&tiled_kernel<2, false, P>);
-    return narrow ? reinterpret_cast<void *>(&tiled_kernel<1, true, P>)
-                  : reinterpret_cast<void *>(&tiled_kernel<1, false, P>);
+        return narrow ? reinterpret_cast<void *>(&tiled_kernel<2, true, P, KC>)
+                      : reinterpret_cast<void *>(&tiled_kernel<2, false, P, KC>);
+    return narrow ? reinterpret_cast<void *>(&tiled_kernel<1, true, P, KC>)
+                  : reinterpret_cast<void *>(&tiled_kernel<1, false, P, KC>);
 }
 
-void *select_ptr(int C, bool narrow, uint32_t P) { return P == 4 ? select_ptr_p<4>(C, narrow) : select_ptr_p<8>(C, narrow); }
+// KC: the variant that reads constant plaintexts (operations marked kOpConst)
+void *select_ptr(int C, bool narrow, uint32_t P, bool kc)
+{
+    if (kc) return P == 4 ? select_ptr_p<4, true>(C, narrow) : select_ptr_p<8, true>(C, narrow);
+    return P == 4 ? select_ptr_p<4, false>(C, narrow) : select_ptr_p<8, false>(C, narrow);
+}
 
 }  // namespace
 
-int tiled_kernel_attributes(int C, bool narrow, uint32_t P, cudaFuncAttributes *attr)
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, cudaFuncAttributes *attr)
 {
-    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P));
+    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc));
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attributes: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
 
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, size_t smem)
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, size_t smem)
 {
     cudaError_t e =
-        cudaFuncSetAttribute(select_ptr(C, narrow, P), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(select_ptr(C, narrow, P, kc), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attribute: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
@@ -622,7 +636,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     dim3 grid(std::min(tiles, resident));
     dim3 block(ts->warps * 32);
     cudaStream_t s = (cudaStream_t)stream;
-    void *fn = select_ptr(ts->C, ts->narrow, ts->batch);
+    void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const);
     void *args[] = {&a};
     cudaError_t e = cudaLaunchKernel(fn, grid, block, args, ts->smem, s);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel launch: %s", cudaGetErrorString(e));

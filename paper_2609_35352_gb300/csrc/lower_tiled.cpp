@@ -44,7 +44,7 @@ struct Seg {
 
 struct OutWork {
     std::vector<Seg> segs;
-    std::vector<std::pair<uint32_t, uint32_t>> raws;  // (source, pt)
+    std::vector<std::pair<uint32_t, uint32_t>> raws;  // (source | kOpConst if constant, pt)
 };
 
 // Estimated issue cost of operations, in warp instructions, and of the
@@ -301,16 +301,19 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
         }
         while (o.size() % P) o.push_back(kOpNop | zero_src);
         // a NOP loads a plaintext tile that another operation of its batch (or
-        // the nearest earlier one) loads too
-        uint32_t last_pt = 0;
+        // the nearest earlier one) loads too (the same words: same index, same
+        // CONST flag)
+        uint32_t last_pt = 0, last_const = 0;
         for (size_t b = 0; b < o.size(); b += P) {
             for (size_t i = b; i < b + P; ++i)
                 if (!(o[i] & kOpNop)) {
                     last_pt = o[i] >> kOpPtShift;
+                    last_const = o[i] & kOpConst;
                     break;
                 }
             for (size_t i = b; i < b + P; ++i)
-                if (o[i] & kOpNop) o[i] = (o[i] & ((1u << kOpPtShift) - 1)) | (last_pt << kOpPtShift);
+                if (o[i] & kOpNop)
+                    o[i] = (o[i] & ((1u << kOpPtShift) - 1) & ~kOpConst) | last_const | (last_pt << kOpPtShift);
         }
     }
     for (uint32_t wi = 0; wi < W; ++wi) {
@@ -546,6 +549,7 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
             if ((op & kOpLast) && pos != P - 1) return "LAST inside a batch";
             // every operation loads a plaintext tile, NOPs included
             if ((op >> kOpPtShift) >= std::max<uint32_t>(n_pt, 1)) return "plaintext index";
+            if ((op & kOpConst) && (op & kOpSeg)) return "SEG marked CONST";
             if (op & kOpNop) {
                 if (op & kOpSeg) return "SEG marked NOP";
                 if ((op & (kOpMaxSources - 1)) != zero) return "NOP source";
@@ -593,8 +597,8 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
 }  // namespace
 
 // kernel_tiled.cu
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, size_t smem);
-int tiled_kernel_attributes(int C, bool narrow, uint32_t P, cudaFuncAttributes *attr);
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, size_t smem);
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, cudaFuncAttributes *attr);
 
 int lower_tiled(fiona_plan *p)
 {
@@ -647,8 +651,8 @@ int lower_tiled(fiona_plan *p)
         std::vector<uint32_t> gl;
         for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
             const fiona_term &t = hp.terms[e];
-            if (t.kind == FIONA_TERM_RAW)
-                groups[j].raws.push_back({t.input, t.pt});
+            if (t.kind == FIONA_TERM_RAW || t.kind == FIONA_TERM_RAW_CONST)
+                groups[j].raws.push_back({t.input | (t.kind == FIONA_TERM_RAW_CONST ? kOpConst : 0u), t.pt});
             else if (t.sign != 0 && std::find(gl.begin(), gl.end(), t.group) == gl.end())
                 gl.push_back(t.group);
         }
@@ -702,6 +706,9 @@ int lower_tiled(fiona_plan *p)
         size_t smem = 0;
         double est = 0;
     };
+    // plans with constant plaintexts run the kernel variant that reads them
+    bool has_const = false;
+    for (const fiona_term &t : hp.terms) has_const |= t.kind == FIONA_TERM_RAW_CONST;
     std::vector<Shape> shapes;
     for (int C : {2, 1})
     for (uint32_t batch : {8u, 4u}) {
@@ -712,7 +719,7 @@ int lower_tiled(fiona_plan *p)
         if (!device) {  // lowering without a GPU: the build's usual figures
             attr.numRegs = 128;
             attr.sharedSizeBytes = 64;
-        } else if (tiled_kernel_attributes(C, narrow, batch, &attr) != FIONA_OK) {
+        } else if (tiled_kernel_attributes(C, narrow, batch, has_const, &attr) != FIONA_OK) {
             continue;
         }
         const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
@@ -836,6 +843,7 @@ int lower_tiled(fiona_plan *p)
     ts->warps = best.W;
     ts->tile = T;
     ts->batch = best.P;
+    ts->has_const = has_const;
     ts->smem = best.smem;
     ts->ctas_per_sm = best.ctas;
     ts->nodes_kept = (uint32_t)lw.nodes.size();
@@ -867,7 +875,7 @@ int lower_tiled(fiona_plan *p)
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
     }
     if (device) {
-        int rc = tiled_configure_kernel(best.C, narrow, best.P, ts->smem);
+        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, ts->smem);
         if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
         if (rc != FIONA_OK) {
             cudaFree(ts->sched.blob);

@@ -56,7 +56,7 @@ extern "C" int fiona_plan_compile(uint32_t n_in, uint32_t n_out, uint32_t n_pt, 
     for (uint64_t e = 0; e < pairs; ++e) {
         const fiona_route &r = routes[e];
         if (r.reserved) return set_error(FIONA_ERR_PLAN, "plan_compile: route %llu reserved field", (unsigned long long)e);
-        if (r.kind == FIONA_TERM_RAW) {
+        if (r.kind == FIONA_TERM_RAW || r.kind == FIONA_TERM_RAW_CONST) {
             if (r.sign != 0 || r.pt >= n_pt)
                 return set_error(FIONA_ERR_PLAN, "plan_compile: raw route %llu malformed", (unsigned long long)e);
         } else if (r.kind == FIONA_TERM_TERNARY) {
@@ -79,7 +79,7 @@ extern "C" int fiona_plan_compile(uint32_t n_in, uint32_t n_out, uint32_t n_pt, 
             t = fiona_term{};
             t.input = i;
             t.kind = (int8_t)r.kind;
-            if (r.kind == FIONA_TERM_RAW) {
+            if (r.kind == FIONA_TERM_RAW || r.kind == FIONA_TERM_RAW_CONST) {
                 t.pt = r.pt;
                 continue;
             }

@@ -51,14 +51,17 @@
 constexpr uint32_t kTiledMaxWarps = 16;
 constexpr uint32_t kPartBit = 0x80000000u;  // job target: partial slot
 
-// operation word: [31:13] plaintext index, [12:9] flags, [8:0] source index
+// operation word: [31:14] plaintext index, [13:9] flags, [8:0] source index.
+// CONST marks a raw term whose plaintext is constant over the coefficients
+// (FIONA_TERM_RAW_CONST): its load reads residue 0 of the limb.
 constexpr uint32_t kOpSrcBits = 9;
 constexpr uint32_t kOpMaxSources = 1u << kOpSrcBits;
 constexpr uint32_t kOpSeg = 1u << 9;
 constexpr uint32_t kOpLast = 1u << 10;
 constexpr uint32_t kOpFold = 1u << 11;
 constexpr uint32_t kOpNop = 1u << 12;
-constexpr uint32_t kOpPtShift = 13;
+constexpr uint32_t kOpConst = 1u << 13;
+constexpr uint32_t kOpPtShift = 14;
 constexpr uint32_t kOpMaxPlaintexts = 1u << (32 - kOpPtShift);
 
 constexpr uint32_t kWarpTableWords = 4;  // op offset, op count, seg offset, target offset
@@ -89,6 +92,7 @@ struct TiledSchedule {
     uint32_t warps = 8;        // warps per CTA
     uint32_t tile = 64;        // coefficients per CTA tile
     uint32_t batch = 8;        // P: operations per batch, plaintext tiles in flight per warp
+    bool has_const = false;    // some operation reads a constant plaintext (kOpConst)
     size_t smem = 0;           // dynamic shared memory per CTA
     uint32_t ctas_per_sm = 0;  // occupancy the lowering planned for
     uint32_t nodes_kept = 0;   // shared sums materialised per tile

@@ -27,7 +27,9 @@ __global__ void fill_kernel(uint64_t *__restrict__ dst, uint64_t total, uint32_t
         if (mode == 1) {
             dst[n] = q - 1;
         } else {
-            const uint64_t x = splitmix_mix(key + (n + 1) * 0x9E3779B97F4A7C15ull);
+            // mode 2: every element of a limb-poly takes the value of its first
+            const uint64_t idx = mode == 2 ? n - n % N : n;
+            const uint64_t x = splitmix_mix(key + (idx + 1) * 0x9E3779B97F4A7C15ull);
             dst[n] = __umul64hi(x, q);
         }
     }
@@ -38,7 +40,7 @@ __global__ void fill_kernel(uint64_t *__restrict__ dst, uint64_t total, uint32_t
 extern "C" int fiona_workload_fill(void *stream, uint64_t *dst, uint64_t outer, uint32_t L,
                                    uint32_t N, const uint64_t *moduli, uint64_t key, int mode)
 {
-    if (!dst || !moduli || L == 0 || L > 64 || N == 0 || (mode != 0 && mode != 1)) return -1;
+    if (!dst || !moduli || L == 0 || L > 64 || N == 0 || mode < 0 || mode > 2) return -1;
     Moduli m{};
     for (uint32_t l = 0; l < L; ++l) m.q[l] = moduli[l];
     const uint64_t total = outer * L * (uint64_t)N;

@@ -50,6 +50,7 @@ STREAM_PLAN = 3
 
 TERM_RAW = 0
 TERM_TERNARY = 1
+TERM_RAW_CONST = 2   # raw term whose plaintext is one value in every slot
 
 # numpy mirrors of the C structs declared in include/fiona.h
 TERM_DTYPE = np.dtype([("input", "<u4"), ("pt", "<u4"), ("group", "<u4"),
@@ -226,7 +227,7 @@ class Plan:
 
     def counts(self) -> Dict[str, int]:
         t = self.terms
-        raw = int(np.sum(t["kind"] == TERM_RAW))
+        raw = int(np.sum((t["kind"] == TERM_RAW) | (t["kind"] == TERM_RAW_CONST)))
         tern = t["kind"] == TERM_TERNARY
         return {
             "raw": raw,
@@ -368,6 +369,7 @@ class Workload:
     plan: Plan
     seed: int
     fill: str = "uniform"        # "uniform" residues, or "max" (every residue q-1)
+    const_pts: int = 0           # plaintexts [0, const_pts) are constant per limb
 
     @property
     def L(self) -> int:
@@ -388,6 +390,9 @@ class Workload:
         if self.fill == "max":
             return np.broadcast_to(q - np.uint64(1), shape).copy()
         flat = np.arange(outer * L * N, dtype=np.uint64).reshape(shape)
+        if stream == STREAM_PLAINTEXTS and self.const_pts:
+            # a constant plaintext repeats its limb's first residue
+            flat[: self.const_pts] = flat[: self.const_pts, :, :1]
         return residues_np(self.key(stream), flat, q)
 
     def host_inputs(self) -> np.ndarray:
@@ -411,6 +416,7 @@ class Workload:
         q = self.moduli_np[l.astype(np.int64)]
         if self.fill == "max":
             return q - np.uint64(1)
+        k = np.where(p < np.uint64(self.const_pts), np.uint64(0), k)
         flat = (p * np.uint64(self.L) + l) * np.uint64(self.N) + k
         return residues_np(self.key(STREAM_PLAINTEXTS), flat, q)
 
@@ -429,7 +435,7 @@ SEED_BASE = 0xF10A0000
 
 # Shapes of the configurations (Sec. 6 layers; Sec. 3.1 weighted sum)
 WORKLOADS = ("tiny", "tiny-dag", "worked-example", "wsum-pmult", "wsum-ternary",
-             "wsum-hybrid", "vgg", "vit", "bert", "overflow60", "overflow50")
+             "wsum-hybrid", "vgg", "vit", "bert", "bert-const", "overflow60", "overflow50")
 
 
 def make_workload(name: str, N: Optional[int] = None, L: Optional[int] = None,
@@ -482,6 +488,13 @@ def make_workload(name: str, N: Optional[int] = None, L: Optional[int] = None,
         n, qs = primes(1 << 16, 12, 50)
         plan = dense_hybrid_plan(PlanRng(seed), 96, 96, 2198, 2198, 488, dag_share=0.30)
         return Workload(name, n, qs, plan, seed)
+    if name == "bert-const":
+        # the BERT layer with its raw weights broadcast to every slot (single-
+        # weight column packing): every raw plaintext is constant per limb
+        seed = SEED_BASE + 4
+        n, qs = primes(1 << 16, 12, 50)
+        plan = dense_hybrid_plan(PlanRng(seed), 96, 96, 2198, 2198, 488, dag_share=0.30)
+        return Workload(name, n, qs, constant_raw_plan(plan), seed, const_pts=plan.counts()["raw"])
     if name in ("overflow60", "overflow50"):
         # worst case for lazy reduction: every residue q-1 and more terms per
         # output than the accumulators hold without a fold (60-bit primes:
@@ -493,6 +506,16 @@ def make_workload(name: str, N: Optional[int] = None, L: Optional[int] = None,
         plan = _overflow_plan(PlanRng(seed), 400 if bits_ == 60 else 2100)
         return Workload(name, n, qs, plan, seed, fill="max")
     raise KeyError(name)
+
+
+def constant_raw_plan(plan: Plan) -> Plan:
+    """The same plan with every raw term marked constant (raw plaintexts
+    come first, so they are plaintexts [0, raw count))."""
+    terms = plan.terms.copy()
+    raw = terms["kind"] == TERM_RAW
+    assert not raw.any() or int(terms["pt"][raw].max()) < int(raw.sum())
+    terms["kind"][raw] = TERM_RAW_CONST
+    return dataclasses.replace(plan, terms=terms)
 
 
 def worked_example_plan() -> Plan:

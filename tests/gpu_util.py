@@ -38,6 +38,8 @@ class DeviceLayer:
             mode = 1 if wl.fill == "max" else 0
             F.device_fill(self.d_in, 2 * p.n_in, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_INPUTS), mode)
             F.device_fill(self.d_pt, p.n_pt, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_PLAINTEXTS), mode)
+            if wl.const_pts:  # constant raw plaintexts come first
+                F.device_fill(self.d_pt, wl.const_pts, wl.L, wl.N, wl.moduli, wl.key(W.STREAM_PLAINTEXTS), 2)
         self.d_out = torch.full((p.n_out * 2 * wl.L * wl.N,), -1, dtype=torch.int64, device="cuda")
 
     def run(self, stream=None) -> None:

@@ -251,3 +251,24 @@ def test_rescale_arguments_on_the_host():
     plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
     assert plan.eval_rescale_status(2, buf, buf, buf, buf) == F.FIONA_ERR_NODEVICE
     assert F.lib().fiona_linear_eval_rescale(None, None, 2, 0, 0, 0, 0) == F.FIONA_ERR_ARG
+
+
+def test_constant_raw_terms_count_one_word_per_limb():
+    """A plaintext read only by FIONA_TERM_RAW_CONST terms moves L words, not
+    L limb-polys; every other count is that of the same layer with plain raw
+    terms."""
+    a = W.make_workload("bert-const", N=1024, L=3)
+    b = W.make_workload("bert", N=1024, L=3)
+    sa = F.Plan(F.Context(a.N, a.moduli, device=F.FIONA_DEVICE_NONE), a.plan).stats()
+    sb = F.Plan(F.Context(b.N, b.moduli, device=F.FIONA_DEVICE_NONE), b.plan).stats()
+    for k in ("n_raw_terms", "n_signed_terms", "n_plaintexts_used", "pmult_grouped", "addsub_shared"):
+        assert sa[k] == sb[k], k
+    n_raw_pts = a.const_pts
+    assert sb["bytes_min"] - sa["bytes_min"] == n_raw_pts * (a.N * a.L * 8 - a.L * 8)
+    # a constant term's plaintext index is checked like a raw one's
+    bad = a.plan.terms.copy()
+    e = int(np.nonzero(bad["kind"] == W.TERM_RAW_CONST)[0][0])
+    bad["pt"][e] = a.plan.n_pt
+    import dataclasses
+    with pytest.raises(F.FionaError):
+        F.Plan(F.Context(a.N, a.moduli, device=F.FIONA_DEVICE_NONE), dataclasses.replace(a.plan, terms=bad))

@@ -203,6 +203,24 @@ def test_closed_form_all_max_residues(name):
             assert np.all(y[j, :, l] == np.uint64((raw + sgn) % q))
 
 
+def test_constant_raw_terms_read_residue_zero():
+    """Kind 2 (constant plaintext) is the raw route on the plaintext whose
+    every coefficient is the limb's first residue: the same outputs as kind 0
+    on that broadcast plaintext, and different ones on the original."""
+    wl = W.make_workload("bert-const", N=1024, L=2)
+    X, P = small_inputs(wl, 16)
+    P = P.copy()
+    P[: wl.const_pts] = W.residues_np(123, np.arange(P[: wl.const_pts].size, dtype=np.uint64).reshape(
+        P[: wl.const_pts].shape), wl.moduli_np.reshape(1, -1, 1))  # not constant
+    got = oracle.linear_eval(wl.plan, wl.moduli, X, P)
+    flat = W.constant_raw_plan(wl.plan)
+    flat.terms["kind"][flat.terms["kind"] == W.TERM_RAW_CONST] = W.TERM_RAW
+    Pb = P.copy()
+    Pb[: wl.const_pts] = P[: wl.const_pts, :, :1]
+    assert np.array_equal(got, oracle.linear_eval(flat, wl.moduli, X, Pb))
+    assert not np.array_equal(got, oracle.linear_eval(flat, wl.moduli, X, P))
+
+
 def test_duplicate_pairs_sum():
     """Two groups on the same (output, input) pair add (plain summation)."""
     qs = W.ntt_primes(1024, 40, 2)

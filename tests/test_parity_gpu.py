@@ -35,6 +35,7 @@ SMALL = [
     ("vgg", 1024, 2),
     ("vit", 2048, 2),
     ("bert", 1024, 1),
+    ("bert-const", 1024, 1),
     ("overflow60", None, None),
     ("overflow50", None, None),
 ]
@@ -64,7 +65,8 @@ def test_elementwise_parity_small(name, N, L, kernel):
 # A fourth field forces the shared sums in play (0: all expanded), a fifth
 # selects batches of 4.
 SHAPES = ["2,16,0", "2,8,1", "1,16,1", "1,4,0", "2,12,1,0", "1,8,0,3", "2,8,1,-1,4", "1,16,0,2,4"]
-SHAPE_CASES = [("tiny-dag", None, None), ("vit", 2048, 2), ("bert", 1024, 1), ("vgg", 1024, 2),
+SHAPE_CASES = [("tiny-dag", None, None), ("vit", 2048, 2), ("bert", 1024, 1), ("bert-const", 1024, 1),
+               ("vgg", 1024, 2),
                ("overflow60", None, None), ("overflow50", None, None)]
 
 
@@ -193,7 +195,7 @@ def test_boundary_residues():
         assert np.array_equal(dl.outputs(), want), kernel
 
 
-FULL = ["wsum-pmult", "wsum-ternary", "wsum-hybrid", "vgg", "vit", "bert"]
+FULL = ["wsum-pmult", "wsum-ternary", "wsum-hybrid", "vgg", "vit", "bert", "bert-const"]
 
 
 @pytest.mark.parametrize("name", FULL)
@@ -207,7 +209,7 @@ def test_full_size_sampled_parity(name):
     dl.run()
     torch.cuda.synchronize()
     rng = np.random.default_rng(42)
-    n_s = 24 if name == "bert" else 64
+    n_s = 24 if name.startswith("bert") else 64
     limbs = rng.integers(0, wl.L, n_s)
     coefs = rng.integers(0, wl.N, n_s)
     coefs[:2] = [0, wl.N - 1]
@@ -241,6 +243,32 @@ def test_device_fill_matches_host_generator():
         p = int(rng.integers(wl.plan.n_pt))
         devp = to_host(dl.d_pt.view(wl.plan.n_pt, 16, wl.N)[p, l].contiguous())[k]
         assert np.array_equal(devp, wl.plaintext_values(p, l, k))
+
+
+def test_constant_plaintexts_are_read_at_residue_zero():
+    """FIONA_TERM_RAW_CONST: a constant plaintext's other residues are never
+    read -- overwriting them changes no output, on either kernel.  The
+    device fill of constant plaintexts matches the host generator."""
+    wl = W.make_workload("bert-const", N=2048, L=2)
+    dl = DeviceLayer(wl, host_inputs=False)
+    torch.cuda.synchronize()
+    n_pt, L, N = wl.plan.n_pt, wl.L, wl.N
+    pts = dl.d_pt.view(n_pt, L, N)
+    k = np.array([0, 1, 17, N - 1])
+    for p in (0, wl.const_pts - 1, wl.const_pts):
+        assert np.array_equal(to_host(pts[p, 1].contiguous())[k], wl.plaintext_values(p, 1, k))
+    want = {}
+    for kernel in ("direct", "tiled"):
+        dl.plan.select_kernel(kernel)
+        dl.run()
+        want[kernel] = dl.outputs().copy()
+    assert np.array_equal(want["direct"], want["tiled"])
+    pts[: wl.const_pts, :, 1:] = -1  # residues that are no residue at all
+    for kernel in ("direct", "tiled"):
+        dl.plan.select_kernel(kernel)
+        dl.d_out.fill_(-1)
+        dl.run()
+        assert np.array_equal(dl.outputs(), want[kernel]), kernel
 
 
 def test_host_buffer_path_matches_device_path():
