@@ -246,6 +246,32 @@ def workload_config(wl: W.Workload, name: str, stats: dict) -> dict:
     }
 
 
+def max_over_ranks(x: float, device: str = "cuda") -> float:
+    """The largest x over the ranks of the default process group (x itself
+    without one): a step takes as long as its slowest rank."""
+    import torch
+    dist = torch.distributed
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier() -> None:
+    """Barrier of the default process group, if there is one."""
+    import torch
+    dist = torch.distributed
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.barrier()
+
+
+def whole_job_rate(units_per_rank_step: float, steps: int, world: int, elapsed_s: float) -> float:
+    """Units all ranks processed per second: every rank processes the same
+    units each step (weak scaling), and elapsed_s is the slowest rank's."""
+    return world * units_per_rank_step * steps / elapsed_s
+
+
 def host_cores() -> int:
     try:
         return len(os.sched_getaffinity(0))
@@ -299,8 +325,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
 
     if rank == 0:
         B.build()
-    if world > 1:
-        torch.distributed.barrier()
+    barrier()
     torch.cuda.set_device(local_rank)
     dev = local_rank
     name = args.workload
@@ -340,8 +365,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     clocks = ClockSampler(dev)
-    if world > 1:
-        torch.distributed.barrier()
+    barrier()
     torch.cuda.synchronize()
     clocks.start()
     t_begin = torch.cuda.Event(enable_timing=True)
@@ -353,18 +377,14 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
         stops[s].record(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
-    if world > 1:
-        torch.distributed.barrier()
+    barrier()
     clk = clocks.stop()
     elapsed_ms = t_begin.elapsed_time(t_end)
     kernel_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(elapsed_ms)
     ms_per_step = elapsed_ms / args.steps
     terms = stats["n_nonzero_terms"]
-    value = world * terms * args.steps / (elapsed_ms / 1e3)
+    value = whole_job_rate(terms, args.steps, world, elapsed_ms / 1e3)
 
     avg_kernel_s = statistics.mean(kernel_ms) / 1e3
     peak, peak_kind = measured_peak()
@@ -387,17 +407,13 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
         e2e_steps = max(3, min(args.steps, args.e2e_steps))
         for _ in range(2):
             plan.eval_host(h_in, d_pt, h_out, d_in, d_out, stream=stream)
-        if world > 1:
-            torch.distributed.barrier()
+        barrier()
         t0 = time.perf_counter()
         for _ in range(e2e_steps):
             plan.eval_host(h_in, d_pt, h_out, d_in, d_out, stream=stream)
         dt = time.perf_counter() - t0
-        if world > 1:
-            t = torch.tensor([dt], device="cuda")
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            dt = float(t.item())
-        e2e = {"value": world * terms * e2e_steps / dt, "unit": UNIT,
+        dt = max_over_ranks(dt)
+        e2e = {"value": whole_job_rate(terms, e2e_steps, world, dt), "unit": UNIT,
                "h2d_bytes_per_step": n_in * 8, "d2h_bytes_per_step": n_out * 8,
                "ms_per_step": 1e3 * dt / e2e_steps, "steps": e2e_steps}
 
@@ -451,8 +467,7 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
 
     if rank == 0:
         B.build()
-    if world > 1:
-        torch.distributed.barrier()
+    barrier()
     torch.cuda.set_device(local_rank)
     dev = local_rank
     name = args.workload
@@ -490,8 +505,7 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     clocks = ClockSampler(dev)
-    if world > 1:
-        torch.distributed.barrier()
+    barrier()
     torch.cuda.synchronize()
     clocks.start()
     for s in range(args.steps):
@@ -499,16 +513,12 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
         ctx.rescale(L, count, d_y, d_o, stream=stream)
         stops[s].record(stream)
     torch.cuda.synchronize()
-    if world > 1:
-        torch.distributed.barrier()
+    barrier()
     clk = clocks.stop()
     step_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
     elapsed_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
-    value = world * count * args.steps / (elapsed_ms / 1e3)
+    elapsed_ms = max_over_ranks(elapsed_ms)
+    value = whole_job_rate(count, args.steps, world, elapsed_ms / 1e3)
     avg_s = statistics.mean(step_ms) / 1e3
     bfly = count * rescale_butterflies(N, L)
     peak_bfly = SM_COUNT * IMAD_PER_CLK_PER_SM * SM_MAX_MHZ * 1e6 / IMAD_SLOTS_PER_BUTTERFLY
@@ -543,8 +553,8 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
         t0 = time.perf_counter()
         for _ in range(e2e_steps):
             one()
-        dt = time.perf_counter() - t0
-        e2e = {"value": world * count * e2e_steps / dt, "unit": unit, "h2d_bytes_per_step": n_y * 8,
+        dt = max_over_ranks(time.perf_counter() - t0)
+        e2e = {"value": whole_job_rate(count, e2e_steps, world, dt), "unit": unit, "h2d_bytes_per_step": n_y * 8,
                "d2h_bytes_per_step": n_o * 8, "ms_per_step": 1e3 * dt / e2e_steps, "steps": e2e_steps}
 
     if rank == 0:
@@ -582,8 +592,7 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
 
     if rank == 0:
         B.build()
-    if world > 1:
-        torch.distributed.barrier()
+    barrier()
     torch.cuda.set_device(local_rank)
     dev = local_rank
     name = args.workload
@@ -629,6 +638,7 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     clocks = ClockSampler(dev)
+    barrier()
     torch.cuda.synchronize()
     clocks.start()
     for a, b, c in ev:
@@ -638,14 +648,15 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
         ctx.encode_coeffs(L, count, d_c, d_o, stream=stream)
         c.record(stream)
     torch.cuda.synchronize()
+    barrier()
     clk = clocks.stop()
     if ctx.device_check(stream) != F.FIONA_OK:
         raise RuntimeError("encoding reported a coefficient out of range")
     step_ms = [a.elapsed_time(c) for a, b, c in ev]
     emb_ms = [a.elapsed_time(b) for a, b, c in ev]
     ntt_ms = [b.elapsed_time(c) for a, b, c in ev]
-    elapsed_ms = sum(step_ms)
-    value = world * count * args.steps / (elapsed_ms / 1e3)
+    elapsed_ms = max_over_ranks(sum(step_ms))
+    value = whole_job_rate(count, args.steps, world, elapsed_ms / 1e3)
     logn = N.bit_length() - 1
     # the embedding is a complex transform of size N/2
     emb_flops = count * (N // 4) * (logn - 1) * FLOPS_PER_COMPLEX_BUTTERFLY
@@ -679,8 +690,8 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
         t0 = time.perf_counter()
         for _ in range(e2e_steps):
             one()
-        dt = time.perf_counter() - t0
-        e2e = {"value": world * count * e2e_steps / dt, "unit": unit, "h2d_bytes_per_step": h_slots.nbytes,
+        dt = max_over_ranks(time.perf_counter() - t0)
+        e2e = {"value": whole_job_rate(count, e2e_steps, world, dt), "unit": unit, "h2d_bytes_per_step": h_slots.nbytes,
                "d2h_bytes_per_step": count * L * N * 8, "ms_per_step": 1e3 * dt / e2e_steps, "steps": e2e_steps}
 
     if rank == 0:
