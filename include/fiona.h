@@ -282,31 +282,38 @@ int fiona_linear_eval_level(const fiona_plan *plan, void *cuda_stream, uint32_t 
  * polys, c0 and c1).  For each poly y, with r the coefficients of its last
  * limb (inverse NTT mod q_{L_cur-1}, canonical in [0, q_{L_cur-1})):
  *   out_l = (y_l - NTT_l(r mod q_l)) * q_{L_cur-1}^{-1}  mod q_l,
- * for l < L_cur - 1, into `out` ([count][L_cur-1][N], canonical).  The NTT
+ * for l < L_cur - 1, into `out` ([count][L_cur-1][N], canonical): the
+ * residues of floor(Y / q_{L_cur-1}) for the CRT value Y of each
+ * coefficient.  With FIONA_RESCALE_ROUND in `flags` the quotient is rounded
+ * to the nearest integer instead, floor((Y + h) / q_{L_cur-1}) with
+ * h = floor(q_{L_cur-1} / 2), as SEAL's rescale does: r is replaced by
+ * r' = (r + h) mod q_{L_cur-1} and the subtracted poly by r' - h.  The NTT
  * form is A[k] = a(psi^(2 brv(k) + 1)) mod q_l, psi the least primitive 2N-th
  * root of unity mod q_l and brv the log2(N)-bit reversal; every modulus must
  * be a prime = 1 mod 2N (FIONA_ERR_MODULUS otherwise).
- * The last limb of every input poly is overwritten with r; the other limbs
+ * The last limb of every input poly is overwritten with r (r' when rounding); the other limbs
  * are only read.  `out` must not overlap `polys`.  Device pointers of the
  * ctx's device, 16-byte aligned.  Asynchronous on `cuda_stream`, except that
  * the first call on a ctx builds its twiddle tables (about 32 N L bytes of
  * device memory, held until fiona_ctx_destroy) synchronously: make it before
  * any stream capture.  Errors: FIONA_ERR_ARG (L_cur outside [2, L], null,
- * misaligned or overlapping buffers), FIONA_ERR_NODEVICE, FIONA_ERR_MODULUS,
- * FIONA_ERR_NOMEM, FIONA_ERR_CUDA. */
+ * misaligned or overlapping buffers, unknown flags), FIONA_ERR_NODEVICE,
+ * FIONA_ERR_MODULUS, FIONA_ERR_NOMEM, FIONA_ERR_CUDA. */
+enum { FIONA_RESCALE_ROUND = 1 };
 int fiona_rescale(const fiona_ctx *ctx, void *cuda_stream, uint32_t L_cur, uint64_t count,
-                  uint64_t *polys, uint64_t *out);
+                  uint64_t *polys, uint64_t *out, uint32_t flags);
 
 /* A layer followed by its rescale: evaluates at level L_eval (as
  * fiona_linear_eval_level) into `work` ([n_out][2][L_eval][N]), then
  * rescales the 2 n_out polys of `work` into `outputs`
  * ([n_out][2][L_eval-1][N]), both on `cuda_stream`.  `work` ends with the
  * un-rescaled layer output except in its last limbs, which hold
- * coefficients.  `outputs` must overlap neither `work` nor `inputs`.
- * Errors as fiona_linear_eval_level and fiona_rescale (L_eval >= 2). */
+ * coefficients.  `outputs` must overlap neither `work` nor `inputs`.  `flags`
+ * as for fiona_rescale.  Errors as fiona_linear_eval_level and fiona_rescale
+ * (L_eval >= 2). */
 int fiona_linear_eval_rescale(const fiona_plan *plan, void *cuda_stream, uint32_t L_eval,
                               const uint64_t *inputs, const uint64_t *plaintexts, uint64_t *work,
-                              uint64_t *outputs);
+                              uint64_t *outputs, uint32_t flags);
 
 /* Plaintext encoding on the GPU (Sec. 2.2 "Ciphertexts and Slots": CKKS
  * packs a vector of numbers into the slots of a plaintext; the layer's gamma

@@ -45,7 +45,7 @@ def _setup(lib: ctypes.CDLL) -> ctypes.CDLL:
         for f in ("oracle_ntt_fast", "oracle_intt_fast"):
             getattr(lib, f).argtypes = [p, u32, u64, u64]
             getattr(lib, f).restype = None
-        lib.oracle_rescale.argtypes = [u64, u32, u32, p, p, p, ctypes.c_int]
+        lib.oracle_rescale.argtypes = [u64, u32, u32, p, p, p, ctypes.c_int, ctypes.c_int]
         lib.oracle_rescale.restype = ctypes.c_int
     if hasattr(lib, "oracle_ckks_embed"):
         lib.oracle_ckks_embed.argtypes = [u32, p, ctypes.c_double, p, u32, p]
@@ -169,13 +169,14 @@ def intt(A: np.ndarray, q: int, fast: bool = True) -> np.ndarray:
     return out
 
 
-def rescale(moduli, polys: np.ndarray, fast: bool = True) -> np.ndarray:
-    """Rescale polys [count][L][N] (NTT form) by the last modulus -> [count][L-1][N]."""
+def rescale(moduli, polys: np.ndarray, fast: bool = True, round: bool = False) -> np.ndarray:
+    """Rescale polys [count][L][N] (NTT form) by the last modulus -> [count][L-1][N]
+    (quotient rounded down, or to nearest with round=True)."""
     y = _c(polys, np.uint64)
     count, L, N = y.shape
     out = np.zeros((count, L - 1, N), np.uint64)
     qs = _c(list(moduli)[:L], np.uint64)
-    rc = load().oracle_rescale(count, N, L, _ptr(qs), _ptr(y), _ptr(out), 1 if fast else 0)
+    rc = load().oracle_rescale(count, N, L, _ptr(qs), _ptr(y), _ptr(out), 1 if fast else 0, 1 if round else 0)
     if rc != 0:
         raise ValueError("oracle_rescale: arguments it cannot evaluate")
     return out

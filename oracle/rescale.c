@@ -21,7 +21,11 @@
  *            canonical in [0, q_{L-1}):
  *              y'_l = (y_l - NTT_l(r mod q_l)) * q_{L-1}^{-1}  mod q_l,
  *            l = 0..L-2, i.e. y' = (Y - (Y mod q_{L-1})) / q_{L-1} for the
- *            integer Y in [0, Q) whose residues are y (coefficient-wise).
+ *            integer Y in [0, Q) whose residues are y (coefficient-wise);
+ *   rounding the same with Y + h in place of Y, h = floor(q_{L-1} / 2), so
+ *            that y' = floor((Y + h) / q_{L-1}), Y / q_{L-1} rounded: in
+ *            coefficient form r' = (r + h) mod q_{L-1} and the subtracted
+ *            poly is r' - h (mod q_l).
  *
  * Two transforms: the definition (an O(N^2) sum, for small N) and the
  * textbook radix-2 transform (Cooley-Tukey forward, Gentleman-Sande
@@ -172,7 +176,7 @@ void oracle_intt_fast(uint64_t *a, uint32_t N, uint64_t q, uint64_t psi)
  * fast != 0 uses the radix-2 transforms, 0 the definitions.  Returns 0, or
  * -1 if an argument cannot be evaluated. */
 int oracle_rescale(uint64_t count, uint32_t N, uint32_t L, const uint64_t *moduli, const uint64_t *in,
-                   uint64_t *out, int fast)
+                   uint64_t *out, int fast, int round)
 {
     if (L < 2 || N < 2 || (N & (N - 1))) return -1;
     uint64_t *psi = (uint64_t *)malloc(sizeof(uint64_t) * L);
@@ -193,9 +197,11 @@ int oracle_rescale(uint64_t count, uint32_t N, uint32_t L, const uint64_t *modul
         } else {
             oracle_intt_direct(y + (uint64_t)(L - 1) * N, r, N, ql, psi[L - 1]);
         }
+        const uint64_t h = round ? ql / 2 : 0;
+        for (uint32_t i = 0; i < N; ++i) r[i] = addm(r[i], h, ql);
         for (uint32_t l = 0; l + 1 < L; ++l) {
             const uint64_t q = moduli[l];
-            for (uint32_t i = 0; i < N; ++i) t[i] = r[i] % q;
+            for (uint32_t i = 0; i < N; ++i) t[i] = subm(r[i] % q, h % q, q);
             if (fast) {
                 oracle_ntt_fast(t, N, q, psi[l]);
             } else {

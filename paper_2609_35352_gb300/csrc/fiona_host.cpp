@@ -885,17 +885,20 @@ static int check_rescale_args(const fiona_ctx *ctx, uint32_t L_cur, uint64_t cou
 }
 
 extern "C" int fiona_rescale(const fiona_ctx *ctx, void *stream, uint32_t L_cur, uint64_t count, uint64_t *polys,
-                             uint64_t *out)
+                             uint64_t *out, uint32_t flags)
 {
+    if (flags & ~(uint32_t)FIONA_RESCALE_ROUND) return set_error(FIONA_ERR_ARG, "rescale: unknown flags 0x%x", flags);
     int rc = check_rescale_args(ctx, L_cur, count, polys, out, "rescale");
     if (rc) return rc;
     DeviceGuard g(ctx->device);
-    return launch_rescale(ctx, stream, L_cur, count, polys, out);
+    return launch_rescale(ctx, stream, L_cur, count, polys, out, flags & FIONA_RESCALE_ROUND);
 }
 
 extern "C" int fiona_linear_eval_rescale(const fiona_plan *p, void *stream, uint32_t L_eval, const uint64_t *in,
-                                         const uint64_t *pt, uint64_t *work, uint64_t *out)
+                                         const uint64_t *pt, uint64_t *work, uint64_t *out, uint32_t flags)
 {
+    if (flags & ~(uint32_t)FIONA_RESCALE_ROUND)
+        return set_error(FIONA_ERR_ARG, "linear_eval_rescale: unknown flags 0x%x", flags);
     int rc = check_eval_args(p, in, pt, work);
     if (rc) return rc;
     const uint64_t count = 2ull * p->hp.n_out;
@@ -908,7 +911,7 @@ extern "C" int fiona_linear_eval_rescale(const fiona_plan *p, void *stream, uint
     DeviceGuard g(p->ctx->device);
     rc = launch_range(p, stream, in, pt, work, 0, L_eval, L_eval);
     if (rc) return rc;
-    return launch_rescale(p->ctx, stream, L_eval, count, work, out);
+    return launch_rescale(p->ctx, stream, L_eval, count, work, out, flags & FIONA_RESCALE_ROUND);
 }
 
 static int check_encode_ctx(const fiona_ctx *ctx, const char *who)

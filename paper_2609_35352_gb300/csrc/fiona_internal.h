@@ -112,7 +112,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
 // rescale.cu.  Rescales `count` polys [count][Lc][N] (the last limb of each
 // is overwritten with its coefficients) into out [count][Lc-1][N].
 int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t count, uint64_t *polys,
-                   uint64_t *out);
+                   uint64_t *out, bool round);
 void free_rescale_tables(const fiona_ctx *ctx);
 namespace fiona_ntt {
 struct NttLimb;

@@ -69,9 +69,9 @@ __device__ __forceinline__ uint64_t reduce_any(uint64_t x, uint64_t q, uint64_t 
 // Modular butterflies.  Values between stages:
 //   forward, general   in [0, 8q): x is brought below 4q before each
 //                      butterfly (x + t, x - t + 4q with t in [0, 4q));
-//   forward, FAST      (q < 2^56, inputs below 4q) no reduction at all: each
+//   forward, FAST      (q < 2^56, inputs below 5q) no reduction at all: each
 //                      stage adds less than 4q to the bound, so after at most
-//                      17 stages values stay below 72q < 2^63;
+//                      17 stages values stay below 73q < 2^63;
 //   inverse            in [0, 4q): x + y is brought below 4q, and
 //                      x - y + 4q is only multiplied.
 template <bool FAST>

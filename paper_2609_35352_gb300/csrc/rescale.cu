@@ -4,7 +4,10 @@
 // the Signed and Raw Routes": one rescale per output).  For a poly y with
 // limbs y_0..y_{Lc-1} in NTT form:
 //   r    = coefficients of y_{Lc-1}       (inverse NTT mod q_{Lc-1})
-//   y'_l = (y_l - NTT_l(r mod q_l)) * q_{Lc-1}^{-1}  mod q_l,   l < Lc-1.
+//   y'_l = (y_l - NTT_l(r mod q_l)) * q_{Lc-1}^{-1}  mod q_l,   l < Lc-1,
+// the quotient of the CRT value Y by q_{Lc-1} rounded down; rounded to the
+// nearest (the variant that adds h = floor(q_{Lc-1} / 2) to Y), r becomes
+// r' = (r + h) mod q_{Lc-1} and the subtracted poly r' - h (mod q_l).
 // NTT form: A[k] = a(psi^(2 brv(k) + 1)) mod q, psi the least primitive
 // 2N-th root of unity mod q (the transform and its passes: ntt.cuh).
 //
@@ -37,6 +40,7 @@ struct Args {
     uint64_t *out;     // [count][Lc-1][N]
     const NttLimb *T;
     uint32_t Lc;
+    uint32_t round;    // 1: nearest quotient (add h = floor(q_{Lc-1} / 2))
 };
 
 // ---------------------------------------------------------------------------
@@ -73,10 +77,11 @@ __global__ void __launch_bounds__(kThreads, 3) k_inv_high(Args A)
     const NttLimb &Tl = A.T[A.Lc - 1];
     const uint64_t q = Tl.q;
     const ulonglong2 ninv = Tl.ninv;
+    const uint64_t h = A.round ? q / 2 : 0;
     inv_high_pass<LOGN>(smem_raw, Tl.inv, first, ModArith<false>{q},
                         [&](uint32_t sub, uint32_t pos) { return g[(size_t)pos * R2 + sub]; },
                         [&](uint32_t sub, uint32_t pos, uint64_t v) {
-                            g[(size_t)pos * R2 + sub] = canon4(mul_shoup_lazy(v, ninv, q), q);
+                            g[(size_t)pos * R2 + sub] = csub(canon4(mul_shoup_lazy(v, ninv, q), q) + h, q);
                         });
 }
 
@@ -96,11 +101,14 @@ __global__ void __launch_bounds__(kThreads, 3) k_fwd_high(Args A)
     uint64_t *o = A.out + (size_t)tr * (1u << LOGN) + first;
     const NttLimb &Tl = A.T[l];
     const uint64_t q = Tl.q, mu = Tl.mu64;
+    // rounding: subtract h mod q_l, as + (q_l - h mod q_l); the loaded value
+    // then stays below 5 q_l (FAST) or 2 q_l
+    const uint64_t hq = A.round ? q - reduce_any(A.T[A.Lc - 1].q / 2, q, mu) : 0;
     fwd_high_pass<LOGN>(
         smem_raw, Tl.fwd, first, ModArith<FAST>{q},
         [&](uint32_t sub, uint32_t pos) {
             const uint64_t v = g[(size_t)pos * R2 + sub];
-            return FAST ? v : reduce_any(v, q, mu);
+            return (FAST ? v : reduce_any(v, q, mu)) + hq;
         },
         [&](uint32_t sub, uint32_t pos, uint64_t v) { o[(size_t)pos * R2 + sub] = v; });
 }
@@ -120,7 +128,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_fwd_low(Args A)
     const NttLimb &Tl = A.T[l];
     const uint64_t q = Tl.q;
     const ulonglong2 qi = Tl.qinv[A.Lc - 1];
-    // transform values: below 72q (FAST) or 8q; M = 128q or 8q bounds them
+    // transform values: below 73q (FAST) or 8q; M = 128q or 8q bounds them
     const uint64_t M = (FAST ? 128 : 8) * q;
     fwd_low_pass<LOGN>(
         smem_raw, Tl.fwd, first, ModArith<FAST>{q},
@@ -243,7 +251,8 @@ int ntt_tables(const fiona_ctx *ctx, const fiona_ntt::NttLimb **limbs)
     return rc;
 }
 
-int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t count, uint64_t *polys, uint64_t *out)
+int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t count, uint64_t *polys, uint64_t *out,
+                   bool round)
 {
     const NttLimb *T = nullptr;
     const int rc = ntt_tables(ctx, &T);
@@ -311,6 +320,7 @@ int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t cou
         a.out = out + p0 * (Lc - 1) * (uint64_t)ctx->N;
         a.T = T;
         a.Lc = Lc;
+        a.round = round ? 1 : 0;
         const uint32_t inv_blocks = (uint32_t)(np << ltiles);
         const uint32_t fwd_blocks = (uint32_t)((np * (Lc - 1)) << ltiles);
         ks[0]<<<inv_blocks, kThreads, smem[0], s>>>(a);

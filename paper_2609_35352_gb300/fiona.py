@@ -29,6 +29,7 @@ FIONA_ERR_NODEVICE = -7
 FIONA_ERR_TIMEOUT = -8
 FIONA_ERR_INTERNAL = -9
 FIONA_DEVICE_NONE = -1
+FIONA_RESCALE_ROUND = 1
 FIONA_KERNEL_AUTO = 0
 FIONA_KERNEL_DIRECT = 1
 FIONA_KERNEL_TILED = 2
@@ -110,9 +111,9 @@ def lib() -> ctypes.CDLL:
         L.fiona_linear_eval_static.argtypes = [p, p, p, p, p]
         L.fiona_linear_eval_level.argtypes = [p, p, u32, p, p, p]
         L.fiona_linear_eval_level.restype = i32
-        L.fiona_rescale.argtypes = [p, p, u32, ctypes.c_uint64, p, p]
+        L.fiona_rescale.argtypes = [p, p, u32, ctypes.c_uint64, p, p, u32]
         L.fiona_rescale.restype = i32
-        L.fiona_linear_eval_rescale.argtypes = [p, p, u32, p, p, p, p]
+        L.fiona_linear_eval_rescale.argtypes = [p, p, u32, p, p, p, p, u32]
         L.fiona_linear_eval_rescale.restype = i32
         L.fiona_ckks_embed.argtypes = [p, p, ctypes.c_uint64, p, ctypes.c_double, p, p]
         L.fiona_ckks_embed.restype = i32
@@ -189,15 +190,17 @@ class Context:
             _check(rc, "fiona_device_check")
         return rc
 
-    def rescale(self, L_cur, count, polys, out, stream=None) -> None:
+    def rescale(self, L_cur, count, polys, out, stream=None, round=False) -> None:
         """fiona_rescale: divide `count` polys ([count][L_cur][N], NTT form)
-        by q_{L_cur-1} into out ([count][L_cur-1][N]); the last limb of each
-        input poly is overwritten."""
-        _check(self.rescale_status(L_cur, count, polys, out, stream), "fiona_rescale")
+        by q_{L_cur-1} into out ([count][L_cur-1][N]), the quotient rounded
+        down (or to nearest with round=True); the last limb of each input
+        poly is overwritten."""
+        _check(self.rescale_status(L_cur, count, polys, out, stream, round), "fiona_rescale")
 
-    def rescale_status(self, L_cur, count, polys, out, stream=None) -> int:
+    def rescale_status(self, L_cur, count, polys, out, stream=None, round=False, flags=None) -> int:
+        f = (FIONA_RESCALE_ROUND if round else 0) if flags is None else int(flags)
         return lib().fiona_rescale(self.handle, stream_handle(stream), int(L_cur), int(count), addr(polys),
-                                   addr(out))
+                                   addr(out), f)
 
     def ckks_embed_status(self, count, slots, scale, coeffs, work, stream=None) -> int:
         """fiona_ckks_embed: slots [count][N/2][2] float64 -> coeffs [count][N]
@@ -299,15 +302,16 @@ class Plan:
         return lib().fiona_linear_eval_level(self.handle, stream_handle(stream), int(L_eval), addr(inputs),
                                              addr(plaintexts), addr(outputs))
 
-    def eval_rescale(self, L_eval, inputs, plaintexts, work, outputs, stream=None) -> None:
+    def eval_rescale(self, L_eval, inputs, plaintexts, work, outputs, stream=None, round=False) -> None:
         """fiona_linear_eval_rescale: the layer at level L_eval into `work`,
         then its rescale into `outputs` ([n_out][2][L_eval-1][N])."""
-        _check(self.eval_rescale_status(L_eval, inputs, plaintexts, work, outputs, stream),
+        _check(self.eval_rescale_status(L_eval, inputs, plaintexts, work, outputs, stream, round),
                "fiona_linear_eval_rescale")
 
-    def eval_rescale_status(self, L_eval, inputs, plaintexts, work, outputs, stream=None) -> int:
+    def eval_rescale_status(self, L_eval, inputs, plaintexts, work, outputs, stream=None, round=False) -> int:
         return lib().fiona_linear_eval_rescale(self.handle, stream_handle(stream), int(L_eval), addr(inputs),
-                                               addr(plaintexts), addr(work), addr(outputs))
+                                               addr(plaintexts), addr(work), addr(outputs),
+                                               FIONA_RESCALE_ROUND if round else 0)
 
     def eval_static(self, inputs, plaintexts, outputs, stream=None) -> int:
         """fiona_linear_eval_static: no device allocation (returns the status)."""

@@ -244,13 +244,14 @@ def test_rescale_arguments_on_the_host():
     """fiona_rescale and fiona_linear_eval_rescale refuse a null ctx or plan
     and a validation-only context before touching any buffer."""
     buf = np.zeros(16, dtype=np.uint64)
-    assert F.lib().fiona_rescale(None, None, 2, 1, F.addr(buf), F.addr(buf)) == F.FIONA_ERR_ARG
+    assert F.lib().fiona_rescale(None, None, 2, 1, F.addr(buf), F.addr(buf), 0) == F.FIONA_ERR_ARG
+    assert F.lib().fiona_rescale(None, None, 2, 1, F.addr(buf), F.addr(buf), 2) == F.FIONA_ERR_ARG
     ctx = ctx_none()
     assert ctx.rescale_status(2, 1, buf, buf) == F.FIONA_ERR_NODEVICE
     wl = W.make_workload("tiny")
     plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
     assert plan.eval_rescale_status(2, buf, buf, buf, buf) == F.FIONA_ERR_NODEVICE
-    assert F.lib().fiona_linear_eval_rescale(None, None, 2, 0, 0, 0, 0) == F.FIONA_ERR_ARG
+    assert F.lib().fiona_linear_eval_rescale(None, None, 2, 0, 0, 0, 0, 0) == F.FIONA_ERR_ARG
 
 
 def test_constant_raw_terms_count_one_word_per_limb():

@@ -169,3 +169,41 @@ def test_eval_rescale_parity(name, N, L, kernel):
         mism = np.argwhere(got != want)
         assert mism.shape[0] == 0, (Le, mism[:5].tolist())
     assert plan.eval_rescale_status(1, to_device(X), to_device(P), work, out) == F.FIONA_ERR_ARG
+
+
+@pytest.mark.parametrize("N,L,bits,count", [(1024, 3, 50, 3), (2048, 4, 60, 2), (65536, 5, 50, 2),
+                                            (131072, 3, 59, 1)])
+def test_rounding_rescale_parity(N, L, bits, count):
+    """FIONA_RESCALE_ROUND: the nearest quotient (oracle round=True, pinned by
+    brute force); the last limb becomes r' = (r + floor(q_last / 2)) mod q_last."""
+    qs = W.ntt_primes(N, bits, L)
+    y = random_polys(N + 7 * L + bits, qs, count, N)
+    ctx = F.Context(N, qs, device=0)
+    d_y = to_device(y)
+    d_out = torch.full((count * (L - 1) * N,), -1, dtype=torch.int64, device="cuda")
+    ctx.rescale(L, count, d_y, d_out, round=True)
+    torch.cuda.synchronize()
+    got = to_host(d_out).reshape(count, L - 1, N)
+    assert np.array_equal(got, oracle.rescale(qs, y, round=True))
+    assert not np.array_equal(got, oracle.rescale(qs, y))
+    ql = qs[-1]
+    last = to_host(d_y).reshape(count, L, N)[:, L - 1]
+    for p in range(count):
+        r = oracle.intt(y[p, L - 1], ql)
+        assert np.array_equal(last[p], (r + np.uint64(ql // 2)) % np.uint64(ql))
+    assert ctx.rescale_status(L, count, d_y, d_out, flags=4) == F.FIONA_ERR_ARG
+
+
+def test_eval_rescale_rounding():
+    wl = W.make_workload("vit", N=2048, L=3)
+    ctx = F.Context(wl.N, wl.moduli, device=0)
+    plan = F.Plan(ctx, wl.plan)
+    p = wl.plan
+    X, P = wl.host_inputs(), wl.host_plaintexts()
+    work = torch.empty(p.n_out * 2 * wl.L * wl.N, dtype=torch.int64, device="cuda")
+    out = torch.empty(p.n_out * 2 * (wl.L - 1) * wl.N, dtype=torch.int64, device="cuda")
+    plan.eval_rescale(wl.L, to_device(X), to_device(P), work, out, round=True)
+    torch.cuda.synchronize()
+    layer = oracle.linear_eval(p, wl.moduli, X, P).reshape(p.n_out * 2, wl.L, wl.N)
+    assert np.array_equal(to_host(out).reshape(p.n_out * 2, wl.L - 1, wl.N),
+                          oracle.rescale(wl.moduli, layer, round=True))

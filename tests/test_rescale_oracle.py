@@ -118,3 +118,33 @@ def test_rescale_of_a_multiple_of_the_last_prime():
     out = oracle.rescale(qs, y)
     for l in range(L - 1):
         assert np.array_equal(oracle.intt(out[0, l], qs[l]), np.array([z % qs[l] for z in Z], np.uint64))
+
+
+@pytest.mark.parametrize("fast", [False, True])
+def test_rounding_rescale_is_the_nearest_quotient(fast):
+    """round=True: the residues of floor((Y + h) / q_last), h = floor(q_last / 2),
+    i.e. Y / q_last rounded to the nearest integer (brute force over Z_Q)."""
+    N, L = 16, 3
+    qs = W.ntt_primes(N, 40, L)
+    rng = np.random.default_rng(12)
+    y = np.zeros((2, L, N), np.uint64)
+    for p in range(2):
+        for l in range(L):
+            y[p, l] = rand_res(rng, qs[l], N)
+    out = oracle.rescale(qs, y, fast=fast, round=True)
+    Q = 1
+    for q in qs:
+        Q *= q
+    ql = qs[-1]
+    for p in range(2):
+        coef = [oracle.intt(y[p, l], qs[l]) for l in range(L)]
+        rcoef = [oracle.intt(out[p, l], qs[l]) for l in range(L - 1)]
+        for k in range(N):
+            Y = 0
+            for l, q in enumerate(qs):
+                Ml = Q // q
+                Y = (Y + int(coef[l][k]) * Ml * pow(Ml, -1, q)) % Q
+            Yp = (Y + ql // 2) // ql
+            assert abs(Yp * ql - Y) <= ql // 2
+            for l in range(L - 1):
+                assert int(rcoef[l][k]) == Yp % qs[l], (p, l, k)
