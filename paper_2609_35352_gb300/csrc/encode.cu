@@ -75,12 +75,12 @@ __device__ __forceinline__ int64_t round_coeff(double x, int *err)
 // embedding, inverse low stages of the size-n transform (LN = log2 n):
 // A[k] gathered from the slots
 template <int LN>
-__global__ void __launch_bounds__(kThreads, 1) k_embed_low(EmbArgs A)
+__global__ void __launch_bounds__(LowPass<LN>::threads, 2) k_embed_low(EmbArgs A)
 {
     using SH = Shape<LN>;
     using PS = LowPass<LN>;
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), p = blockIdx.x >> PS::ltiles;
     const uint32_t first = tile << PS::lsubs;
     const size_t base = (size_t)first << PS::s;
     const double2 *z = A.slots + ((size_t)p << LN);
@@ -94,13 +94,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_embed_low(EmbArgs A)
 // embedding, inverse high stages: x zeta^i, rounded Delta (2/N) Re and Im to
 // coefficients i and i + n
 template <int LN>
-__global__ void __launch_bounds__(kThreads, 2) k_embed_high(EmbArgs A)
+__global__ void __launch_bounds__(HighPass<LN>::threads, 2) k_embed_high(EmbArgs A)
 {
     using SH = Shape<LN>;
     using PS = HighPass<LN>;
     constexpr uint32_t R2 = 1u << (LN - SH::n1);
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), p = blockIdx.x >> PS::ltiles;
     const uint32_t first = tile << PS::lsubs;
     const double2 *g = A.work + ((size_t)p << LN) + first;
     const double2 *tw = A.E.twist + first;
@@ -118,13 +118,13 @@ __global__ void __launch_bounds__(kThreads, 2) k_embed_high(EmbArgs A)
 
 // RNS/NTT form, forward high stages: c mod q_l into out (lazy)
 template <int LOGN, bool FAST>
-__global__ void __launch_bounds__(kThreads, 3) k_enc_high(EncArgs A)
+__global__ void __launch_bounds__(HighPass<LOGN>::threads, 3) k_enc_high(EncArgs A)
 {
     using SH = Shape<LOGN>;
     using PS = HighPass<LOGN>;
     constexpr uint32_t R2 = 1u << (LOGN - SH::n1);
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), tr = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), tr = blockIdx.x >> PS::ltiles;
     const uint32_t p = tr / A.Lc, l = tr % A.Lc;
     const uint32_t first = tile << PS::lsubs;
     const int64_t *c = A.coeffs + ((size_t)p << LOGN) + first;
@@ -146,12 +146,12 @@ __global__ void __launch_bounds__(kThreads, 3) k_enc_high(EncArgs A)
 
 // RNS/NTT form, forward low stages, canonical store
 template <int LOGN, bool FAST>
-__global__ void __launch_bounds__(kThreads, 2) k_enc_low(EncArgs A)
+__global__ void __launch_bounds__(LowPass<LOGN>::threads, 4) k_enc_low(EncArgs A)
 {
     using SH = Shape<LOGN>;
     using PS = LowPass<LOGN>;
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), tr = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), tr = blockIdx.x >> PS::ltiles;
     const uint32_t l = tr % A.Lc;
     const uint32_t first = tile << PS::lsubs;
     uint64_t *o = A.out + ((size_t)tr << LOGN) + ((size_t)first << PS::s);
@@ -227,6 +227,9 @@ struct Kernels {
     EmbKern emb_low, emb_high;
     EncKern enc_high[2], enc_low[2];
     size_t s_emb_low, s_emb_high, s_enc_high, s_enc_low;
+    // log2 tiles per transform and threads per CTA of each pass
+    uint32_t lt_emb_low, lt_emb_high, lt_enc_high, lt_enc_low;
+    uint32_t t_emb_low, t_emb_high, t_enc_high, t_enc_low;
 };
 
 template <int LOGN>
@@ -239,7 +242,15 @@ constexpr Kernels kernels_for()
                    Inst<LOGN>::emb_low,
                    Inst<LOGN>::emb_high,
                    Inst<LOGN>::enc_high,
-                   Inst<LOGN>::enc_low};
+                   Inst<LOGN>::enc_low,
+                   LowPass<LOGN - 1>::ltiles,
+                   HighPass<LOGN - 1>::ltiles,
+                   HighPass<LOGN>::ltiles,
+                   LowPass<LOGN>::ltiles,
+                   LowPass<LOGN - 1>::threads,
+                   HighPass<LOGN - 1>::threads,
+                   HighPass<LOGN>::threads,
+                   LowPass<LOGN>::threads};
 }
 
 const Kernels &kernels(uint32_t n)
@@ -283,7 +294,6 @@ int launch_embed(const fiona_ctx *ctx, void *stream, uint64_t count, const doubl
     if (rc) return rc;
     if (count == 0) return FIONA_OK;
     const Kernels &K = kernels(n);
-    const uint32_t ln = n - 1, ltiles = ln - std::min<uint32_t>(ln, kLogTileMax);
     const uint8_t *tab = static_cast<const uint8_t *>(ctx->d_enc);
     EmbArgs a;
     a.E.cinv = reinterpret_cast<const double2 *>(tab);
@@ -293,15 +303,14 @@ int launch_embed(const fiona_ctx *ctx, void *stream, uint64_t count, const doubl
     a.err = ctx->d_kerr;
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaSuccess;
-    const uint64_t max_polys = ((1ull << 31) - 1) >> ltiles;
+    const uint64_t max_polys = ((1ull << 31) - 1) >> std::max(K.lt_emb_low, K.lt_emb_high);
     for (uint64_t p0 = 0; p0 < count && e == cudaSuccess; p0 += max_polys) {
         const uint64_t np = std::min<uint64_t>(count - p0, max_polys);
         a.slots = reinterpret_cast<const double2 *>(slots) + p0 * (ctx->N / 2);
         a.work = reinterpret_cast<double2 *>(work) + p0 * (ctx->N / 2);
         a.coeffs = coeffs + p0 * ctx->N;
-        const uint32_t blocks = (uint32_t)(np << ltiles);
-        K.emb_low<<<blocks, kThreads, K.s_emb_low, s>>>(a);
-        K.emb_high<<<blocks, kThreads, K.s_emb_high, s>>>(a);
+        K.emb_low<<<(uint32_t)(np << K.lt_emb_low), K.t_emb_low, K.s_emb_low, s>>>(a);
+        K.emb_high<<<(uint32_t)(np << K.lt_emb_high), K.t_emb_high, K.s_emb_high, s>>>(a);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "encode launch: %s", cudaGetErrorString(e));
@@ -324,20 +333,19 @@ int launch_encode_coeffs(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64
     for (uint32_t l = 0; l < Lc; ++l)
         if (ctx->moduli[l] >= (1ull << 56)) fast = false;
     const Kernels &K = kernels(n);
-    const uint32_t ltiles = n - std::min<uint32_t>(n, kLogTileMax);
     EncArgs a;
     a.T = T;
     a.Lc = Lc;
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = cudaSuccess;
-    const uint64_t max_polys = ((1ull << 31) - 1) / ((uint64_t)Lc << ltiles);
+    const uint64_t max_polys = ((1ull << 31) - 1) / ((uint64_t)Lc << std::max(K.lt_enc_high, K.lt_enc_low));
     for (uint64_t p0 = 0; p0 < count && e == cudaSuccess; p0 += max_polys) {
         const uint64_t np = std::min<uint64_t>(count - p0, max_polys);
         a.coeffs = coeffs + p0 * ctx->N;
         a.out = out + p0 * Lc * (uint64_t)ctx->N;
-        const uint32_t blocks = (uint32_t)((np * Lc) << ltiles);
-        K.enc_high[fast]<<<blocks, kThreads, K.s_enc_high, s>>>(a);
-        K.enc_low[fast]<<<blocks, kThreads, K.s_enc_low, s>>>(a);
+        const uint64_t nt = np * Lc;
+        K.enc_high[fast]<<<(uint32_t)(nt << K.lt_enc_high), K.t_enc_high, K.s_enc_high, s>>>(a);
+        K.enc_low[fast]<<<(uint32_t)(nt << K.lt_enc_low), K.t_enc_low, K.s_enc_low, s>>>(a);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "encode launch: %s", cudaGetErrorString(e));

@@ -19,6 +19,9 @@
 //              tile / R1 of them (adjacent columns, so accesses coalesce);
 //   low pass   the other stages, inside blocks of R2 consecutive elements;
 //              a CTA takes tile / R2 blocks.
+// A CTA's tile is 4096 elements in the high pass and 2048 in the low pass
+// (whose CTAs also stage about one twiddle per element: the smaller tile lets
+// more CTAs share an SM); a thread handles 16 elements.
 // A pass runs its stages in rounds of up to 4: in a round each thread holds
 // the 2^K elements of one group in registers, spaced by the round's smallest
 // distance, and applies the round's K stages to them (a group needs 2^K - 1
@@ -34,8 +37,7 @@
 
 namespace fiona_ntt {
 
-constexpr int kLogTileMax = 12;  // at most 4096 elements per CTA
-constexpr uint32_t kThreads = 256;
+constexpr int kLogTileMax = 12;  // at most 4096 elements per CTA (2048 in the low pass)
 constexpr int kLogNMin = 10, kLogNMax = 17;  // the ring dimensions a context accepts
 
 // ---------------------------------------------------------------------------
@@ -126,11 +128,14 @@ struct Shape {
     static constexpr int ltiles = LOGN - lt;                            // log2(tiles per transform)
 };
 
-// A pass over a tile: 2^LSUBS sub-transforms of 2^S positions, in rounds.
-template <int S, int LSUBS, bool HIGH>
+// A pass over a tile: 2^LSUBS sub-transforms of 2^S positions, in rounds,
+// 2^LTILES tiles per transform, 16 elements per thread (at least 64 threads).
+template <int S, int LSUBS, bool HIGH, int LTILES>
 struct PassShape {
     static constexpr int s = S, lsubs = LSUBS, subs = 1 << LSUBS;
     static constexpr int tile = 1 << (S + LSUBS);
+    static constexpr int ltiles = LTILES;
+    static constexpr uint32_t threads = tile / 16 < 64 ? 64 : tile / 16;
     static constexpr int pitch = (1 << S) + 1;
     static constexpr int nr = (S + 3) / 4;
     __host__ __device__ static constexpr int K(int r) { return S / nr + (r < S % nr ? 1 : 0); }
@@ -147,9 +152,15 @@ struct PassShape {
 };
 
 template <int LOGN>
-using HighPass = PassShape<Shape<LOGN>::n1, Shape<LOGN>::lt - Shape<LOGN>::n1, true>;
+using HighPass = PassShape<Shape<LOGN>::n1, Shape<LOGN>::lt - Shape<LOGN>::n1, true, Shape<LOGN>::ltiles>;
+// the low pass: a tile of half the high pass's, but at least one block
 template <int LOGN>
-using LowPass = PassShape<LOGN - Shape<LOGN>::n1, Shape<LOGN>::lt - (LOGN - Shape<LOGN>::n1), false>;
+struct LowShape {
+    static constexpr int s = LOGN - Shape<LOGN>::n1;
+    static constexpr int lt = Shape<LOGN>::lt - 1 > s ? Shape<LOGN>::lt - 1 : s;
+};
+template <int LOGN>
+using LowPass = PassShape<LowShape<LOGN>::s, LowShape<LOGN>::lt - LowShape<LOGN>::s, false, LOGN - LowShape<LOGN>::lt>;
 
 // Group g of round R: sub-transform `sub`, and the element positions
 // (hi << (lD + K)) + (i << lD) + lo, i < 2^K.  High pass: sub-transforms
@@ -158,7 +169,7 @@ template <class PS, int R>
 struct Group {
     static constexpr int K = PS::K(R), J0 = PS::J0(R), LD = PS::s - J0 - K;
     static constexpr int groups = PS::tile >> K;
-    static constexpr int per_thread = (groups + (int)kThreads - 1) / (int)kThreads;
+    static constexpr int per_thread = (groups + (int)PS::threads - 1) / (int)PS::threads;
     uint32_t sub, hi, lo;
     __device__ __forceinline__ explicit Group(uint32_t g)
     {
@@ -231,8 +242,8 @@ __device__ __forceinline__ void round(const typename A::W *stw, const A &ar, Ld 
     typename A::T x[P][E];
 #pragma unroll
     for (int gi = 0; gi < P; ++gi) {
-        const uint32_t g = threadIdx.x + gi * kThreads;
-        if (Gr::groups % kThreads == 0 || g < Gr::groups) {
+        const uint32_t g = threadIdx.x + gi * PS::threads;
+        if (Gr::groups % PS::threads == 0 || g < Gr::groups) {
             const Gr G(g);
 #pragma unroll
             for (int i = 0; i < E; ++i) x[gi][i] = ld(G.sub, G.pos(i));
@@ -241,8 +252,8 @@ __device__ __forceinline__ void round(const typename A::W *stw, const A &ar, Ld 
     between();
 #pragma unroll
     for (int gi = 0; gi < P; ++gi) {
-        const uint32_t g = threadIdx.x + gi * kThreads;
-        if (Gr::groups % kThreads == 0 || g < Gr::groups) {
+        const uint32_t g = threadIdx.x + gi * PS::threads;
+        if (Gr::groups % PS::threads == 0 || g < Gr::groups) {
             const Gr G(g);
             group_stages<PS, R, INV>(x[gi], G, stw, ar);
 #pragma unroll
@@ -284,13 +295,13 @@ __device__ __forceinline__ void stage_twiddles(W *stw, const W *tab, uint32_t fi
 {
     static_assert(sizeof(W) == 16, "twiddles are copied in 16-byte units");
     if constexpr (PS::high) {
-        for (uint32_t e = threadIdx.x; e < (1u << PS::s); e += kThreads) cp_async16(&stw[e], &tab[e]);
+        for (uint32_t e = threadIdx.x; e < (1u << PS::s); e += PS::threads) cp_async16(&stw[e], &tab[e]);
     } else {
         const uint32_t u = (1u << Shape<LOGN>::n1) + first;
 #pragma unroll 1
         for (int j = 0; j < PS::s; ++j) {
             const uint32_t cnt = PS::subs << j, off = cnt - PS::subs;
-            for (uint32_t e = threadIdx.x; e < cnt; e += kThreads)
+            for (uint32_t e = threadIdx.x; e < cnt; e += PS::threads)
                 cp_async16(&stw[off + ((e & ((1u << j) - 1)) << PS::lsubs) + (e >> j)], &tab[(u << j) + e]);
         }
     }
@@ -303,22 +314,22 @@ __device__ __forceinline__ void wait_twiddles()
     __syncthreads();
 }
 
-// A coalesced sweep over the tile's elements e (tile / kThreads per thread):
+// A coalesced sweep over the tile's elements e (tile / threads per thread):
 // every load first, then every store.
 template <class PS, class T, class Ld, class St>
 __device__ __forceinline__ void sweep(Ld ld, St st)
 {
-    constexpr int P = (PS::tile + (int)kThreads - 1) / (int)kThreads;
+    constexpr int P = (PS::tile + (int)PS::threads - 1) / (int)PS::threads;
     T v[P];
 #pragma unroll
     for (int i = 0; i < P; ++i) {
-        const uint32_t e = threadIdx.x + i * kThreads;
-        if (PS::tile % kThreads == 0 || e < PS::tile) v[i] = ld(e);
+        const uint32_t e = threadIdx.x + i * PS::threads;
+        if (PS::tile % PS::threads == 0 || e < PS::tile) v[i] = ld(e);
     }
 #pragma unroll
     for (int i = 0; i < P; ++i) {
-        const uint32_t e = threadIdx.x + i * kThreads;
-        if (PS::tile % kThreads == 0 || e < PS::tile) st(e, v[i]);
+        const uint32_t e = threadIdx.x + i * PS::threads;
+        if (PS::tile % PS::threads == 0 || e < PS::tile) st(e, v[i]);
     }
 }
 

@@ -50,12 +50,12 @@ struct Args {
 
 // inverse, low stages, on the last limb in place
 template <int LOGN>
-__global__ void __launch_bounds__(kThreads, 2) k_inv_low(Args A)
+__global__ void __launch_bounds__(LowPass<LOGN>::threads, 4) k_inv_low(Args A)
 {
     using SH = Shape<LOGN>;
     using PS = LowPass<LOGN>;
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), p = blockIdx.x >> PS::ltiles;
     const uint32_t first = tile << PS::lsubs;
     uint64_t *g = A.polys + ((size_t)p * A.Lc + (A.Lc - 1)) * (1u << LOGN) + ((size_t)first << PS::s);
     const NttLimb &Tl = A.T[A.Lc - 1];
@@ -65,13 +65,13 @@ __global__ void __launch_bounds__(kThreads, 2) k_inv_low(Args A)
 
 // inverse, high stages: stores r = N^-1 x, canonical
 template <int LOGN>
-__global__ void __launch_bounds__(kThreads, 3) k_inv_high(Args A)
+__global__ void __launch_bounds__(HighPass<LOGN>::threads, 3) k_inv_high(Args A)
 {
     using SH = Shape<LOGN>;
     using PS = HighPass<LOGN>;
     constexpr uint32_t R2 = 1u << (LOGN - SH::n1);
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), p = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), p = blockIdx.x >> PS::ltiles;
     const uint32_t first = tile << PS::lsubs;
     uint64_t *g = A.polys + ((size_t)p * A.Lc + (A.Lc - 1)) * (1u << LOGN) + first;
     const NttLimb &Tl = A.T[A.Lc - 1];
@@ -88,13 +88,13 @@ __global__ void __launch_bounds__(kThreads, 3) k_inv_high(Args A)
 // forward, high stages: r (the last limb's coefficients), reduced mod q_l
 // unless FAST, into out
 template <int LOGN, bool FAST>
-__global__ void __launch_bounds__(kThreads, 3) k_fwd_high(Args A)
+__global__ void __launch_bounds__(HighPass<LOGN>::threads, 3) k_fwd_high(Args A)
 {
     using SH = Shape<LOGN>;
     using PS = HighPass<LOGN>;
     constexpr uint32_t R2 = 1u << (LOGN - SH::n1);
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), tr = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), tr = blockIdx.x >> PS::ltiles;
     const uint32_t p = tr / (A.Lc - 1), l = tr % (A.Lc - 1);
     const uint32_t first = tile << PS::lsubs;
     const uint64_t *g = A.polys + ((size_t)p * A.Lc + (A.Lc - 1)) * (1u << LOGN) + first;
@@ -115,12 +115,12 @@ __global__ void __launch_bounds__(kThreads, 3) k_fwd_high(Args A)
 
 // forward, low stages, then y' = (y_l - t) * q_{Lc-1}^-1
 template <int LOGN, bool FAST>
-__global__ void __launch_bounds__(kThreads, 2) k_fwd_low(Args A)
+__global__ void __launch_bounds__(LowPass<LOGN>::threads, 4) k_fwd_low(Args A)
 {
     using SH = Shape<LOGN>;
     using PS = LowPass<LOGN>;
     extern __shared__ __align__(16) uint8_t smem_raw[];
-    const uint32_t tile = blockIdx.x & ((1u << SH::ltiles) - 1), tr = blockIdx.x >> SH::ltiles;
+    const uint32_t tile = blockIdx.x & ((1u << PS::ltiles) - 1), tr = blockIdx.x >> PS::ltiles;
     const uint32_t p = tr / (A.Lc - 1), l = tr % (A.Lc - 1);
     const uint32_t first = tile << PS::lsubs;
     uint64_t *o = A.out + (size_t)tr * (1u << LOGN) + ((size_t)first << PS::s);
@@ -134,7 +134,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_fwd_low(Args A)
         smem_raw, Tl.fwd, first, ModArith<FAST>{q},
         [&] {
             // y is read only by the epilogue: start bringing it into L2 now
-            for (uint32_t e = threadIdx.x * 16; e < PS::tile; e += kThreads * 16)
+            for (uint32_t e = threadIdx.x * 16; e < PS::tile; e += PS::threads * 16)
                 asm volatile("prefetch.global.L2 [%0];\n" ::"l"(y + e));
         },
         [&](uint32_t sub, uint32_t pos) { return o[(sub << PS::s) + pos]; },
@@ -266,7 +266,6 @@ int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t cou
     const uint64_t qlast = ctx->moduli[Lc - 1];
     for (uint32_t l = 0; l + 1 < Lc; ++l)
         if (ctx->moduli[l] >= (1ull << 56) || qlast >= 4 * ctx->moduli[l]) fast = false;
-    const uint32_t lt = std::min<uint32_t>(n, kLogTileMax), ltiles = n - lt;
     const int ix = (int)n - kLogNMin;
     typedef void (*Kern)(Args);
     static const Kern inv_low[] = {k_inv_low<10>, k_inv_low<11>, k_inv_low<12>, k_inv_low<13>,
@@ -283,6 +282,14 @@ int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t cou
          k_fwd_low<14, false>, k_fwd_low<15, false>, k_fwd_low<16, false>, k_fwd_low<17, false>},
         {k_fwd_low<10, true>, k_fwd_low<11, true>, k_fwd_low<12, true>, k_fwd_low<13, true>,
          k_fwd_low<14, true>, k_fwd_low<15, true>, k_fwd_low<16, true>, k_fwd_low<17, true>}};
+    // per pass: tiles per transform (log2) and threads per CTA
+#define FIONA_GEO(P) {P<10>::ltiles, P<11>::ltiles, P<12>::ltiles, P<13>::ltiles, P<14>::ltiles, P<15>::ltiles, P<16>::ltiles, P<17>::ltiles}
+#define FIONA_THR(P) {P<10>::threads, P<11>::threads, P<12>::threads, P<13>::threads, P<14>::threads, P<15>::threads, P<16>::threads, P<17>::threads}
+    static const int low_lt[] = FIONA_GEO(LowPass), high_lt[] = FIONA_GEO(HighPass);
+    static const uint32_t low_thr[] = FIONA_THR(LowPass), high_thr[] = FIONA_THR(HighPass);
+#undef FIONA_GEO
+#undef FIONA_THR
+    const uint32_t lt_low = (uint32_t)low_lt[ix], lt_high = (uint32_t)high_lt[ix];
     const Kern ks[4] = {inv_low[ix], inv_high[ix], fwd_high[fast][ix], fwd_low[fast][ix]};
     typedef ModArith<false> MA;
     static const size_t low_smem[] = {
@@ -311,7 +318,7 @@ int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t cou
         }
     }
     // grid.x < 2^31: transforms * tiles, in chunks of whole polys
-    const uint64_t max_polys = ((1ull << 31) - 1) / ((uint64_t)(Lc - 1) << ltiles);
+    const uint64_t max_polys = ((1ull << 31) - 1) / ((uint64_t)(Lc - 1) << std::max(lt_low, lt_high));
     cudaStream_t s = (cudaStream_t)stream;
     for (uint64_t p0 = 0; p0 < count && e == cudaSuccess; p0 += max_polys) {
         const uint64_t np = std::min<uint64_t>(count - p0, max_polys);
@@ -321,12 +328,11 @@ int launch_rescale(const fiona_ctx *ctx, void *stream, uint32_t Lc, uint64_t cou
         a.T = T;
         a.Lc = Lc;
         a.round = round ? 1 : 0;
-        const uint32_t inv_blocks = (uint32_t)(np << ltiles);
-        const uint32_t fwd_blocks = (uint32_t)((np * (Lc - 1)) << ltiles);
-        ks[0]<<<inv_blocks, kThreads, smem[0], s>>>(a);
-        ks[1]<<<inv_blocks, kThreads, smem[1], s>>>(a);
-        ks[2]<<<fwd_blocks, kThreads, smem[2], s>>>(a);
-        ks[3]<<<fwd_blocks, kThreads, smem[3], s>>>(a);
+        const uint64_t nf = np * (Lc - 1);
+        ks[0]<<<(uint32_t)(np << lt_low), low_thr[ix], smem[0], s>>>(a);
+        ks[1]<<<(uint32_t)(np << lt_high), high_thr[ix], smem[1], s>>>(a);
+        ks[2]<<<(uint32_t)(nf << lt_high), high_thr[ix], smem[2], s>>>(a);
+        ks[3]<<<(uint32_t)(nf << lt_low), low_thr[ix], smem[3], s>>>(a);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "rescale launch: %s", cudaGetErrorString(e));
