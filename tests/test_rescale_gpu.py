@@ -207,3 +207,31 @@ def test_eval_rescale_rounding():
     layer = oracle.linear_eval(p, wl.moduli, X, P).reshape(p.n_out * 2, wl.L, wl.N)
     assert np.array_equal(to_host(out).reshape(p.n_out * 2, wl.L - 1, wl.N),
                           oracle.rescale(wl.moduli, layer, round=True))
+
+
+def test_layer_and_rescale_replay_in_a_cuda_graph():
+    """After a first call (which builds the tables), a layer followed by its
+    rescale is stream-ordered launches only: it captures into a CUDA graph and
+    every replay gives the oracle's residues."""
+    wl = W.make_workload("vit", N=2048, L=3)
+    ctx = F.Context(wl.N, wl.moduli, device=0)
+    plan = F.Plan(ctx, wl.plan)
+    p = wl.plan
+    X, P = wl.host_inputs(), wl.host_plaintexts()
+    d_in, d_pt = to_device(X), to_device(P)
+    work = torch.empty(p.n_out * 2 * wl.L * wl.N, dtype=torch.int64, device="cuda")
+    out = torch.empty(p.n_out * 2 * (wl.L - 1) * wl.N, dtype=torch.int64, device="cuda")
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        plan.eval_rescale(wl.L, d_in, d_pt, work, out, stream=s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        plan.eval_rescale(wl.L, d_in, d_pt, work, out, stream=s)
+    layer = oracle.linear_eval(p, wl.moduli, X, P).reshape(p.n_out * 2, wl.L, wl.N)
+    want = oracle.rescale(wl.moduli, layer)
+    for _ in range(3):
+        out.fill_(-1)
+        g.replay()
+        torch.cuda.synchronize()
+        assert np.array_equal(to_host(out).reshape(p.n_out * 2, wl.L - 1, wl.N), want)
