@@ -64,6 +64,7 @@ direct_kernel(const uint64_t *__restrict__ in, const uint64_t *__restrict__ pt,
     for (uint32_t s = o.seg_begin; s < o.seg_end; ++s) {
         const DirSeg sg = segs[s];
         uint64_t S[2][2] = {{0, 0}, {0, 0}};
+#pragma unroll 4
         for (uint32_t e = sg.op_begin; e < sg.op_end; ++e) {
             const uint32_t w = ops[e];
             const uint32_t i = w & 0x7fffffffu;
@@ -88,6 +89,7 @@ direct_kernel(const uint64_t *__restrict__ in, const uint64_t *__restrict__ pt,
         rns::mac(lo[1][1], hi[1][1], g.y, S[1][1]);
         fold_if_full();
     }
+#pragma unroll 2
     for (uint32_t r = o.raw_begin; r < o.raw_end; ++r) {
         const uint32_t i = raw_in[r];
         // bit 31: a constant plaintext, its limb's residue 0 at every coefficient
