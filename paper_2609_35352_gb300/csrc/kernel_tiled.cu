@@ -18,7 +18,7 @@
 //     before the group's product, then one product by gamma (Sec. 4.2
 //     "Grouping Reconstruction Operations"); per raw term a PMult-MAC of a
 //     plaintext tile and a source.  Plaintext tiles go from HBM straight to
-//     registers: each warp keeps the next P (8 or 4) of its stream in
+//     registers: each warp keeps the next P (16, 8 or 4) of its stream in
 //     flight, across job and tile boundaries, in a register queue indexed at
 //     compile time (the stream is processed in batches of that many
 //     operations).  Signed sums are lazy; products accumulate lazily; the
@@ -329,8 +329,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     constexpr uint32_t VB = C * 8;  // bytes of one lane's words in a tile
     extern __shared__ __align__(16) char sm[];
     __shared__ int s_abort;
-    __shared__ __align__(16) LimbConst s_limb;
-    const uint32_t lim = smem_addr(&s_limb);
+    __shared__ __align__(16) LimbConst s_limb[2];  // per source region
     const uint32_t n_warps = blockDim.x >> 5;
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t n_buf = a.double_buffer ? 2 : 1;
@@ -412,43 +411,56 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
         cp_async_commit();
     };
 
+    // the tile's inputs in region `reg`, once this thread's copies have
+    // landed: narrow plans rewrite them in split form, each thread the words
+    // it copied; and the tile's limb constants
+    auto prepare = [&](uint32_t t, uint32_t reg) {
+        if (threadIdx.x == 0) s_limb[reg] = a.limbs[a.limb0 + t / a.tiles_per_limb];
+        if (!a.n_in) return;
+        cp_async_wait<0>();
+        if (NARROW) {
+            for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x) {
+                ulonglong2 *p = reinterpret_cast<ulonglong2 *>(sm + src0 + reg * a.src_bytes + i * 16);
+                const ulonglong2 x = *p;
+                *p = make_ulonglong2(A::operand(x.x), A::operand(x.y));
+            }
+        }
+    };
+
+    // At the top of each tile its inputs and limb constants are in region
+    // `buf`, published by a barrier.  With two regions the next tile's
+    // copies are started at the top of this tile and prepared at its end,
+    // where warps that finish early would otherwise wait: one barrier per
+    // tile.  With one region the next tile is staged after every warp is
+    // done with this one.
     uint32_t buf = 0;
-    if (a.n_in && tile < total) stage(tile, 0);
+    if (tile < total) {
+        if (a.n_in) stage(tile, 0);
+        prepare(tile, 0);
+    }
+    __syncthreads();
     for (; tile < total; tile += gridDim.x) {
         const uint32_t next = tile + gridDim.x;
         const char *next_ptl = tile_ptl(next);
         const uint32_t next_ko = next_ptl ? tile_koff(next) : 0;
         const uint32_t l = a.limb0 + tile / a.tiles_per_limb;
         const uint32_t k0 = (tile % a.tiles_per_limb) * T;
-        if (threadIdx.x == 0) s_limb = a.limbs[l];  // read after the barrier below
+        const uint32_t lim = smem_addr(&s_limb[buf]);
         const uint32_t sb = src0 + buf * a.src_bytes;  // this tile's source region
         const uint32_t src = sb + lane_off;
 
-        // 1. inputs of this tile: this thread's copies have landed (the next
-        //    tile's, when started here, may still be in flight); narrow plans
-        //    rewrite them in split form; the barrier publishes them
-        if (a.n_in) {
-            if (a.double_buffer && next < total) {
+        // 1. the next tile's inputs: into the other region, or (one region)
+        //    into L2 ahead of their staging
+        if (a.n_in && next < total) {
+            if (a.double_buffer) {
                 stage(next, buf ^ 1);
-                cp_async_wait<1>();
-            } else {
-                cp_async_wait<0>();
-            }
-            if (NARROW) {
-                for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x) {
-                    ulonglong2 *p = reinterpret_cast<ulonglong2 *>(sm + sb + i * 16);
-                    const ulonglong2 x = *p;
-                    *p = make_ulonglong2(A::operand(x.x), A::operand(x.y));
-                }
-            }
-            if (!a.double_buffer && next < total && warp == 0) {
+            } else if (warp == 0) {
                 const uint32_t ln = a.limb0 + next / a.tiles_per_limb;
                 const uint32_t kn = (next % a.tiles_per_limb) * T;
                 for (uint32_t s = lane; s < 2 * a.n_in; s += 32)
                     prefetch_l2(a.in + ((size_t)s * a.L + ln) * a.N + kn, TB);
             }
         }
-        __syncthreads();
 
         // 2. materialised shared sums, children first
         for (uint32_t lev = 0; lev < a.n_levels; ++lev) {
@@ -573,13 +585,26 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
                 stg<C>(dst + (size_t)a.L * a.N, y1);
             }
         }
-        // every warp is done with this tile's region and partial slots; the
-        // proxy fence orders this thread's shared-memory writes before the
-        // bulk copies that will overwrite the region
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        __syncthreads();
-        if (a.n_in && !a.double_buffer && next < total) stage(next, 0);
-        buf ^= a.double_buffer;
+        // 5. the next tile: with two regions, prepare its inputs (their
+        //    copies started at the top of this tile) before the barrier that
+        //    publishes them; with one, stage them once every warp is done
+        //    with this tile's region and partial slots.  The proxy fence
+        //    orders this thread's shared-memory writes before the copies
+        //    that will overwrite the region.
+        if (a.double_buffer) {
+            if (next < total) prepare(next, buf ^ 1);
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncthreads();
+            buf ^= 1;
+        } else {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncthreads();
+            if (next < total) {
+                if (a.n_in) stage(next, 0);
+                prepare(next, 0);
+                __syncthreads();
+            }
+        }
     }
 }
 
@@ -593,9 +618,19 @@ void *select_ptr_p(int C, bool narrow)
                   : reinterpret_cast<void *>(&tiled_kernel<1, false, P, KC>);
 }
 
+// batches of 16: one coefficient per lane only
+template <bool KC>
+void *select_ptr_16(int C, bool narrow)
+{
+    if (C != 1) return nullptr;
+    return narrow ? reinterpret_cast<void *>(&tiled_kernel<1, true, 16, KC>)
+                  : reinterpret_cast<void *>(&tiled_kernel<1, false, 16, KC>);
+}
+
 // KC: the variant that reads constant plaintexts (operations marked kOpConst)
 void *select_ptr(int C, bool narrow, uint32_t P, bool kc)
 {
+    if (P == 16) return kc ? select_ptr_16<true>(C, narrow) : select_ptr_16<false>(C, narrow);
     if (kc) return P == 4 ? select_ptr_p<4, true>(C, narrow) : select_ptr_p<8, true>(C, narrow);
     return P == 4 ? select_ptr_p<4, false>(C, narrow) : select_ptr_p<8, false>(C, narrow);
 }
@@ -604,6 +639,7 @@ void *select_ptr(int C, bool narrow, uint32_t P, bool kc)
 
 int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, cudaFuncAttributes *attr)
 {
+    if (!select_ptr(C, narrow, P, kc)) return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
     cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc));
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attributes: %s", cudaGetErrorString(e));
     return FIONA_OK;
@@ -611,6 +647,7 @@ int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, cudaFuncAtt
 
 int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, size_t smem)
 {
+    if (!select_ptr(C, narrow, P, kc)) return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
     cudaError_t e =
         cudaFuncSetAttribute(select_ptr(C, narrow, P, kc), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attribute: %s", cudaGetErrorString(e));
@@ -637,6 +674,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     dim3 block(ts->warps * 32);
     cudaStream_t s = (cudaStream_t)stream;
     void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const);
+    if (!fn) return set_error(FIONA_ERR_INTERNAL, "tiled kernel: no variant for the schedule's shape");
     void *args[] = {&a};
     cudaError_t e = cudaLaunchKernel(fn, grid, block, args, ts->smem, s);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel launch: %s", cudaGetErrorString(e));

@@ -711,8 +711,9 @@ int lower_tiled(fiona_plan *p)
     for (const fiona_term &t : hp.terms) has_const |= t.kind == FIONA_TERM_RAW_CONST;
     std::vector<Shape> shapes;
     for (int C : {2, 1})
-    for (uint32_t batch : {8u, 4u}) {
+    for (uint32_t batch : {16u, 8u, 4u}) {
         if (ctx->N % (32u * C)) continue;
+        if (batch == 16 && C != 1) continue;  // the kernels with 16 plaintexts in flight per lane
         const uint32_t T = 32u * C, PB = 2 * T * 8;
         const Costs k = costs_for(C, narrow);
         cudaFuncAttributes attr{};
@@ -807,11 +808,12 @@ int lower_tiled(fiona_plan *p)
     // resident warps up to 16 per SM, then 2 coefficients per lane (half the
     // per-operation overhead per coefficient), then more CTAs per SM (their
     // per-tile phases overlap), then batches of 4 with 2 coefficients per
-    // lane and of 8 with one (BERT and ViT ran faster with 4, VGG with 8),
+    // lane and of 16, then 8, with one (BERT and ViT ran faster with 4; VGG
+    // with 16, its deeper plaintext queue keeping more HBM reads in flight),
     // then the cost estimate.
     auto key = [](const Shape &s) {
-        return std::make_tuple(s.dbl ? 1 : 0, std::min<uint32_t>(s.ctas * s.W, 16), s.C, s.ctas,
-                               (s.C == 2) == (s.P == 4) ? 1 : 0, -s.est);
+        const int pref = s.C == 2 ? (s.P == 4 ? 2 : 1) : (s.P == 16 ? 2 : s.P == 8 ? 1 : 0);
+        return std::make_tuple(s.dbl ? 1 : 0, std::min<uint32_t>(s.ctas * s.W, 16), s.C, s.ctas, pref, -s.est);
     };
     Shape best = *std::max_element(shapes.begin(), shapes.end(),
                                    [&](const Shape &a, const Shape &b) { return key(a) < key(b); });

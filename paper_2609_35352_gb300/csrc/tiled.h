@@ -16,7 +16,7 @@
 //        traffic
 // with flags FOLD (reduce the accumulator before this batch) and LAST (this
 // job's result is complete after this batch: reduce, store, clear).  The
-// stream is processed in batches of P operations (P = 8 or 4, the number of
+// stream is processed in batches of P operations (P = 16, 8 or 4, the number of
 // plaintext tiles each warp keeps in flight): every job
 // starts a batch and is padded to whole batches; SEG and FOLD only open a
 // batch (a SEG's signed sum is formed before its batch) and LAST only closes
