@@ -27,6 +27,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <map>
 #include <numeric>
 #include <tuple>
 
@@ -594,6 +595,89 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
     return nullptr;
 }
 
+const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a, uint32_t W, const HostPlan &hp)
+{
+    using Expr = std::vector<std::pair<uint32_t, int64_t>>;  // (input, coefficient), sorted
+    auto add = [](Expr &dst, const Expr &src, int64_t f) {
+        Expr out;
+        size_t i = 0, j = 0;
+        while (i < dst.size() || j < src.size()) {
+            if (j == src.size() || (i < dst.size() && dst[i].first < src[j].first)) {
+                out.push_back(dst[i++]);
+            } else if (i == dst.size() || src[j].first < dst[i].first) {
+                out.push_back({src[j].first, src[j].second * f});
+                ++j;
+            } else {
+                const int64_t v = dst[i].second + src[j].second * f;
+                if (v) out.push_back({dst[i].first, v});
+                ++i;
+                ++j;
+            }
+        }
+        dst.swap(out);
+    };
+    std::vector<Expr> src(a.n_in + a.n_nodes + 1);  // + the zero tile
+    for (uint32_t i = 0; i < a.n_in; ++i) src[i] = {{i, 1}};
+    // a run of n 16-bit indices from word p (each run starts on a new word)
+    auto run = [&](size_t &p, uint32_t n, Expr &e, int64_t f) {
+        for (uint32_t i = 0; i < n; ++i) add(e, src[(w[p + i / 2] >> (16 * (i & 1))) & 0xffffu], f);
+        p += (n + 1) / 2;
+    };
+    // a signed-sum program at word p; p is left past it
+    auto program = [&](size_t &p, Expr &e) {
+        const uint32_t h = w[p++];
+        run(p, h & 0xffffu, e, 1);
+        run(p, h >> 16, e, -1);
+    };
+    for (uint32_t x = 0; x < a.n_nodes; ++x) {
+        size_t p = w[a.o_node_off + x];
+        program(p, src[a.n_in + x]);
+    }
+    // (plaintext, input) -> coefficient, per output and partial slot
+    using Map = std::map<std::pair<uint32_t, uint32_t>, int64_t>;
+    auto put = [](Map &m, const std::pair<uint32_t, uint32_t> &key, int64_t v) {
+        if (!(m[key] += v)) m.erase(key);
+    };
+    std::vector<Map> out(hp.n_out), part(a.n_part);
+    for (uint32_t wi = 0; wi < W; ++wi) {
+        const size_t t = a.o_warp + (size_t)wi * kWarpTableWords;
+        const uint32_t op0 = w[t], n_ops = w[t + 1];
+        size_t sp = w[t + 2], tp = w[t + 3];
+        Map job;
+        for (uint32_t f = 0; f < n_ops; ++f) {
+            const uint32_t op = w[op0 + f], pt = op >> kOpPtShift;
+            if (op & kOpSeg) {
+                Expr e;
+                program(sp, e);
+                for (auto &x : e) put(job, {pt, x.first}, x.second);
+            } else if (!(op & kOpNop)) {
+                for (auto &x : src[op & (kOpMaxSources - 1)]) put(job, {pt, x.first}, x.second);
+            }
+            if (op & kOpLast) {
+                const uint32_t tg = w[tp++];
+                Map &dst = (tg & kPartBit) ? part[tg & ~kPartBit] : out[tg];
+                for (auto &x : job) put(dst, x.first, x.second);
+                job.clear();
+            }
+        }
+    }
+    for (uint32_t r = 0; r < a.n_comb; ++r)
+        for (uint32_t q = w[a.o_comb_off + r]; q < w[a.o_comb_off + r + 1]; ++q)
+            for (auto &x : part[w[a.o_comb_parts + q]]) put(out[w[a.o_comb_out + r]], x.first, x.second);
+    for (uint32_t j = 0; j < hp.n_out; ++j) {
+        Map want;
+        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
+            const fiona_term &tm = hp.terms[e];
+            if (tm.kind == FIONA_TERM_RAW || tm.kind == FIONA_TERM_RAW_CONST)
+                put(want, {tm.pt, tm.input}, 1);
+            else if (tm.sign != 0)
+                put(want, {hp.group_scale_pt[tm.group], tm.input}, tm.sign);
+        }
+        if (want != out[j]) return "an output differs from the plan's terms";
+    }
+    return nullptr;
+}
+
 }  // namespace
 
 // kernel_tiled.cu
@@ -873,6 +957,10 @@ int lower_tiled(fiona_plan *p)
     a.double_buffer = best.dbl ? 1 : 0;
     a.has_pt = hp.n_pt ? 1 : 0;
     if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB, best.P)) {
+        delete ts;
+        return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
+    }
+    if (const char *why = check_linear_map(sc.w, a, best.W, hp)) {
         delete ts;
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
     }

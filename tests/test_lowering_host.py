@@ -1,0 +1,87 @@
+"""The tiled lowering computes the plan's layer, checked on the host.
+
+Plan creation lowers every layer to the tiled kernel's schedule and, before
+accepting it, evaluates that schedule symbolically (shared sums, SEG
+programs, operations, partial slots and their combination) into integer
+coefficients of (plaintext, input) products and compares them with the
+plan's own terms; a difference fails plan creation with
+FIONA_ERR_INTERNAL.  These tests run that check, and the index checks before
+it, on many random layers and every shape the lowering can be forced to, with
+no GPU (validation-only contexts)."""
+import numpy as np
+import pytest
+
+from paper_2609_35352_gb300 import build as B
+from paper_2609_35352_gb300 import fiona as F
+from paper_2609_35352_gb300 import workloads as W
+
+SHAPES = [None, "2,16,0", "2,8,1", "1,16,1", "1,4,0", "2,8,1,-1,4", "1,8,0,3", "1,16,1,-1,16", "2,4,1,-1,8"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    B.build()
+
+
+def random_layer(rng, big=False):
+    """Random route mix: raw, constant raw, ternary with zeros; one to three
+    reconstruction factors per output; shared sums from the plan compiler."""
+    n_in = int(rng.integers(1, 200 if big else 40))
+    n_out = int(rng.integers(1, 40 if big else 20))
+    n_gamma = int(rng.integers(1, 4))
+    p_raw, p_const, p_zero = rng.uniform(0, 0.6), rng.uniform(0, 0.3), rng.uniform(0, 0.2)
+    r = np.zeros((n_out, n_in), F.ROUTE_DTYPE)
+    n_raw = 0
+    for j in range(n_out):
+        for i in range(n_in):
+            u = rng.random()
+            if u < p_raw:
+                kind = W.TERM_RAW_CONST if rng.random() < p_const else W.TERM_RAW
+                r[j, i] = (kind, 0, 0, n_gamma * n_out + n_raw)
+                n_raw += 1
+            else:
+                t = 0 if rng.random() < p_zero else int(rng.choice([-1, 1]))
+                r[j, i] = (W.TERM_TERNARY, t, 0, j * n_gamma + int(rng.integers(n_gamma)))
+    return F.compile_plan(n_in, n_out, n_gamma * n_out + n_raw, r, share=bool(rng.integers(4)),
+                          exact=bool(rng.integers(2)))
+
+
+def lower(desc, N, bits, L):
+    ctx = F.Context(N, W.ntt_primes(N, bits, L), device=F.FIONA_DEVICE_NONE)
+    return F.Plan(ctx, desc)
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_random_layers_lower_exactly(seed, monkeypatch):
+    rng = np.random.default_rng(7000 + seed)
+    shape = SHAPES[seed % len(SHAPES)]
+    if shape:
+        monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+    desc = random_layer(rng, big=seed % 4 == 3)
+    bits = int(rng.choice([40, 50, 59]))  # narrow and wide arithmetic (lazy-sum bounds differ)
+    plan = lower(desc, 4096, bits, 2)     # fails with FIONA_ERR_INTERNAL if the map differs
+    st = plan.stats()
+    assert st["n_terms"] == len(desc.terms)
+
+
+@pytest.mark.parametrize("name", ["tiny", "vgg", "vit", "bert", "bert-const"])
+def test_workloads_lower_exactly(name):
+    wl = W.make_workload(name)
+    plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
+    if name != "tiny":
+        assert plan.stats()["kernel"] == F.FIONA_KERNEL_TILED
+
+
+def test_long_signed_runs_are_cut_and_still_exact():
+    """One output whose signed run is far longer than the 64-word lazy-sum
+    bound of narrow arithmetic (the lowering cuts it into pieces with the
+    same gamma), next to outputs with short runs."""
+    n_in, n_out = 300, 3
+    r = np.zeros((n_out, n_in), F.ROUTE_DTYPE)
+    for i in range(n_in):
+        r[0, i] = (W.TERM_TERNARY, 1 if i % 3 else -1, 0, 0)
+        r[1, i] = (W.TERM_TERNARY, -1 if i % 5 == 0 else 0, 0, 1)
+        r[2, i] = (W.TERM_RAW, 0, 0, 3 + i) if i < 20 else (W.TERM_TERNARY, 1, 0, 2)
+    desc = F.compile_plan(n_in, n_out, 3 + 20, r, share=False)
+    plan = lower(desc, 4096, 50, 2)
+    assert plan.stats()["kernel"] == F.FIONA_KERNEL_TILED
