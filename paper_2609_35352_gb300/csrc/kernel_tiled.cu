@@ -376,25 +376,29 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     // operation words (read-only while the kernel runs: plain loads the
     // compiler may schedule early)
     auto op_word = [&](uint32_t off) -> uint32_t { return *reinterpret_cast<const uint32_t *>(sm + off); };
-    // byte offset of this lane's words in the limb of tile t
-    auto tile_koff = [&](uint32_t t) -> uint32_t { return ((t % a.tiles_per_limb) * T + lane * C) * 8; };
-    // the plaintext words of operation word `w` in the tile at `base` (with
-    // stride 0, offset 0 and the schedule's own address when there is no next
-    // tile: a harmless valid load); a CONST operation reads the limb's first
-    // words instead (base - koff)
-    auto fetch = [&](const char *base, uint32_t koff, uint32_t stride, uint32_t w) -> V<C> {
-        const char *b = KC ? base - ((w & kOpConst) ? koff : 0u) : base;
+    // the first words of plaintext 0 in the limb of the tile whose words
+    // for this lane start at `ptl` (read by CONST operations)
+    auto tile_limb = [&](const char *ptl, uint32_t t) -> const char * {
+        return ptl ? ptl - ((t % a.tiles_per_limb) * T + lane * C) * 8 : nullptr;
+    };
+    // the plaintext words of operation word `w` in the tile at `base`, or
+    // for a CONST operation in the limb at `lbase` (with stride 0 and the
+    // schedule's own address for both when there is no next tile: a
+    // harmless valid load)
+    auto fetch = [&](const char *base, const char *lbase, uint32_t stride, uint32_t w) -> V<C> {
+        const char *b = KC && (w & kOpConst) ? lbase : base;
         return ldg_stream<C>(reinterpret_cast<const uint64_t *>(b + (uint64_t)(w >> kOpPtShift) * stride), pol);
     };
     V<C> r[P];
     uint32_t tile = blockIdx.x;
     const char *cur_ptl = tile_ptl(tile);
-    uint32_t cur_ko = cur_ptl ? tile_koff(tile) : 0;
+    const char *cur_lb = tile_limb(cur_ptl, tile);
     if (n_batches && tile < total) {
         const char *b0 = cur_ptl ? cur_ptl : reinterpret_cast<const char *>(a.sched);
+        const char *l0 = cur_ptl ? cur_lb : b0;
         const uint32_t s0 = cur_ptl ? stride_bytes : 0;
 #pragma unroll
-        for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, cur_ko, s0, op_word(op0 + 4 * i));
+        for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, l0, s0, op_word(op0 + 4 * i));
     }
 
     // every thread: start its 16-byte asynchronous copies of tile `t`'s
@@ -442,7 +446,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     for (; tile < total; tile += gridDim.x) {
         const uint32_t next = tile + gridDim.x;
         const char *next_ptl = tile_ptl(next);
-        const uint32_t next_ko = next_ptl ? tile_koff(next) : 0;
+        const char *next_lb = tile_limb(next_ptl, next);
         const uint32_t l = a.limb0 + tile / a.tiles_per_limb;
         const uint32_t k0 = (tile % a.tiles_per_limb) * T;
         const uint32_t lim = smem_addr(&s_limb[buf]);
@@ -514,11 +518,11 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
         for (uint32_t b = 0; b < n_batches; ++b) {
             const bool wrap = b + 1 == n_batches;
             const char *nb = wrap ? next_ptl : cur_ptl;
-            uint32_t ns = stride_bytes, nko = wrap ? next_ko : cur_ko;
+            const char *nlb = wrap ? next_lb : cur_lb;
+            uint32_t ns = stride_bytes;
             if (!nb) {  // no next tile: a harmless valid load
-                nb = reinterpret_cast<const char *>(a.sched);
+                nb = nlb = reinterpret_cast<const char *>(a.sched);
                 ns = 0;
-                nko = 0;
             }
             const uint32_t cur_off = op0 + b * P * 4, next_off = wrap ? op0 : cur_off + P * 4;
             const uint32_t first = op_word(cur_off);
@@ -558,12 +562,12 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
                     A::mac(acc[0][x], g, s0.x[x]);
                     A::mac(acc[1][x], g, s1.x[x]);
                 }
-                r[i] = fetch(nb, nko, ns, op_word(next_off + 4 * i));
+                r[i] = fetch(nb, nlb, ns, op_word(next_off + 4 * i));
             }
             if (op_word(cur_off + 4 * (P - 1)) & kOpLast) finish();
         }
         cur_ptl = next_ptl;
-        cur_ko = next_ko;
+        cur_lb = next_lb;
 
         // 4. outputs split across warps: add the partial sums
         if (a.n_comb) {
