@@ -4,13 +4,17 @@
 // coefficients per tile, all outputs per tile.  Shared memory holds the
 // schedule (bulk-copied once, completion counted on an mbarrier), the
 // source region(s) and the partial sums.
-//  1. Every thread copies its share of the (c0, c1) tile of every input into
-//     a source region with 16-byte asynchronous copies (cp.async, one commit
-//     group per tile), so each input residue leaves HBM once.  With two
+//  1. The (c0, c1) tile of every input is copied into a source region, so
+//     each input residue leaves HBM once.  With one coefficient per lane one
+//     thread issues one or two TMA tensor copies (the inputs seen as a 3-D
+//     tensor: coefficient, limb, input poly; a box of T coefficients, one
+//     limb and up to 256 polys lands exactly in the region's layout), their
+//     completion counted on the region's mbarrier; with two, every thread
+//     copies its share with 16-byte cp.async (measured: the main loop of
+//     those kernels compiles to fewer instructions that way).  With two
 //     source regions the next tile's copies run during this tile; otherwise
 //     warp 0 prefetches the next tile's inputs into L2.  Narrow plans (every
-//     q < 2^52) rewrite the tiles in radix-2^26 split form (rns.cuh), each
-//     thread the words it copied.
+//     q < 2^52) rewrite the tiles in radix-2^26 split form (rns.cuh).
 //  2. The materialised shared signed sums (Sec. 4.2 "Sharing Signed Sums")
 //     are formed once per tile, level by level, into the same region.
 //  3. Each warp runs its operation stream (tiled.h): per scale group a
@@ -27,9 +31,13 @@
 //  4. Outputs split across warps add their reduced partial sums.
 // The only spin-wait is thread 0's bounded wait for the schedule copy; if it
 // gives up, the CTA raises the context's error flag and stops.
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstring>
+#include <mutex>
 
 #include "tiled.h"
 
@@ -62,6 +70,36 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
         "l"(src), "r"(bytes), "r"(bar)
         : "memory");
+}
+
+// TMA tensor copy of the box at (x, y, z) of the 3-D tensor map `tm` into
+// shared memory at `dst` (128-byte aligned), counted on `bar`.
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm, uint32_t x, uint32_t y, uint32_t z,
+                                            uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(z), "r"(bar)
+        : "memory");
+}
+
+// Bounded wait (no suspend hint: a tile's copies land within microseconds)
+// for phase `parity` of the barrier; false if it gave up after 2^24 tries.
+__device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity)
+{
+    for (uint32_t it = 0; it < (1u << 24); ++it) {
+        uint32_t ok;
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(ok)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (ok) return true;
+    }
+    return false;
 }
 
 // Bulk prefetch of `bytes` (a multiple of 16, 16-byte aligned) into L2.
@@ -319,16 +357,19 @@ __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uin
 }
 
 template <int C, bool NARROW, uint32_t P, bool KC>
-__global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledArgs a)
+__global__ void __launch_bounds__(kTiledMaxWarps * 32)
+    tiled_kernel(const TiledArgs a, const __grid_constant__ CUtensorMap tm_in)
 {
     using A = Arith<NARROW>;
     using Acc = typename A::Acc;
+    constexpr bool TMA = C == 1;  // input tiles by TMA tensor copies
     constexpr uint32_t T = 32 * C;
     constexpr uint32_t TB = T * 8;  // bytes of one poly's tile
     constexpr uint32_t PB = 2 * TB; // bytes of one source (c0, c1)
     constexpr uint32_t VB = C * 8;  // bytes of one lane's words in a tile
-    extern __shared__ __align__(16) char sm[];
+    extern __shared__ __align__(128) char sm[];
     __shared__ int s_abort;
+    if (threadIdx.x == 0) s_abort = 0;
     __shared__ __align__(16) LimbConst s_limb[2];  // per source region
     const uint32_t n_warps = blockDim.x >> 5;
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -337,12 +378,24 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     const uint32_t part_base = src0 + n_buf * a.src_bytes;
     const uint32_t bar_off = part_base + a.n_part * PB;  // the schedule copy's mbarrier
     const uint32_t bar0 = smem_addr(sm) + bar_off;
+    const uint32_t bar_stage = bar0 + 8;  // + 8 * region: the region's input copies have landed
     const uint32_t total = a.n_limbs * a.tiles_per_limb;
     const uint32_t lane_off = lane * VB;
     const uint32_t *sw = reinterpret_cast<const uint32_t *>(sm);
 
-    // the schedule, once per CTA
+    // the schedule, once per CTA (TMA copies want the regions 128-byte
+    // aligned: a misaligned base raises the error flag and copies nothing)
+    if (TMA && threadIdx.x == 0 && (smem_addr(sm) & 127u)) {
+        s_abort = 1;
+        atomicOr(a.err, 1);
+    }
+    __syncthreads();
+    if (s_abort) return;
     if (threadIdx.x == 0) {
+        if (TMA) {
+            mbar_init(bar_stage, 1);
+            mbar_init(bar_stage + 8, 1);
+        }
         mbar_init(bar0, 1);
         mbar_expect_tx(bar0, a.sched_bytes);
         for (uint32_t o = 0; o < a.sched_bytes; o += 32768)
@@ -401,19 +454,32 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
         for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, l0, s0, op_word(op0 + 4 * i));
     }
 
-    // every thread: start its 16-byte asynchronous copies of tile `t`'s
-    // inputs into region `reg` (one commit group per tile)
-    constexpr uint32_t kChunks = TB / 16;  // per source poly
+    // start the copies of tile `t`'s inputs into region `reg`: thread 0's
+    // TMA copies (the boxes cover the 2 n_in polys, the last one ending at
+    // the last poly: an overlap is copied twice, the same words), or every
+    // thread's 16-byte asynchronous copies (one commit group per tile)
+    constexpr uint32_t kChunks = TB / 16;  // 16-byte words per source poly
     const uint32_t n_chunks = 2 * a.n_in * kChunks;
     auto stage = [&](uint32_t t, uint32_t reg) {
         const uint32_t l = a.limb0 + t / a.tiles_per_limb, k0 = (t % a.tiles_per_limb) * T;
         const uint32_t dst = smem_addr(sm) + src0 + reg * a.src_bytes;
-        const char *base = reinterpret_cast<const char *>(a.in + (size_t)l * a.N + k0);
-        const size_t LN8 = (size_t)a.L * a.N * 8;
-        for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x)
-            cp_async16(dst + i * 16, base + (size_t)(i / kChunks) * LN8 + (i % kChunks) * 16);
-        cp_async_commit();
+        if constexpr (TMA) {
+            if (threadIdx.x != 0) return;
+            const uint32_t bar = bar_stage + 8 * reg;
+            mbar_expect_tx(bar, a.n_boxes * a.box_rows * TB);
+            for (uint32_t j = 0; j < a.n_boxes; ++j) {
+                const uint32_t z = min(j * a.box_rows, 2 * a.n_in - a.box_rows);
+                tma_load_3d(dst + z * TB, &tm_in, k0, l, z, bar);
+            }
+        } else {
+            const char *base = reinterpret_cast<const char *>(a.in + (size_t)l * a.N + k0);
+            const size_t LN8 = (size_t)a.L * a.N * 8;
+            for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x)
+                cp_async16(dst + i * 16, base + (size_t)(i / kChunks) * LN8 + (i % kChunks) * 16);
+            cp_async_commit();
+        }
     };
+    uint32_t stage_phase = 0;  // bit r: phase of region r's copy barrier
 
     // the tile's inputs in region `reg`, once this thread's copies have
     // landed: narrow plans rewrite them in split form, each thread the words
@@ -421,7 +487,12 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32) tiled_kernel(const TiledA
     auto prepare = [&](uint32_t t, uint32_t reg) {
         if (threadIdx.x == 0) s_limb[reg] = a.limbs[a.limb0 + t / a.tiles_per_limb];
         if (!a.n_in) return;
-        cp_async_wait<0>();
+        if constexpr (TMA) {
+            if (!mbar_wait_spin(bar_stage + 8 * reg, (stage_phase >> reg) & 1u)) atomicOr(a.err, 1);
+            stage_phase ^= 1u << reg;
+        } else {
+            cp_async_wait<0>();  // this thread's copies; the barrier after publishes everyone's
+        }
         if (NARROW) {
             for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x) {
                 ulonglong2 *p = reinterpret_cast<ulonglong2 *>(sm + src0 + reg * a.src_bytes + i * 16);
@@ -658,6 +729,43 @@ int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, size_t smem)
     return FIONA_OK;
 }
 
+namespace {
+// cuTensorMapEncodeTiled, from the driver the runtime uses (no link to it)
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    });
+    return fn;
+}
+}  // namespace
+
+// The inputs [n_in][2][L][N] as a 3-D tensor (coefficient, limb, poly) with
+// boxes of T coefficients, one limb and `box_rows` polys.
+int tiled_input_map(const TiledArgs &a, uint32_t T, const uint64_t *in, uint32_t layout_L, CUtensorMap *tm)
+{
+    memset(tm, 0, sizeof(*tm));
+    if (!a.n_in) return FIONA_OK;
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (!enc) return set_error(FIONA_ERR_CUDA, "tiled kernel: cuTensorMapEncodeTiled is not available");
+    const cuuint64_t dims[3] = {a.N, layout_L, 2ull * a.n_in};
+    const cuuint64_t strides[2] = {(cuuint64_t)a.N * 8, (cuuint64_t)layout_L * a.N * 8};
+    const cuuint32_t box[3] = {T, 1, a.box_rows};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_UINT64, 3, const_cast<uint64_t *>(in), dims, strides, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return set_error(FIONA_ERR_CUDA, "tiled kernel: input tensor map (error %d)", (int)r);
+    return FIONA_OK;
+}
+
 int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
                  uint64_t *out, uint32_t l0, uint32_t l1, uint32_t layout_L)
 {
@@ -679,7 +787,11 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     cudaStream_t s = (cudaStream_t)stream;
     void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const);
     if (!fn) return set_error(FIONA_ERR_INTERNAL, "tiled kernel: no variant for the schedule's shape");
-    void *args[] = {&a};
+    CUtensorMap tm;  // read by the kernels with one coefficient per lane only
+    memset(&tm, 0, sizeof(tm));
+    if (ts->C == 1)
+        if (const int rc = tiled_input_map(a, ts->tile, in, layout_L, &tm)) return rc;
+    void *args[] = {&a, &tm};
     cudaError_t e = cudaLaunchKernel(fn, grid, block, args, ts->smem, s);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel launch: %s", cudaGetErrorString(e));
     return FIONA_OK;

@@ -337,7 +337,7 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
     w.insert(w.end(), jp.comb_out.begin(), jp.comb_out.end());
     sc.o_comb_parts = (uint32_t)w.size();
     w.insert(w.end(), jp.comb_parts.begin(), jp.comb_parts.end());
-    pad4(w);  // a multiple of 16 bytes
+    while (w.size() % 32) w.push_back(0);  // a multiple of 128 bytes: the regions after it take TMA copies
     return sc;
 }
 
@@ -488,7 +488,10 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
                            uint32_t n_pt, size_t smem, uint32_t PB, uint32_t P)
 {
     const size_t nw = w.size();
-    if (a.sched_bytes != nw * 4 || a.sched_bytes % 16) return "schedule size";
+    if (a.sched_bytes != nw * 4 || a.sched_bytes % 128) return "schedule size";
+    if (a.n_in && (a.box_rows == 0 || a.box_rows > 256 || a.box_rows > 2 * a.n_in ||
+                   (size_t)a.n_boxes * a.box_rows < 2ull * a.n_in || a.n_boxes > 2 * a.n_in))
+        return "input boxes";
     const uint32_t n_src = a.n_in + a.n_nodes, zero = n_src;  // the zero tile follows the sources
     if (n_src + 1 > kOpMaxSources) return "too many sources";
     if ((size_t)a.sched_bytes + (size_t)(a.double_buffer ? 2 : 1) * a.src_bytes + (size_t)a.n_part * PB + 24 >
@@ -955,6 +958,9 @@ int lower_tiled(fiona_plan *p)
     a.n_comb = (uint32_t)jp.comb_out.size();
     a.src_bytes = (hp.n_in + a.n_nodes + 1) * PB;  // + the zero tile
     a.double_buffer = best.dbl ? 1 : 0;
+    // TMA boxes of at most 256 polys covering the 2 n_in input polys
+    a.n_boxes = (2 * hp.n_in + 255) / 256;
+    a.box_rows = a.n_boxes ? (2 * hp.n_in + a.n_boxes - 1) / a.n_boxes : 0;
     a.has_pt = hp.n_pt ? 1 : 0;
     if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB, best.P)) {
         delete ts;

@@ -25,8 +25,9 @@
 // output split across warps whose reduced partial sums are added at the end
 // of the tile.
 //
-// The schedule is one array of 32-bit words, copied once per CTA into shared
-// memory:
+// The schedule is one array of 32-bit words (a multiple of 128 bytes, so that
+// the source regions after it are aligned for TMA), copied once per CTA into
+// shared memory:
 //   level offsets   shared sums of level l are nodes [lev[l], lev[l+1])
 //   node offsets    word offset of each node's program
 //   node programs   n_plus | n_minus << 16, then the plus then the minus
@@ -82,6 +83,8 @@ struct TiledArgs {
     uint32_t tiles_per_limb;
     uint32_t n_in, n_nodes, n_levels, n_part, n_comb;
     uint32_t src_bytes;      // one source region (inputs, shared sums, zero tile)
+    uint32_t box_rows;       // input polys per TMA box (<= 256), n_boxes boxes per tile
+    uint32_t n_boxes;
     uint32_t double_buffer;  // 1: two source regions, next tile staged early
     uint32_t has_pt;         // 0: the plan has no plaintexts (every load reads the schedule)
 };
