@@ -14,7 +14,9 @@
 //     those kernels compiles to fewer instructions that way).  With two
 //     source regions the next tile's copies run during this tile; otherwise
 //     warp 0 prefetches the next tile's inputs into L2.  Narrow plans (every
-//     q < 2^52) rewrite the tiles in radix-2^26 split form (rns.cuh).
+//     q < 2^52) with two coefficients per lane rewrite the tiles in
+//     radix-2^26 split form (rns.cuh); with one, the sources stay canonical
+//     and a product splits the words it reads.
 //  2. The materialised shared signed sums (Sec. 4.2 "Sharing Signed Sums")
 //     are formed once per tile, level by level, into the same region.
 //  3. Each warp runs its operation stream (tiled.h): per scale group a
@@ -244,9 +246,9 @@ struct Arith<false> {
     }
 };
 
-// q < 2^52: every factor in split form (sources in shared memory, the other
-// factor split on the way in); Karatsuba products into three accumulators;
-// packed sums.
+// q < 2^52: every factor in split form (sources split in shared memory or
+// where a product reads them, the other factor split on the way in);
+// Karatsuba products into three accumulators; packed sums of split words.
 template <>
 struct Arith<true> {
     struct Acc {
@@ -336,13 +338,14 @@ __device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32
 }
 
 // Signed sum of the program at byte offset `hdr` (n_plus | n_minus << 16,
-// then the plus run, then the minus run), both polys, as canonical residues.
-// Returns the offset just past the program.
-template <bool NARROW, int C, uint32_t TB>
+// then the plus run, then the minus run), both polys, as canonical residues;
+// SPLIT: the sources are in split form (else canonical, whatever the
+// arithmetic).  Returns the offset just past the program.
+template <bool SPLIT, int C, uint32_t TB>
 __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uint32_t hdr, uint32_t lim,
                                                V<C> &o0, V<C> &o1)
 {
-    using A = Arith<NARROW>;
+    using A = Arith<SPLIT>;
     const uint32_t h = *reinterpret_cast<const uint32_t *>(sm + hdr);
     V<C> p0{}, p1{}, m0{}, m1{};
     uint32_t wp = run_sum<C, TB>(sm, src, hdr + 4, h & 0xffffu, p0, p1);
@@ -363,6 +366,11 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     using A = Arith<NARROW>;
     using Acc = typename A::Acc;
     constexpr bool TMA = C == 1;  // input tiles by TMA tensor copies
+    // narrow sources in shared memory: split form (rewritten once per tile)
+    // with two coefficients per lane; canonical, split where a product reads
+    // them, with one (measured: VGG 2.46 -> 2.36 ms, while the layers with
+    // two coefficients per lane ran 4-5% slower that way)
+    constexpr bool SPLIT = NARROW && C == 2;
     constexpr uint32_t T = 32 * C;
     constexpr uint32_t TB = T * 8;  // bytes of one poly's tile
     constexpr uint32_t PB = 2 * TB; // bytes of one source (c0, c1)
@@ -481,9 +489,9 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     };
     uint32_t stage_phase = 0;  // bit r: phase of region r's copy barrier
 
-    // the tile's inputs in region `reg`, once this thread's copies have
-    // landed: narrow plans rewrite them in split form, each thread the words
-    // it copied; and the tile's limb constants
+    // the tile's inputs in region `reg`, once the copies have landed (with
+    // cp.async each thread rewrites the words it copied); and the tile's
+    // limb constants
     auto prepare = [&](uint32_t t, uint32_t reg) {
         if (threadIdx.x == 0) s_limb[reg] = a.limbs[a.limb0 + t / a.tiles_per_limb];
         if (!a.n_in) return;
@@ -493,7 +501,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         } else {
             cp_async_wait<0>();  // this thread's copies; the barrier after publishes everyone's
         }
-        if (NARROW) {
+        if (SPLIT) {
             for (uint32_t i = threadIdx.x; i < n_chunks; i += blockDim.x) {
                 ulonglong2 *p = reinterpret_cast<ulonglong2 *>(sm + src0 + reg * a.src_bytes + i * 16);
                 const ulonglong2 x = *p;
@@ -541,11 +549,13 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         for (uint32_t lev = 0; lev < a.n_levels; ++lev) {
             for (uint32_t x = sw[a.o_level + lev] + warp; x < sw[a.o_level + lev + 1]; x += n_warps) {
                 V<C> u0, u1;
-                signed_sum<NARROW, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, u0, u1);
+                signed_sum<SPLIT, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, u0, u1);
+                if constexpr (SPLIT) {  // stored in the sources' form
 #pragma unroll
-                for (int x2 = 0; x2 < C; ++x2) {
-                    u0.x[x2] = A::operand(u0.x[x2]);
-                    u1.x[x2] = A::operand(u1.x[x2]);
+                    for (int x2 = 0; x2 < C; ++x2) {
+                        u0.x[x2] = A::operand(u0.x[x2]);
+                        u1.x[x2] = A::operand(u1.x[x2]);
+                    }
                 }
                 const uint32_t dst = src + (a.n_in + x) * PB;
                 sts<C>(sm, dst, u0);
@@ -607,7 +617,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
             V<C> g0, g1;  // the signed sum of this batch's SEG (operand form)
             const bool seg = first & kOpSeg;
             if (seg) {
-                sp = signed_sum<NARROW, C, TB>(sm, src, sp, lim, g0, g1);
+                sp = signed_sum<SPLIT, C, TB>(sm, src, sp, lim, g0, g1);
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
                     g0.x[x] = A::operand(g0.x[x]);
@@ -625,6 +635,13 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
                     const uint32_t so = src + (op & (kOpMaxSources - 1)) * PB;
                     s0 = lds<C>(sm, so);
                     s1 = lds<C>(sm, so + TB);
+                    if constexpr (NARROW && !SPLIT) {  // canonical sources: the product's form here
+#pragma unroll
+                        for (int x = 0; x < C; ++x) {
+                            s0.x[x] = A::operand(s0.x[x]);
+                            s1.x[x] = A::operand(s1.x[x]);
+                        }
+                    }
                 }
 #pragma unroll
                 for (int x = 0; x < C; ++x) {

@@ -173,6 +173,37 @@ def test_edge_plans():
             assert np.array_equal(dl.outputs(), want), (i, kernel)
 
 
+
+@pytest.mark.parametrize("n_in", [1, 200, 259])
+def test_tma_input_boxes(n_in, monkeypatch):
+    """One coefficient per lane stages a tile's 2 n_in input polys with TMA
+    boxes of at most 256 polys: one box (2 polys), two (400 polys, 200 each)
+    and three whose last one overlaps the second (518 polys: boxes of 173 at
+    0, 173 and 345)."""
+    monkeypatch.setenv("FIONA_TILED_SHAPE", "1,4,0")
+    rng = np.random.default_rng(n_in)
+    n_out = 3
+    r = np.zeros((n_out, n_in), F.ROUTE_DTYPE)
+    n_raw = 0
+    for j in range(n_out):
+        for i in range(n_in):
+            if rng.random() < 0.3:
+                r[j, i] = (W.TERM_RAW, 0, 0, n_out + n_raw)
+                n_raw += 1
+            else:
+                r[j, i] = (W.TERM_TERNARY, int(rng.choice([-1, 0, 1])), 0, j)
+    desc = F.compile_plan(n_in, n_out, n_out + n_raw, r, share=False)
+    qs = W.ntt_primes(1024, 50, 2)
+    wl = W.Workload("boxes%d" % n_in, 1024, qs, desc, 4200 + n_in)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel("tiled")
+    assert dl.plan.stats()["tile_coeffs"] == 32
+    want = oracle.linear_eval(desc, qs, dl.X, dl.P)
+    dl.d_out.fill_(-1)
+    dl.run()
+    assert np.array_equal(dl.outputs(), want)
+    assert dl.ctx.device_check() == F.FIONA_OK
+
 def test_boundary_residues():
     """Residues 0, 1, q-1 and random, on 60-bit primes (widest accepted)."""
     qs = W.ntt_primes(1024, 60, 2)
