@@ -26,6 +26,15 @@ extern "C" {
 int fiona_workload_fill(void *cuda_stream, uint64_t *dst, uint64_t outer, uint32_t L, uint32_t N,
                         const uint64_t *moduli, uint64_t key, int mode);
 
+/* Measured integer-multiply roof of the current device: product-accumulates
+ * per second over the whole GPU of the layer kernels' own primitives, one
+ * 50-bit x 50-bit product each -- narrow: three 32x32 -> 64-bit products of
+ * radix-2^26 halves (Karatsuba), the arithmetic of every plan whose moduli
+ * are below 2^52; wide: the 64x64 -> 128-bit product-accumulate.  Runs a few
+ * milliseconds of kernels on the default stream and synchronizes.
+ * Returns 0, or -1 on a null argument, -5 on a CUDA error. */
+int fiona_mul_roof(double *narrow_per_s, double *wide_per_s);
+
 #ifdef __cplusplus
 }
 #endif

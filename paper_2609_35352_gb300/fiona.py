@@ -351,6 +351,8 @@ def workload_lib() -> ctypes.CDLL:
                                           ctypes.c_uint32, ctypes.c_uint32, ctypes.c_void_p,
                                           ctypes.c_uint64, ctypes.c_int]
         W.fiona_workload_fill.restype = ctypes.c_int
+        W.fiona_mul_roof.argtypes = [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
+        W.fiona_mul_roof.restype = ctypes.c_int
         _wlib = W
     return _wlib
 
@@ -362,6 +364,17 @@ def device_fill(dst, outer: int, L: int, N: int, moduli, key: int, mode: int = 0
                                             q.ctypes.data, key, mode)
     if rc != 0:
         raise RuntimeError("fiona_workload_fill failed (%d)" % rc)
+
+
+def mul_roof() -> Dict[str, float]:
+    """fiona_mul_roof: the measured products per second of the narrow
+    (radix-2^26 Karatsuba) and wide (64x64 -> 128) product-accumulates on the
+    current device."""
+    n, w = ctypes.c_double(), ctypes.c_double()
+    rc = workload_lib().fiona_mul_roof(ctypes.byref(n), ctypes.byref(w))
+    if rc != 0:
+        raise RuntimeError("fiona_mul_roof failed (%d)" % rc)
+    return {"narrow": n.value, "wide": w.value}
 
 
 # -- host plan compiler -------------------------------------------------------

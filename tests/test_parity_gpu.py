@@ -335,3 +335,12 @@ def test_check_residues_detects_out_of_range():
     X[3, 1, 2, 77] = wl.moduli[2]  # residue == q
     dl.d_in.copy_(to_device(X))
     assert dl.ctx.check_residues(dl.d_in, 2 * wl.plan.n_in) == F.FIONA_ERR_RANGE
+
+
+def test_mul_roof_measures_the_product_rate():
+    """fiona_mul_roof returns the whole GPU's product-accumulate rates: both
+    positive, within a plausible range for 152 SMs, and the radix-2^26
+    Karatsuba form (three 32-bit products) faster than the 64x64 -> 128 one
+    (four and a carry chain)."""
+    r = F.mul_roof()
+    assert 1e11 < r["wide"] < r["narrow"] < 1e14
