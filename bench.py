@@ -148,16 +148,29 @@ class ClockSampler:
         self.device = device
         self.proc = None
         self.file = None
+        self.skip = 0
 
     def start(self):
+        """Start sampling every 50 ms and return once the first sample is in
+        (at most 3 s): the samples that stop() keeps are those taken after
+        start() returned, i.e. during the timed region."""
         try:
             self.file = tempfile.TemporaryFile(mode="w+")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.device), "--query-gpu=" + self.FIELDS,
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=self.file, stderr=subprocess.DEVNULL)
         except (OSError, ValueError):
             self.proc = None
+            return
+        deadline = time.time() + 3.0
+        while time.time() < deadline and self.proc.poll() is None:
+            self.file.seek(0)
+            lines = self.file.read().splitlines()
+            if lines:
+                self.skip = len(lines)
+                break
+            time.sleep(0.01)
 
     def stop(self) -> dict:
         if self.proc is None:
@@ -173,7 +186,7 @@ class ClockSampler:
         reasons = set()
         names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
                  "sw_power_cap"]
-        for line in self.file.read().splitlines():
+        for line in self.file.read().splitlines()[self.skip:]:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) < 9:
                 continue
@@ -284,8 +297,10 @@ def run_reference(args, rank: int, world: int) -> None:
         return
     cores = host_cores()
     wl = W.make_workload(args.workload)
-    # sized so that warmup + steps stay within about two minutes
-    budget = max(0.5, min(5.0, 120.0 / max(1, args.steps + args.warmup)))
+    # sized so that warmup + steps stay within about two minutes (the
+    # worker-side time of each step is what is measured; at least one
+    # position per core)
+    budget = max(0.02, min(5.0, 120.0 / max(1, args.steps + args.warmup)))
     smp = OracleSampler(args.workload, cores, budget)
     for _ in range(args.warmup):
         smp.step()
@@ -725,7 +740,7 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(WORKLOAD_TEXT))
