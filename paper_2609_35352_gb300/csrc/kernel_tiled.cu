@@ -20,9 +20,9 @@
 //  2. The materialised shared signed sums (Sec. 4.2 "Sharing Signed Sums")
 //     are formed once per tile, level by level, into the same region.
 //  3. Each warp runs its operation stream (tiled.h): per scale group a
-//     signed sum over sources, its additions spread over the operations
-//     before the group's product, then one product by gamma (Sec. 4.2
-//     "Grouping Reconstruction Operations"); per raw term a PMult-MAC of a
+//     signed sum over sources, formed before the batch its product opens,
+//     then one product by gamma (Sec. 4.2 "Grouping Reconstruction
+//     Operations"); per raw term a PMult-MAC of a
 //     plaintext tile and a source.  Plaintext tiles go from HBM straight to
 //     registers: each warp keeps the next P (16, 8 or 4) of its stream in
 //     flight, across job and tile boundaries, in a register queue indexed at
@@ -31,8 +31,13 @@
 //     signed and raw routes are added before the single final reduction
 //     (Sec. 4.2 "Combining the Signed and Raw Routes").
 //  4. Outputs split across warps add their reduced partial sums.
-// The only spin-wait is thread 0's bounded wait for the schedule copy; if it
-// gives up, the CTA raises the context's error flag and stops.
+//  5. The next tile's inputs are prepared (with two regions: their copies,
+//     started at the top of this tile, waited for and rewritten) before the
+//     one barrier per tile that publishes them.
+// The spin-waits are bounded: thread 0's wait for the schedule copy (if it
+// gives up, the CTA raises the context's error flag and stops) and each
+// thread's wait for a region's TMA copies (if it gives up, the flag is
+// raised and the tile computed from whatever the region holds).
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
