@@ -344,3 +344,21 @@ def test_mul_roof_measures_the_product_rate():
     (four and a carry chain)."""
     r = F.mul_roof()
     assert 1e11 < r["wide"] < r["narrow"] < 1e14
+
+
+@pytest.mark.parametrize("bits,L", [(50, 3), (59, 2)])
+def test_largest_ring_dimension(bits, L):
+    """The tiny layer (8 inputs, 4 outputs, signed, raw and DAG-free) at the
+    largest ring dimension the context accepts, N = 2^17, on both kernels,
+    narrow (50-bit) and wide (59-bit) arithmetic: element by element."""
+    N = 1 << 17
+    qs = W.ntt_primes(N, bits, L)
+    base = W.make_workload("tiny")
+    wl = W.Workload("tiny-2^17", N, qs, base.plan, base.seed + bits)
+    dl = DeviceLayer(wl)
+    want = oracle.linear_eval(base.plan, qs, dl.X, dl.P)
+    for kernel in ("direct", "tiled"):
+        dl.plan.select_kernel(kernel)
+        dl.d_out.fill_(-1)
+        dl.run()
+        assert np.array_equal(dl.outputs(), want), kernel
