@@ -21,7 +21,7 @@
 namespace {
 
 constexpr int kChains = 4;
-constexpr int kSteps = 2048;
+constexpr int kSteps = 256;
 
 template <bool NARROW>
 __global__ void __launch_bounds__(256) roof_kernel(const uint64_t *seed, uint64_t *sink)
@@ -59,7 +59,7 @@ double rate(int sms, const uint64_t *seed, uint64_t *sink)
     cudaEvent_t e0, e1;
     cudaEventCreate(&e0);
     cudaEventCreate(&e1);
-    const int reps = 5;
+    const int reps = 3;
     cudaEventRecord(e0);
     for (int r = 0; r < reps; ++r) roof_kernel<NARROW><<<grid, block>>>(seed, sink);
     cudaEventRecord(e1);
