@@ -414,14 +414,17 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
                 "kernel_ms_median": statistics.median(kernel_ms)}
     # the secondary roof: 50-bit x 50-bit products against the measured rate
     # of the same product-accumulate (fiona_mul_roof), outside the timed region
-    roof = F.mul_roof()
     narrow = max(wl.moduli) < (1 << 52)
-    mul_peak = roof["narrow" if narrow else "wide"]
     mul_achieved = stats["wide_products"] / avg_kernel_s
+    try:
+        mul_peak = F.mul_roof()["narrow" if narrow else "wide"]
+    except RuntimeError as e:  # the line keeps its HBM figures without it
+        mul_peak, why = None, str(e)
     alu = {"bound": "alu", "unit": "products/s", "achieved": mul_achieved, "peak": mul_peak,
-           "frac": mul_achieved / mul_peak,
-           "peak_kind": "measured (fiona_mul_roof: the %s product-accumulate on every SM)"
-                        % ("radix-2^26 Karatsuba" if narrow else "64x64->128"),
+           "frac": mul_achieved / mul_peak if mul_peak else None,
+           "peak_kind": ("measured (fiona_mul_roof: the %s product-accumulate on every SM)"
+                         % ("radix-2^26 Karatsuba" if narrow else "64x64->128")) if mul_peak else
+                        "unavailable: " + why,
            "products_per_launch": stats["wide_products"]}
 
     # end to end: host inputs -> result on the host, plaintexts resident
