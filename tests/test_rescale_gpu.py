@@ -209,13 +209,19 @@ def test_eval_rescale_rounding():
                           oracle.rescale(wl.moduli, layer, round=True))
 
 
-def test_layer_and_rescale_replay_in_a_cuda_graph():
+@pytest.mark.parametrize("shape,tile", [(None, 64), ("1,8,1", 32)])
+def test_layer_and_rescale_replay_in_a_cuda_graph(shape, tile, monkeypatch):
     """After a first call (which builds the tables), a layer followed by its
     rescale is stream-ordered launches only: it captures into a CUDA graph and
-    every replay gives the oracle's residues."""
+    every replay gives the oracle's residues -- with input tiles staged by
+    cp.async (two coefficients per lane) and by TMA tensor copies, whose
+    tensor map is a kernel parameter captured with the launch (one)."""
+    if shape:
+        monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
     wl = W.make_workload("vit", N=2048, L=3)
     ctx = F.Context(wl.N, wl.moduli, device=0)
     plan = F.Plan(ctx, wl.plan)
+    assert plan.stats()["tile_coeffs"] == tile
     p = wl.plan
     X, P = wl.host_inputs(), wl.host_plaintexts()
     d_in, d_pt = to_device(X), to_device(P)
