@@ -49,7 +49,7 @@ def random_layer(rng):
     return F.compile_plan(n_in, n_out, n_gamma * n_out + n_raw, r, share=bool(rng.integers(4)), exact=exact)
 
 
-@pytest.mark.parametrize("seed", range(12))
+@pytest.mark.parametrize("seed", range(40))
 def test_random_layers(seed, monkeypatch):
     rng = np.random.default_rng(1000 + seed)
     shape = SHAPES[seed % len(SHAPES)]
@@ -78,7 +78,7 @@ def test_random_layers(seed, monkeypatch):
     assert dl.ctx.device_check() == F.FIONA_OK
 
 
-@pytest.mark.parametrize("seed", range(8))
+@pytest.mark.parametrize("seed", range(16))
 def test_random_rescales(seed):
     rng = np.random.default_rng(2000 + seed)
     N = int(rng.choice([1024, 2048, 4096, 16384]))
