@@ -370,6 +370,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
 {
     using A = Arith<NARROW>;
     using Acc = typename A::Acc;
+    static_assert(P % 4 == 0, "operation words are read four at a time");
     constexpr bool TMA = C == 1;  // input tiles by TMA tensor copies
     // narrow sources in shared memory: split form (rewritten once per tile)
     // with two coefficients per lane; canonical, split where a product reads
@@ -629,9 +630,19 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
                     g1.x[x] = A::operand(g1.x[x]);
                 }
             }
+            // this batch's and the next batch's operation words, four at a
+            // time with 16-byte loads (every stream and batch starts on a
+            // 16-byte boundary)
+            uint4 cw4, nw4;
 #pragma unroll
             for (uint32_t i = 0; i < P; ++i) {
-                const uint32_t op = i == 0 ? first : op_word(cur_off + 4 * i);
+                if (i % 4 == 0) {
+                    cw4 = *reinterpret_cast<const uint4 *>(sm + cur_off + 4 * i);
+                    nw4 = *reinterpret_cast<const uint4 *>(sm + next_off + 4 * i);
+                }
+                const uint32_t cwi = i % 4 == 0 ? cw4.x : i % 4 == 1 ? cw4.y : i % 4 == 2 ? cw4.z : cw4.w;
+                const uint32_t nwi = i % 4 == 0 ? nw4.x : i % 4 == 1 ? nw4.y : i % 4 == 2 ? nw4.z : nw4.w;
+                const uint32_t op = i == 0 ? first : cwi;
                 V<C> s0, s1;
                 if (i == 0 && seg) {
                     s0 = g0;
@@ -655,9 +666,9 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
                     A::mac(acc[0][x], g, s0.x[x]);
                     A::mac(acc[1][x], g, s1.x[x]);
                 }
-                r[i] = fetch(nb, nlb, ns, op_word(next_off + 4 * i));
+                r[i] = fetch(nb, nlb, ns, nwi);
             }
-            if (op_word(cur_off + 4 * (P - 1)) & kOpLast) finish();
+            if (cw4.w & kOpLast) finish();  // the batch's last word
         }
         cur_ptl = next_ptl;
         cur_lb = next_lb;
