@@ -50,7 +50,7 @@ from paper_2609_35352_gb300 import workloads as W  # noqa: E402
 
 METRIC = "hybrid linear layer ciphertext-terms/s and HBM GB/s (% of GB300 peak), N=2^16"
 UNIT = "ciphertext-terms/s"
-DEFAULT_WORKLOAD = "wsum-hybrid"
+DEFAULT_WORKLOAD = "bert"
 WORKLOAD_TEXT = {
     "wsum-pmult": "64-ciphertext weighted sum -> 1 output, all PMult",
     "wsum-ternary": "64-ciphertext weighted sum -> 1 output, all ternary (one scale PMult)",
@@ -61,29 +61,54 @@ WORKLOAD_TEXT = {
     "bert-const": "the bert layer with every raw weight broadcast to all slots (constant raw plaintexts)",
 }
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0  # GB300 HBM3e, the ~8 TB/s the target is stated against
 
 
 # ----------------------------------------------------------------------------
 # CPU oracle on a sample (spawned workers; never forked after CUDA init)
 # ----------------------------------------------------------------------------
-def _oracle_worker(task):
-    name, limb, coefs = task
+_WORKER_BYTES = 32 << 20  # bound on the sampled residues one worker holds
+
+
+def _oracle_time(state) -> float:
     import oracle
+    p, q, X, P = state
+    t0 = time.perf_counter()
+    oracle.linear_eval(p, q, X, P)
+    return time.perf_counter() - t0
+
+
+def _oracle_state(name: str, limb: int, coefs: list):
+    """The residues of one limb and some coefficients of a workload: every
+    input (both polys) and every plaintext."""
     wl = W.make_workload(name)
     p = wl.plan
     k = np.asarray(coefs, dtype=np.uint64)
     X = wl.input_values(np.arange(p.n_in).reshape(-1, 1, 1), np.arange(2).reshape(1, -1, 1),
                         limb, k.reshape(1, 1, -1)).reshape(p.n_in, 2, 1, -1)
     P = wl.plaintext_values(np.arange(p.n_pt).reshape(-1, 1), limb, k.reshape(1, -1))
-    P = P.reshape(p.n_pt, 1, -1)
-    t0 = time.perf_counter()
-    oracle.linear_eval(p, [wl.moduli[limb]], X, P)
-    return time.perf_counter() - t0, len(coefs)
+    return p, [wl.moduli[limb]], X, P.reshape(p.n_pt, 1, -1)
+
+
+def _oracle_worker(conn, name, limb, coefs):
+    """One spawned process with a fixed task: it generates its positions'
+    residues once (untimed), then times the oracle on them each time it is
+    asked, until it receives None."""
+    import oracle
+    oracle.build()
+    state = _oracle_state(name, limb, coefs)
+    conn.send(("ready", len(coefs)))
+    while conn.recv() is not None:
+        conn.send((_oracle_time(state), len(coefs)))
+    conn.close()
 
 
 class OracleSampler:
-    """Runs the oracle over `positions` sampled (limb, coefficient) positions
-    per step, split over `cores` spawned processes."""
+    """Runs the oracle over sampled (limb, coefficient) positions of a layer
+    on `cores` spawned processes, each with its own fixed positions (the same
+    every step; their residues generated once, untimed).  The sample is sized
+    to about `budget_s` seconds of oracle time per process and step, and to at
+    most _WORKER_BYTES of residues per process."""
 
     def __init__(self, name: str, cores: int, budget_s: float):
         import oracle
@@ -91,33 +116,34 @@ class OracleSampler:
         self.name = name
         self.wl = W.make_workload(name)
         self.cores = cores
-        self.pool = mp.get_context("spawn").Pool(cores)
-        # calibrate: one worker, a few positions
-        dt, n = self.pool.apply(_oracle_worker, ((name, 0, list(range(8))),))
-        per_pos = dt / n
-        total = int(budget_s * cores / per_pos)
-        full = self.wl.L * self.wl.N
-        self.positions = max(cores, min(total, full))
-        self.per_core = max(1, self.positions // cores)
+        # calibrate here (not timed in the line): a few positions, one process
+        state = _oracle_state(name, 0, list(range(8)))
+        _oracle_time(state)
+        per_pos = max(_oracle_time(state) / 8, 1e-7)
+        p = self.wl.plan
+        values_per_pos = 2 * p.n_in + p.n_pt
+        per_core = min(int(budget_s / per_pos), _WORKER_BYTES // (8 * values_per_pos), self.wl.N)
+        self.per_core = max(1, per_core)
         self.positions = self.per_core * cores
-        self.step_no = 0
-
-    def tasks(self):
+        ctx = mp.get_context("spawn")
+        self.procs, self.conns = [], []
         wl = self.wl
-        out = []
-        base = self.step_no * self.positions
-        for c in range(self.cores):
-            start = (base + c * self.per_core) % (wl.L * wl.N)
-            flat = (start + np.arange(self.per_core)) % (wl.L * wl.N)
-            limb = int(flat[0] // wl.N)
-            # keep each task inside one limb
-            coefs = [int(x % wl.N) for x in flat if int(x // wl.N) == limb]
-            out.append((self.name, limb, coefs))
-        self.step_no += 1
-        return out
+        for c in range(cores):
+            limb = c % wl.L
+            start = ((c // wl.L) * self.per_core) % max(1, wl.N - self.per_core + 1)
+            a, b = ctx.Pipe()
+            pr = ctx.Process(target=_oracle_worker,
+                             args=(b, name, limb, list(range(start, start + self.per_core))), daemon=True)
+            pr.start()
+            self.procs.append(pr)
+            self.conns.append(a)
+        for a in self.conns:
+            a.recv()  # ready
 
     def step(self):
-        res = self.pool.map(_oracle_worker, self.tasks())
+        for a in self.conns:
+            a.send(1)
+        res = [a.recv() for a in self.conns]
         wall = max(r[0] for r in res)
         pos = sum(r[1] for r in res)
         return wall, pos
@@ -128,82 +154,167 @@ class OracleSampler:
 
     def sample_text(self, pos: int) -> str:
         return ("oracle on %d sampled (limb, coefficient) positions of %d per step "
-                "(all outputs, both polys), %d spawned processes; terms/s scaled by the "
-                "sampled fraction" % (pos, self.wl.L * self.wl.N, self.cores))
+                "(all outputs, both polys), %d spawned processes, the slowest one's time; "
+                "terms/s scaled by the sampled fraction" % (pos, self.wl.L * self.wl.N, self.cores))
 
     def close(self):
-        self.pool.terminate()
-        self.pool.join()
+        for a in self.conns:
+            try:
+                a.send(None)
+            except OSError:
+                pass
+        for pr in self.procs:
+            pr.join(timeout=5)
+            if pr.is_alive():
+                pr.terminate()
 
 
 # ----------------------------------------------------------------------------
 # clocks during the timed region
 # ----------------------------------------------------------------------------
+# NVML clock-event reason bits (nvml.h)
+_NVML_REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+                 0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+
+class _Nvml:
+    """Read-only NVML queries through ctypes (the driver's libnvidia-ml):
+    SM clock, its maximum, power draw and the active clock-event reasons of
+    one device.  Raises OSError when NVML cannot be used."""
+
+    def __init__(self, device: int):
+        import ctypes
+        self.ct = ctypes
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        self.lib = lib
+        self.h = ctypes.c_void_p()
+        ok = False
+        try:  # the CUDA device's own identity (CUDA and NVML orders may differ)
+            import torch
+            props = torch.cuda.get_device_properties(device)
+            uuid = getattr(props, "uuid", None)
+            if uuid is not None:
+                u = str(uuid)
+                u = u if u.startswith("GPU-") else "GPU-" + u
+                ok = lib.nvmlDeviceGetHandleByUUID(u.encode(), ctypes.byref(self.h)) == 0
+            if not ok and hasattr(props, "pci_bus_id"):
+                bus = "%08x:%02x:%02x.0" % (props.pci_domain_id, props.pci_bus_id, props.pci_device_id)
+                ok = lib.nvmlDeviceGetHandleByPciBusId_v2(bus.encode(), ctypes.byref(self.h)) == 0
+        except Exception:  # noqa: BLE001 - fall back to the index
+            ok = False
+        if not ok and lib.nvmlDeviceGetHandleByIndex_v2(device, ctypes.byref(self.h)) != 0:
+            raise OSError("no NVML handle for device %d" % device)
+        self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            lib.nvmlDeviceGetCurrentClocksThrottleReasons
+
+    def sample(self):
+        ct = self.ct
+        sm, smax, mw = ct.c_uint(), ct.c_uint(), ct.c_uint()
+        bits = ct.c_ulonglong()
+        if self.lib.nvmlDeviceGetClockInfo(self.h, 1, ct.byref(sm)) != 0:  # NVML_CLOCK_SM
+            return None
+        self.lib.nvmlDeviceGetMaxClockInfo(self.h, 1, ct.byref(smax))
+        if self.lib.nvmlDeviceGetPowerUsage(self.h, ct.byref(mw)) != 0:
+            mw.value = 0
+        if self.reasons_fn(self.h, ct.byref(bits)) != 0:
+            bits.value = 0
+        return float(sm.value), float(smax.value), mw.value / 1000.0, int(bits.value)
+
+
 class ClockSampler:
+    """SM clock, power and throttle reasons of one GPU while the timed region
+    runs.  NVML is polled every 2 ms from a thread, and once synchronously at
+    start() and at mark_end() (both inside the timed region, the GPU busy with
+    queued work), so that even a region of a few milliseconds has samples.
+    Without NVML, nvidia-smi samples every 20 ms instead."""
+
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, device: int):
         self.device = device
+        self.samples = []  # (sm_mhz, max_mhz, watts, reason names)
+        self.nvml = None
+        self.thread = None
+        self.stop_flag = False
         self.proc = None
         self.file = None
         self.skip = 0
+        self.source = "nvml"
+        try:
+            self.nvml = _Nvml(device)
+        except (OSError, AttributeError):
+            self.nvml = None
+            self.source = "nvidia-smi"
+
+    def _take(self):
+        s = self.nvml.sample()
+        if s is not None:
+            names = [n for b, n in _NVML_REASONS.items() if s[3] & b]
+            self.samples.append((s[0], s[1], s[2], names))
+
+    def _loop(self):
+        while not self.stop_flag:
+            self._take()
+            time.sleep(0.002)
 
     def start(self):
-        """Start sampling every 50 ms and return once the first sample is in
-        (at most 3 s): the samples that stop() keeps are those taken after
-        start() returned, i.e. during the timed region."""
+        """Call right after the timed region's first launch is queued."""
+        if self.nvml is not None:
+            import threading
+            self._take()
+            self.thread = threading.Thread(target=self._loop, daemon=True)
+            self.thread.start()
+            return
         try:
             self.file = tempfile.TemporaryFile(mode="w+")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.device), "--query-gpu=" + self.FIELDS,
-                 "--format=csv,noheader,nounits", "-lms", "50"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=self.file, stderr=subprocess.DEVNULL)
         except (OSError, ValueError):
             self.proc = None
-            return
-        deadline = time.time() + 3.0
-        while time.time() < deadline and self.proc.poll() is None:
-            self.file.seek(0)
-            lines = self.file.read().splitlines()
-            if lines:
-                self.skip = len(lines)
-                break
-            time.sleep(0.01)
+
+    def mark_end(self):
+        """Call after the last launch is queued, before the final synchronize."""
+        if self.nvml is not None:
+            self._take()
 
     def stop(self) -> dict:
-        if self.proc is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"],
-                    "samples": 0}
-        self.proc.terminate()
-        try:
-            self.proc.wait(timeout=5)
-        except subprocess.TimeoutExpired:
-            self.proc.kill()
-        self.file.seek(0)
-        sm, smax, power = [], [], []
-        reasons = set()
-        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
-                 "sw_power_cap"]
-        for line in self.file.read().splitlines()[self.skip:]:
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 9:
-                continue
+        if self.nvml is not None:
+            self.stop_flag = True
+            if self.thread is not None:
+                self.thread.join(timeout=2)
+        elif self.proc is not None:
+            self.proc.terminate()
             try:
-                sm.append(float(parts[1]))
-                smax.append(float(parts[2]))
-                power.append(float(parts[3]))
-            except ValueError:
-                continue
-            for n, v in zip(names[1:], parts[5:9]):
-                if v.lower() == "active":
-                    reasons.add(n)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
-                "reasons": sorted(reasons), "samples": len(sm),
-                "power_w_max": max(power)}
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.file.seek(0)
+            names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+            for line in self.file.read().splitlines():
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    vals = float(parts[1]), float(parts[2]), float(parts[3])
+                except ValueError:
+                    continue
+                self.samples.append(vals + ([n for n, v in zip(names, parts[5:9]) if v.lower() == "active"],))
+        else:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no clock source (NVML, nvidia-smi)"],
+                    "samples": 0, "source": None}
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "source": self.source}
+        sm = [x[0] for x in self.samples]
+        reasons = sorted(set(r for x in self.samples for r in x[3]))
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(x[1] for x in self.samples),
+                "sm_mhz_min": min(sm), "reasons": reasons, "samples": len(sm),
+                "power_w_max": max(x[2] for x in self.samples), "source": self.source}
 
 
 # ----------------------------------------------------------------------------
@@ -246,16 +357,19 @@ def profiled_traffic(workload: str, kernel: str):
     return ent.get("dram_bytes_per_launch")
 
 
-def workload_config(wl: W.Workload, name: str, stats: dict) -> dict:
+def workload_config(wl: W.Workload, name: str) -> dict:
+    """The workload, from the plan description alone: both arms print the
+    same dict for the same layer."""
+    c = wl.plan.counts()
+    bytes_min = W.min_bytes(wl.plan, wl.L, wl.N)
     return {
         "workload": "%s (%s): N=2^%d, L=%d RNS limbs of %d-bit primes, %d inputs -> %d outputs"
                     % (name, WORKLOAD_TEXT.get(name, name), wl.N.bit_length() - 1, wl.L,
                        max(wl.moduli).bit_length(), wl.plan.n_in, wl.plan.n_out),
         "N": wl.N, "L": wl.L, "n_in": wl.plan.n_in, "n_out": wl.plan.n_out,
-        "nonzero_terms": stats["n_nonzero_terms"], "raw_terms": stats["n_raw_terms"],
-        "signed_terms": stats["n_signed_terms"], "shared_sums": stats["n_nodes"],
-        "bytes_min_per_step": stats["bytes_min"],
-        "l2": "inputs larger than L2 (%.2f GB read per step, L2 129 MB)" % (stats["bytes_min"] / 1e9),
+        "nonzero_terms": c["nonzero"], "raw_terms": c["raw"], "signed_terms": c["plus"] + c["minus"],
+        "shared_sums": wl.plan.n_nodes, "bytes_min_per_step": bytes_min,
+        "l2": "inputs larger than L2 (%.2f GB read per step, L2 129 MB)" % (bytes_min / 1e9),
     }
 
 
@@ -313,13 +427,7 @@ def run_reference(args, rank: int, world: int) -> None:
     wall = sum(walls)
     frac = sum(poss) / (wl.L * wl.N)
     value = frac * wl.plan.counts()["nonzero"] / wall
-    stats = {"n_nonzero_terms": wl.plan.counts()["nonzero"], "n_raw_terms": wl.plan.counts()["raw"],
-             "n_signed_terms": wl.plan.counts()["plus"] + wl.plan.counts()["minus"],
-             "n_nodes": wl.plan.n_nodes,
-             "bytes_min_per_step": None,
-             "bytes_min": 0}
-    cfg = workload_config(wl, args.workload, stats)
-    cfg.pop("l2")
+    cfg = workload_config(wl, args.workload)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup,
@@ -352,9 +460,13 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     if rank == 0 and world == 1 and not args.no_cpu and args.limbs is None:
         cores = host_cores()
         smp = OracleSampler(name, cores, args.cpu_budget)
-        w, pos = smp.step()
-        cpu = {"value": smp.throughput(w, pos), "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": smp.sample_text(pos)}
+        walls, poss = [], []
+        while not walls or sum(walls) < args.cpu_budget:  # about cpu_budget s on every core
+            w, pos = smp.step()
+            walls.append(w)
+            poss.append(pos)
+        cpu = {"value": smp.throughput(sum(walls), sum(poss)), "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": smp.sample_text(poss[0]) + ", %d steps" % len(walls)}
         smp.close()
 
     ctx = F.Context(wl.N, wl.moduli, device=dev)
@@ -382,7 +494,6 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     clocks = ClockSampler(dev)
     barrier()
     torch.cuda.synchronize()
-    clocks.start()
     t_begin = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_begin.record(stream)
@@ -390,7 +501,10 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
         starts[s].record(stream)
         plan.eval(d_in, d_pt, d_out, stream=stream)
         stops[s].record(stream)
+        if s == 0:
+            clocks.start()
     t_end.record(stream)
+    clocks.mark_end()
     torch.cuda.synchronize()
     barrier()
     clk = clocks.stop()
@@ -407,6 +521,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     kernel = "tiled" if stats["kernel"] == 2 else "direct"
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak,
+                "peak_nominal": NOMINAL_HBM_GBS, "frac_nominal": achieved / NOMINAL_HBM_GBS,
                 "traffic": profiled_traffic(name, kernel) if args.limbs is None else None,
                 "kernel": kernel,
                 "peak_kind": peak_kind,
@@ -447,12 +562,10 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
                "ms_per_step": 1e3 * dt / e2e_steps, "steps": e2e_steps}
 
     if rank == 0:
-        cfg = workload_config(wl, name, stats)
-        cfg["parallelism"] = "replicas x%d (independent layer per GPU)" % world
-        cfg["kernel"] = kernel
-        cfg["tile_coeffs"] = stats["tile_coeffs"]
-        cfg["warps_per_cta"] = stats["warps_per_cta"]
-        cfg["ctas_per_sm"] = stats["ctas_per_sm"]
+        cfg = workload_config(wl, name)
+        if cfg["bytes_min_per_step"] != stats["bytes_min"]:
+            raise RuntimeError("minimal bytes: the library counts %d, the plan description %d"
+                               % (stats["bytes_min"], cfg["bytes_min_per_step"]))
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
@@ -462,6 +575,11 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
             "hbm_gbs": achieved, "hbm_frac": achieved / peak,
             "roofline": roofline, "alu": alu, "cpu_baseline": cpu, "e2e": e2e,
             "clocks": clk, "gpu_launches": args.steps,
+            "parallelism": "replicas x%d (independent layer per GPU)" % world,
+            "kernel": {"name": kernel, "tile_coeffs": stats["tile_coeffs"],
+                       "warps_per_cta": stats["warps_per_cta"], "ctas_per_sm": stats["ctas_per_sm"],
+                       "shared_sums_formed": stats["nodes_materialized"],
+                       "addsub_executed": stats.get("addsub_executed")},
         }
         print(json.dumps(line), flush=True)
     plan.close()
@@ -537,11 +655,13 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
     clocks = ClockSampler(dev)
     barrier()
     torch.cuda.synchronize()
-    clocks.start()
     for s in range(args.steps):
         starts[s].record(stream)
         ctx.rescale(L, count, d_y, d_o, stream=stream)
         stops[s].record(stream)
+        if s == 0:
+            clocks.start()
+    clocks.mark_end()
     torch.cuda.synchronize()
     barrier()
     clk = clocks.stop()
@@ -670,13 +790,15 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
     clocks = ClockSampler(dev)
     barrier()
     torch.cuda.synchronize()
-    clocks.start()
-    for a, b, c in ev:
+    for i, (a, b, c) in enumerate(ev):
         a.record(stream)
         ctx.ckks_embed(count, d_slots, scale, d_c, d_w, stream=stream)
         b.record(stream)
         ctx.encode_coeffs(L, count, d_c, d_o, stream=stream)
         c.record(stream)
+        if i == 0:
+            clocks.start()
+    clocks.mark_end()
     torch.cuda.synchronize()
     barrier()
     clk = clocks.stop()

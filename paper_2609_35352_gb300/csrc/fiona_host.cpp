@@ -432,15 +432,22 @@ static int upload(fiona_plan *p, const std::vector<std::pair<const void *, size_
     return FIONA_OK;
 }
 
-static int lower_direct(fiona_plan *p)
-{
-    const HostPlan &hp = p->hp;
-    std::vector<DirOut> outs(hp.n_out);
+// The direct kernel's schedule of a plan: per output its scale-group segments
+// (each a run of signed operations, bit 31 = subtract) and its raw terms
+// (input, plaintext with bit 31 = constant plaintext).
+struct DirectSchedule {
+    std::vector<DirOut> outs;
     std::vector<DirSeg> segs;
     std::vector<uint32_t> ops, raw_in, raw_pt;
+};
+
+static DirectSchedule direct_schedule(const HostPlan &hp)
+{
+    DirectSchedule d;
+    d.outs.resize(hp.n_out);
     for (uint32_t j = 0; j < hp.n_out; ++j) {
-        DirOut &o = outs[j];
-        o.seg_begin = (uint32_t)segs.size();
+        DirOut &o = d.outs[j];
+        o.seg_begin = (uint32_t)d.segs.size();
         std::vector<uint32_t> seen;
         for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
             const fiona_term &t = hp.terms[e];
@@ -449,31 +456,37 @@ static int lower_direct(fiona_plan *p)
             seen.push_back(t.group);
             DirSeg sg{};
             sg.scale_pt = hp.group_scale_pt[t.group];
-            sg.op_begin = (uint32_t)ops.size();
+            sg.op_begin = (uint32_t)d.ops.size();
             for (uint32_t f = e; f < hp.term_offsets[j + 1]; ++f) {
                 const fiona_term &u = hp.terms[f];
                 if (u.kind == FIONA_TERM_TERNARY && u.group == t.group && u.sign != 0)
-                    ops.push_back(u.input | (u.sign < 0 ? 0x80000000u : 0u));
+                    d.ops.push_back(u.input | (u.sign < 0 ? 0x80000000u : 0u));
             }
-            sg.op_end = (uint32_t)ops.size();
-            segs.push_back(sg);
+            sg.op_end = (uint32_t)d.ops.size();
+            d.segs.push_back(sg);
         }
-        o.seg_end = (uint32_t)segs.size();
-        o.raw_begin = (uint32_t)raw_in.size();
+        o.seg_end = (uint32_t)d.segs.size();
+        o.raw_begin = (uint32_t)d.raw_in.size();
         for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
             const fiona_term &t = hp.terms[e];
             if (t.kind != FIONA_TERM_RAW && t.kind != FIONA_TERM_RAW_CONST) continue;
-            raw_in.push_back(t.input);
-            raw_pt.push_back(t.pt | (t.kind == FIONA_TERM_RAW_CONST ? 0x80000000u : 0u));
+            d.raw_in.push_back(t.input);
+            d.raw_pt.push_back(t.pt | (t.kind == FIONA_TERM_RAW_CONST ? 0x80000000u : 0u));
         }
-        o.raw_end = (uint32_t)raw_in.size();
+        o.raw_end = (uint32_t)d.raw_in.size();
     }
+    return d;
+}
+
+static int lower_direct(fiona_plan *p)
+{
+    const DirectSchedule d = direct_schedule(p->hp);
     std::vector<size_t> off;
-    int rc = upload(p, {{outs.data(), outs.size() * sizeof(DirOut)},
-                        {segs.data(), segs.size() * sizeof(DirSeg)},
-                        {ops.data(), ops.size() * 4},
-                        {raw_in.data(), raw_in.size() * 4},
-                        {raw_pt.data(), raw_pt.size() * 4}},
+    int rc = upload(p, {{d.outs.data(), d.outs.size() * sizeof(DirOut)},
+                        {d.segs.data(), d.segs.size() * sizeof(DirSeg)},
+                        {d.ops.data(), d.ops.size() * 4},
+                        {d.raw_in.data(), d.raw_in.size() * 4},
+                        {d.raw_pt.data(), d.raw_pt.size() * 4}},
                     off);
     if (rc) return rc;
     uint8_t *b = (uint8_t *)p->sched.blob;
@@ -486,50 +499,17 @@ static int lower_direct(fiona_plan *p)
 }
 
 // Host image for fiona_linear_eval_static: the limb constants and the direct
-// schedule (same layout as lower_direct's), each part 16-byte aligned.
+// schedule (the same parts as lower_direct's), each part 16-byte aligned.
 static void build_static_image(fiona_plan *p)
 {
-    const HostPlan &hp = p->hp;
-    std::vector<DirOut> outs(hp.n_out);
-    std::vector<DirSeg> segs;
-    std::vector<uint32_t> ops, raw_in, raw_pt;
-    for (uint32_t j = 0; j < hp.n_out; ++j) {
-        DirOut &o = outs[j];
-        o.seg_begin = (uint32_t)segs.size();
-        std::vector<uint32_t> seen;
-        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
-            const fiona_term &t = hp.terms[e];
-            if (t.kind != FIONA_TERM_TERNARY || t.sign == 0) continue;
-            if (std::find(seen.begin(), seen.end(), t.group) != seen.end()) continue;
-            seen.push_back(t.group);
-            DirSeg sg{};
-            sg.scale_pt = hp.group_scale_pt[t.group];
-            sg.op_begin = (uint32_t)ops.size();
-            for (uint32_t f = e; f < hp.term_offsets[j + 1]; ++f) {
-                const fiona_term &u = hp.terms[f];
-                if (u.kind == FIONA_TERM_TERNARY && u.group == t.group && u.sign != 0)
-                    ops.push_back(u.input | (u.sign < 0 ? 0x80000000u : 0u));
-            }
-            sg.op_end = (uint32_t)ops.size();
-            segs.push_back(sg);
-        }
-        o.seg_end = (uint32_t)segs.size();
-        o.raw_begin = (uint32_t)raw_in.size();
-        for (uint32_t e = hp.term_offsets[j]; e < hp.term_offsets[j + 1]; ++e) {
-            const fiona_term &t = hp.terms[e];
-            if (t.kind != FIONA_TERM_RAW && t.kind != FIONA_TERM_RAW_CONST) continue;
-            raw_in.push_back(t.input);
-            raw_pt.push_back(t.pt | (t.kind == FIONA_TERM_RAW_CONST ? 0x80000000u : 0u));
-        }
-        o.raw_end = (uint32_t)raw_in.size();
-    }
+    const DirectSchedule d = direct_schedule(p->hp);
     const std::pair<const void *, size_t> parts[6] = {
         {p->ctx->limbs.data(), p->ctx->limbs.size() * sizeof(LimbConst)},
-        {outs.data(), outs.size() * sizeof(DirOut)},
-        {segs.data(), segs.size() * sizeof(DirSeg)},
-        {ops.data(), ops.size() * 4},
-        {raw_in.data(), raw_in.size() * 4},
-        {raw_pt.data(), raw_pt.size() * 4}};
+        {d.outs.data(), d.outs.size() * sizeof(DirOut)},
+        {d.segs.data(), d.segs.size() * sizeof(DirSeg)},
+        {d.ops.data(), d.ops.size() * 4},
+        {d.raw_in.data(), d.raw_in.size() * 4},
+        {d.raw_pt.data(), d.raw_pt.size() * 4}};
     size_t total = 0;
     for (int i = 0; i < 6; ++i) {
         p->static_off[i] = total;
@@ -852,10 +832,10 @@ extern "C" int fiona_linear_eval_static(const fiona_plan *p, void *stream, const
                          "the %zu-byte static area; use fiona_linear_eval",
                          p->static_image.size(), kStaticAreaBytes);
     if (p->hp.n_out == 0) return FIONA_OK;
-    if (p->ctx->device != FIONA_DEVICE_NONE) {
-        DeviceGuard g(p->ctx->device);
-        return launch_direct_static(p, stream, in, pt, out);
-    }
+    // a validation-only context runs on the current device (see the header)
+    if (p->ctx->device == FIONA_DEVICE_NONE) return launch_direct_static(p, stream, in, pt, out);
+    DeviceGuard g(p->ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "linear_eval_static: cannot select device %d", p->ctx->device);
     return launch_direct_static(p, stream, in, pt, out);
 }
 

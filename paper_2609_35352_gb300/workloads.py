@@ -238,6 +238,22 @@ class Plan:
         }
 
 
+def min_bytes(plan: Plan, L: int, N: int) -> int:
+    """Minimal HBM bytes of one evaluation: each input read by a nonzero term
+    (both polys), each plaintext a raw term or a used scale group reads, and
+    each output, one limb-poly of N * 8 bytes per limb, moved once; a
+    plaintext read only as a constant (TERM_RAW_CONST) counts one residue per
+    limb.  A count, the same as fiona_plan_stats.bytes_min."""
+    t = plan.terms
+    raw = (t["kind"] == TERM_RAW) | (t["kind"] == TERM_RAW_CONST)
+    signed = (t["kind"] == TERM_TERNARY) & (t["sign"] != 0)
+    inputs = set(int(i) for i in t["input"][raw | signed])
+    whole = set(int(p) for p in t["pt"][t["kind"] == TERM_RAW])
+    whole |= set(int(plan.group_scale_pt[g]) for g in set(int(g) for g in t["group"][signed]))
+    const = set(int(p) for p in t["pt"][t["kind"] == TERM_RAW_CONST]) - whole
+    return L * N * 8 * (2 * len(inputs) + len(whole) + 2 * plan.n_out) + len(const) * L * 8
+
+
 def build_plan(n_in: int, n_out: int, per_output: List[List[Tuple[int, int, int, int, int]]],
                 n_pt: int, group_scale_pt: List[int], group_output: List[int],
                 nodes: List[List[Tuple[int, int, int]]],

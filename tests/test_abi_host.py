@@ -273,3 +273,14 @@ def test_constant_raw_terms_count_one_word_per_limb():
     import dataclasses
     with pytest.raises(F.FionaError):
         F.Plan(F.Context(a.N, a.moduli, device=F.FIONA_DEVICE_NONE), dataclasses.replace(a.plan, terms=bad))
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny-dag", "worked-example", "wsum-hybrid", "vgg", "vit", "bert",
+                                  "bert-const"])
+def test_minimal_bytes_counted_alike(name):
+    """The benchmark's configuration counts the minimal bytes from the plan
+    description alone (so that both of its arms print the same dict); the
+    count equals fiona_plan_stats.bytes_min."""
+    wl = W.make_workload(name)
+    s = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan).stats()
+    assert W.min_bytes(wl.plan, wl.L, wl.N) == s["bytes_min"]

@@ -44,6 +44,13 @@ def test_reference_arm_line():
     e2e = line["e2e"]
     assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
     assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
+    # the configuration is the workload's alone: the library arm prints the same dict
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2609_35352_gb300 import workloads as W
+    assert line["config"] == bench.workload_config(W.make_workload(bench.DEFAULT_WORKLOAD),
+                                                   bench.DEFAULT_WORKLOAD)
+    assert line["config"]["bytes_min_per_step"] > 0 and "l2" in line["config"]
 
 
 @pytest.mark.gpu
@@ -63,3 +70,7 @@ def test_library_arm_line():
     clk = line["clocks"]
     for k in ("sm_mhz", "sm_max_mhz", "reasons"):
         assert k in clk
+    assert clk["samples"] >= 2 and clk["sm_mhz"] > 0  # taken inside the timed region
+    assert roof["peak_nominal"] > roof["peak"] * 0.9 and 0 < roof["frac_nominal"] < roof["frac"] * 1.2
+    ref = run_bench("--impl", "reference", "--steps", "1", "--warmup", "3")
+    assert ref["config"] == line["config"]

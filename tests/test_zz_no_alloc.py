@@ -31,8 +31,10 @@ def device_buffers(wl):
 
 
 @pytest.mark.parametrize("name,N,L", [("tiny-dag", None, None), ("vit", 2048, 2),
-                                      ("overflow60", None, None)])
+                                      ("overflow60", None, None), ("bert-const", 1024, 2)])
 def test_static_entry_matches_linear_eval(name, N, L):
+    """bert-const: constant raw plaintexts, which the kernel reads through
+    their limb's first residue."""
     wl = W.make_workload(name, N=N, L=L)
     d_in, d_pt, n_out = device_buffers(wl)
     ref_ctx = F.Context(wl.N, wl.moduli, device=0)
@@ -49,6 +51,25 @@ def test_static_entry_matches_linear_eval(name, N, L):
         assert plan.eval_static(d_in, d_pt, got, stream=stream) == F.FIONA_OK, F.last_error()
         torch.cuda.synchronize()
         assert torch.equal(got, want), "call %d differs from fiona_linear_eval" % call
+
+
+def test_static_entry_matches_the_oracle():
+    """The static entry point against the CPU oracle directly, on the
+    host-generated residues of a small layer with a two-level DAG."""
+    import oracle
+    oracle.build()
+    wl = W.make_workload("tiny-dag")
+    X, P = wl.host_inputs(), wl.host_plaintexts()
+    want = oracle.linear_eval(wl.plan, wl.moduli, X, P)
+    d_in = torch.from_numpy(X.view(np.int64)).cuda()
+    d_pt = torch.from_numpy(P.view(np.int64)).cuda()
+    ctx = F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE)
+    plan = F.Plan(ctx, wl.plan)
+    got = torch.full((wl.plan.n_out * 2 * wl.L * wl.N,), -1, dtype=torch.int64, device="cuda")
+    assert plan.eval_static(d_in, d_pt, got) == F.FIONA_OK, F.last_error()
+    torch.cuda.synchronize()
+    got = got.cpu().numpy().view(np.uint64).reshape(want.shape)
+    assert np.array_equal(got, want)
 
 
 def test_static_entry_rejects_layers_beyond_the_area():
