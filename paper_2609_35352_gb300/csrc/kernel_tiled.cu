@@ -34,10 +34,11 @@
 //  5. The next tile's inputs are prepared (with two regions: their copies,
 //     started at the top of this tile, waited for and rewritten) before the
 //     one barrier per tile that publishes them.
-// The spin-waits are bounded: thread 0's wait for the schedule copy (if it
-// gives up, the CTA raises the context's error flag and stops) and each
-// thread's wait for a region's TMA copies (if it gives up, the flag is
-// raised and the tile computed from whatever the region holds).
+// The spin-waits are bounded: thread 0's wait for the schedule copy and each
+// thread's wait for a region's TMA copies.  One that gives up raises the
+// context's error flag; the CTA then stops at its next barrier (thread 0
+// first waits, bounded again, for the copies it issued), leaving the tiles
+// it did not reach unwritten.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -47,8 +48,11 @@
 #include <mutex>
 
 #include "tiled.h"
+#include "tile_math.cuh"
 
 namespace {
+
+using namespace tile;
 
 constexpr uint32_t kWaitLimit = 2000;
 constexpr uint32_t kWaitHintNs = 1000000;
@@ -156,212 +160,6 @@ __device__ __forceinline__ uint64_t evict_first_policy()
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
     return pol;
-}
-
-// The limb's constants, read from shared memory where they are needed
-// (kept out of registers between uses).
-__device__ __forceinline__ LimbConst load_limb(uint32_t addr)
-{
-    LimbConst m;
-    asm volatile("ld.shared.v2.u64 {%0, %1}, [%2];" : "=l"(m.q), "=l"(m.mu_hi) : "r"(addr));
-    asm volatile("ld.shared.v2.u64 {%0, %1}, [%2+16];" : "=l"(m.mu_lo), "=l"(m.mu64) : "r"(addr));
-    return m;
-}
-
-template <int C>
-struct V {
-    uint64_t x[C];
-};
-
-// one lane's C plaintext words, not cached in L1
-template <int C>
-__device__ __forceinline__ V<C> ldg_stream(const uint64_t *p, uint64_t pol)
-{
-    V<C> v;
-    if constexpr (C == 2)
-        asm("ld.global.nc.L1::no_allocate.L2::cache_hint.v2.u64 {%0, %1}, [%2], %3;"
-            : "=l"(v.x[0]), "=l"(v.x[1])
-            : "l"(p), "l"(pol));
-    else
-        asm("ld.global.nc.L1::no_allocate.L2::cache_hint.u64 %0, [%1], %2;"
-            : "=l"(v.x[0])
-            : "l"(p), "l"(pol));
-    return v;
-}
-
-// shared memory through byte offsets from the dynamic shared array
-template <int C>
-__device__ __forceinline__ V<C> lds(const char *sm, uint32_t off)
-{
-    V<C> v;
-    if constexpr (C == 2) {
-        const ulonglong2 t = *reinterpret_cast<const ulonglong2 *>(sm + off);
-        v.x[0] = t.x;
-        v.x[1] = t.y;
-    } else {
-        v.x[0] = *reinterpret_cast<const uint64_t *>(sm + off);
-    }
-    return v;
-}
-
-template <int C>
-__device__ __forceinline__ void sts(char *sm, uint32_t off, const V<C> &v)
-{
-    if constexpr (C == 2)
-        *reinterpret_cast<ulonglong2 *>(sm + off) = make_ulonglong2(v.x[0], v.x[1]);
-    else
-        *reinterpret_cast<uint64_t *>(sm + off) = v.x[0];
-}
-
-template <int C>
-__device__ __forceinline__ void stg(uint64_t *p, const V<C> &v)
-{
-    if constexpr (C == 2)
-        *reinterpret_cast<ulonglong2 *>(p) = make_ulonglong2(v.x[0], v.x[1]);
-    else
-        *p = v.x[0];
-}
-
-// ---------------------------------------------------------------------------
-// Arithmetic policies.  "Operand form" is how source residues sit in shared
-// memory: canonical for Wide, split for Narrow.
-// ---------------------------------------------------------------------------
-template <bool NARROW>
-struct Arith;
-
-// Any q < 2^60: 128-bit products (lo, hi), plain 64-bit sums.
-template <>
-struct Arith<false> {
-    struct Acc {
-        uint64_t lo, hi;
-    };
-    __device__ static uint64_t operand(uint64_t a) { return a; }
-    __device__ static void zero(Acc &a) { a.lo = a.hi = 0; }
-    __device__ static void mac(Acc &a, uint64_t x, uint64_t y) { rns::mac(a.lo, a.hi, x, y); }
-    __device__ static uint64_t reduce(const Acc &a, const LimbConst &m) { return rns::reduce128(a.lo, a.hi, m); }
-    __device__ static void fold(Acc &a, const LimbConst &m)
-    {
-        a.lo = reduce(a, m);
-        a.hi = 0;
-    }
-    // canonical residue of P - M, each a plain sum within the lazy-sum bound
-    __device__ static uint64_t signed_value(uint64_t p, uint64_t mm, const LimbConst &m)
-    {
-        return rns::sub_mod(rns::reduce64(p, m), rns::reduce64(mm, m), m.q);
-    }
-};
-
-// q < 2^52: every factor in split form (sources split in shared memory or
-// where a product reads them, the other factor split on the way in);
-// Karatsuba products into three accumulators; packed sums of split words.
-template <>
-struct Arith<true> {
-    struct Acc {
-        uint64_t lo, x, hi;
-    };
-    __device__ static uint64_t operand(uint64_t a) { return rns::split26(a); }
-    __device__ static void zero(Acc &a) { a.lo = a.x = a.hi = 0; }
-    // both factors in operand (split) form
-    __device__ static void mac(Acc &a, uint64_t x, uint64_t y) { rns::mac26(a.lo, a.x, a.hi, x, y); }
-    __device__ static uint64_t reduce(const Acc &a, const LimbConst &m) { return rns::reduce26(a.lo, a.x, a.hi, m); }
-    __device__ static void fold(Acc &a, const LimbConst &m)
-    {
-        a.lo = reduce(a, m);
-        a.x = a.lo;  // the middle term x - lo - hi stays 0
-        a.hi = 0;
-    }
-    // P - M + 64q is below 2^59 (each packed sum reads back below 2^58)
-    __device__ static uint64_t signed_value(uint64_t p, uint64_t mm, const LimbConst &m)
-    {
-        const uint64_t k = (uint64_t)rns::kNarrowSumBudget * m.q;
-        return rns::reduce64(rns::unsplit_sum(p) + k - rns::unsplit_sum(mm), m);
-    }
-};
-
-// Sum of the n source tiles (both polys) named by the 16-bit indices packed
-// two per word from schedule byte offset `wp`; `src` = this lane's offset in
-// the source region.  K indices per step (each decoded once, its two polys
-// read at offsets 0 and TB), their loads independent, and the next step's
-// index words requested before this step's additions (the last request may
-// read words past the run: they lie inside the dynamic shared memory, which
-// continues with the source region, and are not used).  Returns the offset
-// just past the run's words.
-template <int C, uint32_t TB>
-__device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32_t wp, uint32_t n, V<C> &s0,
-                                            V<C> &s1)
-{
-    constexpr uint32_t PB = 2 * TB;
-    constexpr uint32_t K = C == 1 ? 8 : 2;  // 2K loads of C words in flight
-    constexpr uint32_t NW = K / 2;          // index words per step
-    uint32_t k = 0;
-    if (n >= K) {
-        uint32_t w[NW];
-#pragma unroll
-        for (uint32_t j = 0; j < NW; ++j) w[j] = *reinterpret_cast<const uint32_t *>(sm + wp + 4 * j);
-        for (; k + K <= n; k += K, wp += 4 * NW) {
-            V<C> a[K], b[K];
-#pragma unroll
-            for (uint32_t j = 0; j < K; ++j) {
-                const uint32_t o = src + ((j & 1) ? (w[j / 2] >> 16) : (w[j / 2] & 0xffffu)) * PB;
-                a[j] = lds<C>(sm, o);
-                b[j] = lds<C>(sm, o + TB);
-            }
-#pragma unroll
-            for (uint32_t j = 0; j < NW; ++j) w[j] = *reinterpret_cast<const uint32_t *>(sm + wp + 4 * NW + 4 * j);
-#pragma unroll
-            for (int x = 0; x < C; ++x) {
-#pragma unroll
-                for (uint32_t j = 0; j + 1 < K; j += 2) {  // three-input additions
-                    s0.x[x] = s0.x[x] + a[j].x[x] + a[j + 1].x[x];
-                    s1.x[x] = s1.x[x] + b[j].x[x] + b[j + 1].x[x];
-                }
-            }
-        }
-    }
-    for (; k + 2 <= n; k += 2, wp += 4) {
-        const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp);
-        const uint32_t o0 = src + (w & 0xffffu) * PB, o1 = src + (w >> 16) * PB;
-        const V<C> a0 = lds<C>(sm, o0), a1 = lds<C>(sm, o1), b0 = lds<C>(sm, o0 + TB), b1 = lds<C>(sm, o1 + TB);
-#pragma unroll
-        for (int x = 0; x < C; ++x) {
-            s0.x[x] += a0.x[x] + a1.x[x];
-            s1.x[x] += b0.x[x] + b1.x[x];
-        }
-    }
-    if (k < n) {
-        const uint32_t w = *reinterpret_cast<const uint32_t *>(sm + wp);
-        const uint32_t o0 = src + (w & 0xffffu) * PB;
-        const V<C> a0 = lds<C>(sm, o0), b0 = lds<C>(sm, o0 + TB);
-#pragma unroll
-        for (int x = 0; x < C; ++x) {
-            s0.x[x] += a0.x[x];
-            s1.x[x] += b0.x[x];
-        }
-        wp += 4;
-    }
-    return wp;
-}
-
-// Signed sum of the program at byte offset `hdr` (n_plus | n_minus << 16,
-// then the plus run, then the minus run), both polys, as canonical residues;
-// SPLIT: the sources are in split form (else canonical, whatever the
-// arithmetic).  Returns the offset just past the program.
-template <bool SPLIT, int C, uint32_t TB>
-__device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uint32_t hdr, uint32_t lim,
-                                               V<C> &o0, V<C> &o1)
-{
-    using A = Arith<SPLIT>;
-    const uint32_t h = *reinterpret_cast<const uint32_t *>(sm + hdr);
-    V<C> p0{}, p1{}, m0{}, m1{};
-    uint32_t wp = run_sum<C, TB>(sm, src, hdr + 4, h & 0xffffu, p0, p1);
-    wp = run_sum<C, TB>(sm, src, wp, h >> 16, m0, m1);
-    const LimbConst m = load_limb(lim);
-#pragma unroll
-    for (int x = 0; x < C; ++x) {
-        o0.x[x] = A::signed_value(p0.x[x], m0.x[x], m);
-        o1.x[x] = A::signed_value(p1.x[x], m1.x[x], m);
-    }
-    return wp;
 }
 
 template <int C, bool NARROW, uint32_t P, bool KC>
@@ -494,6 +292,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         }
     };
     uint32_t stage_phase = 0;  // bit r: phase of region r's copy barrier
+    uint32_t failed = 0;       // 1 + region + 2 * phase of a copy wait that gave up
 
     // the tile's inputs in region `reg`, once the copies have landed (with
     // cp.async each thread rewrites the words it copied); and the tile's
@@ -502,7 +301,11 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         if (threadIdx.x == 0) s_limb[reg] = a.limbs[a.limb0 + t / a.tiles_per_limb];
         if (!a.n_in) return;
         if constexpr (TMA) {
-            if (!mbar_wait_spin(bar_stage + 8 * reg, (stage_phase >> reg) & 1u)) atomicOr(a.err, 1);
+            if (!mbar_wait_spin(bar_stage + 8 * reg, (stage_phase >> reg) & 1u)) {
+                s_abort = 1;  // the CTA stops after the next barrier
+                atomicOr(a.err, 1);
+                failed = 1 + reg + 2 * ((stage_phase >> reg) & 1u);
+            }
             stage_phase ^= 1u << reg;
         } else {
             cp_async_wait<0>();  // this thread's copies; the barrier after publishes everyone's
@@ -523,11 +326,20 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     // tile.  With one region the next tile is staged after every warp is
     // done with this one.
     uint32_t buf = 0;
+    // after a copy wait gave up: every thread stops at the same barrier, once
+    // thread 0 has waited (bounded again) for the copies it issued
+    auto stop = [&]() {
+        if (TMA && threadIdx.x == 0 && failed) mbar_wait_spin(bar_stage + 8 * ((failed - 1) & 1), (failed - 1) >> 1);
+    };
     if (tile < total) {
         if (a.n_in) stage(tile, 0);
         prepare(tile, 0);
     }
     __syncthreads();
+    if (s_abort) {
+        stop();
+        return;
+    }
     for (; tile < total; tile += gridDim.x) {
         const uint32_t next = tile + gridDim.x;
         const char *next_ptl = tile_ptl(next);
@@ -713,6 +525,10 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
                 __syncthreads();
             }
         }
+        if (s_abort) {
+            stop();
+            return;
+        }
     }
 }
 
@@ -782,15 +598,16 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
 
 // The inputs [n_in][2][L][N] as a 3-D tensor (coefficient, limb, poly) with
 // boxes of T coefficients, one limb and `box_rows` polys.
-int tiled_input_map(const TiledArgs &a, uint32_t T, const uint64_t *in, uint32_t layout_L, CUtensorMap *tm)
+int input_tensor_map(uint32_t N, uint32_t layout_L, uint32_t n_in, uint32_t T, uint32_t box_rows,
+                     const uint64_t *in, CUtensorMap *tm)
 {
     memset(tm, 0, sizeof(*tm));
-    if (!a.n_in) return FIONA_OK;
+    if (!n_in) return FIONA_OK;
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (!enc) return set_error(FIONA_ERR_CUDA, "tiled kernel: cuTensorMapEncodeTiled is not available");
-    const cuuint64_t dims[3] = {a.N, layout_L, 2ull * a.n_in};
-    const cuuint64_t strides[2] = {(cuuint64_t)a.N * 8, (cuuint64_t)layout_L * a.N * 8};
-    const cuuint32_t box[3] = {T, 1, a.box_rows};
+    const cuuint64_t dims[3] = {N, layout_L, 2ull * n_in};
+    const cuuint64_t strides[2] = {(cuuint64_t)N * 8, (cuuint64_t)layout_L * N * 8};
+    const cuuint32_t box[3] = {T, 1, box_rows};
     const cuuint32_t estr[3] = {1, 1, 1};
     const CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_UINT64, 3, const_cast<uint64_t *>(in), dims, strides, box, estr,
                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
@@ -799,11 +616,16 @@ int tiled_input_map(const TiledArgs &a, uint32_t T, const uint64_t *in, uint32_t
     return FIONA_OK;
 }
 
+// kernel_ws.cu
+int launch_ws(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt, uint64_t *out, uint32_t l0,
+              uint32_t l1, uint32_t layout_L);
+
 int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const uint64_t *pt,
                  uint64_t *out, uint32_t l0, uint32_t l1, uint32_t layout_L)
 {
     const TiledSchedule *ts = p->tiled;
     if (!ts) return set_error(FIONA_ERR_ARG, "tiled kernel not available for this plan");
+    if (ts->ws) return launch_ws(p, stream, in, pt, out, l0, l1, layout_L);
     if (l1 <= l0) return FIONA_OK;
     TiledArgs a = ts->args;
     a.in = in;
@@ -823,7 +645,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     CUtensorMap tm;  // read by the kernels with one coefficient per lane only
     memset(&tm, 0, sizeof(tm));
     if (ts->C == 1)
-        if (const int rc = tiled_input_map(a, ts->tile, in, layout_L, &tm)) return rc;
+        if (const int rc = input_tensor_map(a.N, layout_L, a.n_in, ts->tile, a.box_rows, in, &tm)) return rc;
     void *args[] = {&a, &tm};
     cudaError_t e = cudaLaunchKernel(fn, grid, block, args, ts->smem, s);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel launch: %s", cudaGetErrorString(e));

@@ -209,6 +209,7 @@ struct Sched {
     std::vector<uint32_t> w;
     uint32_t o_level = 0, o_node_off = 0, o_warp = 0, o_comb_off = 0, o_comb_out = 0, o_comb_parts = 0;
     uint64_t pt_ops = 0;  // plaintext tiles fetched per tile
+    uint32_t prefix_words = 0;  // words before the operation streams when they come last
 };
 
 void pad4(std::vector<uint32_t> &w)
@@ -217,7 +218,7 @@ void pad4(std::vector<uint32_t> &w)
 }
 
 Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const std::vector<Seg> &nodes, uint32_t W,
-             uint32_t mac_budget, uint32_t zero_index, uint32_t P)
+             uint32_t mac_budget, uint32_t zero_index, uint32_t P, bool ops_last = false)
 {
     Sched sc;
     auto &w = sc.w;
@@ -317,12 +318,15 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
                     o[i] = (o[i] & ((1u << kOpPtShift) - 1) & ~kOpConst) | last_const | (last_pt << kOpPtShift);
         }
     }
-    for (uint32_t wi = 0; wi < W; ++wi) {
-        pad4(w);
-        w[sc.o_warp + wi * kWarpTableWords + 0] = (uint32_t)w.size();
-        w[sc.o_warp + wi * kWarpTableWords + 1] = (uint32_t)ops[wi].size();
-        w.insert(w.end(), ops[wi].begin(), ops[wi].end());
-    }
+    auto put_ops = [&]() {
+        for (uint32_t wi = 0; wi < W; ++wi) {
+            pad4(w);
+            w[sc.o_warp + wi * kWarpTableWords + 0] = (uint32_t)w.size();
+            w[sc.o_warp + wi * kWarpTableWords + 1] = (uint32_t)ops[wi].size();
+            w.insert(w.end(), ops[wi].begin(), ops[wi].end());
+        }
+    };
+    if (!ops_last) put_ops();
     for (uint32_t wi = 0; wi < W; ++wi) {
         w[sc.o_warp + wi * kWarpTableWords + 2] = (uint32_t)w.size();
         w.insert(w.end(), segw[wi].begin(), segw[wi].end());
@@ -338,6 +342,11 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
     sc.o_comb_parts = (uint32_t)w.size();
     w.insert(w.end(), jp.comb_parts.begin(), jp.comb_parts.end());
     while (w.size() % 32) w.push_back(0);  // a multiple of 128 bytes: the regions after it take TMA copies
+    sc.prefix_words = (uint32_t)w.size();
+    if (ops_last) {  // the operation streams after the part copied to shared memory
+        put_ops();
+        while (w.size() % 32) w.push_back(0);
+    }
     return sc;
 }
 
@@ -686,6 +695,147 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
 // kernel_tiled.cu
 int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, size_t smem);
 int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, cudaFuncAttributes *attr);
+// kernel_ws.cu
+int ws_kernel_attributes(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, cudaFuncAttributes *attr);
+int ws_configure_kernel(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, size_t smem);
+
+namespace {
+
+// Lowering for the warp-specialised kernel (kernel_ws.cu): two coefficients
+// per lane, W consumer warps plus a stager warp, one or two source regions,
+// a ring of D groups of P plaintext slots per consumer warp.  The shape: the
+// most consumer warps per SM (up to 16), then the most plaintext bytes in
+// flight per SM (up to 64 KB, where HBM reads saturate), then two source
+// regions, then deeper rings.  Tuning override FIONA_WS_SHAPE="W,regions,D".
+int lower_ws(fiona_plan *p, const NodeInfo &ni, const std::vector<OutWork> &groups, uint32_t budget,
+             uint32_t mac_budget, bool narrow, bool has_const, bool device)
+{
+    const HostPlan &hp = p->hp;
+    const fiona_ctx *ctx = p->ctx;
+    constexpr uint32_t P = 4, T = 64, TB = T * 8, PB = 2 * TB;
+    if (ctx->N % T) return set_error(FIONA_ERR_ARG, "ws kernel: N is not a multiple of %u", T);
+    const Costs k = costs_for(2, narrow);
+    const std::vector<uint32_t> no_rank;
+    const Lowered lw = resolve(hp, ni, groups, no_rank, 0, budget);  // shared sums expanded
+    const size_t per_sm = 228 * 1024;
+    int fw = 0, fb = 0, fd = 0;
+    const char *env = getenv("FIONA_WS_SHAPE");
+    const bool forced = env && sscanf(env, "%d,%d,%d", &fw, &fb, &fd) == 3;
+    struct Pick {
+        uint32_t W = 0, nbuf = 0, D = 0, ctas = 0;
+        size_t smem = 0;
+        std::tuple<uint32_t, uint32_t, uint32_t, uint32_t> key{};
+    } best;
+    for (uint32_t W : {16u, 15u, 12u, 8u, 4u})
+        for (uint32_t D : {4u, 3u}) {
+            cudaFuncAttributes attr{};
+            if (!device) {
+                attr.numRegs = W > 15 ? 96 : 128;
+                attr.sharedSizeBytes = 128;
+            } else if (ws_kernel_attributes(narrow, P, has_const, W, D, &attr) != FIONA_OK) {
+                continue;
+            }
+            const size_t smem_cap = (ctx->smem_optin ? ctx->smem_optin : 227 * 1024) - attr.sharedSizeBytes - 64;
+            const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
+            for (uint32_t nbuf : {2u, 1u}) {
+                if (forced && (W != (uint32_t)fw || nbuf != (uint32_t)fb || D != (uint32_t)fd)) continue;
+                const JobPlan jp = build_jobs(lw.work, W, k, P);
+                const Sched sc = encode(jp, lw.level_off, lw.nodes, W, mac_budget, hp.n_in, P);
+                const uint32_t src_bytes = (hp.n_in + 1) * PB;
+                const WsLayout lay((uint32_t)sc.w.size() * 4, nbuf, src_bytes, jp.n_part, W, D, P, TB);
+                if (lay.total > smem_cap) continue;
+                const uint32_t threads = (W + 1) * 32;
+                const uint32_t warps_alloc = (threads / 32 + 3) & ~3u;  // registers go to warps in fours
+                const uint32_t ctas = std::min({(uint32_t)(per_sm / (lay.total + attr.sharedSizeBytes + 1024)),
+                                                65536u / (warps_alloc * 32 * regs), 2048u / threads});
+                if (!ctas) continue;
+                const uint32_t ring = std::min<uint32_t>(ctas * W * (D - 1) * P * TB, 64 * 1024);
+                const auto key = std::make_tuple(std::min(ctas * W, 16u), ring, nbuf, D);
+                if (best.W == 0 || key > best.key) best = {W, nbuf, D, ctas, lay.total, key};
+            }
+        }
+    if (!best.W) return set_error(FIONA_ERR_ARG, "ws kernel: the input tiles do not fit in shared memory");
+    const JobPlan jp = build_jobs(lw.work, best.W, k, P);
+    const Sched sc = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in, P);
+
+    TiledSchedule *ts = new (std::nothrow) TiledSchedule;
+    if (!ts) return set_error(FIONA_ERR_NOMEM, "ws schedule: host allocation");
+    ts->ws = true;
+    ts->C = 2;
+    ts->narrow = narrow;
+    ts->warps = best.W;
+    ts->tile = T;
+    ts->batch = P;
+    ts->has_const = has_const;
+    ts->smem = best.smem;
+    ts->ctas_per_sm = best.ctas;
+    ts->nodes_kept = 0;
+    ts->nodes_expanded = (uint32_t)ni.ids.size();
+    ts->ring = best.D;
+    WsArgs &a = ts->ws_args;
+    a.limbs = ctx->d_limbs;
+    a.err = ctx->d_kerr;
+    a.wait_ns = 2000000000ull;
+    a.smem_sched_bytes = (uint32_t)sc.w.size() * 4;
+    a.o_warp = sc.o_warp;
+    a.o_comb_off = sc.o_comb_off;
+    a.o_comb_out = sc.o_comb_out;
+    a.o_comb_parts = sc.o_comb_parts;
+    a.N = ctx->N;
+    a.L = ctx->L;
+    a.pt_stride = ctx->L * ctx->N;
+    a.tiles_per_limb = ctx->N / T;
+    a.n_in = hp.n_in;
+    a.n_part = jp.n_part;
+    a.n_comb = (uint32_t)jp.comb_out.size();
+    a.src_bytes = (hp.n_in + 1) * PB;
+    a.n_boxes = (2 * hp.n_in + 255) / 256;
+    a.box_rows = a.n_boxes ? (2 * hp.n_in + a.n_boxes - 1) / a.n_boxes : 0;
+    a.n_buf = best.nbuf;
+    a.has_pt = hp.n_pt ? 1 : 0;
+    a.flags = 0;
+    if (const char *t = getenv("FIONA_TEST_WS_TIMEOUT")) {  // test only: a wait that runs out
+        if (atoi(t) > 0) {
+            a.flags |= kWsFlagExtraTx;
+            a.wait_ns = 2000000ull;
+        }
+    }
+    // the schedule checks of the tiled kernel, on a mirror of its arguments
+    TiledArgs m{};
+    m.sched_bytes = (uint32_t)(sc.w.size() * 4);
+    m.o_level = sc.o_level;
+    m.o_node_off = sc.o_node_off;
+    m.o_warp = sc.o_warp;
+    m.o_comb_off = sc.o_comb_off;
+    m.o_comb_out = sc.o_comb_out;
+    m.o_comb_parts = sc.o_comb_parts;
+    m.n_in = hp.n_in;
+    m.n_part = jp.n_part;
+    m.n_comb = a.n_comb;
+    m.src_bytes = a.src_bytes;
+    m.box_rows = a.box_rows;
+    m.n_boxes = a.n_boxes;
+    const char *why = check_schedule(sc.w, m, best.W, hp.n_out, hp.n_pt, (size_t)1 << 30, PB, P);
+    if (!why) why = check_linear_map(sc.w, m, best.W, hp);
+    if (why) {
+        delete ts;
+        return set_error(FIONA_ERR_INTERNAL, "ws schedule check failed: %s", why);
+    }
+    if (device) {
+        int rc = ws_configure_kernel(narrow, P, has_const, best.W, best.D, ts->smem);
+        if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
+        if (rc != FIONA_OK) {
+            cudaFree(ts->sched.blob);
+            delete ts;
+            return rc;
+        }
+        a.sched = (const uint32_t *)ts->sched.blob;
+    }
+    p->tiled = ts;
+    return FIONA_OK;
+}
+
+}  // namespace
 
 int lower_tiled(fiona_plan *p)
 {
@@ -757,6 +907,14 @@ int lower_tiled(fiona_plan *p)
             groups[j].segs.push_back(std::move(sg));
         }
     }
+
+    // -- the warp-specialised kernel (FIONA_TILED_WS=1)
+    if (const char *env = getenv("FIONA_TILED_WS"))
+        if (atoi(env) > 0) {
+            bool has_const = false;
+            for (const fiona_term &t : hp.terms) has_const |= t.kind == FIONA_TERM_RAW_CONST;
+            return lower_ws(p, ni, groups, budget, mac_budget, narrow, has_const, device);
+        }
 
     // -- forming shared sums once per tile is a phase of its own (a barrier per
     //    DAG level, no plaintext traffic issued meanwhile): measured on the ViT

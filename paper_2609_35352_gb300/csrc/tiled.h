@@ -89,6 +89,56 @@ struct TiledArgs {
     uint32_t has_pt;         // 0: the plan has no plaintexts (every load reads the schedule)
 };
 
+// Warp-specialised variant (kernel_ws.cu), two coefficients per lane.  The
+// block is W consumer warps (the operation streams, as above) and one stager
+// warp that copies each tile's inputs by TMA and, for narrow plans, rewrites
+// them in split form.  Each consumer warp copies its own plaintext tiles
+// with per-lane asynchronous copies into a ring of D groups of P slots in
+// shared memory, D - 1 batches ahead of its use.  The schedule is copied to
+// shared memory whole (`smem_sched_bytes`).
+constexpr uint32_t kWsMaxWarps = 16;  // consumer warps
+constexpr uint32_t kWsFlagExtraTx = 1;  // test only: the first input copy expects 16 bytes that never come
+
+struct WsArgs {
+    const uint64_t *in;
+    const uint64_t *pt;
+    uint64_t *out;
+    const LimbConst *limbs;
+    const uint32_t *sched;   // schedule words (global), copied to shared memory
+    int *err;                // set to 1 when a bounded wait gives up
+    uint64_t wait_ns;        // bound of every wait
+    uint32_t smem_sched_bytes;
+    uint32_t o_warp, o_comb_off, o_comb_out, o_comb_parts;
+    uint32_t N, L;
+    uint32_t pt_stride;      // L * N
+    uint32_t limb0, n_limbs;
+    uint32_t tiles_per_limb;
+    uint32_t n_in, n_part, n_comb;
+    uint32_t src_bytes;      // one source region (inputs, zero tile)
+    uint32_t box_rows, n_boxes;
+    uint32_t n_buf;          // source regions (1 or 2)
+    uint32_t has_pt;
+    uint32_t flags;          // kWsFlag*
+};
+
+// Shared-memory layout of the warp-specialised kernel (byte offsets), the
+// same on the host and in the kernel.
+struct WsLayout {
+    uint32_t src0, part0, ring0, bar0, total;
+#if defined(__CUDACC__)
+    __host__ __device__
+#endif
+    WsLayout(uint32_t sched_bytes, uint32_t n_buf, uint32_t src_bytes, uint32_t n_part, uint32_t W, uint32_t D,
+             uint32_t P, uint32_t TB)
+    {
+        src0 = sched_bytes;
+        part0 = src0 + n_buf * src_bytes;
+        ring0 = part0 + 2 * n_part * 2 * TB;
+        bar0 = ring0 + W * D * P * TB;
+        total = bar0 + 8 * 8;
+    }
+};
+
 struct TiledSchedule {
     int C = 2;                 // coefficients per lane
     bool narrow = false;       // every modulus < 2^52: radix-2^26 arithmetic
@@ -102,4 +152,7 @@ struct TiledSchedule {
     uint32_t nodes_expanded = 0;  // shared sums expanded into their uses
     DeviceSchedule sched;
     TiledArgs args{};          // device pointers (data pointers unset)
+    bool ws = false;           // the warp-specialised kernel runs this plan
+    uint32_t ring = 0;         // its plaintext ring depth D (groups of P slots per warp)
+    WsArgs ws_args{};
 };
