@@ -188,7 +188,8 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     const uint32_t n_buf = a.double_buffer ? 2 : 1;
     const uint32_t src0 = a.sched_bytes;  // byte offsets in `sm`
     const uint32_t part_base = src0 + n_buf * a.src_bytes;
-    const uint32_t bar_off = part_base + a.n_part * PB;  // the schedule copy's mbarrier
+    const uint32_t slot_base = part_base + a.n_part * PB;  // warp slots: n_slots tile pairs per warp
+    const uint32_t bar_off = slot_base + a.n_slots * PB;  // the schedule copy's mbarrier
     const uint32_t bar0 = smem_addr(sm) + bar_off;
     const uint32_t bar_stage = bar0 + 8;  // + 8 * region: the region's input copies have landed
     const uint32_t total = a.n_limbs * a.tiles_per_limb;
@@ -231,6 +232,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     const uint32_t wt = a.o_warp + warp * kWarpTableWords;
     const uint32_t op0 = sw[wt] * 4, n_batches = sw[wt + 1] / P;
     const uint32_t seg0 = sw[wt + 2] * 4, tg0 = sw[wt + 3];
+    const uint32_t slots = slot_base + sw[wt + 4] * PB + lane_off;  // this lane's words of its warp's slot 0
     const uint64_t pol = evict_first_policy();
     const uint32_t stride_bytes = a.pt_stride * 8;  // L * N * 8 < 2^32 (lowering)
     auto tile_ptl = [&](uint32_t t) -> const char * {
@@ -367,7 +369,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         for (uint32_t lev = 0; lev < a.n_levels; ++lev) {
             for (uint32_t x = sw[a.o_level + lev] + warp; x < sw[a.o_level + lev + 1]; x += n_warps) {
                 V<C> u0, u1;
-                signed_sum<SPLIT, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, u0, u1);
+                signed_sum<SPLIT, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, 0, u0, u1);
                 if constexpr (SPLIT) {  // stored in the sources' form
 #pragma unroll
                     for (int x2 = 0; x2 < C; ++x2) {
@@ -435,7 +437,24 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
             V<C> g0, g1;  // the signed sum of this batch's SEG (operand form)
             const bool seg = first & kOpSeg;
             if (seg) {
-                sp = signed_sum<SPLIT, C, TB>(sm, src, sp, lim, g0, g1);
+                // shared signed sums this warp forms for its own later uses
+                // (Sec. 4.2 "Sharing Signed Sums"), then this group's sum
+                const uint32_t nf = first & (kOpMaxSources - 1);
+                for (uint32_t f = 0; f < nf; ++f) {
+                    const uint32_t dst = slots + sw[sp >> 2] * PB;
+                    V<C> u0, u1;
+                    sp = signed_sum<SPLIT, C, TB>(sm, src, sp + 4, lim, slots, u0, u1);
+                    if constexpr (SPLIT) {  // stored in the sources' form
+#pragma unroll
+                        for (int x = 0; x < C; ++x) {
+                            u0.x[x] = A::operand(u0.x[x]);
+                            u1.x[x] = A::operand(u1.x[x]);
+                        }
+                    }
+                    sts<C>(sm, dst, u0);
+                    sts<C>(sm, dst + TB, u1);
+                }
+                sp = signed_sum<SPLIT, C, TB>(sm, src, sp, lim, slots, g0, g1);
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
                     g0.x[x] = A::operand(g0.x[x]);

@@ -65,7 +65,7 @@ __global__ void __launch_bounds__((MAXW + 1) * 32, 1)
     __shared__ __align__(16) LimbConst s_limb[2];
     const uint32_t W = (blockDim.x >> 5) - 1;  // consumer warps
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const WsLayout lay(a.smem_sched_bytes, a.n_buf, a.src_bytes, a.n_part, W, D, P, TB);
+    const WsLayout lay(a.smem_sched_bytes, a.n_buf, a.src_bytes, a.n_part, W, D, P, TB, a.n_slots);
     const uint32_t smb = smem_addr(sm);
     const uint32_t bar_sched = smb + lay.bar0;
     auto bar_loaded = [&](uint32_t r) { return bar_sched + 8 + 8 * r; };
@@ -181,6 +181,7 @@ __global__ void __launch_bounds__((MAXW + 1) * 32, 1)
     const uint32_t op0 = sw[wt] * 4, n_batches = sw[wt + 1] / P;
     const uint32_t seg0 = sw[wt + 2] * 4, tg0 = sw[wt + 3];
     const uint32_t ring_w = lay.ring0 + warp * D * P * TB + lane_off;  // byte offset in `sm`
+    const uint32_t slots = lay.slot0 + sw[wt + 4] * PB + lane_off;  // this lane's words of its warp's slot 0
     const uint64_t pol = evict_first_policy();
     // the prefetch cursor: batch pf_b of tile pf_tile, D - 1 batches ahead;
     // pf_lb / pf_tb: the tile's limb of plaintext 0 and this lane's words in
@@ -275,7 +276,24 @@ __global__ void __launch_bounds__((MAXW + 1) * 32, 1)
             V<C> g0, g1;  // the signed sum of this batch's SEG (operand form)
             const bool seg = hw[0] & kOpSeg;
             if (seg) {
-                sp = signed_sum<SPLIT, C, TB>(sm, src, sp, lim, g0, g1);
+                // shared signed sums this warp forms for its own later uses
+                // (Sec. 4.2 "Sharing Signed Sums"), then this group's sum
+                const uint32_t nf = hw[0] & (kOpMaxSources - 1);
+                for (uint32_t f = 0; f < nf; ++f) {
+                    const uint32_t dst = slots + sw[sp >> 2] * PB;
+                    V<C> u0, u1;
+                    sp = signed_sum<SPLIT, C, TB>(sm, src, sp + 4, lim, slots, u0, u1);
+                    if constexpr (SPLIT) {
+#pragma unroll
+                        for (int x = 0; x < C; ++x) {
+                            u0.x[x] = A::operand(u0.x[x]);
+                            u1.x[x] = A::operand(u1.x[x]);
+                        }
+                    }
+                    sts<C>(sm, dst, u0);
+                    sts<C>(sm, dst + TB, u1);
+                }
+                sp = signed_sum<SPLIT, C, TB>(sm, src, sp, lim, slots, g0, g1);
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
                     g0.x[x] = A::operand(g0.x[x]);

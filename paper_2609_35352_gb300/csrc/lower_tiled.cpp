@@ -27,6 +27,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <functional>
 #include <map>
 #include <numeric>
 #include <tuple>
@@ -37,11 +38,28 @@ namespace {
 
 constexpr uint32_t kNodeTag = 0x80000000u;  // operand naming a shared sum
 
+// A signed-sum program formed by a warp into one of its slots.
+struct Form {
+    uint32_t slot;
+    std::vector<uint32_t> plus, minus;             // source indices
+    std::vector<uint32_t> plus_slots, minus_slots; // warp slots
+};
+
 // One SEG operation (after cuts) or the unresolved operand list of a group.
 struct Seg {
     uint32_t scale_pt;
-    std::vector<uint32_t> plus, minus;  // source indices
+    std::vector<uint32_t> plus, minus;              // source indices
+    std::vector<uint32_t> plus_slots, minus_slots;  // warp slots (shared sums this warp formed)
+    std::vector<Form> forms;                        // sums formed into slots before this one
 };
+
+// operands a SEG reads, its formations included
+size_t seg_operands(const Seg &s)
+{
+    size_t n = s.plus.size() + s.minus.size() + s.plus_slots.size() + s.minus_slots.size();
+    for (const Form &f : s.forms) n += f.plus.size() + f.minus.size() + f.plus_slots.size() + f.minus_slots.size();
+    return n;
+}
 
 struct OutWork {
     std::vector<Seg> segs;
@@ -70,7 +88,7 @@ Costs costs_for(int C, bool narrow)
 double work_cost(const OutWork &w, const Costs &k, size_t P)
 {  // P: operations per batch
     double c = k.last + k.raw * (double)w.raws.size();
-    for (auto &s : w.segs) c += k.seg + k.operand * (double)(s.plus.size() + s.minus.size());
+    for (auto &s : w.segs) c += k.seg * (1.0 + 0.5 * (double)s.forms.size()) + k.operand * (double)seg_operands(s);
     // NOP padding: each SEG opens a batch, the job fills its last one
     const size_t ops = w.segs.size() + w.raws.size();
     size_t slots = 0;
@@ -130,15 +148,69 @@ std::vector<OutWork> split_work(const OutWork &w, uint32_t P, const Costs &k, si
     return chunk;
 }
 
+// Outputs that share signed sums (Sec. 4.2 "Sharing Signed Sums"): per
+// shared sum of the plan, the distinct outputs whose groups use it, and what
+// keeping it saves.  Used to place such outputs on one warp, which can then
+// form the sum once per tile for all of them.
+struct Sharing {
+    std::vector<std::vector<uint32_t>> users;  // per plan node
+    std::vector<double> benefit;               // per plan node
+};
+
+// Clusters of outputs for W warps: the users of each shared sum (best saving
+// first) are merged while the merged cost stays within one warp's share.
+// Returns a cluster id per output (-1: on its own).
+std::vector<int> clusters_for(const std::vector<OutWork> &work, uint32_t W, const Costs &k, size_t batch,
+                              const Sharing *sh)
+{
+    std::vector<int> cl(work.size(), -1);
+    if (!sh || work.empty()) return cl;
+    std::vector<double> cost(work.size());
+    double total = 0;
+    for (size_t j = 0; j < work.size(); ++j) total += cost[j] = work_cost(work[j], k, batch);
+    double cmax = 0;
+    for (double c : cost) cmax = std::max(cmax, c);
+    const double cap = std::max(total / W, 2 * cmax);  // a pair of outputs always fits
+    std::vector<uint32_t> parent(work.size());
+    std::iota(parent.begin(), parent.end(), 0);
+    std::vector<double> ccost = cost;
+    std::function<uint32_t(uint32_t)> find = [&](uint32_t x) { return parent[x] == x ? x : parent[x] = find(parent[x]); };
+    std::vector<uint32_t> order(sh->users.size());
+    std::iota(order.begin(), order.end(), 0);
+    std::stable_sort(order.begin(), order.end(), [&](uint32_t x, uint32_t y) { return sh->benefit[x] > sh->benefit[y]; });
+    for (uint32_t nd : order) {
+        const auto &us = sh->users[nd];
+        if (us.size() < 2 || sh->benefit[nd] <= 0) continue;
+        std::vector<uint32_t> roots;
+        for (uint32_t u : us) {
+            const uint32_t r = find(u);
+            if (std::find(roots.begin(), roots.end(), r) == roots.end()) roots.push_back(r);
+        }
+        if (roots.size() < 2) continue;
+        double c = 0;
+        for (uint32_t r : roots) c += ccost[r];
+        if (c > cap) continue;
+        for (size_t i = 1; i < roots.size(); ++i) parent[roots[i]] = roots[0];
+        ccost[roots[0]] = c;
+    }
+    std::vector<uint32_t> size(work.size(), 0);
+    for (size_t j = 0; j < work.size(); ++j) ++size[find((uint32_t)j)];
+    for (size_t j = 0; j < work.size(); ++j)
+        if (size[find((uint32_t)j)] > 1) cl[j] = (int)find((uint32_t)j);
+    return cl;
+}
+
 // Jobs for W warps: every output worth splitting is cut into `split` parts
-// (more if it costs more than a fair share, total / W), then all jobs are
-// assigned largest first to the least-loaded warp.  `makespan` receives the
-// largest warp load.
+// (more if it costs more than a fair share, total / W), except outputs
+// clustered with others (`cl`), which stay whole and together; then the
+// units (a cluster's jobs, or one job) are assigned largest first to the
+// least-loaded warp.  `makespan` receives the largest warp load.
 JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Costs &k, uint32_t split,
-                         double &makespan, size_t batch)
+                         double &makespan, size_t batch, const std::vector<int> &cl)
 {
     JobPlan jp;
     std::vector<Job> jobs;
+    std::vector<int> job_cluster;
     jp.comb_off.assign(1, 0);
     double total = 0;
     for (auto &w : work) total += work_cost(w, k, batch);
@@ -148,8 +220,9 @@ JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Cos
         uint32_t P = (uint32_t)std::max(1.0, std::round(c / std::max(share, 1.0)));
         P = std::min(W, std::max(P, split));
         // a part must be worth its partial slot and final addition
-        if (P <= 1 || c < 4 * k.last) {
+        if (P <= 1 || c < 4 * k.last || cl[j] >= 0) {
             jobs.push_back({j, work[j]});
+            job_cluster.push_back(cl[j]);
             continue;
         }
         std::vector<OutWork> chunk = split_work(work[j], P, k, batch);
@@ -157,35 +230,55 @@ JobPlan build_jobs_split(const std::vector<OutWork> &work, uint32_t W, const Cos
         for (auto &ch : chunk) {
             if (ch.segs.empty() && ch.raws.empty()) continue;
             jobs.push_back({kPartBit | jp.n_part, std::move(ch)});
+            job_cluster.push_back(-1);
             jp.comb_parts.push_back(jp.n_part++);
         }
         jp.comb_off.push_back((uint32_t)jp.comb_parts.size());
     }
-    std::vector<uint32_t> order(jobs.size());
-    std::iota(order.begin(), order.end(), 0);
-    std::vector<double> jc(jobs.size());
+    // units: the jobs of one cluster, or a single job
+    std::vector<std::vector<uint32_t>> units;
+    std::map<int, uint32_t> unit_of;
+    for (uint32_t i = 0; i < jobs.size(); ++i) {
+        if (job_cluster[i] < 0) {
+            units.push_back({i});
+            continue;
+        }
+        auto it = unit_of.find(job_cluster[i]);
+        if (it == unit_of.end()) {
+            unit_of[job_cluster[i]] = (uint32_t)units.size();
+            units.push_back({i});
+        } else {
+            units[it->second].push_back(i);
+        }
+    }
+    std::vector<double> jc(jobs.size()), uc(units.size(), 0);
     for (size_t i = 0; i < jobs.size(); ++i) jc[i] = work_cost(jobs[i].w, k, batch);
-    std::stable_sort(order.begin(), order.end(), [&](uint32_t a, uint32_t b) { return jc[a] > jc[b]; });
+    for (size_t u = 0; u < units.size(); ++u)
+        for (uint32_t i : units[u]) uc[u] += jc[i];
+    std::vector<uint32_t> order(units.size());
+    std::iota(order.begin(), order.end(), 0);
+    std::stable_sort(order.begin(), order.end(), [&](uint32_t a, uint32_t b) { return uc[a] > uc[b]; });
     std::vector<double> load(W, 0);
     jp.per_warp.assign(W, {});
-    for (uint32_t o : order) {
+    for (uint32_t u : order) {
         const uint32_t wi = (uint32_t)(std::min_element(load.begin(), load.end()) - load.begin());
-        jp.per_warp[wi].push_back(std::move(jobs[o]));
-        load[wi] += jc[o];
+        for (uint32_t i : units[u]) jp.per_warp[wi].push_back(std::move(jobs[i]));
+        load[wi] += uc[u];
     }
     makespan = *std::max_element(load.begin(), load.end());
     return jp;
 }
 
 // The split (1 to 4 parts per output) with the smallest largest warp load;
-// a finer split must gain at least 3% to be taken.
-JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t W, const Costs &k, size_t batch)
+// a finer split must gain at least 3% to be taken.  With `sh`, outputs that
+// share signed sums are clustered onto warps first.
+JobPlan build_jobs_with(const std::vector<OutWork> &work, uint32_t W, const Costs &k, size_t batch,
+                        const std::vector<int> &cl, double &best_ms)
 {
-    double best_ms = 0;
-    JobPlan best = build_jobs_split(work, W, k, 1, best_ms, batch);
+    JobPlan best = build_jobs_split(work, W, k, 1, best_ms, batch, cl);
     for (uint32_t split = 2; split <= 4; ++split) {
         double ms = 0;
-        JobPlan jp = build_jobs_split(work, W, k, split, ms, batch);
+        JobPlan jp = build_jobs_split(work, W, k, split, ms, batch, cl);
         if (ms < 0.97 * best_ms) {
             best_ms = ms;
             best = std::move(jp);
@@ -194,14 +287,118 @@ JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t W, const Costs &k,
     return best;
 }
 
+// Brings the users of shared sums onto one warp by swapping whole outputs of
+// similar cost between warps, a sum at a time (best saving first), keeping
+// every warp's load within `limit`; outputs already brought together stay.
+void colocate(JobPlan &jp, const std::vector<OutWork> &work, const Costs &k, size_t batch, const Sharing &sh,
+              double limit)
+{
+    const uint32_t W = (uint32_t)jp.per_warp.size();
+    std::vector<int> warp_of(work.size(), -1), pinned(work.size(), 0);
+    std::vector<double> load(W, 0), cost(work.size(), 0);
+    for (uint32_t wi = 0; wi < W; ++wi)
+        for (const Job &jb : jp.per_warp[wi]) {
+            const double c = work_cost(jb.w, k, batch);
+            load[wi] += c;
+            if (!(jb.target & kPartBit)) {
+                warp_of[jb.target] = (int)wi;
+                cost[jb.target] = c;
+            }
+        }
+    std::vector<uint32_t> order(sh.users.size());
+    std::iota(order.begin(), order.end(), 0);
+    std::stable_sort(order.begin(), order.end(), [&](uint32_t x, uint32_t y) { return sh.benefit[x] > sh.benefit[y]; });
+    for (uint32_t nd : order) {
+        const auto &us = sh.users[nd];
+        if (us.size() < 2 || sh.benefit[nd] <= 0) continue;
+        bool whole = true;
+        for (uint32_t u : us) whole &= warp_of[u] >= 0;
+        if (!whole) continue;
+        // the warp already holding most of the users (pinned ones first)
+        std::vector<int> votes(W, 0);
+        for (uint32_t u : us) votes[warp_of[u]] += 1 + 4 * pinned[u];
+        const uint32_t t = (uint32_t)(std::max_element(votes.begin(), votes.end()) - votes.begin());
+        std::vector<std::pair<uint32_t, uint32_t>> swaps;  // (user, partner on t)
+        std::vector<double> ld = load;
+        std::vector<int> taken(work.size(), 0);
+        bool ok = true;
+        for (uint32_t u : us) {
+            if ((uint32_t)warp_of[u] == t) continue;
+            if (pinned[u]) {
+                ok = false;
+                break;
+            }
+            const uint32_t from = (uint32_t)warp_of[u];
+            int best = -1;
+            double bd = 0;
+            for (size_t v = 0; v < work.size(); ++v) {
+                if (warp_of[v] != (int)t || pinned[v] || taken[v] ||
+                    std::find(us.begin(), us.end(), (uint32_t)v) != us.end())
+                    continue;
+                const double lt = ld[t] - cost[v] + cost[u], lf = ld[from] - cost[u] + cost[v];
+                if (lt > limit || lf > limit) continue;
+                const double d = std::fabs(cost[v] - cost[u]);
+                if (best < 0 || d < bd) {
+                    best = (int)v;
+                    bd = d;
+                }
+            }
+            if (best < 0) {
+                ok = false;
+                break;
+            }
+            taken[best] = 1;
+            ld[t] += cost[u] - cost[best];
+            ld[from] += cost[best] - cost[u];
+            swaps.push_back({u, (uint32_t)best});
+        }
+        if (!ok) continue;
+        for (auto &sp : swaps) {
+            const uint32_t from = (uint32_t)warp_of[sp.first];
+            warp_of[sp.second] = (int)from;
+            warp_of[sp.first] = (int)t;
+        }
+        load = ld;
+        for (uint32_t u : us) pinned[u] = 1;
+    }
+    // rebuild the warps' job lists (parts stay where they were; outputs that
+    // share a warp follow one another in index order)
+    std::vector<std::vector<Job>> pw(W);
+    for (uint32_t wi = 0; wi < W; ++wi)
+        for (Job &jb : jp.per_warp[wi])
+            if (jb.target & kPartBit) pw[wi].push_back(std::move(jb));
+    for (size_t j = 0; j < work.size(); ++j)
+        if (warp_of[j] >= 0) pw[warp_of[j]].push_back({(uint32_t)j, work[j]});
+    jp.per_warp = std::move(pw);
+}
+
+// ... then the users of shared sums are brought together by swaps within 1%
+// of the largest warp load (warp balance is worth more than the additions a
+// shared sum saves).
+JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t W, const Costs &k, size_t batch,
+                   const Sharing *sh = nullptr)
+{
+    double ms = 0;
+    JobPlan jp = build_jobs_with(work, W, k, batch, std::vector<int>(work.size(), -1), ms);
+    if (sh) colocate(jp, work, k, batch, *sh, 1.01 * ms);
+    return jp;
+}
+
 // Program words of a signed sum: n_plus | n_minus << 16, then each run as
 // 16-bit indices, two per word.
-void put_program(std::vector<uint32_t> &w, const std::vector<uint32_t> &plus, const std::vector<uint32_t> &minus)
+void put_program(std::vector<uint32_t> &w, const std::vector<uint32_t> &plus, const std::vector<uint32_t> &minus,
+                 const std::vector<uint32_t> &plus_slots = {}, const std::vector<uint32_t> &minus_slots = {})
 {
     w.push_back((uint32_t)plus.size() | ((uint32_t)minus.size() << 16));
     for (const auto *run : {&plus, &minus})
         for (size_t i = 0; i < run->size(); i += 2)
-            w.push_back((*run)[i] | (i + 1 < run->size() ? (*run)[i + 1] << 16 : 0u));
+            w.push_back(run->at(i) | (i + 1 < run->size() ? run->at(i + 1) << 16 : 0u));
+    // the slot word: counts, then up to six 4-bit slot numbers (plus first)
+    uint32_t sw = (uint32_t)plus_slots.size() | ((uint32_t)minus_slots.size() << 4);
+    uint32_t j = 0;
+    for (const auto *ss : {&plus_slots, &minus_slots})
+        for (uint32_t sl : *ss) sw |= (sl & 15u) << (8 + 4 * j++);
+    w.push_back(sw);
 }
 
 // The whole schedule (see tiled.h).
@@ -209,7 +406,6 @@ struct Sched {
     std::vector<uint32_t> w;
     uint32_t o_level = 0, o_node_off = 0, o_warp = 0, o_comb_off = 0, o_comb_out = 0, o_comb_parts = 0;
     uint64_t pt_ops = 0;  // plaintext tiles fetched per tile
-    uint32_t prefix_words = 0;  // words before the operation streams when they come last
 };
 
 void pad4(std::vector<uint32_t> &w)
@@ -218,7 +414,7 @@ void pad4(std::vector<uint32_t> &w)
 }
 
 Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const std::vector<Seg> &nodes, uint32_t W,
-             uint32_t mac_budget, uint32_t zero_index, uint32_t P, bool ops_last = false)
+             uint32_t mac_budget, uint32_t zero_index, uint32_t P, const std::vector<uint32_t> *warp_slots = nullptr)
 {
     Sched sc;
     auto &w = sc.w;
@@ -271,8 +467,12 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
             for (size_t p = first; k < segs.size() || r < raws.size(); ++p) {
                 if (p % P == 0 && k < segs.size() && seg_at[(p - b0) / P]) {
                     const Seg &sg = segs[k++];
-                    put_program(segw[wi], sg.plus, sg.minus);
-                    o.push_back((sg.scale_pt << kOpPtShift) | kOpSeg);
+                    for (const Form &f : sg.forms) {
+                        segw[wi].push_back(f.slot);
+                        put_program(segw[wi], f.plus, f.minus, f.plus_slots, f.minus_slots);
+                    }
+                    put_program(segw[wi], sg.plus, sg.minus, sg.plus_slots, sg.minus_slots);
+                    o.push_back((sg.scale_pt << kOpPtShift) | kOpSeg | (uint32_t)sg.forms.size());
                 } else {
                     o.push_back(raw_or_nop());  // a NOP while a SEG waits for its batch
                 }
@@ -318,15 +518,14 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
                     o[i] = (o[i] & ((1u << kOpPtShift) - 1) & ~kOpConst) | last_const | (last_pt << kOpPtShift);
         }
     }
-    auto put_ops = [&]() {
-        for (uint32_t wi = 0; wi < W; ++wi) {
-            pad4(w);
-            w[sc.o_warp + wi * kWarpTableWords + 0] = (uint32_t)w.size();
-            w[sc.o_warp + wi * kWarpTableWords + 1] = (uint32_t)ops[wi].size();
-            w.insert(w.end(), ops[wi].begin(), ops[wi].end());
-        }
-    };
-    if (!ops_last) put_ops();
+    for (uint32_t wi = 0, first = 0; wi < W; ++wi) {
+        pad4(w);
+        w[sc.o_warp + wi * kWarpTableWords + 0] = (uint32_t)w.size();
+        w[sc.o_warp + wi * kWarpTableWords + 1] = (uint32_t)ops[wi].size();
+        w[sc.o_warp + wi * kWarpTableWords + 4] = first;
+        if (warp_slots) first += (*warp_slots)[wi];
+        w.insert(w.end(), ops[wi].begin(), ops[wi].end());
+    }
     for (uint32_t wi = 0; wi < W; ++wi) {
         w[sc.o_warp + wi * kWarpTableWords + 2] = (uint32_t)w.size();
         w.insert(w.end(), segw[wi].begin(), segw[wi].end());
@@ -342,11 +541,6 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
     sc.o_comb_parts = (uint32_t)w.size();
     w.insert(w.end(), jp.comb_parts.begin(), jp.comb_parts.end());
     while (w.size() % 32) w.push_back(0);  // a multiple of 128 bytes: the regions after it take TMA copies
-    sc.prefix_words = (uint32_t)w.size();
-    if (ops_last) {  // the operation streams after the part copied to shared memory
-        put_ops();
-        while (w.size() % 32) w.push_back(0);
-    }
     return sc;
 }
 
@@ -478,6 +672,191 @@ Lowered resolve(const HostPlan &hp, const NodeInfo &ni, const std::vector<OutWor
     return lw;
 }
 
+// Shared signed sums formed by the warps that use them (Sec. 4.2 "Sharing
+// Signed Sums").  For each warp, every shared sum that the warp's outputs use
+// at least twice is formed once per tile, by that warp, into one of its
+// slots, right before the first scale group that needs it, and read from
+// there by every later use on the warp; a sum's own program may read sums
+// formed before it.  Slots are reused once a sum has no use left in the
+// tile.  Sums a warp uses once, or that would need more than `max_slots`
+// slots, more than six slot operands in one program or runs beyond
+// `budget`, are expanded into their terms (the same residues).  Rewrites the
+// jobs' scale groups (whole outputs only; parts of split outputs keep their
+// expanded terms) and returns the slots per warp and the sums formed per
+// tile.
+struct LocalResult {
+    uint32_t n_slots = 0;              // slots of all warps
+    uint32_t formed = 0;               // sums formed per tile, all warps
+    std::vector<uint32_t> warp_slots;  // per warp
+};
+
+LocalResult localize(JobPlan &jp, const std::vector<OutWork> &groups, const NodeInfo &ni, uint32_t budget,
+                     uint32_t max_slots)
+{
+    LocalResult res;
+    res.warp_slots.assign(jp.per_warp.size(), 0);
+    const size_t n_nodes = ni.kids.size();
+    for (size_t wi = 0; wi < jp.per_warp.size(); ++wi) {
+        auto &jobs = jp.per_warp[wi];
+        std::vector<uint32_t> uses(n_nodes, 0);
+        for (const Job &jb : jobs) {
+            if (jb.target & kPartBit) continue;
+            for (const Seg &g : groups[jb.target].segs)
+                for (const auto *l : {&g.plus, &g.minus})
+                    for (uint32_t o : *l)
+                        if (o & kNodeTag) ++uses[o & ~kNodeTag];
+        }
+        std::vector<char> local(n_nodes, 0);
+        bool any = false;
+        for (size_t k = 0; k < n_nodes; ++k)
+            if (uses[k] >= 2) local[k] = any = 1;
+        if (!any) continue;
+        // operands of an unresolved list against the local set
+        struct Res {
+            std::vector<uint32_t> plus, minus, np, nm;  // sources; local sums (plan node ids)
+        };
+        std::function<void(uint32_t, int, Res &)> expand = [&](uint32_t o, int sign, Res &r) {
+            if (!(o & kNodeTag)) {
+                (sign < 0 ? r.minus : r.plus).push_back(o);
+                return;
+            }
+            const uint32_t k = o & ~kNodeTag;
+            if (local[k]) {
+                (sign < 0 ? r.nm : r.np).push_back(k);
+                return;
+            }
+            for (auto &c : ni.kids[k]) expand(c.first, sign * c.second, r);
+        };
+        for (int round = 0; round < 64; ++round) {
+            // every scale group of the warp's whole outputs, in stream order
+            std::vector<Res> segres;
+            std::vector<uint32_t> seg_job, seg_grp;
+            for (uint32_t ji = 0; ji < jobs.size(); ++ji) {
+                if (jobs[ji].target & kPartBit) continue;
+                const auto &gs = groups[jobs[ji].target].segs;
+                for (uint32_t gi = 0; gi < gs.size(); ++gi) {
+                    Res r;
+                    for (uint32_t o : gs[gi].plus) expand(o, +1, r);
+                    for (uint32_t o : gs[gi].minus) expand(o, -1, r);
+                    segres.push_back(std::move(r));
+                    seg_job.push_back(ji);
+                    seg_grp.push_back(gi);
+                }
+            }
+            std::vector<Res> nodres(n_nodes);
+            for (size_t k = 0; k < n_nodes; ++k)
+                if (local[k])
+                    for (auto &c : ni.kids[k]) expand(c.first, c.second, nodres[k]);
+            // formation points (children first) and last uses
+            std::vector<int> formed_at(n_nodes, -1), last(n_nodes, -1);
+            std::vector<std::vector<uint32_t>> forms(segres.size());
+            std::function<void(uint32_t, int)> need = [&](uint32_t k, int si) {
+                last[k] = std::max(last[k], si);
+                if (formed_at[k] >= 0) return;
+                for (uint32_t c : nodres[k].np) need(c, si);
+                for (uint32_t c : nodres[k].nm) need(c, si);
+                formed_at[k] = si;
+                forms[si].push_back(k);
+            };
+            for (int si = 0; si < (int)segres.size(); ++si) {
+                for (uint32_t k : segres[si].np) need(k, si);
+                for (uint32_t k : segres[si].nm) need(k, si);
+            }
+            // constraints: six slot operands a program, runs within the budget
+            int bad = -1;
+            auto check = [&](const Res &r, bool is_node) {
+                if (r.np.size() + r.nm.size() > 6) return false;
+                if (is_node && (r.plus.size() + r.np.size() > budget || r.minus.size() + r.nm.size() > budget))
+                    return false;
+                return true;
+            };
+            for (size_t k = 0; k < n_nodes && bad < 0; ++k)
+                if (local[k] && formed_at[k] >= 0 && !check(nodres[k], true)) bad = (int)k;
+            for (size_t si = 0; si < segres.size() && bad < 0; ++si)
+                if (!check(segres[si], false)) {
+                    const auto &r = segres[si];
+                    bad = (int)(r.np.empty() ? r.nm.back() : r.np.back());
+                }
+            // slots by lifetime
+            std::vector<int> slot(n_nodes, -1);
+            uint32_t live_max = 0;
+            if (bad < 0) {
+                std::vector<char> busy(16, 0);
+                for (int si = 0; si < (int)segres.size() && bad < 0; ++si) {
+                    for (uint32_t k : forms[si]) {
+                        int f = -1;
+                        for (uint32_t x = 0; x < max_slots; ++x)
+                            if (!busy[x]) {
+                                f = (int)x;
+                                break;
+                            }
+                        if (f < 0) {
+                            bad = (int)k;
+                            break;
+                        }
+                        busy[f] = 1;
+                        slot[k] = f;
+                        live_max = std::max(live_max, (uint32_t)f + 1);
+                    }
+                    for (size_t k = 0; k < n_nodes; ++k)
+                        if (slot[k] >= 0 && last[k] == si && busy[slot[k]]) busy[slot[k]] = 0;
+                }
+            }
+            if (bad >= 0) {  // expand the offending sum and try again
+                local[bad] = 0;
+                continue;
+            }
+            // rewrite the scale groups of the warp's whole outputs
+            std::vector<std::vector<Seg>> newsegs(jobs.size());
+            for (size_t si = 0; si < segres.size(); ++si) {
+                const Res &r = segres[si];
+                const uint32_t ji = seg_job[si];
+                const Seg &g = groups[jobs[ji].target].segs[seg_grp[si]];
+                std::vector<Form> fs;
+                for (uint32_t k : forms[si]) {
+                    Form f;
+                    f.slot = (uint32_t)slot[k];
+                    f.plus = nodres[k].plus;
+                    f.minus = nodres[k].minus;
+                    for (uint32_t c : nodres[k].np) f.plus_slots.push_back((uint32_t)slot[c]);
+                    for (uint32_t c : nodres[k].nm) f.minus_slots.push_back((uint32_t)slot[c]);
+                    fs.push_back(std::move(f));
+                }
+                std::vector<uint32_t> ps, ms;
+                for (uint32_t k : r.np) ps.push_back((uint32_t)slot[k]);
+                for (uint32_t k : r.nm) ms.push_back((uint32_t)slot[k]);
+                if (r.plus.empty() && r.minus.empty() && ps.empty() && ms.empty() && fs.empty()) continue;
+                size_t pb = 0, mb = 0;
+                bool first = true;
+                do {  // runs of at most `budget` operands, slot operands in the first piece
+                    Seg piece;
+                    piece.scale_pt = g.scale_pt;
+                    if (first) {
+                        piece.plus_slots = ps;
+                        piece.minus_slots = ms;
+                        piece.forms = std::move(fs);
+                    }
+                    const size_t pe = std::min(r.plus.size(), pb + budget - piece.plus_slots.size());
+                    const size_t me = std::min(r.minus.size(), mb + budget - piece.minus_slots.size());
+                    piece.plus.assign(r.plus.begin() + pb, r.plus.begin() + pe);
+                    piece.minus.assign(r.minus.begin() + mb, r.minus.begin() + me);
+                    pb = pe;
+                    mb = me;
+                    first = false;
+                    newsegs[ji].push_back(std::move(piece));
+                } while (pb < r.plus.size() || mb < r.minus.size());
+            }
+            for (uint32_t ji = 0; ji < jobs.size(); ++ji)
+                if (!(jobs[ji].target & kPartBit)) jobs[ji].w.segs = std::move(newsegs[ji]);
+            for (size_t k = 0; k < n_nodes; ++k) res.formed += formed_at[k] >= 0 ? 1 : 0;
+            res.warp_slots[wi] = live_max;
+            res.n_slots += live_max;
+            break;
+        }
+    }
+    return res;
+}
+
 int upload_blob(TiledSchedule *ts, const std::vector<uint32_t> &words)
 {
     const size_t bytes = std::max<size_t>(words.size() * 4, 256);
@@ -503,7 +882,8 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
         return "input boxes";
     const uint32_t n_src = a.n_in + a.n_nodes, zero = n_src;  // the zero tile follows the sources
     if (n_src + 1 > kOpMaxSources) return "too many sources";
-    if ((size_t)a.sched_bytes + (size_t)(a.double_buffer ? 2 : 1) * a.src_bytes + (size_t)a.n_part * PB + 24 >
+    if ((size_t)a.sched_bytes + (size_t)(a.double_buffer ? 2 : 1) * a.src_bytes + (size_t)a.n_part * PB +
+            (size_t)a.n_slots * PB + 24 >
         smem)
         return "shared-memory layout";
     if (a.src_bytes != (n_src + 1) * PB) return "source region size";
@@ -512,8 +892,9 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
         v = w[i];
         return true;
     };
-    // a signed-sum program at word `o` whose indices must be below `lim`
-    auto program = [&](size_t o, uint32_t lim, size_t end, size_t &next) -> bool {
+    // a signed-sum program at word `o` whose indices must be below `lim` and
+    // whose slot numbers below `slot_lim`
+    auto program = [&](size_t o, uint32_t lim, size_t end, size_t &next, uint32_t slot_lim) -> bool {
         uint32_t h;
         if (o >= end || !at(o, h)) return false;
         const uint32_t np = h & 0xffffu, nm = h >> 16;
@@ -527,7 +908,13 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
                 ++p;
             }
         }
-        next = p;
+        uint32_t sw;
+        if (p >= end || !at(p, sw)) return false;
+        const uint32_t ns = (sw & 15u) + ((sw >> 4) & 15u);
+        if (ns > 6 || (ns < 6 && (sw >> (8 + 4 * ns)) != 0)) return false;
+        for (uint32_t j = 0; j < ns; ++j)
+            if (((sw >> (8 + 4 * j)) & 15u) >= slot_lim) return false;
+        next = p + 1;
         return true;
     };
     // levels and node programs
@@ -542,7 +929,7 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
             uint32_t off;
             size_t next;
             // a node reads inputs and nodes of lower levels only
-            if (!at(a.o_node_off + x, off) || !program(off, a.n_in + w[a.o_level + l], a.o_warp, next))
+            if (!at(a.o_node_off + x, off) || !program(off, a.n_in + w[a.o_level + l], a.o_warp, next, 0))
                 return "node program";
         }
     // warp streams
@@ -551,6 +938,10 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
         if (t + kWarpTableWords > nw) return "warp table";
         const uint32_t op0 = w[t], n_ops = w[t + 1], seg0 = w[t + 2], tg0 = w[t + 3];
         if (op0 % 4 || n_ops % P || (size_t)op0 + n_ops > nw) return "op stream";
+        // this warp's slots: from its first to the next warp's first (or the end)
+        const uint32_t sl0 = w[t + 4], sl1 = wi + 1 < W ? w[t + kWarpTableWords + 4] : a.n_slots;
+        if (sl1 < sl0 || sl1 > a.n_slots) return "warp slot table";
+        const uint32_t n_wslots = sl1 - sl0;
         size_t sp = seg0, tp = tg0;
         const size_t seg_end = wi + 1 < W ? w[t + kWarpTableWords + 2] : w[a.o_warp + 3];
         const size_t tg_end = wi + 1 < W ? w[t + kWarpTableWords + 3] : a.o_comb_off;
@@ -568,7 +959,13 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
                 if ((op & (kOpMaxSources - 1)) != zero) return "NOP source";
             } else if (op & kOpSeg) {
                 size_t next;
-                if (!program(sp, n_src, seg_end, next)) return "segment program";
+                for (uint32_t f = 0; f < (op & (kOpMaxSources - 1)); ++f) {  // formations into warp slots
+                    uint32_t slot;
+                    if (sp >= seg_end || !at(sp, slot) || slot >= n_wslots) return "formation slot";
+                    if (!program(sp + 1, n_src, seg_end, next, n_wslots)) return "formation program";
+                    sp = next;
+                }
+                if (!program(sp, n_src, seg_end, next, n_wslots)) return "segment program";
                 sp = next;
                 open = true;
             } else {
@@ -635,11 +1032,15 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
         for (uint32_t i = 0; i < n; ++i) add(e, src[(w[p + i / 2] >> (16 * (i & 1))) & 0xffffu], f);
         p += (n + 1) / 2;
     };
+    std::vector<Expr> slot(std::max<uint32_t>(a.n_slots, 1));  // the current warp's slots
     // a signed-sum program at word p; p is left past it
     auto program = [&](size_t &p, Expr &e) {
         const uint32_t h = w[p++];
         run(p, h & 0xffffu, e, 1);
         run(p, h >> 16, e, -1);
+        const uint32_t sw = w[p++];
+        const uint32_t nps = sw & 15u, ns = nps + ((sw >> 4) & 15u);
+        for (uint32_t j = 0; j < ns; ++j) add(e, slot[(sw >> (8 + 4 * j)) & 15u], j < nps ? 1 : -1);
     };
     for (uint32_t x = 0; x < a.n_nodes; ++x) {
         size_t p = w[a.o_node_off + x];
@@ -656,9 +1057,16 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
         const uint32_t op0 = w[t], n_ops = w[t + 1];
         size_t sp = w[t + 2], tp = w[t + 3];
         Map job;
+        for (auto &x : slot) x.clear();  // a warp's slots are its own
         for (uint32_t f = 0; f < n_ops; ++f) {
             const uint32_t op = w[op0 + f], pt = op >> kOpPtShift;
             if (op & kOpSeg) {
+                for (uint32_t g = 0; g < (op & (kOpMaxSources - 1)); ++g) {
+                    const uint32_t sl = w[sp++];
+                    Expr u;
+                    program(sp, u);
+                    slot[sl] = std::move(u);
+                }
                 Expr e;
                 program(sp, e);
                 for (auto &x : e) put(job, {pt, x.first}, x.second);
@@ -742,7 +1150,7 @@ int lower_ws(fiona_plan *p, const NodeInfo &ni, const std::vector<OutWork> &grou
                 const JobPlan jp = build_jobs(lw.work, W, k, P);
                 const Sched sc = encode(jp, lw.level_off, lw.nodes, W, mac_budget, hp.n_in, P);
                 const uint32_t src_bytes = (hp.n_in + 1) * PB;
-                const WsLayout lay((uint32_t)sc.w.size() * 4, nbuf, src_bytes, jp.n_part, W, D, P, TB);
+                const WsLayout lay((uint32_t)sc.w.size() * 4, nbuf, src_bytes, jp.n_part, W, D, P, TB, 0);
                 if (lay.total > smem_cap) continue;
                 const uint32_t threads = (W + 1) * 32;
                 const uint32_t warps_alloc = (threads / 32 + 3) & ~3u;  // registers go to warps in fours
@@ -938,6 +1346,20 @@ int lower_tiled(fiona_plan *p)
         if (save < 0.30 * opnds) rank.clear();
     }
 
+    // -- outputs sharing signed sums, to be placed on one warp each
+    Sharing sharing;
+    sharing.users.resize(hp.n_nodes);
+    sharing.benefit = ni.benefit;
+    for (uint32_t j = 0; j < hp.n_out; ++j)
+        for (const Seg &g : groups[j].segs)
+            for (const auto *l : {&g.plus, &g.minus})
+                for (uint32_t o : *l)
+                    if (o & kNodeTag) {
+                        auto &us = sharing.users[o & ~kNodeTag];
+                        if (us.empty() || us.back() != j) us.push_back(j);
+                    }
+    const Sharing *sh = ni.ids.empty() ? nullptr : &sharing;
+
     // -- shape search
     const size_t smem_cap = (ctx->smem_optin ? ctx->smem_optin : 227 * 1024) - 256;
     const size_t per_sm = 228 * 1024;
@@ -969,14 +1391,20 @@ int lower_tiled(fiona_plan *p)
             continue;
         }
         const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
-        for (uint32_t W : {16u, 12u, 8u, 4u}) {
+        for (uint32_t W : {16u, 12u, 8u, 4u, 2u, 1u}) {
+            // one or two warps only when the tuning override asks for them
+            if (W < 4) {
+                const char *env = getenv("FIONA_TILED_SHAPE");
+                int fc = 0, fw = 0;
+                if (!env || sscanf(env, "%d,%d", &fc, &fw) != 2 || fw != (int)W) continue;
+            }
             for (bool dbl : {true, false}) {
                 if (dbl && hp.n_in == 0) continue;
                 const uint32_t nbuf = dbl ? 2 : 1;
                 // most shared sums that fit: smem grows with each kept sum
                 auto smem_for = [&](uint32_t keep, Lowered &lw, JobPlan &jp, Sched &sc) {
                     lw = resolve(hp, ni, groups, rank, keep, budget);
-                    jp = build_jobs(lw.work, W, k, batch);
+                    jp = build_jobs(lw.work, W, k, batch, keep ? nullptr : sh);
                     sc = encode(jp, lw.level_off, lw.nodes, W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(),
                                 batch);
                     const uint32_t n_src = hp.n_in + (uint32_t)lw.nodes.size() + 1;  // + the zero tile
@@ -1077,12 +1505,66 @@ int lower_tiled(fiona_plan *p)
     const uint32_t T = 32u * best.C, PB = 2 * T * 8;
     const Costs k = costs_for(best.C, narrow);
     const Lowered lw = resolve(hp, ni, groups, rank, best.keep, budget);
-    const JobPlan jp = build_jobs(lw.work, best.W, k, best.P);
-    const Sched sc =
-        encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(), best.P);
+    JobPlan jp = build_jobs(lw.work, best.W, k, best.P, best.keep ? nullptr : sh);
+    // shared sums formed by the warps that use them, when no sum is formed
+    // for the whole block and the warps' slots fit in shared memory
+    LocalResult loc;
+    // (a tuning override with a fourth field selects the block-level sums instead)
+    if (!best.keep && sh && !force_keep && !getenv("FIONA_NO_WARP_SUMS")) {
+        for (uint32_t max_slots = 8; max_slots >= 1; max_slots /= 2) {
+            JobPlan jt = jp;
+            LocalResult r = localize(jt, groups, ni, budget, max_slots);
+            const Sched st = encode(jt, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in, best.P, &r.warp_slots);
+            const size_t sm = st.w.size() * 4 + (size_t)(hp.n_in + 1) * PB * (best.dbl ? 2 : 1) +
+                              (size_t)jt.n_part * PB + (size_t)r.n_slots * PB + 32;
+            if (getenv("FIONA_TILED_DEBUG"))
+                fprintf(stderr, "warp sums: max_slots=%u formed=%u slots=%u smem=%zu cap=%zu\n", max_slots, r.formed,
+                        r.n_slots, sm, smem_cap);
+            if (!r.formed) break;
+            // warps whose slots do not fit give up theirs (largest first)
+            size_t over = sm > smem_cap - 64 ? sm - (smem_cap - 64) : 0;
+            const size_t per_cta = per_sm / std::max(best.ctas, 1u);
+            if (sm + 1024 > per_cta) over = std::max(over, sm + 1024 - per_cta);
+            if (over && max_slots > 1) continue;
+            if (over) {  // one slot a warp: drop warps until the rest fit
+                std::vector<uint32_t> keep_w(best.W, 1);
+                size_t freed = 0;
+                for (uint32_t wi = 0; wi < best.W && freed < over; ++wi)
+                    if (r.warp_slots[wi]) {
+                        keep_w[wi] = 0;
+                        freed += PB;
+                    }
+                if (freed < over) break;
+                JobPlan jk = jp;
+                std::vector<std::vector<Job>> saved = jk.per_warp;
+                r = localize(jk, groups, ni, budget, 1);
+                for (uint32_t wi = 0; wi < best.W; ++wi)
+                    if (!keep_w[wi]) {  // this warp keeps its expanded groups
+                        jk.per_warp[wi] = saved[wi];
+                        r.n_slots -= r.warp_slots[wi];
+                        r.warp_slots[wi] = 0;
+                    }
+                r.formed = 0;  // recount from the schedule below
+                jt = std::move(jk);
+            }
+            jp = std::move(jt);
+            loc = r;
+            break;
+        }
+    }
+    const Sched sc = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(),
+                            best.P, loc.warp_slots.empty() ? nullptr : &loc.warp_slots);
+    if (!loc.warp_slots.empty()) {  // sums formed per tile, from the schedule's formations
+        loc.formed = 0;
+        for (uint32_t wi = 0; wi < best.W; ++wi) {
+            const uint32_t op0 = sc.w[sc.o_warp + wi * kWarpTableWords];
+            const uint32_t n = sc.w[sc.o_warp + wi * kWarpTableWords + 1];
+            for (uint32_t f = 0; f < n; ++f)
+                if (sc.w[op0 + f] & kOpSeg) loc.formed += sc.w[op0 + f] & (kOpMaxSources - 1);
+        }
+    }
     best.smem = sc.w.size() * 4 + (size_t)(hp.n_in + lw.nodes.size() + 1) * PB * (best.dbl ? 2 : 1) +
-                (size_t)jp.n_part * PB + 32;
-
+                (size_t)jp.n_part * PB + (size_t)loc.n_slots * PB + 32;
     TiledSchedule *ts = new (std::nothrow) TiledSchedule;
     if (!ts) return set_error(FIONA_ERR_NOMEM, "tiled schedule: host allocation");
     ts->C = best.C;
@@ -1093,9 +1575,10 @@ int lower_tiled(fiona_plan *p)
     ts->has_const = has_const;
     ts->smem = best.smem;
     ts->ctas_per_sm = best.ctas;
-    ts->nodes_kept = (uint32_t)lw.nodes.size();
-    ts->nodes_expanded = (uint32_t)ni.ids.size() - ts->nodes_kept;
+    ts->nodes_kept = (uint32_t)lw.nodes.size() + loc.formed;
+    ts->nodes_expanded = (uint32_t)ni.ids.size() - std::min<uint32_t>((uint32_t)ni.ids.size(), ts->nodes_kept);
     TiledArgs &a = ts->args;
+    a.n_slots = loc.n_slots;
     a.o_level = sc.o_level;
     a.o_node_off = sc.o_node_off;
     a.o_warp = sc.o_warp;

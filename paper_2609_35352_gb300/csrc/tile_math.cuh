@@ -193,27 +193,44 @@ __device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32
     return wp;
 }
 
-// Signed sum of the program at byte offset `hdr` (n_plus | n_minus << 16,
-// then the plus run, then the minus run), both polys, as canonical residues;
-// SPLIT: the sources are in split form (else canonical, whatever the
-// arithmetic).  Returns the offset just past the program.
+// Signed sum of the program at byte offset `hdr`, both polys, as canonical
+// residues; SPLIT: the sources are in split form (else canonical, whatever
+// the arithmetic).  A program is n_plus | n_minus << 16, the plus run, the
+// minus run, then one slot word: n_plus_slots | n_minus_slots << 4 and up to
+// six 4-bit slot numbers from bit 8 (plus slots first).  A slot is a tile
+// pair of this warp's slot area at byte offset `slots` (this lane's words
+// of slot 0), holding a shared signed sum the warp formed earlier.  Returns
+// the offset just past the program.
 template <bool SPLIT, int C, uint32_t TB>
 __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uint32_t hdr, uint32_t lim,
-                                               V<C> &o0, V<C> &o1)
+                                               uint32_t slots, V<C> &o0, V<C> &o1)
 {
     using A = Arith<SPLIT>;
+    constexpr uint32_t PB = 2 * TB;
     const uint32_t h = *reinterpret_cast<const uint32_t *>(sm + hdr);
     V<C> p0{}, p1{}, m0{}, m1{};
     uint32_t wp = run_sum<C, TB>(sm, src, hdr + 4, h & 0xffffu, p0, p1);
     wp = run_sum<C, TB>(sm, src, wp, h >> 16, m0, m1);
+    const uint32_t sw = *reinterpret_cast<const uint32_t *>(sm + wp);
+    const uint32_t nps = sw & 15u, ns = nps + ((sw >> 4) & 15u);
+    for (uint32_t j = 0; j < ns; ++j) {
+        const uint32_t o = slots + ((sw >> (8 + 4 * j)) & 15u) * PB;
+        const V<C> a = lds<C>(sm, o), b = lds<C>(sm, o + TB);
+        V<C> &t0 = j < nps ? p0 : m0;
+        V<C> &t1 = j < nps ? p1 : m1;
+#pragma unroll
+        for (int x = 0; x < C; ++x) {
+            t0.x[x] += a.x[x];
+            t1.x[x] += b.x[x];
+        }
+    }
     const LimbConst m = load_limb(lim);
 #pragma unroll
     for (int x = 0; x < C; ++x) {
         o0.x[x] = A::signed_value(p0.x[x], m0.x[x], m);
         o1.x[x] = A::signed_value(p1.x[x], m1.x[x], m);
     }
-    return wp;
+    return wp + 4;
 }
-
 
 }  // namespace tile

@@ -34,14 +34,18 @@
 //                   source indices, two 16-bit indices per word (each run
 //                   starts on a new word)
 //   warp table      per warp: op stream offset, op count (a multiple of the
-//                   prefetch depth), segment stream offset, target offset
+//                   prefetch depth), segment stream offset, target offset,
+//                   first warp slot (then padding to eight words)
 //   op streams      one word per operation (layout below)
 //   segment streams per SEG operation, in order: a program as above
 //   target streams  per job: output index, or kPartBit | partial slot
 //   combine lists   per split output: its partial slots
 // Source index s names the tile pair (c0, c1) at s * 2T words of the source
 // region: inputs first, then the materialised shared sums in level order,
-// then the zero tile.
+// then the zero tile.  Programs name warp slots in their slot word (see
+// tile_math.cuh signed_sum); a warp's slots are tile pairs of its own, after
+// the partial slots, written and read only by that warp (each lane its own
+// coefficients).
 #pragma once
 #include <stdint.h>
 
@@ -54,7 +58,10 @@ constexpr uint32_t kPartBit = 0x80000000u;  // job target: partial slot
 
 // operation word: [31:14] plaintext index, [13:9] flags, [8:0] source index.
 // CONST marks a raw term whose plaintext is constant over the coefficients
-// (FIONA_TERM_RAW_CONST): its load reads residue 0 of the limb.
+// (FIONA_TERM_RAW_CONST): its load reads residue 0 of the limb.  A SEG's
+// [8:0] is instead the number of shared signed sums the warp forms into its
+// slots before the SEG's own sum: its segment-stream entry is that many
+// (slot number, program) pairs, then the SEG's program.
 constexpr uint32_t kOpSrcBits = 9;
 constexpr uint32_t kOpMaxSources = 1u << kOpSrcBits;
 constexpr uint32_t kOpSeg = 1u << 9;
@@ -65,7 +72,8 @@ constexpr uint32_t kOpConst = 1u << 13;
 constexpr uint32_t kOpPtShift = 14;
 constexpr uint32_t kOpMaxPlaintexts = 1u << (32 - kOpPtShift);
 
-constexpr uint32_t kWarpTableWords = 4;  // op offset, op count, seg offset, target offset
+// per warp: op offset, op count, seg offset, target offset, first slot
+constexpr uint32_t kWarpTableWords = 8;
 
 struct TiledArgs {
     const uint64_t *in;
@@ -87,6 +95,8 @@ struct TiledArgs {
     uint32_t n_boxes;
     uint32_t double_buffer;  // 1: two source regions, next tile staged early
     uint32_t has_pt;         // 0: the plan has no plaintexts (every load reads the schedule)
+    uint32_t n_slots;        // warp slots of the CTA (shared signed sums a warp forms for itself);
+                             // a warp's own start at the slot its table entry names
 };
 
 // Warp-specialised variant (kernel_ws.cu), two coefficients per lane.  The
@@ -119,22 +129,24 @@ struct WsArgs {
     uint32_t n_buf;          // source regions (1 or 2)
     uint32_t has_pt;
     uint32_t flags;          // kWsFlag*
+    uint32_t n_slots;        // warp slots of the CTA (a warp's own start where its table entry says)
 };
 
 // Shared-memory layout of the warp-specialised kernel (byte offsets), the
 // same on the host and in the kernel.
 struct WsLayout {
-    uint32_t src0, part0, ring0, bar0, total;
+    uint32_t src0, part0, ring0, slot0, bar0, total;
 #if defined(__CUDACC__)
     __host__ __device__
 #endif
     WsLayout(uint32_t sched_bytes, uint32_t n_buf, uint32_t src_bytes, uint32_t n_part, uint32_t W, uint32_t D,
-             uint32_t P, uint32_t TB)
+             uint32_t P, uint32_t TB, uint32_t S)
     {
         src0 = sched_bytes;
         part0 = src0 + n_buf * src_bytes;
         ring0 = part0 + 2 * n_part * 2 * TB;
-        bar0 = ring0 + W * D * P * TB;
+        slot0 = ring0 + W * D * P * TB;
+        bar0 = slot0 + S * 2 * TB;
         total = bar0 + 8 * 8;
     }
 };

@@ -85,3 +85,21 @@ def test_long_signed_runs_are_cut_and_still_exact():
     desc = F.compile_plan(n_in, n_out, 3 + 20, r, share=False)
     plan = lower(desc, 4096, 50, 2)
     assert plan.stats()["kernel"] == F.FIONA_KERNEL_TILED
+
+
+def test_warp_formed_sums_lower_exactly(monkeypatch):
+    """Random compiled layers on one, two or four warps, so that the users of
+    shared signed sums often share a warp: the warps form those sums into
+    their slots (nested sums included, children first), and the symbolic
+    check of every schedule against the plan's terms passes (plan creation
+    fails otherwise).  Sums are formed wherever their slots fit without
+    lowering the planned occupancy, which most of these layers allow."""
+    formed = []
+    for seed in range(24):
+        rng = np.random.default_rng(9100 + seed)
+        monkeypatch.setenv("FIONA_TILED_SHAPE", ["2,1,1", "2,2,0", "1,2,1", "1,4,0"][seed % 4])
+        desc = random_layer(rng, big=False)
+        bits = int(rng.choice([40, 50, 59]))
+        plan = lower(desc, 4096, bits, 2)
+        formed.append(plan.stats()["nodes_materialized"])
+    assert sum(1 for f in formed if f > 0) >= 12, formed

@@ -362,3 +362,28 @@ def test_largest_ring_dimension(bits, L):
         dl.d_out.fill_(-1)
         dl.run()
         assert np.array_equal(dl.outputs(), want), kernel
+
+
+@pytest.mark.parametrize("name,N,L,shape", [("tiny-dag", None, None, "2,1,1"), ("tiny-dag", None, None, "1,2,0"),
+                                            ("worked-example", None, None, "2,1,1"),
+                                            ("vit", 2048, 2, "2,4,1"), ("vit", 2048, 2, "1,4,1,-1,16"),
+                                            ("bert", 1024, 1, "2,8,1"), ("bert", 1024, 1, None),
+                                            ("overflow60", None, None, "2,2,1")])
+def test_warp_formed_sums(name, N, L, shape, monkeypatch):
+    """Shared signed sums formed once per tile by the warp whose outputs use
+    them (Sec. 4.2 "Sharing Signed Sums"), read back from the warp's slots:
+    the plan reports them formed and every residue equals the oracle's."""
+    if shape:
+        monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+    wl = W.make_workload(name, N=N, L=L)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel("tiled")
+    st = dl.plan.stats()
+    if name != "overflow60":
+        assert st["nodes_materialized"] > 0, st
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    for _ in range(2):
+        dl.run()
+        mism = np.argwhere(dl.outputs() != want)
+        assert mism.shape[0] == 0, "first mismatches (j, c, l, k): %s" % mism[:5].tolist()
+    assert dl.ctx.device_check() == F.FIONA_OK
