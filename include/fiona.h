@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define FIONA_ABI_VERSION 1
+#define FIONA_ABI_VERSION 2
 
 typedef struct fiona_ctx fiona_ctx;   /* N, RNS moduli, per-limb constants on one device */
 typedef struct fiona_plan fiona_plan; /* one validated, lowered linear layer */
@@ -153,9 +153,14 @@ typedef struct fiona_plan_stats_t {
     uint32_t smem_bytes;          /* dynamic shared memory per CTA                          */
     uint32_t ctas_per_sm;         /* occupancy the lowering planned for                     */
     uint32_t kernel;              /* variant in use: FIONA_KERNEL_DIRECT or FIONA_KERNEL_TILED */
-    uint32_t nodes_materialized;  /* TILED: shared sums formed once per tile (the others are
-                                     expanded into their uses: same residues, more Add/Sub) */
-    uint32_t reserved[4];
+    uint32_t nodes_materialized;  /* TILED: shared sums formed once per tile, by the block or
+                                     by the warp whose outputs use them (a sum several warps
+                                     use counts once per warp); the others are expanded into
+                                     their uses: same residues, more Add/Sub */
+    uint32_t addsub_executed;     /* Add/Sub of the kernel in use, in the units of addsub_flat:
+                                     each sum of n operands it forms (shared sums, scale groups,
+                                     an output's products, its partial sums) counts n - 1 */
+    uint32_t reserved[3];
 } fiona_plan_stats_t;
 
 /* Create a context for ring dimension N (a power of two, 2^10 <= N <= 2^17)

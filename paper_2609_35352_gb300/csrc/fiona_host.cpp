@@ -572,6 +572,7 @@ static int select_kernel(fiona_plan *p, int which)
         s.smem_bytes = (uint32_t)p->tiled->smem;
         s.ctas_per_sm = p->tiled->ctas_per_sm;
         s.nodes_materialized = p->tiled->nodes_kept;
+        s.addsub_executed = p->tiled->addsub;
     } else {
         s.kernel = FIONA_KERNEL_DIRECT;
         s.tile_coeffs = 256;
@@ -579,6 +580,7 @@ static int select_kernel(fiona_plan *p, int which)
         s.smem_bytes = 0;
         s.ctas_per_sm = 0;
         s.nodes_materialized = 0;
+        s.addsub_executed = (uint32_t)std::min<uint64_t>(s.addsub_flat, 0xffffffffu);
     }
     return FIONA_OK;
 }

@@ -857,6 +857,50 @@ LocalResult localize(JobPlan &jp, const std::vector<OutWork> &groups, const Node
     return res;
 }
 
+// Add/Sub a schedule performs per evaluation, in the units of the paper's
+// counts (a sum of n operands costs n - 1): the shared sums formed for the
+// block and by warps, every scale group's signed sum, each job's products
+// added together, and the partial sums of split outputs.
+uint32_t count_addsub(const std::vector<uint32_t> &w, const TiledArgs &a, uint32_t W)
+{
+    uint64_t n = 0;
+    auto program = [&](size_t &p) {  // operands of the program at word p; p is left past it
+        const uint32_t h = w[p++];
+        const uint32_t np = h & 0xffffu, nm = h >> 16;
+        p += (np + 1) / 2 + (nm + 1) / 2;
+        const uint32_t sw = w[p++];
+        return (uint64_t)np + nm + (sw & 15u) + ((sw >> 4) & 15u);
+    };
+    for (uint32_t x = 0; x < a.n_nodes; ++x) {
+        size_t p = w[a.o_node_off + x];
+        n += program(p) - 1;
+    }
+    for (uint32_t wi = 0; wi < W; ++wi) {
+        const size_t t = a.o_warp + (size_t)wi * kWarpTableWords;
+        const uint32_t op0 = w[t], n_ops = w[t + 1];
+        size_t sp = w[t + 2];
+        uint64_t products = 0;
+        for (uint32_t f = 0; f < n_ops; ++f) {
+            const uint32_t op = w[op0 + f];
+            if (op & kOpSeg) {
+                for (uint32_t g = 0; g < (op & (kOpMaxSources - 1)); ++g) {
+                    ++sp;  // the slot
+                    n += program(sp) - 1;
+                }
+                const uint64_t k = program(sp);
+                if (k) n += k - 1;
+            }
+            if (!(op & kOpNop)) ++products;
+            if (op & kOpLast) {
+                if (products) n += products - 1;
+                products = 0;
+            }
+        }
+    }
+    for (uint32_t r = 0; r < a.n_comb; ++r) n += w[a.o_comb_off + r + 1] - w[a.o_comb_off + r] - 1;
+    return (uint32_t)std::min<uint64_t>(n, 0xffffffffu);
+}
+
 int upload_blob(TiledSchedule *ts, const std::vector<uint32_t> &words)
 {
     const size_t bytes = std::max<size_t>(words.size() * 4, 256);
@@ -1224,6 +1268,7 @@ int lower_ws(fiona_plan *p, const NodeInfo &ni, const std::vector<OutWork> &grou
     m.box_rows = a.box_rows;
     m.n_boxes = a.n_boxes;
     const char *why = check_schedule(sc.w, m, best.W, hp.n_out, hp.n_pt, (size_t)1 << 30, PB, P);
+    ts->addsub = count_addsub(sc.w, m, best.W);
     if (!why) why = check_linear_map(sc.w, m, best.W, hp);
     if (why) {
         delete ts;
@@ -1603,6 +1648,7 @@ int lower_tiled(fiona_plan *p)
     a.n_boxes = (2 * hp.n_in + 255) / 256;
     a.box_rows = a.n_boxes ? (2 * hp.n_in + a.n_boxes - 1) / a.n_boxes : 0;
     a.has_pt = hp.n_pt ? 1 : 0;
+    ts->addsub = count_addsub(sc.w, a, best.W);
     if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB, best.P)) {
         delete ts;
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);

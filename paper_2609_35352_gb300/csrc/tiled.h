@@ -160,6 +160,7 @@ struct TiledSchedule {
     bool has_const = false;    // some operation reads a constant plaintext (kOpConst)
     size_t smem = 0;           // dynamic shared memory per CTA
     uint32_t ctas_per_sm = 0;  // occupancy the lowering planned for
+    uint32_t addsub = 0;       // Add/Sub per evaluation (fiona_plan_stats.addsub_executed)
     uint32_t nodes_kept = 0;   // shared sums materialised per tile
     uint32_t nodes_expanded = 0;  // shared sums expanded into their uses
     DeviceSchedule sched;

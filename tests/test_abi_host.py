@@ -36,7 +36,7 @@ def test_library_exports_every_declared_symbol(header, path):
         assert hasattr(lib, n), n
     if header == "fiona.h":
         assert set(F.EXPORTED) <= set(names)
-        assert F.lib().fiona_abi_version() == 1
+        assert F.lib().fiona_abi_version() == 2
 
 
 def ctx_none(N=1024, bits=40, L=3):
@@ -284,3 +284,25 @@ def test_minimal_bytes_counted_alike(name):
     wl = W.make_workload(name)
     s = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan).stats()
     assert W.min_bytes(wl.plan, wl.L, wl.N) == s["bytes_min"]
+
+
+def test_executed_addsub_reaches_the_papers_shared_count(monkeypatch):
+    """The worked example (Sec. 4.2) on one warp: the kernel forms U = A_1 - A_3
+    once and both outputs read it, so the Add/Sub it executes equal the
+    paper's count with sharing (one subtraction saved: 5 -> 4); every other
+    plan lies between the shared and the flat count, and the direct kernel
+    executes the flat count."""
+    monkeypatch.setenv("FIONA_TILED_SHAPE", "2,1,1")
+    wl = W.make_workload("worked-example")
+    plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
+    s = plan.stats()
+    assert s["nodes_materialized"] == 1
+    assert s["addsub_executed"] == s["addsub_shared"] == 4 and s["addsub_flat"] == 5
+    monkeypatch.delenv("FIONA_TILED_SHAPE")
+    for name in ("tiny-dag", "vit", "bert", "vgg"):
+        wl = W.make_workload(name)
+        plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
+        s = plan.stats()
+        assert s["addsub_shared"] <= s["addsub_executed"] <= s["addsub_flat"], (name, s)
+        plan.select_kernel("direct")
+        assert plan.stats()["addsub_executed"] == s["addsub_flat"]
