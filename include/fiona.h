@@ -203,6 +203,31 @@ int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out, uint3
                       uint32_t n_uses, const fiona_sum_use *uses, fiona_plan **out);
 void fiona_plan_destroy(fiona_plan *plan); /* NULL is a no-op */
 
+/* A layer whose plaintexts are encoded at several scales (Sec. 4.2,
+ * "Combining the Signed and Raw Routes": an output's signed and raw routes
+ * are added before its one rescale only when their plaintexts share a scale;
+ * with different scales each must be rescaled on its own).  pt_class[p] in
+ * [0, n_class) is the scale class of plaintext p (a scale group's class is
+ * that of its gamma, a raw term's that of its plaintext).  Output j of the
+ * description becomes n_class results: result j * n_class + s holds the
+ * scale groups and raw terms of output j whose plaintexts have class s,
+ * combined (a class with no term of output j gives a result of zeros).  The
+ * plan then evaluates like any other with n_out * n_class outputs: the output
+ * buffer of fiona_linear_eval (and its variants) is [n_out][n_class][2][L][N],
+ * and fiona_plan_stats counts those results as outputs.  Other arguments and
+ * errors as fiona_plan_create; FIONA_ERR_ARG if n_class is 0 or above 255,
+ * pt_class is null while n_pt > 0, or n_out * n_class exceeds 65535;
+ * FIONA_ERR_PLAN if a class is >= n_class.  n_class = 1 is
+ * fiona_plan_create. */
+int fiona_plan_create_classes(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out, uint32_t n_pt,
+                              const uint32_t *term_offsets, const fiona_term *terms,
+                              uint32_t n_groups, const uint32_t *group_scale_pt,
+                              const uint32_t *group_output,
+                              uint32_t n_nodes, const uint32_t *node_offsets,
+                              const fiona_sum_child *children,
+                              uint32_t n_uses, const fiona_sum_use *uses,
+                              uint32_t n_class, const uint8_t *pt_class, fiona_plan **out);
+
 /* Route of the weights of output j on input i, for the plan compiler.
  * 8 bytes. */
 typedef struct fiona_route {

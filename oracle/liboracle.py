@@ -32,6 +32,8 @@ def _setup(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.oracle_linear_eval.argtypes = [u64, u32, p, u32, u32, u32, p, p, p, p, p, p,
                                        u32, p, p, p, p]
     lib.oracle_linear_eval.restype = ctypes.c_int
+    lib.oracle_linear_eval_classes.argtypes = [u64, u32, p, u32, u32, u32, p, p, p, p, p, p,
+                                               u32, p, u32, p, p, p, p]
     lib.oracle_linear_eval_dag.argtypes = [u64, u32, p, u32, u32, u32, p, p, p, p, p, p,
                                            u32, p, u32, p, p, p, p, u32, p, p, p, p,
                                            p, p, p]
@@ -104,6 +106,30 @@ def linear_eval(plan, moduli, inputs: np.ndarray, plaintexts: np.ndarray,
                                 _ptr(inputs), _ptr(plaintexts), _ptr(out))
     if rc != 0:
         raise ValueError("oracle rejected the plan")
+    return out
+
+
+def linear_eval_classes(plan, moduli, pt_class, n_class: int, inputs: np.ndarray, plaintexts: np.ndarray,
+                        lib: Optional[ctypes.CDLL] = None) -> np.ndarray:
+    """Evaluation with plaintext scale classes: returns [n_out][n_class][2][L][n],
+    output j's terms of class s (by their plaintext) in [j][s]."""
+    lib = lib or load()
+    q = _c(moduli, np.uint64)
+    L = q.shape[0]
+    inputs = _c(inputs, np.uint64)
+    plaintexts = _c(plaintexts, np.uint64)
+    n = inputs.shape[-1] if inputs.ndim == 4 else plaintexts.shape[-1]
+    assert inputs.shape == (plan.n_in, 2, L, n), inputs.shape
+    assert plaintexts.shape == (plan.n_pt, L, n), plaintexts.shape
+    cls = _c(pt_class, np.uint8)
+    assert cls.shape == (plan.n_pt,)
+    out = np.zeros((plan.n_out, n_class, 2, L, n), dtype=np.uint64)
+    arrs = _term_arrays(plan)
+    rc = lib.oracle_linear_eval_classes(n, L, _ptr(q), plan.n_in, plan.n_out, plan.n_pt,
+                                        *[_ptr(a) for a in arrs[:6]], plan.n_groups, _ptr(arrs[6]),
+                                        n_class, _ptr(cls), _ptr(inputs), _ptr(plaintexts), _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle rejected the plan or its classes")
     return out
 
 

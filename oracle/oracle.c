@@ -26,6 +26,14 @@
  * Every operation is reduced at once with 128-bit '%' (schoolbook).  Nothing
  * is blocked, fused, reordered or reduced lazily.
  *
+ * oracle_linear_eval_classes evaluates a layer whose plaintexts carry scale
+ * classes (encoded at different scales).  The two routes of an output are
+ * added only when their plaintexts share a scale (Sec. 4.2, "Combining the
+ * Signed and Raw Routes": the routes are combined before the one rescale of
+ * the output, which needs one common scale), so each (output j, class s) is
+ * its own result: the sum above restricted to the scale groups whose gamma
+ * has class s and the raw terms whose plaintext has class s.
+ *
  * oracle_linear_eval_dag evaluates the same layer through the DAG of shared
  * signed sums (Sec. 4.2, "Sharing Signed Sums", Eq. "shared-example"): each
  * shared sum U is formed once, and an output that uses sigma*U adds it to its
@@ -34,7 +42,7 @@
  * Layouts (row-major uint64):
  *   inputs      [n_in ][2][L][n_coef]
  *   plaintexts  [n_pt ][L][n_coef]
- *   outputs     [n_out][2][L][n_coef]
+ *   outputs     [n_out][2][L][n_coef]   ([n_out][n_class][2][L][n_coef] with classes)
  * Terms of output j are term_*[term_offsets[j] .. term_offsets[j+1]).
  * kind 0 = raw route (uses term_pt), kind 1 = signed route (term_sign in
  * {-1,0,+1}, term_group = scale group whose plaintext is group_scale_pt[g]),
@@ -87,7 +95,7 @@ static uint64_t eval_one(uint32_t j, uint32_t c, uint32_t l, uint64_t k,
                          const uint32_t *group_scale_pt,
                          const uint64_t *inputs, const uint64_t *plaintexts,
                          const uint8_t *covered, const uint64_t *extra_signed,
-                         const uint8_t *group_has_use)
+                         const uint8_t *group_has_use, const uint8_t *pt_class, uint32_t want_class)
 {
     uint64_t y = 0;
     uint32_t e0 = term_offsets[j], e1 = term_offsets[j + 1];
@@ -97,6 +105,8 @@ static uint64_t eval_one(uint32_t j, uint32_t c, uint32_t l, uint64_t k,
         if (term_kind[e] != 1)
             continue;
         uint32_t g = term_group[e];
+        if (pt_class && pt_class[group_scale_pt[g]] != want_class)
+            continue;
         /* visit each scale group once: at its first term in this output */
         int first = 1;
         for (uint32_t f = e0; f < e; ++f)
@@ -127,6 +137,8 @@ static uint64_t eval_one(uint32_t j, uint32_t c, uint32_t l, uint64_t k,
     /* raw route: one PMult per raw group, added at the same scale */
     for (uint32_t e = e0; e < e1; ++e) {
         if (term_kind[e] != 0 && term_kind[e] != 2)
+            continue;
+        if (pt_class && pt_class[term_pt[e]] != want_class)
             continue;
         uint64_t a = inputs[in_idx(term_input[e], c, l, k, L, n_coef)];
         uint64_t p = plaintexts[pt_idx(term_pt[e], l, term_kind[e] == 2 ? 0 : k, L, n_coef)];
@@ -185,7 +197,37 @@ int oracle_linear_eval(uint64_t n_coef, uint32_t L, const uint64_t *moduli,
                     outputs[in_idx(j, c, l, k, L, n_coef)] =
                         eval_one(j, c, l, k, L, n_coef, moduli[l], term_offsets, term_input,
                                  term_kind, term_sign, term_pt, term_group, group_scale_pt,
-                                 inputs, plaintexts, NULL, NULL, NULL);
+                                 inputs, plaintexts, NULL, NULL, NULL, NULL, 0);
+    return 0;
+}
+
+int oracle_linear_eval_classes(uint64_t n_coef, uint32_t L, const uint64_t *moduli,
+                               uint32_t n_in, uint32_t n_out, uint32_t n_pt,
+                               const uint32_t *term_offsets, const uint32_t *term_input,
+                               const int8_t *term_kind, const int8_t *term_sign,
+                               const uint32_t *term_pt, const uint32_t *term_group,
+                               uint32_t n_groups, const uint32_t *group_scale_pt,
+                               uint32_t n_class, const uint8_t *pt_class,
+                               const uint64_t *inputs, const uint64_t *plaintexts,
+                               uint64_t *outputs)
+{
+    if (check_common(L, moduli, n_in, n_out, n_pt, term_offsets, term_input, term_kind,
+                     term_sign, term_pt, term_group, n_groups, group_scale_pt))
+        return -1;
+    if (n_class == 0)
+        return -1;
+    for (uint32_t p = 0; p < n_pt; ++p)
+        if (pt_class[p] >= n_class)
+            return -1;
+    for (uint32_t j = 0; j < n_out; ++j)
+        for (uint32_t s = 0; s < n_class; ++s)
+            for (uint32_t c = 0; c < 2; ++c)
+                for (uint32_t l = 0; l < L; ++l)
+                    for (uint64_t k = 0; k < n_coef; ++k)
+                        outputs[in_idx(j * n_class + s, c, l, k, L, n_coef)] =
+                            eval_one(j, c, l, k, L, n_coef, moduli[l], term_offsets, term_input,
+                                     term_kind, term_sign, term_pt, term_group, group_scale_pt,
+                                     inputs, plaintexts, NULL, NULL, NULL, pt_class, s);
     return 0;
 }
 
@@ -308,7 +350,7 @@ int oracle_linear_eval_dag(uint64_t n_coef, uint32_t L, const uint64_t *moduli,
                     outputs[in_idx(j, c, l, k, L, n_coef)] =
                         eval_one(j, c, l, k, L, n_coef, q, term_offsets, term_input, term_kind,
                                  term_sign, term_pt, term_group, group_scale_pt, inputs,
-                                 plaintexts, covered, extra, has_use);
+                                 plaintexts, covered, extra, has_use, NULL, 0);
                 }
             }
     }

@@ -709,6 +709,60 @@ extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n
     return FIONA_OK;
 }
 
+// Plaintext scale classes: output j of the description becomes results
+// j * n_class + s, each holding the terms of j whose plaintext has class s
+// (a scale group by its gamma); the validation and lowering are those of the
+// expanded layer (Sec. 4.2 "Combining the Signed and Raw Routes": routes are
+// combined within one scale only).
+extern "C" int fiona_plan_create_classes(const fiona_ctx *ctx, uint32_t n_in, uint32_t n_out, uint32_t n_pt,
+                                         const uint32_t *term_offsets, const fiona_term *terms,
+                                         uint32_t n_groups, const uint32_t *group_scale_pt,
+                                         const uint32_t *group_output, uint32_t n_nodes,
+                                         const uint32_t *node_offsets, const fiona_sum_child *children,
+                                         uint32_t n_uses, const fiona_sum_use *uses, uint32_t n_class,
+                                         const uint8_t *pt_class, fiona_plan **out)
+{
+    if (n_class == 0 || n_class > 255) return set_error(FIONA_ERR_ARG, "plan_create_classes: n_class %u", n_class);
+    if (n_class == 1)
+        return fiona_plan_create(ctx, n_in, n_out, n_pt, term_offsets, terms, n_groups, group_scale_pt,
+                                 group_output, n_nodes, node_offsets, children, n_uses, uses, out);
+    if (!ctx || !out || !term_offsets) return set_error(FIONA_ERR_ARG, "plan_create_classes: null argument");
+    if (n_pt && !pt_class) return set_error(FIONA_ERR_ARG, "plan_create_classes: null pt_class");
+    if ((uint64_t)n_out * n_class > 65535) return set_error(FIONA_ERR_ARG, "plan_create_classes: too many results");
+    if ((n_groups && (!group_scale_pt || !group_output)) || (n_uses && !uses))
+        return set_error(FIONA_ERR_ARG, "plan_create_classes: null array with nonzero count");
+    const uint64_t n_terms = term_offsets[n_out];
+    if (n_terms && !terms) return set_error(FIONA_ERR_ARG, "plan_create_classes: null terms");
+    for (uint32_t pi = 0; pi < n_pt; ++pi)
+        if (pt_class[pi] >= n_class)
+            return set_error(FIONA_ERR_PLAN, "plaintext %u has class %u >= %u", pi, pt_class[pi], n_class);
+    // the class of a plaintext index (out-of-range indices are left to the
+    // validation of the expanded plan)
+    auto cls = [&](uint32_t pt) -> uint32_t { return pt < n_pt ? pt_class[pt] : 0; };
+    auto gcls = [&](uint32_t g) -> uint32_t { return g < n_groups ? cls(group_scale_pt[g]) : 0; };
+    for (uint32_t j = 0; j < n_out; ++j)
+        if (term_offsets[j + 1] < term_offsets[j]) return set_error(FIONA_ERR_PLAN, "term_offsets decrease");
+    std::vector<uint32_t> offs(1, 0);
+    std::vector<fiona_term> ts;
+    ts.reserve(n_terms);
+    for (uint32_t j = 0; j < n_out; ++j)
+        for (uint32_t s = 0; s < n_class; ++s) {
+            for (uint32_t e = term_offsets[j]; e < term_offsets[j + 1]; ++e) {
+                const fiona_term &t = terms[e];
+                const uint32_t c = t.kind == FIONA_TERM_TERNARY ? gcls(t.group) : cls(t.pt);
+                if (c == s) ts.push_back(t);
+            }
+            offs.push_back((uint32_t)ts.size());
+        }
+    std::vector<uint32_t> gout(n_groups);
+    for (uint32_t g = 0; g < n_groups; ++g)
+        gout[g] = group_output[g] < n_out ? group_output[g] * n_class + gcls(g) : n_out * n_class;
+    std::vector<fiona_sum_use> us(uses, uses + n_uses);
+    for (auto &u : us) u.output = u.output < n_out ? u.output * n_class + gcls(u.group) : n_out * n_class;
+    return fiona_plan_create(ctx, n_in, n_out * n_class, n_pt, offs.data(), ts.data(), n_groups, group_scale_pt,
+                             gout.data(), n_nodes, node_offsets, children, n_uses, us.data(), out);
+}
+
 extern "C" void fiona_plan_destroy(fiona_plan *p)
 {
     if (!p) return;

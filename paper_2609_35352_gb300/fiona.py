@@ -35,7 +35,8 @@ FIONA_KERNEL_DIRECT = 1
 FIONA_KERNEL_TILED = 2
 KERNELS = {"auto": FIONA_KERNEL_AUTO, "direct": FIONA_KERNEL_DIRECT, "tiled": FIONA_KERNEL_TILED}
 
-EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona_plan_destroy",
+EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona_plan_create_classes",
+            "fiona_plan_destroy",
             "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host",
             "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version",
             "fiona_plan_select_kernel", "fiona_device_check", "fiona_linear_eval_static",
@@ -89,6 +90,8 @@ def lib() -> ctypes.CDLL:
         L.fiona_plan_create.argtypes = [p, u32, u32, u32, p, p, u32, p, p, u32, p, p, u32, p,
                                         ctypes.POINTER(p)]
         L.fiona_plan_create.restype = i32
+        L.fiona_plan_create_classes.argtypes = [p, u32, u32, u32, p, p, u32, p, p, u32, p, p, u32, p, u32, p, p]
+        L.fiona_plan_create_classes.restype = i32
         L.fiona_plan_destroy.argtypes = [p]
         L.fiona_plan_destroy.restype = None
         L.fiona_plan_stats.argtypes = [p, ctypes.POINTER(PlanStats)]
@@ -249,7 +252,10 @@ class Plan:
     n_out, n_pt, term_offsets, terms, group_scale_pt, group_output,
     node_offsets, children and uses (see workloads.Plan)."""
 
-    def __init__(self, ctx: Context, desc):
+    def __init__(self, ctx: Context, desc, pt_class=None, n_class: int = 1):
+        """With pt_class (a scale class per plaintext, < n_class): the plan of
+        fiona_plan_create_classes, whose n_out * n_class results are laid out
+        [n_out][n_class][2][L][N]."""
         self.ctx = ctx
         self._keep = []
 
@@ -266,14 +272,25 @@ class Plan:
         us = np.ascontiguousarray(desc.uses)
         n_nodes = max(int(noffs.shape[0]) - 1, 0)
         h = ctypes.c_void_p()
-        rc = lib().fiona_plan_create(ctx.handle, desc.n_in, desc.n_out, desc.n_pt, ptr(offs),
-                                     ptr(terms), int(gsp.shape[0]), ptr(gsp), ptr(gout),
-                                     n_nodes, ptr(noffs) if n_nodes else None, ptr(ch),
-                                     int(us.shape[0]), ptr(us), ctypes.byref(h))
+        if pt_class is None:
+            rc = lib().fiona_plan_create(ctx.handle, desc.n_in, desc.n_out, desc.n_pt, ptr(offs),
+                                         ptr(terms), int(gsp.shape[0]), ptr(gsp), ptr(gout),
+                                         n_nodes, ptr(noffs) if n_nodes else None, ptr(ch),
+                                         int(us.shape[0]), ptr(us), ctypes.byref(h))
+            where = "fiona_plan_create"
+        else:
+            cls = _arr(pt_class, np.uint8)
+            rc = lib().fiona_plan_create_classes(ctx.handle, desc.n_in, desc.n_out, desc.n_pt, ptr(offs),
+                                                 ptr(terms), int(gsp.shape[0]), ptr(gsp), ptr(gout),
+                                                 n_nodes, ptr(noffs) if n_nodes else None, ptr(ch),
+                                                 int(us.shape[0]), ptr(us), int(n_class), ptr(cls),
+                                                 ctypes.byref(h))
+            where = "fiona_plan_create_classes"
         self._keep = []
-        _check(rc, "fiona_plan_create")
+        _check(rc, where)
         self.handle = h
-        self.n_in, self.n_out, self.n_pt = desc.n_in, desc.n_out, desc.n_pt
+        self.n_in, self.n_pt = desc.n_in, desc.n_pt
+        self.n_out = desc.n_out * (1 if pt_class is None else int(n_class))
 
     def stats(self) -> Dict[str, int]:
         s = PlanStats()

@@ -238,6 +238,43 @@ class Plan:
         }
 
 
+def scale_classes(plan: Plan, n_class: int = 2, kind: str = "routes", seed: int = 0) -> np.ndarray:
+    """A scale class per plaintext (uint8, < n_class), for a layer whose
+    plaintexts are encoded at several scales.  "routes": the scale groups'
+    gamma plaintexts in class 0, the raw weights in class 1 (the two routes
+    at different scales); "random": seeded uniform classes."""
+    cls = np.zeros(plan.n_pt, dtype=np.uint8)
+    if n_class < 2:
+        return cls
+    if kind == "routes":
+        t = plan.terms
+        raw = t["pt"][(t["kind"] == TERM_RAW) | (t["kind"] == TERM_RAW_CONST)]
+        cls[np.unique(raw).astype(np.int64)] = 1
+        cls[np.unique(plan.group_scale_pt).astype(np.int64)] = 0
+    else:
+        rng = PlanRng(seed ^ 0x5CA1E, STREAM_PLAN)
+        for p in range(plan.n_pt):
+            cls[p] = rng.below(n_class)
+    return cls
+
+
+def class_subplan(plan: Plan, pt_class: np.ndarray, s: int) -> Plan:
+    """The layer restricted to the terms whose plaintext (a scale group's
+    gamma for signed terms) has class s; every output kept, the DAG dropped."""
+    t = plan.terms
+    per_output = []
+    for j in range(plan.n_out):
+        rows = []
+        for e in range(int(plan.term_offsets[j]), int(plan.term_offsets[j + 1])):
+            pt = int(plan.group_scale_pt[t["group"][e]]) if t["kind"][e] == TERM_TERNARY else int(t["pt"][e])
+            if int(pt_class[pt]) == s:
+                rows.append((int(t["input"][e]), int(t["kind"][e]), int(t["sign"][e]), int(t["pt"][e]),
+                             int(t["group"][e])))
+        per_output.append(rows)
+    return build_plan(plan.n_in, plan.n_out, per_output, plan.n_pt, list(plan.group_scale_pt),
+                      list(plan.group_output), [], [])
+
+
 def min_bytes(plan: Plan, L: int, N: int) -> int:
     """Minimal HBM bytes of one evaluation: each input read by a nonzero term
     (both polys), each plaintext a raw term or a used scale group reads, and

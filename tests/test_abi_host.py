@@ -306,3 +306,28 @@ def test_executed_addsub_reaches_the_papers_shared_count(monkeypatch):
         assert s["addsub_shared"] <= s["addsub_executed"] <= s["addsub_flat"], (name, s)
         plan.select_kernel("direct")
         assert plan.stats()["addsub_executed"] == s["addsub_flat"]
+
+
+def test_scale_class_plans():
+    """fiona_plan_create_classes: argument checks, and the plan of a layer
+    with two plaintext scales is that of its n_out * 2 results (each output's
+    terms split by their plaintext's class, the counts preserved)."""
+    wl = W.make_workload("tiny-dag")
+    ctx = F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE)
+    cls = W.scale_classes(wl.plan, 2, "random", seed=3)
+    plan = F.Plan(ctx, wl.plan, pt_class=cls, n_class=2)
+    s, s1 = plan.stats(), F.Plan(ctx, wl.plan).stats()
+    assert s["n_out"] == 2 * wl.plan.n_out and plan.n_out == 2 * wl.plan.n_out
+    for k in ("n_terms", "n_raw_terms", "n_signed_terms", "n_skipped_terms", "n_scale_groups_used"):
+        assert s[k] == s1[k], k
+    assert s["rescale_combined"] >= s1["rescale_combined"]
+    one = F.Plan(ctx, wl.plan, pt_class=np.zeros(wl.plan.n_pt, np.uint8), n_class=1).stats()
+    assert one == s1
+    with pytest.raises(F.FionaError) as e:
+        F.Plan(ctx, wl.plan, pt_class=cls, n_class=0)
+    assert e.value.status == F.FIONA_ERR_ARG
+    bad = cls.copy()
+    bad[0] = 2
+    with pytest.raises(F.FionaError) as e:
+        F.Plan(ctx, wl.plan, pt_class=bad, n_class=2)
+    assert e.value.status == F.FIONA_ERR_PLAN

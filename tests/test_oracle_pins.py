@@ -245,6 +245,45 @@ def test_dag_equals_flat_reduced_bert():
 
 
 # -- planted mistakes ----------------------------------------------------------
+@pytest.mark.parametrize("name,kind,n_class", [("tiny", "routes", 2), ("tiny-dag", "random", 3),
+                                               ("worked-example", "random", 2)])
+def test_scale_classes(name, kind, n_class):
+    """Plaintexts at several scales (Sec. 4.2 "Combining the Signed and Raw
+    Routes": routes combine within one scale): each class's result equals the
+    brute-force evaluation over Z_Q of the layer restricted to that class's
+    terms (a sub-plan built by filtering the term list), and the class
+    results sum to the one-scale evaluation of the whole layer."""
+    wl = W.make_workload(name)
+    X, P = small_inputs(wl, 6)
+    cls = W.scale_classes(wl.plan, n_class, kind, seed=3)
+    assert len(set(cls.tolist())) > 1
+    y = oracle.linear_eval_classes(wl.plan, wl.moduli, cls, n_class, X, P)
+    for s_ in range(n_class):
+        sub = W.class_subplan(wl.plan, cls, s_)
+        assert np.array_equal(y[:, s_], crt.eval_over_ZQ(sub, wl.moduli, X, P)), s_
+    q = np.array(wl.moduli, dtype=object).reshape(1, 1, -1, 1)
+    total = (y.astype(object).sum(axis=1) % q).astype(np.uint64)
+    assert np.array_equal(total, oracle.linear_eval(wl.plan, wl.moduli, X, P))
+    one = oracle.linear_eval_classes(wl.plan, wl.moduli, np.zeros(wl.plan.n_pt, np.uint8), 1, X, P)
+    assert np.array_equal(one[:, 0], oracle.linear_eval(wl.plan, wl.moduli, X, P))
+
+
+def test_planted_class_mistake_is_caught(tmp_path):
+    """The raw route's class test taken out of the oracle: the per-class
+    brute force catches it."""
+    src = open(os.path.join(os.path.dirname(oracle.__file__), "oracle.c")).read()
+    old = "if (pt_class && pt_class[term_pt[e]] != want_class)"
+    assert old in src
+    path = tmp_path / "mutant.c"
+    path.write_text(src.replace(old, "if (0)"))
+    lib = oracle.load_variant(str(path), str(tmp_path / "libmutant.so"))
+    wl = W.make_workload("tiny")
+    X, P = small_inputs(wl, 6)
+    cls = W.scale_classes(wl.plan, 2, "routes")
+    y = oracle.linear_eval_classes(wl.plan, wl.moduli, cls, 2, X, P, lib=lib)
+    assert not np.array_equal(y[:, 0], crt.eval_over_ZQ(W.class_subplan(wl.plan, cls, 0), wl.moduli, X, P))
+
+
 MUTATIONS = {
     "sign_flip": ("s = sub_mod(s, a, q);", "s = add_mod(s, a, q);"),
     "dropped_raw": ("y = add_mod(y, mul_mod(p, a, q), q);", "(void)p; (void)a;"),

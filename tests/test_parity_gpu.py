@@ -387,3 +387,28 @@ def test_warp_formed_sums(name, N, L, shape, monkeypatch):
         mism = np.argwhere(dl.outputs() != want)
         assert mism.shape[0] == 0, "first mismatches (j, c, l, k): %s" % mism[:5].tolist()
     assert dl.ctx.device_check() == F.FIONA_OK
+
+
+@pytest.mark.parametrize("kernel", ["direct", "tiled"])
+@pytest.mark.parametrize("name,N,L,kind,n_class", [("tiny", None, None, "routes", 2),
+                                                   ("tiny-dag", None, None, "random", 3),
+                                                   ("vit", 2048, 2, "random", 2),
+                                                   ("bert-const", 1024, 1, "routes", 2)])
+def test_scale_class_parity(name, N, L, kind, n_class, kernel):
+    """Plaintexts at several scales (fiona_plan_create_classes): every
+    (output, class) result [n_out][n_class][2][L][N] equals the oracle's."""
+    wl = W.make_workload(name, N=N, L=L)
+    cls = W.scale_classes(wl.plan, n_class, kind, seed=5)
+    ctx = F.Context(wl.N, wl.moduli, device=0)
+    plan = F.Plan(ctx, wl.plan, pt_class=cls, n_class=n_class)
+    plan.select_kernel(kernel)
+    X, P = wl.host_inputs(), wl.host_plaintexts()
+    p = wl.plan
+    d_out = torch.full((p.n_out * n_class * 2 * wl.L * wl.N,), -1, dtype=torch.int64, device="cuda")
+    plan.eval(to_device(X), to_device(P), d_out)
+    torch.cuda.synchronize()
+    got = to_host(d_out).reshape(p.n_out, n_class, 2, wl.L, wl.N)
+    want = oracle.linear_eval_classes(p, wl.moduli, cls, n_class, X, P)
+    mism = np.argwhere(got != want)
+    assert mism.shape[0] == 0, "first mismatches (j, s, c, l, k): %s" % mism[:5].tolist()
+    assert ctx.device_check() == F.FIONA_OK
