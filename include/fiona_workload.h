@@ -35,6 +35,14 @@ int fiona_workload_fill(void *cuda_stream, uint64_t *dst, uint64_t outer, uint32
  * Returns 0, or -1 on a null argument, -5 on a CUDA error. */
 int fiona_mul_roof(double *narrow_per_s, double *wide_per_s);
 
+/* Measured butterfly roof of the current device: forward NTT butterflies per
+ * second over the whole GPU of the rescale's own butterfly (one product by a
+ * twiddle with Shoup's precomputed quotient, a sum and a difference); fast:
+ * without the conditional subtraction (every modulus below 2^56), general:
+ * with it.  Runs a few milliseconds of kernels on the default stream and
+ * synchronizes.  Returns 0, or -1 on a null argument, -5 on a CUDA error. */
+int fiona_bfly_roof(double *fast_per_s, double *general_per_s);
+
 #ifdef __cplusplus
 }
 #endif

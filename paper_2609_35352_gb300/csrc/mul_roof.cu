@@ -16,6 +16,7 @@
 #include <cuda_runtime.h>
 
 #include "fiona_workload.h"
+#include "ntt.cuh"
 #include "rns.cuh"
 
 namespace {
@@ -72,7 +73,92 @@ double rate(int sms, const uint64_t *seed, uint64_t *sink)
     return products / (ms * 1e-3);
 }
 
+// Forward NTT butterflies of the rescale (fiona_ntt::ModArith::ct: one
+// product by a twiddle with Shoup's precomputed quotient, a sum and a
+// difference), FAST = without the conditional subtraction (every modulus
+// below 2^56), in kChains independent chains per thread; the twiddle changes
+// every step so that nothing folds away.
+template <bool FAST>
+__global__ void __launch_bounds__(256) bfly_kernel(const uint64_t *seed, uint64_t *sink)
+{
+    const fiona_ntt::ModArith<FAST> ar{(seed[0] >> 14) | 1};
+    uint64_t x[kChains], y[kChains];
+    ulonglong2 w[kChains];
+#pragma unroll
+    for (int c = 0; c < kChains; ++c) {
+        x[c] = seed[(threadIdx.x + c) & 63] >> 14;
+        y[c] = seed[(threadIdx.x + 7 * c + 1) & 63] >> 14;
+        w[c] = make_ulonglong2(seed[(threadIdx.x + 3 * c + 2) & 63] >> 14, seed[(threadIdx.x + 5 * c + 3) & 63]);
+    }
+    for (int s = 0; s < kSteps; ++s) {
+#pragma unroll
+        for (int c = 0; c < kChains; ++c) {
+            ar.ct(x[c], y[c], w[c]);
+            w[c].x ^= y[c] & 0xF;
+        }
+    }
+    uint64_t r = 0;
+#pragma unroll
+    for (int c = 0; c < kChains; ++c) r += x[c] ^ y[c] ^ w[c].x;
+    sink[blockIdx.x * blockDim.x + threadIdx.x] = r;
+}
+
+template <bool FAST>
+double bfly_rate(int sms, const uint64_t *seed, uint64_t *sink)
+{
+    const dim3 grid(sms * 8), block(256);
+    bfly_kernel<FAST><<<grid, block>>>(seed, sink);  // warm-up
+    cudaEvent_t e0, e1;
+    cudaEventCreate(&e0);
+    cudaEventCreate(&e1);
+    const int reps = 3;
+    cudaEventRecord(e0);
+    for (int r = 0; r < reps; ++r) bfly_kernel<FAST><<<grid, block>>>(seed, sink);
+    cudaEventRecord(e1);
+    float ms = 0;
+    const bool ok = cudaEventSynchronize(e1) == cudaSuccess && cudaEventElapsedTime(&ms, e0, e1) == cudaSuccess;
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    if (!ok || ms <= 0) return 0;
+    return (double)reps * grid.x * block.x * kSteps * kChains / (ms * 1e-3);
+}
+
+// device buffers of the roof measurements: 64 seed words and one sink word
+// per thread of the grid
+int roof_buffers(int *sms, uint64_t **seed, uint64_t **sink)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || *sms <= 0)
+        return -5;
+    if (cudaMalloc(seed, 64 * sizeof(uint64_t)) != cudaSuccess) return -5;
+    if (cudaMalloc(sink, (size_t)*sms * 8 * 256 * sizeof(uint64_t)) != cudaSuccess) {
+        cudaFree(*seed);
+        return -5;
+    }
+    uint64_t h[64];
+    uint64_t x = 0x9E3779B97F4A7C15ull;
+    for (auto &v : h) v = (x = x * 6364136223846793005ull + 1442695040888963407ull);
+    return cudaMemcpy(*seed, h, sizeof(h), cudaMemcpyHostToDevice) == cudaSuccess ? 0 : -5;
+}
+
 }  // namespace
+
+extern "C" int fiona_bfly_roof(double *fast_per_s, double *general_per_s)
+{
+    if (!fast_per_s || !general_per_s) return -1;
+    int sms = 0;
+    uint64_t *seed = nullptr, *sink = nullptr;
+    int rc = roof_buffers(&sms, &seed, &sink);
+    if (rc == 0) {
+        *fast_per_s = bfly_rate<true>(sms, seed, sink);
+        *general_per_s = bfly_rate<false>(sms, seed, sink);
+        if (*fast_per_s <= 0 || *general_per_s <= 0 || cudaGetLastError() != cudaSuccess) rc = -5;
+    }
+    cudaFree(seed);
+    cudaFree(sink);
+    return rc;
+}
 
 extern "C" int fiona_mul_roof(double *narrow_per_s, double *wide_per_s)
 {

@@ -371,6 +371,8 @@ def workload_lib() -> ctypes.CDLL:
         W.fiona_workload_fill.restype = ctypes.c_int
         W.fiona_mul_roof.argtypes = [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
         W.fiona_mul_roof.restype = ctypes.c_int
+        W.fiona_bfly_roof.argtypes = [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
+        W.fiona_bfly_roof.restype = ctypes.c_int
         _wlib = W
     return _wlib
 
@@ -393,6 +395,16 @@ def mul_roof() -> Dict[str, float]:
     if rc != 0:
         raise RuntimeError("fiona_mul_roof failed (%d)" % rc)
     return {"narrow": n.value, "wide": w.value}
+
+
+def bfly_roof() -> Dict[str, float]:
+    """fiona_bfly_roof: the measured forward NTT butterflies per second of the
+    rescale's butterfly, fast (moduli below 2^56) and general."""
+    f, g = ctypes.c_double(), ctypes.c_double()
+    rc = workload_lib().fiona_bfly_roof(ctypes.byref(f), ctypes.byref(g))
+    if rc != 0:
+        raise RuntimeError("fiona_bfly_roof failed (%d)" % rc)
+    return {"fast": f.value, "general": g.value}
 
 
 # -- host plan compiler -------------------------------------------------------
