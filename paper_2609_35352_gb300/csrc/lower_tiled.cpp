@@ -314,10 +314,13 @@ void colocate(JobPlan &jp, const std::vector<OutWork> &work, const Costs &k, siz
         bool whole = true;
         for (uint32_t u : us) whole &= warp_of[u] >= 0;
         if (!whole) continue;
-        // the warp already holding most of the users (pinned ones first)
+        // the warp already holding most of the users (pinned ones first); of
+        // those, the least loaded (it will also form the sum)
         std::vector<int> votes(W, 0);
         for (uint32_t u : us) votes[warp_of[u]] += 1 + 4 * pinned[u];
-        const uint32_t t = (uint32_t)(std::max_element(votes.begin(), votes.end()) - votes.begin());
+        uint32_t t = 0;
+        for (uint32_t wi = 1; wi < W; ++wi)
+            if (votes[wi] > votes[t] || (votes[wi] == votes[t] && load[wi] < load[t])) t = wi;
         std::vector<std::pair<uint32_t, uint32_t>> swaps;  // (user, partner on t)
         std::vector<double> ld = load;
         std::vector<int> taken(work.size(), 0);
