@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define FIONA_ABI_VERSION 2
+#define FIONA_ABI_VERSION 3
 
 typedef struct fiona_ctx fiona_ctx;   /* N, RNS moduli, per-limb constants on one device */
 typedef struct fiona_plan fiona_plan; /* one validated, lowered linear layer */
@@ -160,7 +160,10 @@ typedef struct fiona_plan_stats_t {
     uint32_t addsub_executed;     /* Add/Sub of the kernel in use, in the units of addsub_flat:
                                      each sum of n operands it forms (shared sums, scale groups,
                                      an output's products, its partial sums) counts n - 1 */
-    uint32_t reserved[3];
+    uint32_t tensor_core_sums;    /* TILED: scale-group signed sums formed per tile as one
+                                     contraction on the tensor cores (the groups' terms, shared
+                                     sums expanded, exact in fp16 chunks); 0: on the ALUs      */
+    uint32_t reserved[2];
 } fiona_plan_stats_t;
 
 /* Create a context for ring dimension N (a power of two, 2^10 <= N <= 2^17)

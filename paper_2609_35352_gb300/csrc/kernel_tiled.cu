@@ -47,6 +47,7 @@
 #include <cstring>
 #include <mutex>
 
+#include "tc_signed.cuh"
 #include "tiled.h"
 #include "tile_math.cuh"
 
@@ -162,10 +163,11 @@ __device__ __forceinline__ uint64_t evict_first_policy()
     return pol;
 }
 
-template <int C, bool NARROW, uint32_t P, bool KC>
+template <int C, bool NARROW, uint32_t P, bool KC, bool TC = false>
 __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     tiled_kernel(const TiledArgs a, const __grid_constant__ CUtensorMap tm_in)
 {
+    static_assert(!TC || (C == 1 && NARROW), "tensor-core sums: one coefficient per lane, narrow moduli");
     using A = Arith<NARROW>;
     using Acc = typename A::Acc;
     static_assert(P % 4 == 0, "operation words are read four at a time");
@@ -183,6 +185,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     __shared__ int s_abort;
     if (threadIdx.x == 0) s_abort = 0;
     __shared__ __align__(16) LimbConst s_limb[2];  // per source region
+    __shared__ uint32_t s_tmem;                    // TC: the CTA's tensor memory
     const uint32_t n_warps = blockDim.x >> 5;
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t n_buf = a.double_buffer ? 2 : 1;
@@ -192,6 +195,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     const uint32_t bar_off = slot_base + a.n_slots * PB;  // the schedule copy's mbarrier
     const uint32_t bar0 = smem_addr(sm) + bar_off;
     const uint32_t bar_stage = bar0 + 8;  // + 8 * region: the region's input copies have landed
+    const uint32_t bar_tc = bar0 + 24;    // TC: the tile's contraction is complete
     const uint32_t total = a.n_limbs * a.tiles_per_limb;
     const uint32_t lane_off = lane * VB;
     const uint32_t *sw = reinterpret_cast<const uint32_t *>(sm);
@@ -226,6 +230,13 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         const uint32_t reg = i / (PB / 16), o = i % (PB / 16);
         *reinterpret_cast<ulonglong2 *>(sm + src0 + reg * a.src_bytes + a.src_bytes - PB + o * 16) =
             make_ulonglong2(0, 0);
+    }
+    // TC: the tensor memory (published by the first tile's barrier) and the
+    // contraction's barrier
+    if constexpr (TC) {
+        if (warp == 0) tcs::tmem_alloc(smem_addr(&s_tmem), a.tc_cols);
+        if (threadIdx.x == 0) mbar_init(bar_tc, 1);
+        tcs::fence_before();
     }
 
     // ---- this warp's operation stream and its plaintext queue
@@ -295,6 +306,8 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     };
     uint32_t stage_phase = 0;  // bit r: phase of region r's copy barrier
     uint32_t failed = 0;       // 1 + region + 2 * phase of a copy wait that gave up
+    uint32_t tc_phase = 0;     // TC: phase of the contraction's barrier
+    uint32_t tc_failed = 0;    // TC: 1 + phase of a contraction wait that gave up
 
     // the tile's inputs in region `reg`, once the copies have landed (with
     // cp.async each thread rewrites the words it copied); and the tile's
@@ -330,14 +343,30 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     uint32_t buf = 0;
     // after a copy wait gave up: every thread stops at the same barrier, once
     // thread 0 has waited (bounded again) for the copies it issued
+    // (and for the tensor cores' work in flight), then frees the CTA's
+    // tensor memory
+    uint32_t tmem = 0;
+    auto release = [&]() {
+        if constexpr (TC) {
+            tcs::fence_after();
+            if (warp == 0) tcs::tmem_dealloc(tmem, a.tc_cols);
+        }
+    };
     auto stop = [&]() {
         if (TMA && threadIdx.x == 0 && failed) mbar_wait_spin(bar_stage + 8 * ((failed - 1) & 1), (failed - 1) >> 1);
+        if (TC && threadIdx.x == 0 && tc_failed) mbar_wait_spin(bar_tc, tc_failed - 1);
+        if constexpr (TC) __syncthreads();
+        release();
     };
     if (tile < total) {
         if (a.n_in) stage(tile, 0);
         prepare(tile, 0);
     }
     __syncthreads();
+    if constexpr (TC) {
+        tcs::fence_after();
+        tmem = s_tmem;
+    }
     if (s_abort) {
         stop();
         return;
@@ -365,8 +394,41 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
             }
         }
 
+        // 2. TC: the scale groups' signed sums, as one contraction on the
+        //    tensor cores (tc_signed.cuh): every warp converts its share of
+        //    the inputs into tensor memory, one thread issues the
+        //    contraction, and every warp turns its share of the products
+        //    into canonical residues, stored as the group sources
+        if constexpr (TC) {
+            const TcGeometry geo{a.tc_k, a.tc_n};
+            const uint32_t q4 = warp & 3, kq = warp >> 2, nq = n_warps >> 2;
+            const uint32_t tq = tmem + ((32u * q4) << 16);
+            const uint32_t row = sb + tcs::row_poly(q4) * TB + tcs::row_coef(q4, lane) * 8;
+            tcs::convert(sm, row, PB, a.n_in, geo, tq, kq, nq);
+            tcs::wait_st();
+            tcs::fence_before();
+            __syncthreads();
+            tcs::fence_after();
+            if (threadIdx.x == 0) tcs::issue(tmem, smem_addr(sm) + a.o_tcw * 4, geo, bar_tc);
+            if (!mbar_wait_spin(bar_tc, tc_phase)) {
+                s_abort = 1;  // the CTA stops after this tile's last barrier
+                atomicOr(a.err, 1);
+                tc_failed = 1 + tc_phase;
+            }
+            tc_phase ^= 1;
+            tcs::fence_after();
+            const LimbConst m = load_limb(lim);
+            const uint64_t bias = (uint64_t)a.tc_wabs * m.q;
+            const float *magic = reinterpret_cast<const float *>(sm + a.o_tcm * 4);
+            tcs::epilogue(tq, geo, a.tc_groups, magic, bias, m, lane, kq, nq, [&](uint32_t g, uint64_t v) {
+                *reinterpret_cast<uint64_t *>(sm + row + (a.n_in + g) * PB) = v;
+            });
+            tcs::fence_before();
+            __syncthreads();
+        }
         // 2. materialised shared sums, children first
-        for (uint32_t lev = 0; lev < a.n_levels; ++lev) {
+        const uint32_t n_levels = TC ? 0 : a.n_levels;  // TC: its one level is the contraction
+        for (uint32_t lev = 0; lev < n_levels; ++lev) {
             for (uint32_t x = sw[a.o_level + lev] + warp; x < sw[a.o_level + lev + 1]; x += n_warps) {
                 V<C> u0, u1;
                 signed_sum<SPLIT, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, 0, u0, u1);
@@ -549,6 +611,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
             return;
         }
     }
+    release();
 }
 
 template <uint32_t P, bool KC>
@@ -570,9 +633,16 @@ void *select_ptr_16(int C, bool narrow)
                   : reinterpret_cast<void *>(&tiled_kernel<1, false, 16, KC>);
 }
 
-// KC: the variant that reads constant plaintexts (operations marked kOpConst)
-void *select_ptr(int C, bool narrow, uint32_t P, bool kc)
+// KC: the variant that reads constant plaintexts (operations marked kOpConst);
+// TC: the signed sums on the tensor cores (one coefficient per lane, narrow
+// moduli, batches of 16)
+void *select_ptr(int C, bool narrow, uint32_t P, bool kc, bool tc = false)
 {
+    if (tc) {
+        if (C != 1 || !narrow || P != 16) return nullptr;
+        return kc ? reinterpret_cast<void *>(&tiled_kernel<1, true, 16, true, true>)
+                  : reinterpret_cast<void *>(&tiled_kernel<1, true, 16, false, true>);
+    }
     if (P == 16) return kc ? select_ptr_16<true>(C, narrow) : select_ptr_16<false>(C, narrow);
     if (kc) return P == 4 ? select_ptr_p<4, true>(C, narrow) : select_ptr_p<8, true>(C, narrow);
     return P == 4 ? select_ptr_p<4, false>(C, narrow) : select_ptr_p<8, false>(C, narrow);
@@ -580,19 +650,21 @@ void *select_ptr(int C, bool narrow, uint32_t P, bool kc)
 
 }  // namespace
 
-int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, cudaFuncAttributes *attr)
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr)
 {
-    if (!select_ptr(C, narrow, P, kc)) return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
-    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc));
+    if (!select_ptr(C, narrow, P, kc, tc))
+        return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
+    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc, tc));
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attributes: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
 
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, size_t smem)
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem)
 {
-    if (!select_ptr(C, narrow, P, kc)) return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
-    cudaError_t e =
-        cudaFuncSetAttribute(select_ptr(C, narrow, P, kc), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (!select_ptr(C, narrow, P, kc, tc))
+        return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
+    cudaError_t e = cudaFuncSetAttribute(select_ptr(C, narrow, P, kc, tc),
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attribute: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
@@ -659,7 +731,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     dim3 grid(std::min(tiles, resident));
     dim3 block(ts->warps * 32);
     cudaStream_t s = (cudaStream_t)stream;
-    void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const);
+    void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const, ts->tc);
     if (!fn) return set_error(FIONA_ERR_INTERNAL, "tiled kernel: no variant for the schedule's shape");
     CUtensorMap tm;  // read by the kernels with one coefficient per lane only
     memset(&tm, 0, sizeof(tm));

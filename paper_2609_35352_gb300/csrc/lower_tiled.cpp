@@ -860,6 +860,163 @@ LocalResult localize(JobPlan &jp, const std::vector<OutWork> &groups, const Node
     return res;
 }
 
+// The scale groups' signed sums as one tensor-core contraction per tile
+// (tc_signed.cuh): every used group of every output (shared sums expanded
+// into their terms) becomes one materialised source, the group's column of
+// the weight matrix W, formed per tile before the operation streams run; the
+// group's product by gamma is then an ordinary operation on that source.
+struct TcPlan {
+    bool ok = false;
+    std::vector<OutWork> work;  // per output: its raw terms, then one operation per group source
+    std::vector<Seg> nodes;     // the group sums, over inputs only
+    uint32_t K = 0, N = 0;      // contraction length (inputs, padded to 16) and width (groups, padded to 8)
+    uint32_t wabs = 0;          // largest sum of |weights| of a group
+    uint32_t cols = 0;          // tensor memory columns a CTA allocates (a power of two)
+};
+
+// exact fp16 bits of an integer |v| <= 2048
+uint16_t fp16_of_int(int v)
+{
+    if (v == 0) return 0;
+    const uint16_t sgn = v < 0 ? 0x8000 : 0;
+    const uint32_t a = (uint32_t)(v < 0 ? -v : v);
+    int e = 0;
+    while ((a >> (e + 1)) != 0) ++e;
+    return (uint16_t)(sgn | ((e + 15) << 10) | ((a << (10 - e)) & 0x3FFu));
+}
+
+// net weight of each input in a program's plus and minus lists
+std::vector<int> net_weights(const Seg &s, uint32_t n_in)
+{
+    std::vector<int> w(n_in, 0);
+    for (uint32_t i : s.plus) ++w[i];
+    for (uint32_t i : s.minus) --w[i];
+    return w;
+}
+
+TcPlan plan_tc(const HostPlan &hp, const NodeInfo &ni, const std::vector<OutWork> &groups, uint64_t q_max)
+{
+    TcPlan tc;
+    const uint32_t n_in = hp.n_in;
+    const std::vector<int32_t> none(hp.n_nodes, -1);
+    const Resolver rv{ni, none};
+    tc.work.resize(groups.size());
+    for (size_t j = 0; j < groups.size(); ++j) {
+        tc.work[j].raws = groups[j].raws;
+        for (const Seg &g : groups[j].segs) {
+            Seg s;
+            s.scale_pt = g.scale_pt;
+            for (uint32_t op : g.plus) rv.add(op, +1, s.plus, s.minus);
+            for (uint32_t op : g.minus) rv.add(op, -1, s.plus, s.minus);
+            const std::vector<int> w = net_weights(s, n_in);
+            if (std::all_of(w.begin(), w.end(), [](int x) { return x == 0; })) continue;
+            tc.work[j].raws.push_back({n_in + (uint32_t)tc.nodes.size(), s.scale_pt});
+            tc.nodes.push_back(std::move(s));
+        }
+    }
+    const uint32_t ng = (uint32_t)tc.nodes.size();
+    if (!ng || n_in + ng + 1 > kOpMaxSources) return tc;
+    tc.K = (n_in + 15) & ~15u;
+    tc.N = std::max(8u, (ng + 7) & ~7u);
+    if (tc.N > 256) return tc;
+    const TcGeometry geo{tc.K, tc.N};
+    if (geo.cols() > 512) return tc;
+    tc.cols = 32;
+    while (tc.cols < geo.cols()) tc.cols *= 2;
+    for (const Seg &s : tc.nodes) {
+        int cs = 0;
+        uint32_t ab = 0;
+        for (int x : net_weights(s, n_in)) {
+            if (x > 2048 || x < -2048) return tc;
+            cs += x;
+            ab += (uint32_t)std::abs(x);
+        }
+        // exact chunk sums in fp32 (2047 * ab < 2^24), the magic constant
+        // exact (|1024 cs| < 2^22), S + wabs * q below 2^64
+        if (ab > 8191 || std::abs(cs) >= 4096) return tc;
+        tc.wabs = std::max(tc.wabs, ab);
+    }
+    if ((unsigned __int128)2 * tc.wabs * q_max >= ((unsigned __int128)1 << 64)) return tc;
+    tc.ok = true;
+    return tc;
+}
+
+// Append W (fp16, K-major core matrices, tc_signed.cuh) and the groups'
+// magic constants to the schedule; returns their word offsets.
+void append_tc(std::vector<uint32_t> &w, const TcPlan &tc, uint32_t n_in, uint32_t &o_w, uint32_t &o_magic)
+{
+    const TcGeometry geo{tc.K, tc.N};
+    pad4(w);
+    o_w = (uint32_t)w.size();
+    w.resize(w.size() + geo.w_bytes() / 4, 0);
+    for (uint32_t n = 0; n < tc.nodes.size(); ++n) {
+        const std::vector<int> wt = net_weights(tc.nodes[n], n_in);
+        for (uint32_t k = 0; k < n_in; ++k) {
+            const uint32_t b = (n / 8) * geo.sbo() + (k / 8) * 128 + (n % 8) * 16 + (k % 8) * 2;
+            w[o_w + b / 4] |= (uint32_t)fp16_of_int(wt[k]) << (16 * ((b / 2) & 1));
+        }
+    }
+    o_magic = (uint32_t)w.size();
+    for (uint32_t n = 0; n < tc.nodes.size(); ++n) {
+        const std::vector<int> wt = net_weights(tc.nodes[n], n_in);
+        const int cs = std::accumulate(wt.begin(), wt.end(), 0);
+        const float magic = 12582912.0f - 1024.0f * (float)cs;
+        uint32_t bits;
+        memcpy(&bits, &magic, 4);
+        w.push_back(bits);
+    }
+    while (w.size() % 32) w.push_back(0);
+}
+
+// Check the contraction's tables against the node programs the schedule
+// holds (the sums the linear-map check verified): every weight, the padding
+// zero, each magic constant, the bound wabs, and the layout.
+const char *check_tc(const std::vector<uint32_t> &w, const TiledArgs &a)
+{
+    if (!a.tc_groups) return nullptr;
+    if (a.tc_groups != a.n_nodes || a.n_levels != 1) return "tensor-core sums: node count";
+    const TcGeometry geo{a.tc_k, a.tc_n};
+    if (a.tc_k % 16 || a.tc_k < a.n_in || a.tc_n % 8 || a.tc_n < std::max(a.tc_groups, 8u) || a.tc_n > 256 ||
+        geo.cols() > a.tc_cols || a.tc_cols > 512 || (a.tc_cols & (a.tc_cols - 1)) || a.tc_cols < 32)
+        return "tensor-core sums: geometry";
+    if (a.o_tcw % 4 || (size_t)a.o_tcw + geo.w_bytes() / 4 > a.o_tcm || (size_t)a.o_tcm + a.tc_groups > w.size())
+        return "tensor-core sums: layout";
+    for (uint32_t n = 0; n < a.tc_n; ++n) {
+        std::vector<int> want(a.tc_k, 0);
+        if (n < a.tc_groups) {  // the node program: plus run, minus run, inputs only
+            size_t p = w[a.o_node_off + n];
+            const uint32_t h = w[p++];
+            for (int sign : {1, -1}) {
+                const uint32_t cnt = sign > 0 ? (h & 0xffffu) : (h >> 16);
+                for (uint32_t i = 0; i < cnt; ++i) {
+                    const uint32_t idx = (w[p + i / 2] >> (16 * (i & 1))) & 0xffffu;
+                    if (idx >= a.n_in) return "tensor-core sums: a node reads a non-input";
+                    want[idx] += sign;
+                }
+                p += (cnt + 1) / 2;
+            }
+            if (w[p] != 0) return "tensor-core sums: a node reads warp slots";
+        }
+        int cs = 0;
+        uint32_t ab = 0;
+        for (uint32_t k = 0; k < a.tc_k; ++k) {
+            const uint32_t b = (n / 8) * geo.sbo() + (k / 8) * 128 + (n % 8) * 16 + (k % 8) * 2;
+            const uint16_t h = (uint16_t)(w[a.o_tcw + b / 4] >> (16 * ((b / 2) & 1)));
+            if (std::abs(want[k]) > 2048 || h != fp16_of_int(want[k])) return "tensor-core sums: weight";
+            cs += want[k];
+            ab += (uint32_t)std::abs(want[k]);
+        }
+        if (n < a.tc_groups) {
+            const float magic = 12582912.0f - 1024.0f * (float)cs;
+            uint32_t bits;
+            memcpy(&bits, &magic, 4);
+            if (w[a.o_tcm + n] != bits || std::abs(cs) >= 4096 || ab > 8191 || ab > a.tc_wabs)
+                return "tensor-core sums: constants";
+        }
+    }
+    return nullptr;
+}
+
 // Add/Sub a schedule performs per evaluation, in the units of the paper's
 // counts (a sum of n operands costs n - 1): the shared sums formed for the
 // block and by warps, every scale group's signed sum, each job's products
@@ -930,7 +1087,7 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
     const uint32_t n_src = a.n_in + a.n_nodes, zero = n_src;  // the zero tile follows the sources
     if (n_src + 1 > kOpMaxSources) return "too many sources";
     if ((size_t)a.sched_bytes + (size_t)(a.double_buffer ? 2 : 1) * a.src_bytes + (size_t)a.n_part * PB +
-            (size_t)a.n_slots * PB + 24 >
+            (size_t)a.n_slots * PB + (a.tc_groups ? 32 : 24) >
         smem)
         return "shared-memory layout";
     if (a.src_bytes != (n_src + 1) * PB) return "source region size";
@@ -1148,8 +1305,8 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
 }  // namespace
 
 // kernel_tiled.cu
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, size_t smem);
-int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, cudaFuncAttributes *attr);
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem);
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr);
 // kernel_ws.cu
 int ws_kernel_attributes(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, cudaFuncAttributes *attr);
 int ws_configure_kernel(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, size_t smem);
@@ -1435,7 +1592,7 @@ int lower_tiled(fiona_plan *p)
         if (!device) {  // lowering without a GPU: the build's usual figures
             attr.numRegs = 128;
             attr.sharedSizeBytes = 64;
-        } else if (tiled_kernel_attributes(C, narrow, batch, has_const, &attr) != FIONA_OK) {
+        } else if (tiled_kernel_attributes(C, narrow, batch, has_const, false, &attr) != FIONA_OK) {
             continue;
         }
         const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
@@ -1552,11 +1709,66 @@ int lower_tiled(fiona_plan *p)
     }
     const uint32_t T = 32u * best.C, PB = 2 * T * 8;
     const Costs k = costs_for(best.C, narrow);
-    const Lowered lw = resolve(hp, ni, groups, rank, best.keep, budget);
-    JobPlan jp = build_jobs(lw.work, best.W, k, best.P, best.keep ? nullptr : sh);
+    const uint32_t nbuf = best.dbl ? 2 : 1;
+    Lowered lw;
+    JobPlan jp;
+    LocalResult loc;
+    Sched sc;
+    // -- the scale groups' signed sums as one tensor-core contraction per
+    //    tile (one coefficient per lane, every q < 2^50, batches of 16, warps
+    //    in fours: one per tensor-memory quarter), when its sources, W and
+    //    the schedule fit and FIONA_TILED_TC=1 asks for it.  Not the default:
+    //    measured on the VGG layer, the contraction's phase (conversion to
+    //    fp16 chunks 3.3k cycles a tile, 45 dependent MMAs 4.3k, epilogue
+    //    1.8k) costs more than the shared-memory sums it replaces, which
+    //    overlap the plaintext loads (3.45 against 2.34 ms a launch)
+    bool use_tc = false;
+    TcPlan tc;
+    uint32_t o_tcw = 0, o_tcm = 0;
+    {
+        const char *env = getenv("FIONA_TILED_TC");
+        const bool allow = env && atoi(env) != 0;
+        if (allow && !force_keep && best.C == 1 && narrow && best.P == 16 && best.W % 4 == 0 &&
+            ctx->q_max < (1ull << 50))
+            tc = plan_tc(hp, ni, groups, ctx->q_max);
+        cudaFuncAttributes attr{};
+        if (!device) {
+            attr.numRegs = 128;
+            attr.sharedSizeBytes = 64;
+        } else if (tc.ok && tiled_kernel_attributes(1, true, best.P, has_const, true, &attr) != FIONA_OK) {
+            tc.ok = false;
+        }
+        if (tc.ok) {
+            const uint32_t ng = (uint32_t)tc.nodes.size();
+            Lowered lt;
+            lt.work = tc.work;
+            lt.nodes = tc.nodes;
+            lt.level_off = {0, ng};
+            lt.n_levels = 1;
+            JobPlan jt = build_jobs(lt.work, best.W, k, best.P, nullptr);
+            Sched st = encode(jt, lt.level_off, lt.nodes, best.W, mac_budget, hp.n_in + ng, best.P);
+            append_tc(st.w, tc, hp.n_in, o_tcw, o_tcm);
+            const size_t smem = st.w.size() * 4 + (size_t)(hp.n_in + ng + 1) * PB * nbuf + (size_t)jt.n_part * PB + 32;
+            const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
+            const uint32_t ctas = std::min({(uint32_t)(per_sm / (smem + attr.sharedSizeBytes + 1024)),
+                                            2048 / (best.W * 32), 65536 / (best.W * 32 * regs), 512 / tc.cols});
+            if (getenv("FIONA_TILED_DEBUG"))
+                fprintf(stderr, "tensor-core sums: groups=%u K=%u N=%u cols=%u smem=%zu ctas=%u\n", ng, tc.K, tc.N,
+                        tc.cols, smem, ctas);
+            if (smem + attr.sharedSizeBytes <= smem_cap && ctas >= 1) {
+                use_tc = true;
+                lw = std::move(lt);
+                jp = std::move(jt);
+                sc = std::move(st);
+                best.ctas = ctas;
+            }
+        }
+    }
+    if (!use_tc) {
+    lw = resolve(hp, ni, groups, rank, best.keep, budget);
+    jp = build_jobs(lw.work, best.W, k, best.P, best.keep ? nullptr : sh);
     // shared sums formed by the warps that use them, when no sum is formed
     // for the whole block and the warps' slots fit in shared memory
-    LocalResult loc;
     // (a tuning override with a fourth field selects the block-level sums instead)
     if (!best.keep && sh && !force_keep && !getenv("FIONA_NO_WARP_SUMS")) {
         for (uint32_t max_slots = 8; max_slots >= 1; max_slots /= 2) {
@@ -1600,8 +1812,8 @@ int lower_tiled(fiona_plan *p)
             break;
         }
     }
-    const Sched sc = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(),
-                            best.P, loc.warp_slots.empty() ? nullptr : &loc.warp_slots);
+    sc = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(), best.P,
+                loc.warp_slots.empty() ? nullptr : &loc.warp_slots);
     if (!loc.warp_slots.empty()) {  // sums formed per tile, from the schedule's formations
         loc.formed = 0;
         for (uint32_t wi = 0; wi < best.W; ++wi) {
@@ -1611,8 +1823,9 @@ int lower_tiled(fiona_plan *p)
                 if (sc.w[op0 + f] & kOpSeg) loc.formed += sc.w[op0 + f] & (kOpMaxSources - 1);
         }
     }
-    best.smem = sc.w.size() * 4 + (size_t)(hp.n_in + lw.nodes.size() + 1) * PB * (best.dbl ? 2 : 1) +
-                (size_t)jp.n_part * PB + (size_t)loc.n_slots * PB + 32;
+    }  // !use_tc
+    best.smem = sc.w.size() * 4 + (size_t)(hp.n_in + lw.nodes.size() + 1) * PB * nbuf + (size_t)jp.n_part * PB +
+                (size_t)loc.n_slots * PB + 32;
     TiledSchedule *ts = new (std::nothrow) TiledSchedule;
     if (!ts) return set_error(FIONA_ERR_NOMEM, "tiled schedule: host allocation");
     ts->C = best.C;
@@ -1623,7 +1836,10 @@ int lower_tiled(fiona_plan *p)
     ts->has_const = has_const;
     ts->smem = best.smem;
     ts->ctas_per_sm = best.ctas;
-    ts->nodes_kept = (uint32_t)lw.nodes.size() + loc.formed;
+    ts->tc = use_tc;
+    // (the group sums of the tensor-core variant are not shared sums: every
+    // shared sum is expanded into them)
+    ts->nodes_kept = use_tc ? 0 : (uint32_t)lw.nodes.size() + loc.formed;
     ts->nodes_expanded = (uint32_t)ni.ids.size() - std::min<uint32_t>((uint32_t)ni.ids.size(), ts->nodes_kept);
     TiledArgs &a = ts->args;
     a.n_slots = loc.n_slots;
@@ -1651,6 +1867,15 @@ int lower_tiled(fiona_plan *p)
     a.n_boxes = (2 * hp.n_in + 255) / 256;
     a.box_rows = a.n_boxes ? (2 * hp.n_in + a.n_boxes - 1) / a.n_boxes : 0;
     a.has_pt = hp.n_pt ? 1 : 0;
+    if (use_tc) {
+        a.tc_groups = (uint32_t)tc.nodes.size();
+        a.tc_k = tc.K;
+        a.tc_n = tc.N;
+        a.tc_cols = tc.cols;
+        a.tc_wabs = tc.wabs;
+        a.o_tcw = o_tcw;
+        a.o_tcm = o_tcm;
+    }
     ts->addsub = count_addsub(sc.w, a, best.W);
     if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB, best.P)) {
         delete ts;
@@ -1660,8 +1885,12 @@ int lower_tiled(fiona_plan *p)
         delete ts;
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
     }
+    if (const char *why = check_tc(sc.w, a)) {
+        delete ts;
+        return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
+    }
     if (device) {
-        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, ts->smem);
+        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, use_tc, ts->smem);
         if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
         if (rc != FIONA_OK) {
             cudaFree(ts->sched.blob);

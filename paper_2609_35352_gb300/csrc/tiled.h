@@ -40,6 +40,8 @@
 //   segment streams per SEG operation, in order: a program as above
 //   target streams  per job: output index, or kPartBit | partial slot
 //   combine lists   per split output: its partial slots
+//   (tensor-core sums only) W as fp16 core matrices, then one fp32 constant
+//                   per group (tc_signed.cuh)
 // Source index s names the tile pair (c0, c1) at s * 2T words of the source
 // region: inputs first, then the materialised shared sums in level order,
 // then the zero tile.  Programs name warp slots in their slot word (see
@@ -50,6 +52,7 @@
 #include <stdint.h>
 
 #include "fiona_internal.h"
+#include "tc_geometry.h"
 
 // most warps per CTA (the kernels are built for it: at most 128 registers a
 // thread; a bound of 20 warps measured slower, its register cap spills)
@@ -97,6 +100,14 @@ struct TiledArgs {
     uint32_t has_pt;         // 0: the plan has no plaintexts (every load reads the schedule)
     uint32_t n_slots;        // warp slots of the CTA (shared signed sums a warp forms for itself);
                              // a warp's own start at the slot its table entry names
+    // tensor-core signed sums (tc_signed.cuh; tc_groups = 0: none): the
+    // n_nodes = tc_groups level-0 nodes are formed as one contraction per
+    // tile, by the kernel variant built for it, instead of by their programs
+    uint32_t tc_groups;
+    uint32_t tc_k, tc_n;     // TcGeometry
+    uint32_t tc_cols;        // tensor memory columns a CTA allocates
+    uint32_t tc_wabs;        // largest sum of |weights| of a group: S + tc_wabs * q > 0
+    uint32_t o_tcw, o_tcm;   // word offsets of W (fp16 image) and of the groups' magic constants
 };
 
 // Warp-specialised variant (kernel_ws.cu), two coefficients per lane.  The
@@ -165,6 +176,7 @@ struct TiledSchedule {
     uint32_t nodes_expanded = 0;  // shared sums expanded into their uses
     DeviceSchedule sched;
     TiledArgs args{};          // device pointers (data pointers unset)
+    bool tc = false;           // the scale groups' signed sums run on the tensor cores (args.tc_groups)
     bool ws = false;           // the warp-specialised kernel runs this plan
     uint32_t ring = 0;         // its plaintext ring depth D (groups of P slots per warp)
     WsArgs ws_args{};

@@ -65,8 +65,9 @@ class PlanStats(ctypes.Structure):
         "n_inputs_used", "n_plaintexts_used", "bytes_min", "wide_products")] + \
         [(n, ctypes.c_uint32) for n in (
             "N", "L", "n_in", "n_out", "n_pt", "n_groups", "tile_coeffs", "warps_per_cta",
-            "smem_bytes", "ctas_per_sm", "kernel", "nodes_materialized", "addsub_executed")] + \
-        [("reserved", ctypes.c_uint32 * 3)]
+            "smem_bytes", "ctas_per_sm", "kernel", "nodes_materialized", "addsub_executed",
+                  "tensor_core_sums")] + \
+        [("reserved", ctypes.c_uint32 * 2)]
 
     def as_dict(self) -> Dict[str, int]:
         return {n: int(getattr(self, n)) for n, _ in self._fields_ if n != "reserved"}

@@ -103,3 +103,35 @@ def test_warp_formed_sums_lower_exactly(monkeypatch):
         plan = lower(desc, 4096, bits, 2)
         formed.append(plan.stats()["nodes_materialized"])
     assert sum(1 for f in formed if f > 0) >= 12, formed
+
+
+def test_tensor_core_sums_lower_exactly(monkeypatch):
+    """FIONA_TILED_TC=1: every used scale group's signed sum becomes one
+    group source formed by the tensor-core contraction; plan creation checks
+    the schedule's linear map (the group programs) and decodes the fp16
+    weight image and the groups' constants back against those programs
+    (failing with FIONA_ERR_INTERNAL otherwise).  Random compiled layers with
+    one coefficient per lane and batches of 16 (shared sums expanded into the
+    groups), the VGG layer, and the layers that cannot take it: moduli of 59
+    bits, and BERT's 96 groups (tensor memory holds at most 28 next to its
+    96 inputs)."""
+    monkeypatch.setenv("FIONA_TILED_TC", "1")
+    taken = 0
+    for seed in range(16):
+        rng = np.random.default_rng(9300 + seed)
+        monkeypatch.setenv("FIONA_TILED_SHAPE", ["1,4,1,-1,16", "1,8,0,-1,16", "1,16,1,-1,16"][seed % 3])
+        desc = random_layer(rng, big=seed % 2 == 1)
+        plan = lower(desc, 4096, int(rng.choice([40, 50])), 2)
+        taken += plan.stats()["tensor_core_sums"] > 0
+    # (the others: a single output, which runs the direct kernel, or more
+    # groups than tensor memory holds next to the inputs' chunks)
+    assert taken >= 8
+    monkeypatch.delenv("FIONA_TILED_SHAPE")
+    for name, want in (("vgg", 16), ("bert", 0), ("overflow60", 0)):
+        wl = W.make_workload(name)
+        plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
+        assert plan.stats()["tensor_core_sums"] == want, name
+    monkeypatch.delenv("FIONA_TILED_TC")
+    wl = W.make_workload("vgg")
+    plan = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan)
+    assert plan.stats()["tensor_core_sums"] == 0  # the ALU sums are the default

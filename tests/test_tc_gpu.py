@@ -1,0 +1,87 @@
+"""GPU parity of the tiled kernel's tensor-core signed sums (tc_signed.cuh):
+every scale group's signed sum formed per tile as one contraction of the
+inputs (cut into 10-bit fp16 chunks) with the layer's ternary weights on the
+tensor cores, then reduced exactly (Sec. 4.2 "Grouping Reconstruction
+Operations": the sum is the same element of Z_q however it is formed).  The
+bar is bit-exact equality with the CPU oracle."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+pytestmark = pytest.mark.gpu
+
+import oracle  # noqa: E402
+from paper_2609_35352_gb300 import build as B  # noqa: E402
+from paper_2609_35352_gb300 import fiona as F  # noqa: E402
+from paper_2609_35352_gb300 import workloads as W  # noqa: E402
+
+from gpu_util import DeviceLayer  # noqa: E402
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    B.build()
+
+
+# (layer, N, L, shape override "C,W,regions,keep,P" or None): warps per
+# tensor-memory quarter 1 to 4, one and two source regions, several tiles per
+# CTA (the contraction's barrier and tensor memory reused), residues q - 1
+# everywhere (overflow50), shared sums expanded into the groups (vit,
+# tiny-dag), a single output (wsum-ternary), inputs not a multiple of 16
+# (vit: 32, tiny-dag: 8 -> zero rows of W).
+CASES = [
+    ("vgg", 1024, 2, None),
+    ("vgg", 4096, 3, "1,16,1,-1,16"),
+    ("vgg", 4096, 3, "1,12,1,-1,16"),
+    ("vgg", 2048, 2, "1,8,0,-1,16"),
+    ("vgg", 2048, 2, "1,4,1,-1,16"),
+    ("overflow50", None, None, "1,16,1,-1,16"),
+    ("vit", 2048, 2, "1,16,1,-1,16"),
+    ("tiny-dag", None, None, "1,4,1,-1,16"),
+    ("tiny", None, None, "1,8,0,-1,16"),
+    ("wsum-ternary", 1024, 3, "1,4,1,-1,16"),
+]
+
+
+@pytest.mark.parametrize("name,N,L,shape", CASES)
+def test_tensor_core_sums_parity(name, N, L, shape, monkeypatch):
+    monkeypatch.setenv("FIONA_TILED_TC", "1")
+    if shape:
+        monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+    wl = W.make_workload(name, N=N, L=L)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel("tiled")
+    st = dl.plan.stats()
+    assert st["tensor_core_sums"] > 0, st
+    if shape:
+        f = [int(v) for v in shape.split(",")]
+        assert (st["tile_coeffs"], st["warps_per_cta"]) == (32 * f[0], f[1]), st
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    for _ in range(2):  # the second launch on a dirty output buffer
+        dl.run()
+        mism = np.argwhere(dl.outputs() != want)
+        assert mism.shape[0] == 0, "first mismatches (j, c, l, k): %s" % mism[:5].tolist()
+    assert dl.ctx.device_check() == F.FIONA_OK
+
+
+def test_tensor_core_sums_match_the_alu_sums(monkeypatch):
+    """The same layer with the sums on the ALUs (the default) gives the same
+    residues, on inputs the device generator fills."""
+    wl = W.make_workload("vgg", N=4096, L=2)
+    monkeypatch.setenv("FIONA_TILED_TC", "1")
+    dl = DeviceLayer(wl, host_inputs=False)
+    dl.plan.select_kernel("tiled")
+    assert dl.plan.stats()["tensor_core_sums"] == 16
+    dl.run()
+    got_tc = dl.outputs().copy()
+    monkeypatch.delenv("FIONA_TILED_TC")
+    alu = F.Plan(dl.ctx, wl.plan)
+    alu.select_kernel("tiled")
+    assert alu.stats()["tensor_core_sums"] == 0
+    dl.d_out.fill_(-1)
+    alu.eval(dl.d_in, dl.d_pt, dl.d_out)
+    assert np.array_equal(dl.outputs(), got_tc)
+    assert dl.ctx.device_check() == F.FIONA_OK
