@@ -225,10 +225,14 @@ class _Nvml:
 
 class ClockSampler:
     """SM clock, power and throttle reasons of one GPU while the timed region
-    runs.  NVML is polled every 2 ms from a thread, and once synchronously at
-    start() and at mark_end() (both inside the timed region, the GPU busy with
-    queued work), so that even a region of a few milliseconds has samples.
-    Without NVML, nvidia-smi samples every 20 ms instead."""
+    runs.  NVML is polled every millisecond from a thread started before the
+    region (an NVML query can take a millisecond: none runs on the launching
+    thread before the last launch is queued, so the GPU never waits for one);
+    mark_begin() after the first launch is queued opens the window, a
+    synchronous sample at mark_end() (the GPU still busy with queued work)
+    closes it, and stop(t_done) keeps the samples taken from the first launch
+    to the final synchronize.  Without NVML, nvidia-smi samples every 20 ms
+    instead."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -243,6 +247,7 @@ class ClockSampler:
         self.proc = None
         self.file = None
         self.skip = 0
+        self.t_begin = None
         self.source = "nvml"
         try:
             self.nvml = _Nvml(device)
@@ -251,21 +256,21 @@ class ClockSampler:
             self.source = "nvidia-smi"
 
     def _take(self):
+        t0 = time.monotonic()
         s = self.nvml.sample()
         if s is not None:
             names = [n for b, n in _NVML_REASONS.items() if s[3] & b]
-            self.samples.append((s[0], s[1], s[2], names))
+            self.samples.append((s[0], s[1], s[2], names, t0))
 
     def _loop(self):
         while not self.stop_flag:
             self._take()
-            time.sleep(0.002)
+            time.sleep(0.001)
 
     def start(self):
-        """Call right after the timed region's first launch is queued."""
+        """Call before the timed region."""
         if self.nvml is not None:
             import threading
-            self._take()
             self.thread = threading.Thread(target=self._loop, daemon=True)
             self.thread.start()
             return
@@ -278,16 +283,24 @@ class ClockSampler:
         except (OSError, ValueError):
             self.proc = None
 
+    def mark_begin(self):
+        """Call right after the timed region's first launch is queued."""
+        self.t_begin = time.monotonic()
+
     def mark_end(self):
         """Call after the last launch is queued, before the final synchronize."""
         if self.nvml is not None:
             self._take()
 
-    def stop(self) -> dict:
+    def stop(self, t_done=None) -> dict:
+        """`t_done`: time.monotonic() right after the region's final synchronize."""
         if self.nvml is not None:
             self.stop_flag = True
             if self.thread is not None:
                 self.thread.join(timeout=2)
+            lo = self.t_begin if self.t_begin is not None else float("-inf")
+            hi = t_done if t_done is not None else float("inf")
+            self.samples = [x for x in self.samples if lo <= x[4] <= hi]
         elif self.proc is not None:
             self.proc.terminate()
             try:
@@ -329,7 +342,8 @@ def measured_peak():
 
 
 KERNEL_FILES = {"direct": ["kernel_direct.cu", "rns.cuh"],
-                "tiled": ["kernel_tiled.cu", "tiled.h", "lower_tiled.cpp", "rns.cuh"]}
+                "tiled": ["kernel_tiled.cu", "tiled.h", "lower_tiled.cpp", "rns.cuh", "tile_math.cuh",
+                          "tc_signed.cuh", "tc_geometry.h"]}
 
 
 def kernel_source_hash(kernel: str) -> str:
@@ -492,6 +506,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     clocks = ClockSampler(dev)
+    clocks.start()
     barrier()
     torch.cuda.synchronize()
     t_begin = torch.cuda.Event(enable_timing=True)
@@ -502,12 +517,13 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
         plan.eval(d_in, d_pt, d_out, stream=stream)
         stops[s].record(stream)
         if s == 0:
-            clocks.start()
+            clocks.mark_begin()
     t_end.record(stream)
     clocks.mark_end()
     torch.cuda.synchronize()
+    t_done = time.monotonic()
     barrier()
-    clk = clocks.stop()
+    clk = clocks.stop(t_done)
     elapsed_ms = t_begin.elapsed_time(t_end)
     kernel_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
     elapsed_ms = max_over_ranks(elapsed_ms)
@@ -653,6 +669,7 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     stops = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     clocks = ClockSampler(dev)
+    clocks.start()
     barrier()
     torch.cuda.synchronize()
     for s in range(args.steps):
@@ -660,11 +677,12 @@ def run_rescale(args, rank: int, world: int, local_rank: int) -> None:
         ctx.rescale(L, count, d_y, d_o, stream=stream)
         stops[s].record(stream)
         if s == 0:
-            clocks.start()
+            clocks.mark_begin()
     clocks.mark_end()
     torch.cuda.synchronize()
+    t_done = time.monotonic()
     barrier()
-    clk = clocks.stop()
+    clk = clocks.stop(t_done)
     step_ms = [a.elapsed_time(b) for a, b in zip(starts, stops)]
     elapsed_ms = sum(step_ms)
     elapsed_ms = max_over_ranks(elapsed_ms)
@@ -799,6 +817,7 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     clocks = ClockSampler(dev)
+    clocks.start()
     barrier()
     torch.cuda.synchronize()
     for i, (a, b, c) in enumerate(ev):
@@ -808,11 +827,12 @@ def run_encode(args, rank: int, world: int, local_rank: int) -> None:
         ctx.encode_coeffs(L, count, d_c, d_o, stream=stream)
         c.record(stream)
         if i == 0:
-            clocks.start()
+            clocks.mark_begin()
     clocks.mark_end()
     torch.cuda.synchronize()
+    t_done = time.monotonic()
     barrier()
-    clk = clocks.stop()
+    clk = clocks.stop(t_done)
     if ctx.device_check(stream) != F.FIONA_OK:
         raise RuntimeError("encoding reported a coefficient out of range")
     step_ms = [a.elapsed_time(c) for a, b, c in ev]
