@@ -432,9 +432,9 @@ int fiona_check_residues(const fiona_ctx *ctx, void *cuda_stream, const uint64_t
 
 /* Report kernel-side failures of earlier calls on this context:
  * synchronises `cuda_stream`, then returns FIONA_ERR_TIMEOUT if a tiled
- * kernel gave up waiting for its bulk copies (every such wait is bounded; the
- * CTA then stops: the outputs of that evaluation are undefined, the context
- * stays usable), FIONA_ERR_RANGE if an encoding met a
+ * kernel gave up waiting for its bulk copies or its tensor-core contraction
+ * (every such wait is bounded; the CTA then stops: the outputs of that
+ * evaluation are undefined, the context stays usable), FIONA_ERR_RANGE if an encoding met a
  * coefficient out of range (fiona_ckks_embed), FIONA_ERR_CUDA on a CUDA
  * error, FIONA_OK otherwise; the flags are cleared. */
 int fiona_device_check(const fiona_ctx *ctx, void *cuda_stream);

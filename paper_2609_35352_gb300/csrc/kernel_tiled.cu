@@ -34,11 +34,15 @@
 //  5. The next tile's inputs are prepared (with two regions: their copies,
 //     started at the top of this tile, waited for and rewritten) before the
 //     one barrier per tile that publishes them.
-// The spin-waits are bounded: thread 0's wait for the schedule copy and each
-// thread's wait for a region's TMA copies.  One that gives up raises the
-// context's error flag; the CTA then stops at its next barrier (thread 0
-// first waits, bounded again, for the copies it issued), leaving the tiles
-// it did not reach unwritten.
+// The waits are bounded: thread 0's wait for the schedule copy (about two
+// seconds), and each thread's wait for a region's TMA copies and for the
+// tensor-core contraction (TiledArgs::wait_ns, measured on the global
+// timer; a wait also ends once another thread of the CTA gave up).  One
+// that gives up raises the context's error flag; the CTA then stops at its
+// next barrier (thread 0 first waits, bounded again, for the copies and the
+// contraction it issued, and the CTA frees its tensor memory).  The tile in
+// progress is computed from whatever its region holds, and the tiles the
+// CTA did not reach stay unwritten: outputs are undefined after a timeout.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -47,6 +51,7 @@
 #include <cstring>
 #include <mutex>
 
+#include "async.cuh"
 #include "tc_signed.cuh"
 #include "tiled.h"
 #include "tile_math.cuh"
@@ -96,23 +101,9 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm,
         : "memory");
 }
 
-// Bounded wait (no suspend hint: a tile's copies land within microseconds)
-// for phase `parity` of the barrier; false if it gave up after 2^24 tries.
-__device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity)
-{
-    for (uint32_t it = 0; it < (1u << 24); ++it) {
-        uint32_t ok;
-        asm volatile(
-            "{\n\t.reg .pred p;\n\t"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-            "selp.u32 %0, 1, 0, p;\n\t}"
-            : "=r"(ok)
-            : "r"(bar), "r"(parity)
-            : "memory");
-        if (ok) return true;
-    }
-    return false;
-}
+// bound of thread 0's wait, when a CTA stops, for the copies and the
+// contraction it issued
+constexpr uint64_t kDrainNs = 20000000;
 
 // Bulk prefetch of `bytes` (a multiple of 16, 16-byte aligned) into L2.
 __device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes)
@@ -291,7 +282,9 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         if constexpr (TMA) {
             if (threadIdx.x != 0) return;
             const uint32_t bar = bar_stage + 8 * reg;
-            mbar_expect_tx(bar, a.n_boxes * a.box_rows * TB);
+            // (test only: the CTA's first copy expects 16 bytes that never come)
+            const uint32_t extra = (a.test_flags & kTiledFlagExtraTx) && t == blockIdx.x ? 16 : 0;
+            mbar_expect_tx(bar, a.n_boxes * a.box_rows * TB + extra);
             for (uint32_t j = 0; j < a.n_boxes; ++j) {
                 const uint32_t z = min(j * a.box_rows, 2 * a.n_in - a.box_rows);
                 tma_load_3d(dst + z * TB, &tm_in, k0, l, z, bar);
@@ -316,7 +309,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         if (threadIdx.x == 0) s_limb[reg] = a.limbs[a.limb0 + t / a.tiles_per_limb];
         if (!a.n_in) return;
         if constexpr (TMA) {
-            if (!mbar_wait_spin(bar_stage + 8 * reg, (stage_phase >> reg) & 1u)) {
+            if (!async::mbar_wait_bounded(bar_stage + 8 * reg, (stage_phase >> reg) & 1u, &s_abort, a.wait_ns)) {
                 s_abort = 1;  // the CTA stops after the next barrier
                 atomicOr(a.err, 1);
                 failed = 1 + reg + 2 * ((stage_phase >> reg) & 1u);
@@ -353,8 +346,10 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
         }
     };
     auto stop = [&]() {
-        if (TMA && threadIdx.x == 0 && failed) mbar_wait_spin(bar_stage + 8 * ((failed - 1) & 1), (failed - 1) >> 1);
-        if (TC && threadIdx.x == 0 && tc_failed) mbar_wait_spin(bar_tc, tc_failed - 1);
+        const int never = 0;
+        if (TMA && threadIdx.x == 0 && failed)
+            async::mbar_wait_bounded(bar_stage + 8 * ((failed - 1) & 1), (failed - 1) >> 1, &never, kDrainNs);
+        if (TC && threadIdx.x == 0 && tc_failed) async::mbar_wait_bounded(bar_tc, tc_failed - 1, &never, kDrainNs);
         if constexpr (TC) __syncthreads();
         release();
     };
@@ -410,7 +405,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
             __syncthreads();
             tcs::fence_after();
             if (threadIdx.x == 0) tcs::issue(tmem, smem_addr(sm) + a.o_tcw * 4, geo, bar_tc);
-            if (!mbar_wait_spin(bar_tc, tc_phase)) {
+            if (!async::mbar_wait_bounded(bar_tc, tc_phase, &s_abort, a.wait_ns)) {
                 s_abort = 1;  // the CTA stops after this tile's last barrier
                 atomicOr(a.err, 1);
                 tc_failed = 1 + tc_phase;
@@ -426,9 +421,10 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
             tcs::fence_before();
             __syncthreads();
         }
-        // 2. materialised shared sums, children first
-        const uint32_t n_levels = TC ? 0 : a.n_levels;  // TC: its one level is the contraction
-        for (uint32_t lev = 0; lev < n_levels; ++lev) {
+        // 2. materialised shared sums, children first (TC: its one level is
+        //    the contraction)
+        if constexpr (!TC)
+        for (uint32_t lev = 0; lev < a.n_levels; ++lev) {
             for (uint32_t x = sw[a.o_level + lev] + warp; x < sw[a.o_level + lev + 1]; x += n_warps) {
                 V<C> u0, u1;
                 signed_sum<SPLIT, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, 0, u0, u1);

@@ -1876,6 +1876,13 @@ int lower_tiled(fiona_plan *p)
         a.o_tcw = o_tcw;
         a.o_tcm = o_tcm;
     }
+    a.wait_ns = 2000000000ull;
+    if (const char *t = getenv("FIONA_TEST_TILED_TIMEOUT")) {  // test only: a copy wait that runs out
+        if (atoi(t) > 0 && best.C == 1 && hp.n_in) {
+            a.test_flags |= kTiledFlagExtraTx;
+            a.wait_ns = 2000000ull;
+        }
+    }
     ts->addsub = count_addsub(sc.w, a, best.W);
     if (const char *why = check_schedule(sc.w, a, best.W, hp.n_out, hp.n_pt, ts->smem, PB, best.P)) {
         delete ts;

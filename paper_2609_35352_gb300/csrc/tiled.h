@@ -77,6 +77,8 @@ constexpr uint32_t kOpMaxPlaintexts = 1u << (32 - kOpPtShift);
 
 // per warp: op offset, op count, seg offset, target offset, first slot
 constexpr uint32_t kWarpTableWords = 8;
+// test only: the first input copy of each CTA expects 16 bytes that never come
+constexpr uint32_t kTiledFlagExtraTx = 1;
 
 struct TiledArgs {
     const uint64_t *in;
@@ -108,6 +110,8 @@ struct TiledArgs {
     uint32_t tc_cols;        // tensor memory columns a CTA allocates
     uint32_t tc_wabs;        // largest sum of |weights| of a group: S + tc_wabs * q > 0
     uint32_t o_tcw, o_tcm;   // word offsets of W (fp16 image) and of the groups' magic constants
+    uint64_t wait_ns;        // bound of the waits for input copies and for the contraction
+    uint32_t test_flags;     // kTiledFlag* (0 outside tests)
 };
 
 // Warp-specialised variant (kernel_ws.cu), two coefficients per lane.  The

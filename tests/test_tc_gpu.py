@@ -85,3 +85,32 @@ def test_tensor_core_sums_match_the_alu_sums(monkeypatch):
     alu.eval(dl.d_in, dl.d_pt, dl.d_out)
     assert np.array_equal(dl.outputs(), got_tc)
     assert dl.ctx.device_check() == F.FIONA_OK
+
+
+@pytest.mark.parametrize("tc,shape", [("0", "1,16,1,-1,16"), ("1", "1,16,1,-1,16"), ("0", "1,8,0,-1,16")])
+def test_tiled_copy_wait_runs_out(tc, shape, monkeypatch):
+    """A test-only plan (FIONA_TEST_TILED_TIMEOUT) whose first input copy per
+    CTA expects 16 bytes more than its TMA boxes bring, with waits bounded at
+    2 ms: every thread's wait for the tile runs out, the CTA stops (thread 0
+    waits, bounded, for its copies; the tensor-core variant frees its tensor
+    memory), fiona_device_check reports FIONA_ERR_TIMEOUT once, and the next
+    evaluation on the same context is exact."""
+    monkeypatch.setenv("FIONA_TILED_TC", tc)
+    monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+    monkeypatch.setenv("FIONA_TEST_TILED_TIMEOUT", "1")
+    wl = W.make_workload("vgg", N=2048, L=2)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel("tiled")
+    assert (dl.plan.stats()["tensor_core_sums"] > 0) == (tc == "1")
+    dl.run()
+    torch.cuda.synchronize()
+    assert dl.ctx.device_check() == F.FIONA_ERR_TIMEOUT
+    assert dl.ctx.device_check() == F.FIONA_OK  # the flag was cleared
+    monkeypatch.delenv("FIONA_TEST_TILED_TIMEOUT")
+    plan = F.Plan(dl.ctx, wl.plan)
+    plan.select_kernel("tiled")
+    plan.eval(dl.d_in, dl.d_pt, dl.d_out)
+    torch.cuda.synchronize()
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    assert np.array_equal(dl.outputs(), want)
+    assert dl.ctx.device_check() == F.FIONA_OK
