@@ -389,8 +389,9 @@ int fiona_encode(const fiona_ctx *ctx, void *cuda_stream, uint32_t L_cur, uint64
  * `d_inputs`, evaluates with the device-resident `d_plaintexts` (the model's
  * weights stay on the GPU), and copies the result through `d_outputs` to
  * `h_outputs` (host, [n_out][2][L][N]).  The work is split into limb chunks
- * so the copies of one chunk overlap the kernel of another (RNS limbs are
- * independent).  Synchronous: returns when h_outputs holds the result.
+ * (one limb each, at most 16 chunks) so the copies of one chunk overlap the
+ * kernel of another (RNS limbs are independent).  Synchronous: returns when
+ * h_outputs holds the result.
  * Errors as fiona_linear_eval. */
 int fiona_linear_eval_host(const fiona_plan *plan, void *cuda_stream, const uint64_t *h_inputs,
                            const uint64_t *d_plaintexts, uint64_t *h_outputs,

@@ -839,8 +839,11 @@ extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const u
     const size_t pitch = (size_t)L * N * 8;
     cudaStream_t s = (cudaStream_t)stream;
     cudaStream_t sin = (cudaStream_t)p->copy_in_stream, sout = (cudaStream_t)p->copy_out_stream;
-    const uint32_t chunks = std::min<uint32_t>(L, 4);
-    cudaEvent_t ev[2 * 4 + 1];
+    // one limb per chunk (at most 16 chunks): the pipeline's fill and drain
+    // (the first chunk's input copy, the last one's output copy) stay short
+    constexpr uint32_t kMaxChunks = 16;
+    const uint32_t chunks = std::min<uint32_t>(L, kMaxChunks);
+    cudaEvent_t ev[2 * kMaxChunks + 1];
     int made = 0;
     cudaError_t e = cudaSuccess;
     for (int i = 0; i < 2 * (int)chunks + 1 && e == cudaSuccess; ++i, ++made)
