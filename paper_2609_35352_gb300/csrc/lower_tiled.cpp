@@ -1774,7 +1774,33 @@ int lower_tiled(fiona_plan *p)
         for (uint32_t max_slots = 8; max_slots >= 1; max_slots /= 2) {
             JobPlan jt = jp;
             LocalResult r = localize(jt, groups, ni, budget, max_slots);
-            const Sched st = encode(jt, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in, best.P, &r.warp_slots);
+            Sched st = encode(jt, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in, best.P, &r.warp_slots);
+            // when some warps have more operation slots than others, those
+            // set the tile's length: a formation there (its run sums,
+            // reduction and store before the batch that needs it) lengthens
+            // every tile, so those warps keep their groups expanded (measured
+            // on the ViT layer: 0.943 ms with two of its four formations on
+            // such warps, 0.906 ms with none formed)
+            std::vector<uint32_t> crit;
+            if (r.formed && !getenv("FIONA_WARP_SUMS_ANYWHERE")) {
+                uint32_t most = 0, least = ~0u;
+                for (uint32_t wi = 0; wi < best.W; ++wi) {
+                    most = std::max(most, st.w[st.o_warp + wi * kWarpTableWords + 1]);
+                    least = std::min(least, st.w[st.o_warp + wi * kWarpTableWords + 1]);
+                }
+                for (uint32_t wi = 0; wi < best.W && least < most; ++wi)
+                    if (r.warp_slots[wi] && st.w[st.o_warp + wi * kWarpTableWords + 1] == most) crit.push_back(wi);
+                if (!crit.empty()) {
+                    for (uint32_t wi : crit) {  // this warp keeps its expanded groups
+                        jt.per_warp[wi] = jp.per_warp[wi];
+                        r.n_slots -= r.warp_slots[wi];
+                        r.warp_slots[wi] = 0;
+                    }
+                    r.formed = 0;
+                    for (uint32_t wi = 0; wi < best.W; ++wi) r.formed += r.warp_slots[wi] ? 1 : 0;
+                    st = encode(jt, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in, best.P, &r.warp_slots);
+                }
+            }
             const size_t sm = st.w.size() * 4 + (size_t)(hp.n_in + 1) * PB * (best.dbl ? 2 : 1) +
                               (size_t)jt.n_part * PB + (size_t)r.n_slots * PB + 32;
             if (getenv("FIONA_TILED_DEBUG"))
@@ -1798,6 +1824,7 @@ int lower_tiled(fiona_plan *p)
                 JobPlan jk = jp;
                 std::vector<std::vector<Job>> saved = jk.per_warp;
                 r = localize(jk, groups, ni, budget, 1);
+                for (uint32_t wi : crit) keep_w[wi] = 0;
                 for (uint32_t wi = 0; wi < best.W; ++wi)
                     if (!keep_w[wi]) {  // this warp keeps its expanded groups
                         jk.per_warp[wi] = saved[wi];
