@@ -16,7 +16,7 @@ from paper_2609_35352_gb300 import build as B  # noqa: E402
 from paper_2609_35352_gb300 import fiona as F  # noqa: E402
 from paper_2609_35352_gb300 import workloads as W  # noqa: E402
 
-from gpu_util import DeviceLayer  # noqa: E402
+from gpu_util import DeviceLayer, oracle_at, to_host  # noqa: E402
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -114,3 +114,36 @@ def test_tiled_copy_wait_runs_out(tc, shape, monkeypatch):
     want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
     assert np.array_equal(dl.outputs(), want)
     assert dl.ctx.device_check() == F.FIONA_OK
+
+
+def test_tensor_core_sums_full_size(monkeypatch):
+    """The full VGG layer (N = 2^16, 20 limbs, inputs filled on the device)
+    with the tensor-core sums: outputs at sampled (limb, coefficient)
+    coordinates equal the oracle's, every residue is canonical, and every
+    residue equals the ALU sums' result."""
+    monkeypatch.setenv("FIONA_TILED_TC", "1")
+    wl = W.make_workload("vgg")
+    dl = DeviceLayer(wl, host_inputs=False)
+    dl.plan.select_kernel("tiled")
+    assert dl.plan.stats()["tensor_core_sums"] == 16
+    dl.run()
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(43)
+    limbs = rng.integers(0, wl.L, 48)
+    coefs = rng.integers(0, wl.N, 48)
+    coefs[:2] = [0, wl.N - 1]
+    want = oracle_at(wl, limbs, coefs)
+    out = dl.d_out.view(wl.plan.n_out, 2, wl.L, wl.N)
+    got = to_host(out[:, :, torch.from_numpy(limbs).cuda(), torch.from_numpy(coefs).cuda()].contiguous())
+    assert np.array_equal(got.reshape(want.shape), want)
+    assert dl.ctx.check_residues(dl.d_out, wl.plan.n_out * 2) == F.FIONA_OK
+    assert dl.ctx.device_check() == F.FIONA_OK
+    first = dl.d_out.clone()
+    monkeypatch.delenv("FIONA_TILED_TC")
+    alu = F.Plan(dl.ctx, wl.plan)
+    alu.select_kernel("tiled")
+    assert alu.stats()["tensor_core_sums"] == 0
+    dl.d_out.fill_(-1)
+    alu.eval(dl.d_in, dl.d_pt, dl.d_out)
+    torch.cuda.synchronize()
+    assert torch.equal(first, dl.d_out)
