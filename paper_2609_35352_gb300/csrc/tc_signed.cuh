@@ -5,13 +5,16 @@
 // All scale groups' signed sums of a tile (Sec. 4.2 "Grouping
 // Reconstruction Operations") form the product S = A W of the tile's inputs
 // A (rows: the 64 (poly, coefficient) pairs; columns: the inputs) and the
-// layer's ternary weight matrix W (inputs x groups, entries t in {-1, 0,
-// +1}).  Residues have 50 bits; each is cut into five 10-bit chunks v, held
-// exactly in fp16 as 1024 + v (exponent of 1024, mantissa v), so
+// layer's weight matrix W (inputs x groups: each input's net sign in the
+// group, t in {-1, 0, +1}, or a small integer where expanded shared sums
+// repeat an input).  Residues have 50 bits; each is cut into five 10-bit
+// chunks v, held exactly in fp16 as 1024 + v (exponent of 1024, mantissa
+// v), so
 //   S = sum_j 2^(10 j) (A_j W - 1024 * colsum(W))
 // where A_j holds chunk j.  The tensor cores compute each A_j W with f32
 // accumulation, exact because every partial sum is an integer below 2^24
-// (at most 2047 * K for K inputs).  The chunk matrices go to tensor memory
+// (at most 2047 * sum |w| over a group; the lowering checks the bound).  The
+// chunk matrices go to tensor memory
 // (TMEM, the A operand; M = 64 rows, 16 rows per warp quarter: row 16 q + l
 // in lane 32 q + l), W sits in shared memory in the canonical K-major layout
 // without swizzle (core matrices of 8 rows x 16 bytes), and each D_j = A_j W
@@ -47,15 +50,8 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols)
 __device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// eight 32-bit columns of this warp's lanes from column `col` (TMEM address
-// `taddr` = lane << 16 | column)
-__device__ __forceinline__ void st8(uint32_t taddr, const uint32_t (&v)[8])
-{
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
-                 "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
-                 : "memory");
-}
-
+// four 32-bit columns of this warp's lanes from the TMEM address `taddr`
+// (lane << 16 | column)
 __device__ __forceinline__ void st4(uint32_t taddr, const uint32_t (&v)[4])
 {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(v[0]), "r"(v[1]),
@@ -65,6 +61,7 @@ __device__ __forceinline__ void st4(uint32_t taddr, const uint32_t (&v)[4])
 
 __device__ __forceinline__ void wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
+// four 32-bit columns of this warp's lanes from `taddr` (complete after wait_ld)
 __device__ __forceinline__ void ld4(uint32_t taddr, uint32_t (&v)[4])
 {
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"

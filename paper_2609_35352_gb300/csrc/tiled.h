@@ -20,8 +20,9 @@
 // plaintext tiles each warp keeps in flight): every job
 // starts a batch and is padded to whole batches; SEG and FOLD only open a
 // batch (a SEG's signed sum is formed before its batch) and LAST only closes
-// one.  (Measured: letting jobs end mid-batch, to pad less, costs more in the
-// loop than the padding it saves.)  A job is one output, or one part of an
+// one.  (Measured: a LAST test on every operation, so that jobs could end
+// inside a batch and pad less, slows the loop by 15-50%, more than the
+// padding it could save.)  A job is one output, or one part of an
 // output split across warps whose reduced partial sums are added at the end
 // of the tile.
 //
