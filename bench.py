@@ -595,7 +595,8 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
             "kernel": {"name": kernel, "tile_coeffs": stats["tile_coeffs"],
                        "warps_per_cta": stats["warps_per_cta"], "ctas_per_sm": stats["ctas_per_sm"],
                        "shared_sums_formed": stats["nodes_materialized"],
-                       "addsub_executed": stats.get("addsub_executed")},
+                       "addsub_executed": stats.get("addsub_executed"),
+                       "tensor_core_sums": stats.get("tensor_core_sums")},
         }
         print(json.dumps(line), flush=True)
     plan.close()
