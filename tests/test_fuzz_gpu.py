@@ -78,6 +78,34 @@ def test_random_layers(seed, monkeypatch):
     assert dl.ctx.device_check() == F.FIONA_OK
 
 
+@pytest.mark.parametrize("seed", range(24))
+def test_random_layers_tensor_core_sums(seed, monkeypatch):
+    """Random compiled layers (shared sums expanded into the groups, so the
+    weights are small integers, not only +-1), 40- and 50-bit primes, one
+    coefficient per lane, 4, 8 or 16 warps: the signed sums on the tensor
+    cores against the oracle, bit-exact, where the plan takes them."""
+    rng = np.random.default_rng(3000 + seed)
+    monkeypatch.setenv("FIONA_TILED_TC", "1")
+    monkeypatch.setenv("FIONA_TILED_SHAPE", ["1,4,1,-1,16", "1,8,0,-1,16", "1,16,1,-1,16"][seed % 3])
+    desc = random_layer(rng)
+    N = int(rng.choice([1024, 2048]))
+    bits = int(rng.choice([40, 50]))
+    L = int(rng.integers(1, 4))
+    wl = W.Workload("fuzz-tc", N, W.ntt_primes(N, bits, L), desc, 7000 + seed)
+    dl = DeviceLayer(wl)
+    try:
+        dl.plan.select_kernel("tiled")
+    except F.FionaError:
+        pytest.skip("the forced shape does not fit this layer")
+    if dl.plan.stats()["tensor_core_sums"] == 0:
+        pytest.skip("no signed sums, or more groups than tensor memory holds")
+    want = oracle.linear_eval(desc, wl.moduli, dl.X, dl.P)
+    dl.run()
+    mism = np.argwhere(dl.outputs() != want)
+    assert mism.shape[0] == 0, (seed, mism[:5].tolist())
+    assert dl.ctx.device_check() == F.FIONA_OK
+
+
 @pytest.mark.parametrize("seed", range(16))
 def test_random_rescales(seed):
     rng = np.random.default_rng(2000 + seed)
