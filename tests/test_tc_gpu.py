@@ -147,3 +147,28 @@ def test_tensor_core_sums_full_size(monkeypatch):
     alu.eval(dl.d_in, dl.d_pt, dl.d_out)
     torch.cuda.synchronize()
     assert torch.equal(first, dl.d_out)
+
+
+def test_tensor_core_sums_with_scale_classes(monkeypatch):
+    """Plaintexts at two scales (fiona_plan_create_classes: one result per
+    output and class, groups split by their scale plaintext's class) with the
+    tensor-core sums: every (output, class) result equals the oracle's."""
+    from gpu_util import to_device
+    monkeypatch.setenv("FIONA_TILED_TC", "1")
+    monkeypatch.setenv("FIONA_TILED_SHAPE", "1,4,1,-1,16")
+    wl = W.make_workload("tiny")
+    cls = W.scale_classes(wl.plan, 2, "routes", seed=5)
+    ctx = F.Context(wl.N, wl.moduli, device=0)
+    plan = F.Plan(ctx, wl.plan, pt_class=cls, n_class=2)
+    plan.select_kernel("tiled")
+    assert plan.stats()["tensor_core_sums"] > 0
+    X, P = wl.host_inputs(), wl.host_plaintexts()
+    p = wl.plan
+    d_out = torch.full((p.n_out * 2 * 2 * wl.L * wl.N,), -1, dtype=torch.int64, device="cuda")
+    plan.eval(to_device(X), to_device(P), d_out)
+    torch.cuda.synchronize()
+    got = to_host(d_out).reshape(p.n_out, 2, 2, wl.L, wl.N)
+    want = oracle.linear_eval_classes(p, wl.moduli, cls, 2, X, P)
+    mism = np.argwhere(got != want)
+    assert mism.shape[0] == 0, "first mismatches (j, s, c, l, k): %s" % mism[:5].tolist()
+    assert ctx.device_check() == F.FIONA_OK
