@@ -190,6 +190,7 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
     const uint32_t total = a.n_limbs * a.tiles_per_limb;
     const uint32_t lane_off = lane * VB;
     const uint32_t *sw = reinterpret_cast<const uint32_t *>(sm);
+    const uint32_t zero = a.zero;  // 0, unknown to the compiler (rns::mac26)
 
     // the schedule, once per CTA (TMA copies want the regions 128-byte
     // aligned: a misaligned base raises the error flag and copies nothing)
@@ -552,8 +553,8 @@ __global__ void __launch_bounds__(kTiledMaxWarps * 32)
                 for (int x = 0; x < C; ++x) {
                     // a CONST plaintext is its limb's residue 0 at every coefficient
                     const uint64_t g = A::operand((KC && x > 0 && (op & kOpConst)) ? r[i].x[0] : r[i].x[x]);
-                    A::mac(acc[0][x], g, s0.x[x]);
-                    A::mac(acc[1][x], g, s1.x[x]);
+                    A::mac(acc[0][x], g, s0.x[x], zero);
+                    A::mac(acc[1][x], g, s1.x[x], zero);
                 }
                 r[i] = fetch(nb, nlb, ns, nwi);
             }

@@ -1904,6 +1904,7 @@ int lower_tiled(fiona_plan *p)
         a.o_tcm = o_tcm;
     }
     a.wait_ns = 2000000000ull;
+    a.zero = 0;
     if (const char *t = getenv("FIONA_TEST_TILED_TIMEOUT")) {  // test only: a copy wait that runs out
         if (atoi(t) > 0 && best.C == 1 && hp.n_in) {
             a.test_flags |= kTiledFlagExtraTx;

@@ -25,7 +25,7 @@ constexpr int kChains = 4;
 constexpr int kSteps = 256;
 
 template <bool NARROW>
-__global__ void __launch_bounds__(256) roof_kernel(const uint64_t *seed, uint64_t *sink)
+__global__ void __launch_bounds__(256) roof_kernel(const uint64_t *seed, uint64_t *sink, uint32_t zero)
 {
     uint64_t a[kChains], b[kChains], lo[kChains], mid[kChains], hi[kChains];
 #pragma unroll
@@ -39,7 +39,7 @@ __global__ void __launch_bounds__(256) roof_kernel(const uint64_t *seed, uint64_
 #pragma unroll
         for (int c = 0; c < kChains; ++c) {
             if (NARROW)
-                rns::mac26(lo[c], mid[c], hi[c], a[c], b[c]);
+                rns::mac26(lo[c], mid[c], hi[c], a[c], b[c], zero);  // as the layer kernels call it
             else
                 rns::mac(lo[c], hi[c], a[c], b[c]);
             // the next step's operands depend on this step (stay in split form)
@@ -56,13 +56,13 @@ template <bool NARROW>
 double rate(int sms, const uint64_t *seed, uint64_t *sink)
 {
     const dim3 grid(sms * 8), block(256);
-    roof_kernel<NARROW><<<grid, block>>>(seed, sink);  // warm-up
+    roof_kernel<NARROW><<<grid, block>>>(seed, sink, 0);  // warm-up
     cudaEvent_t e0, e1;
     cudaEventCreate(&e0);
     cudaEventCreate(&e1);
     const int reps = 3;
     cudaEventRecord(e0);
-    for (int r = 0; r < reps; ++r) roof_kernel<NARROW><<<grid, block>>>(seed, sink);
+    for (int r = 0; r < reps; ++r) roof_kernel<NARROW><<<grid, block>>>(seed, sink, 0);
     cudaEventRecord(e1);
     float ms = 0;
     const bool ok = cudaEventSynchronize(e1) == cudaSuccess && cudaEventElapsedTime(&ms, e0, e1) == cudaSuccess;

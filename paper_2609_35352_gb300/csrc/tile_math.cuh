@@ -88,7 +88,7 @@ struct Arith<false> {
     };
     __device__ static uint64_t operand(uint64_t a) { return a; }
     __device__ static void zero(Acc &a) { a.lo = a.hi = 0; }
-    __device__ static void mac(Acc &a, uint64_t x, uint64_t y) { rns::mac(a.lo, a.hi, x, y); }
+    __device__ static void mac(Acc &a, uint64_t x, uint64_t y, uint32_t /*zero*/ = 0) { rns::mac(a.lo, a.hi, x, y); }
     __device__ static uint64_t reduce(const Acc &a, const LimbConst &m) { return rns::reduce128(a.lo, a.hi, m); }
     __device__ static void fold(Acc &a, const LimbConst &m)
     {
@@ -112,8 +112,12 @@ struct Arith<true> {
     };
     __device__ static uint64_t operand(uint64_t a) { return rns::split26(a); }
     __device__ static void zero(Acc &a) { a.lo = a.x = a.hi = 0; }
-    // both factors in operand (split) form
-    __device__ static void mac(Acc &a, uint64_t x, uint64_t y) { rns::mac26(a.lo, a.x, a.hi, x, y); }
+    // both factors in operand (split) form; `zero` as in rns::mac26 (a
+    // literal 0 folds the half sums back into two-input additions)
+    __device__ static void mac(Acc &a, uint64_t x, uint64_t y, uint32_t zero = 0)
+    {
+        rns::mac26(a.lo, a.x, a.hi, x, y, zero);
+    }
     __device__ static uint64_t reduce(const Acc &a, const LimbConst &m) { return rns::reduce26(a.lo, a.x, a.hi, m); }
     __device__ static void fold(Acc &a, const LimbConst &m)
     {

@@ -113,6 +113,7 @@ struct TiledArgs {
     uint32_t o_tcw, o_tcm;   // word offsets of W (fp16 image) and of the groups' magic constants
     uint64_t wait_ns;        // bound of the waits for input copies and for the contraction
     uint32_t test_flags;     // kTiledFlag* (0 outside tests)
+    uint32_t zero;           // always 0, read at run time (rns::mac26)
 };
 
 // Warp-specialised variant (kernel_ws.cu), two coefficients per lane.  The
