@@ -397,6 +397,26 @@ int fiona_linear_eval_host(const fiona_plan *plan, void *cuda_stream, const uint
                            const uint64_t *d_plaintexts, uint64_t *h_outputs,
                            uint64_t *d_inputs, uint64_t *d_outputs);
 
+/* The same evaluation, queued only: returns once the copies and kernels are
+ * enqueued.  fiona_linear_eval_host_join(plan, cuda_stream) then makes
+ * `cuda_stream` wait for the plan's output copies queued so far; h_outputs
+ * holds the result once `cuda_stream` has completed after the join
+ * (cudaStreamSynchronize, or an event recorded on it).  The input copies of a
+ * call wait for the work queued on `cuda_stream` before the call (which
+ * includes the kernels of the calls before it, not their output copies).
+ * Consecutive calls on one plan may reuse the same device buffers: each limb
+ * chunk's input copy waits for the previous call's kernel on that chunk and
+ * its kernel for the previous call's output copy of it, so a burst of calls
+ * overlaps one query's input copies with the previous query's output copies
+ * (the two directions of the host link run at once).  The host buffers
+ * belong to a call until its join has completed; the calls on one plan come
+ * from one host thread at a time.  Errors as fiona_linear_eval (a CUDA error
+ * may also surface at the synchronisation). */
+int fiona_linear_eval_host_async(const fiona_plan *plan, void *cuda_stream, const uint64_t *h_inputs,
+                                 const uint64_t *d_plaintexts, uint64_t *h_outputs,
+                                 uint64_t *d_inputs, uint64_t *d_outputs);
+int fiona_linear_eval_host_join(const fiona_plan *plan, void *cuda_stream);
+
 /* Evaluate the layer without allocating any device memory.  The paper has no
  * counterpart: this entry point exists for callers that cannot call
  * cudaMalloc at the time they evaluate -- for example a serving runtime that

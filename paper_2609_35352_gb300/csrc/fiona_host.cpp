@@ -533,6 +533,14 @@ static void release_device(fiona_plan *p)
     if (p->copy_in_stream) cudaStreamDestroy((cudaStream_t)p->copy_in_stream);
     if (p->copy_out_stream) cudaStreamDestroy((cudaStream_t)p->copy_out_stream);
     p->copy_in_stream = p->copy_out_stream = nullptr;
+    for (void **set : {p->ev_in, p->ev_kernel, p->ev_out})
+        for (uint32_t c = 0; c < fiona_plan::kHostChunks; ++c)
+            if (set[c]) {
+                cudaEventDestroy((cudaEvent_t)set[c]);
+                set[c] = nullptr;
+            }
+    if (p->ev_start) cudaEventDestroy((cudaEvent_t)p->ev_start);
+    p->ev_start = nullptr;
 }
 
 // The tiled schedule is optional: a plan whose tile does not fit in shared
@@ -689,6 +697,10 @@ extern "C" int fiona_plan_create(const fiona_ctx *ctx, uint32_t n_in, uint32_t n
             if (e == cudaSuccess)
                 e = cudaStreamCreateWithFlags((cudaStream_t *)&p->copy_out_stream,
                                               cudaStreamNonBlocking);
+            for (void **set : {p->ev_in, p->ev_kernel, p->ev_out})
+                for (uint32_t c = 0; c < fiona_plan::kHostChunks && e == cudaSuccess; ++c)
+                    e = cudaEventCreateWithFlags((cudaEvent_t *)&set[c], cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventCreateWithFlags((cudaEvent_t *)&p->ev_start, cudaEventDisableTiming);
             if (e != cudaSuccess) rc = cuda_fail(e, "plan_create: stream");
         }
         if (rc) {
@@ -825,56 +837,100 @@ extern "C" int fiona_linear_eval_level(const fiona_plan *p, void *stream, uint32
     return launch_range(p, stream, in, pt, out, 0, L_eval, L_eval);
 }
 
-extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const uint64_t *h_in,
-                                      const uint64_t *d_pt, uint64_t *h_out, uint64_t *d_in,
-                                      uint64_t *d_out)
+// Queue the host-buffer evaluation: per limb chunk (one limb each, at most
+// kHostChunks), its input copy on the plan's input stream, its kernel on
+// `stream`, its output copy on the plan's output stream, each ordered after
+// the step before it and after the previous call's use of the same chunk of
+// d_in (its kernel) and d_out (its output copy); with `join`, `stream` ends
+// waiting for the last output copy (a queued call leaves that to
+// fiona_linear_eval_host_join, so that the next call's input copies, which
+// wait for the work on `stream` before them, need not wait for these output
+// copies too).
+static int eval_host_enqueue(const fiona_plan *p, cudaStream_t s, const uint64_t *h_in, const uint64_t *d_pt,
+                             uint64_t *h_out, uint64_t *d_in, uint64_t *d_out, bool join)
 {
-    int rc = check_eval_args(p, d_in, d_pt, d_out);
-    if (rc) return rc;
-    if ((p->hp.n_in && !h_in) || !h_out)
-        return set_error(FIONA_ERR_ARG, "linear_eval_host: null host buffer");
-    if (p->hp.n_out == 0) return FIONA_OK;
-    DeviceGuard g(p->ctx->device);
     const uint32_t L = p->ctx->L, N = p->ctx->N;
     const size_t pitch = (size_t)L * N * 8;
-    cudaStream_t s = (cudaStream_t)stream;
     cudaStream_t sin = (cudaStream_t)p->copy_in_stream, sout = (cudaStream_t)p->copy_out_stream;
-    // one limb per chunk (at most 16 chunks): the pipeline's fill and drain
-    // (the first chunk's input copy, the last one's output copy) stay short
-    constexpr uint32_t kMaxChunks = 16;
-    const uint32_t chunks = std::min<uint32_t>(L, kMaxChunks);
-    cudaEvent_t ev[2 * kMaxChunks + 1];
-    int made = 0;
-    cudaError_t e = cudaSuccess;
-    for (int i = 0; i < 2 * (int)chunks + 1 && e == cudaSuccess; ++i, ++made)
-        e = cudaEventCreateWithFlags(&ev[i], cudaEventDisableTiming);
-    // the copy streams must not run ahead of work already queued on `stream`
-    if (e == cudaSuccess) e = cudaEventRecord(ev[2 * chunks], s);
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(sin, ev[2 * chunks], 0);
-    for (uint32_t c = 0; c < chunks && e == cudaSuccess && rc == FIONA_OK; ++c) {
+    const uint32_t chunks = std::min<uint32_t>(L, fiona_plan::kHostChunks);
+    auto ev = [](void *const *set, uint32_t c) { return (cudaEvent_t)set[c]; };
+    // the copies must not run ahead of work already queued on `stream`
+    cudaError_t e = cudaEventRecord((cudaEvent_t)p->ev_start, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(sin, (cudaEvent_t)p->ev_start, 0);
+    for (uint32_t c = 0; c < chunks && e == cudaSuccess; ++c) {
         const uint32_t l0 = L * c / chunks, l1 = L * (c + 1) / chunks;
         const size_t width = (size_t)(l1 - l0) * N * 8;
+        if ((e = cudaStreamWaitEvent(sin, ev(p->ev_kernel, c), 0)) != cudaSuccess) break;
         if (p->hp.n_in) {
             e = cudaMemcpy2DAsync(d_in + (size_t)l0 * N, pitch, h_in + (size_t)l0 * N, pitch, width,
                                   (size_t)p->hp.n_in * 2, cudaMemcpyHostToDevice, sin);
             if (e != cudaSuccess) break;
         }
-        if ((e = cudaEventRecord(ev[2 * c], sin)) != cudaSuccess) break;
-        if ((e = cudaStreamWaitEvent(s, ev[2 * c], 0)) != cudaSuccess) break;
-        rc = launch_range(p, s, d_in, d_pt, d_out, l0, l1, L);
-        if (rc) break;
-        if ((e = cudaEventRecord(ev[2 * c + 1], s)) != cudaSuccess) break;
-        if ((e = cudaStreamWaitEvent(sout, ev[2 * c + 1], 0)) != cudaSuccess) break;
+        if ((e = cudaEventRecord(ev(p->ev_in, c), sin)) != cudaSuccess) break;
+        if ((e = cudaStreamWaitEvent(s, ev(p->ev_in, c), 0)) != cudaSuccess) break;
+        if ((e = cudaStreamWaitEvent(s, ev(p->ev_out, c), 0)) != cudaSuccess) break;
+        if (const int rc = launch_range(p, s, d_in, d_pt, d_out, l0, l1, L)) return rc;
+        if ((e = cudaEventRecord(ev(p->ev_kernel, c), s)) != cudaSuccess) break;
+        if ((e = cudaStreamWaitEvent(sout, ev(p->ev_kernel, c), 0)) != cudaSuccess) break;
         e = cudaMemcpy2DAsync(h_out + (size_t)l0 * N, pitch, d_out + (size_t)l0 * N, pitch, width,
                               (size_t)p->hp.n_out * 2, cudaMemcpyDeviceToHost, sout);
+        if (e == cudaSuccess) e = cudaEventRecord(ev(p->ev_out, c), sout);
     }
-    cudaError_t e2 = cudaStreamSynchronize(sout);
-    cudaError_t e3 = cudaStreamSynchronize(sin);
-    for (int i = 0; i < made; ++i) cudaEventDestroy(ev[i]);
-    if (rc) return rc;
+    if (e == cudaSuccess && join) e = cudaStreamWaitEvent(s, ev(p->ev_out, chunks - 1), 0);
     if (e != cudaSuccess) return cuda_fail(e, "linear_eval_host");
+    return FIONA_OK;
+}
+
+static int check_host_args(const fiona_plan *p, const uint64_t *h_in, const uint64_t *d_pt, const uint64_t *h_out,
+                           const uint64_t *d_in, const uint64_t *d_out)
+{
+    int rc = check_eval_args(p, d_in, d_pt, d_out);
+    if (rc) return rc;
+    if ((p->hp.n_in && !h_in) || !h_out) return set_error(FIONA_ERR_ARG, "linear_eval_host: null host buffer");
+    return FIONA_OK;
+}
+
+extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const uint64_t *h_in,
+                                      const uint64_t *d_pt, uint64_t *h_out, uint64_t *d_in,
+                                      uint64_t *d_out)
+{
+    if (const int rc = check_host_args(p, h_in, d_pt, h_out, d_in, d_out)) return rc;
+    if (p->hp.n_out == 0) return FIONA_OK;
+    DeviceGuard g(p->ctx->device);
+    cudaStream_t s = (cudaStream_t)stream;
+    const int rc = eval_host_enqueue(p, s, h_in, d_pt, h_out, d_in, d_out, true);
+    // whatever was queued completes before the call returns
+    const cudaError_t e = cudaStreamSynchronize(s);
+    const cudaError_t e2 = cudaStreamSynchronize((cudaStream_t)p->copy_out_stream);
+    const cudaError_t e3 = cudaStreamSynchronize((cudaStream_t)p->copy_in_stream);
+    if (rc) return rc;
+    if (e != cudaSuccess) return cuda_fail(e, "linear_eval_host: sync");
     if (e2 != cudaSuccess) return cuda_fail(e2, "linear_eval_host: sync");
     if (e3 != cudaSuccess) return cuda_fail(e3, "linear_eval_host: sync");
+    return FIONA_OK;
+}
+
+extern "C" int fiona_linear_eval_host_async(const fiona_plan *p, void *stream, const uint64_t *h_in,
+                                            const uint64_t *d_pt, uint64_t *h_out, uint64_t *d_in,
+                                            uint64_t *d_out)
+{
+    if (const int rc = check_host_args(p, h_in, d_pt, h_out, d_in, d_out)) return rc;
+    if (p->hp.n_out == 0) return FIONA_OK;
+    DeviceGuard g(p->ctx->device);
+    return eval_host_enqueue(p, (cudaStream_t)stream, h_in, d_pt, h_out, d_in, d_out, false);
+}
+
+extern "C" int fiona_linear_eval_host_join(const fiona_plan *p, void *stream)
+{
+    if (!p) return set_error(FIONA_ERR_ARG, "linear_eval_host_join: null plan");
+    if (p->ctx->device == FIONA_DEVICE_NONE)
+        return set_error(FIONA_ERR_NODEVICE, "linear_eval_host_join: validation-only context");
+    if (p->hp.n_out == 0) return FIONA_OK;
+    DeviceGuard g(p->ctx->device);
+    const uint32_t chunks = std::min<uint32_t>(p->ctx->L, fiona_plan::kHostChunks);
+    // the output copies run in order on one stream: the last chunk's is the last
+    const cudaError_t e = cudaStreamWaitEvent((cudaStream_t)stream, (cudaEvent_t)p->ev_out[chunks - 1], 0);
+    if (e != cudaSuccess) return cuda_fail(e, "linear_eval_host_join");
     return FIONA_OK;
 }
 

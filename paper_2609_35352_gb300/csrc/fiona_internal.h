@@ -83,9 +83,16 @@ struct fiona_plan {
     const uint32_t *d_raw_pt = nullptr;
     // tiled schedule
     TiledSchedule *tiled = nullptr;
-    // streams for fiona_linear_eval_host
+    // streams for fiona_linear_eval_host(_async), and per limb chunk the
+    // events of its last input copy, kernel and output copy: a call orders
+    // each chunk after the previous call's use of the same device buffers
+    static constexpr uint32_t kHostChunks = 16;
     void *copy_in_stream = nullptr;
     void *copy_out_stream = nullptr;
+    void *ev_in[kHostChunks] = {};
+    void *ev_kernel[kHostChunks] = {};
+    void *ev_out[kHostChunks] = {};
+    void *ev_start = nullptr;
     // host image of the direct schedule and the limb constants, copied into
     // the library's fixed device area by fiona_linear_eval_static
     std::vector<uint8_t> static_image;

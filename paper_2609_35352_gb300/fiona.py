@@ -37,7 +37,8 @@ KERNELS = {"auto": FIONA_KERNEL_AUTO, "direct": FIONA_KERNEL_DIRECT, "tiled": FI
 
 EXPORTED = ("fiona_ctx_create", "fiona_ctx_destroy", "fiona_plan_create", "fiona_plan_create_classes",
             "fiona_plan_destroy",
-            "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host",
+            "fiona_plan_stats", "fiona_linear_eval", "fiona_linear_eval_host", "fiona_linear_eval_host_async",
+            "fiona_linear_eval_host_join",
             "fiona_check_residues", "fiona_status_str", "fiona_last_error", "fiona_abi_version",
             "fiona_plan_select_kernel", "fiona_device_check", "fiona_linear_eval_static",
             "fiona_linear_eval_level", "fiona_plan_compile", "fiona_rescale",
@@ -101,6 +102,10 @@ def lib() -> ctypes.CDLL:
         L.fiona_linear_eval.restype = i32
         L.fiona_linear_eval_host.argtypes = [p, p, p, p, p, p, p]
         L.fiona_linear_eval_host.restype = i32
+        L.fiona_linear_eval_host_async.argtypes = [p, p, p, p, p, p, p]
+        L.fiona_linear_eval_host_async.restype = i32
+        L.fiona_linear_eval_host_join.argtypes = [p, p]
+        L.fiona_linear_eval_host_join.restype = i32
         L.fiona_check_residues.argtypes = [p, p, p, ctypes.c_uint64]
         L.fiona_check_residues.restype = i32
         L.fiona_status_str.argtypes = [i32]
@@ -343,6 +348,18 @@ class Plan:
         _check(lib().fiona_linear_eval_host(self.handle, stream_handle(stream), addr(h_inputs),
                                             addr(d_plaintexts), addr(h_outputs), addr(d_inputs),
                                             addr(d_outputs)), "fiona_linear_eval_host")
+
+    def eval_host_async(self, h_inputs, d_plaintexts, h_outputs, d_inputs, d_outputs,
+                        stream=None) -> None:
+        """fiona_linear_eval_host_async: queued only; the result is in
+        h_outputs once `stream` has completed after eval_host_join."""
+        _check(lib().fiona_linear_eval_host_async(self.handle, stream_handle(stream), addr(h_inputs),
+                                                  addr(d_plaintexts), addr(h_outputs), addr(d_inputs),
+                                                  addr(d_outputs)), "fiona_linear_eval_host_async")
+
+    def eval_host_join(self, stream=None) -> None:
+        """fiona_linear_eval_host_join: `stream` waits for the queued output copies."""
+        _check(lib().fiona_linear_eval_host_join(self.handle, stream_handle(stream)), "fiona_linear_eval_host_join")
 
     def close(self) -> None:
         if getattr(self, "handle", None):

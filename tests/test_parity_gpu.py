@@ -315,6 +315,39 @@ def test_host_buffer_path_matches_device_path():
     assert np.array_equal(h_out.numpy().view(np.uint64).reshape(want.shape), want)
 
 
+def test_host_buffer_queries_queued_back_to_back():
+    """fiona_linear_eval_host_async: three queries with different inputs,
+    queued back to back on the same device buffers (each limb chunk of a
+    query ordered after the previous query's kernel and output copy of that
+    chunk), into three host outputs: after one synchronisation every output
+    equals the device path's result for its own inputs."""
+    wl = W.make_workload("vit", N=4096, L=5)
+    dl = DeviceLayer(wl)
+    p = wl.plan
+    rng = np.random.default_rng(11)
+    qs = np.asarray(wl.moduli, dtype=np.uint64)
+    wants, h_ins, h_outs = [], [], []
+    for k in range(3):
+        X = (rng.integers(0, 2**62, dl.X.shape, dtype=np.uint64) % qs[None, None, :, None]).astype(np.uint64)
+        d_x = torch.from_numpy(X.view(np.int64).reshape(-1)).cuda()
+        dl.d_out.fill_(-1)
+        dl.plan.eval(d_x, dl.d_pt, dl.d_out)
+        wants.append(dl.outputs().copy())
+        h_ins.append(torch.from_numpy(X.view(np.int64).reshape(-1)).pin_memory())
+        h_outs.append(torch.full((wants[-1].size,), -1, dtype=torch.int64).pin_memory())
+    d_in2 = torch.zeros_like(dl.d_in)
+    d_out2 = torch.zeros_like(dl.d_out)
+    stream = torch.cuda.Stream()
+    for k in range(3):
+        dl.plan.eval_host_async(h_ins[k], dl.d_pt, h_outs[k], d_in2, d_out2, stream=stream)
+    dl.plan.eval_host_join(stream=stream)
+    stream.synchronize()
+    for k in range(3):
+        got = h_outs[k].numpy().view(np.uint64).reshape(wants[k].shape)
+        assert np.array_equal(got, wants[k]), k
+    assert dl.ctx.device_check() == F.FIONA_OK
+
+
 def test_stream_and_alignment_errors():
     wl = W.make_workload("tiny")
     dl = DeviceLayer(wl)
