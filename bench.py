@@ -342,8 +342,8 @@ def measured_peak():
 
 
 KERNEL_FILES = {"direct": ["kernel_direct.cu", "rns.cuh"],
-                "tiled": ["kernel_tiled.cu", "tiled.h", "lower_tiled.cpp", "rns.cuh", "tile_math.cuh",
-                          "tc_signed.cuh", "tc_geometry.h"]}
+                "tiled": ["kernel_tiled.cu", "kernel_tiled_off.cu", "tiled_kernel.cuh", "tiled.h", "lower_tiled.cpp",
+                          "rns.cuh", "tile_math.cuh", "async.cuh", "tc_signed.cuh", "tc_geometry.h"]}
 
 
 def kernel_source_hash(kernel: str) -> str:
@@ -607,7 +607,8 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
                        "warps_per_cta": stats["warps_per_cta"], "ctas_per_sm": stats["ctas_per_sm"],
                        "shared_sums_formed": stats["nodes_materialized"],
                        "addsub_executed": stats.get("addsub_executed"),
-                       "tensor_core_sums": stats.get("tensor_core_sums")},
+                       "tensor_core_sums": stats.get("tensor_core_sums"),
+                       "source_offsets": stats.get("source_offsets")},
         }
         print(json.dumps(line), flush=True)
     plan.close()

@@ -163,7 +163,11 @@ typedef struct fiona_plan_stats_t {
     uint32_t tensor_core_sums;    /* TILED: scale-group signed sums formed per tile as one
                                      contraction on the tensor cores (the groups' terms, shared
                                      sums expanded, exact in fp16 chunks); 0: on the ALUs      */
-    uint32_t reserved[2];
+    uint32_t source_offsets;      /* TILED: 1 if the schedule's signed-sum runs hold source byte
+                                     offsets (one addition per source address), 0 if 16-bit
+                                     indices packed two per word (used when the larger offset
+                                     schedule does not fit in shared memory)                   */
+    uint32_t reserved;
 } fiona_plan_stats_t;
 
 /* Create a context for ring dimension N (a power of two, 2^10 <= N <= 2^17)

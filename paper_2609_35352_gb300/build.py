@@ -26,7 +26,7 @@ FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", 
 
 LIBRARIES = {
     "libfiona.so": ["fiona_host.cpp", "lower_tiled.cpp", "plan_compile.cpp", "kernel_direct.cu",
-                    "kernel_tiled.cu", "kernel_ws.cu", "rescale.cu", "encode.cu"],
+                    "kernel_tiled.cu", "kernel_tiled_off.cu", "kernel_ws.cu", "rescale.cu", "encode.cu"],
     "libfiona_workload.so": ["workload_fill.cu", "mul_roof.cu"],
 }
 

@@ -582,6 +582,7 @@ static int select_kernel(fiona_plan *p, int which)
         s.nodes_materialized = p->tiled->nodes_kept;
         s.addsub_executed = p->tiled->addsub;
         s.tensor_core_sums = p->tiled->tc ? p->tiled->args.tc_groups : 0;
+        s.source_offsets = p->tiled->args.src_offsets;
     } else {
         s.kernel = FIONA_KERNEL_DIRECT;
         s.tile_coeffs = 256;
@@ -591,6 +592,7 @@ static int select_kernel(fiona_plan *p, int which)
         s.nodes_materialized = 0;
         s.addsub_executed = (uint32_t)std::min<uint64_t>(s.addsub_flat, 0xffffffffu);
         s.tensor_core_sums = 0;
+        s.source_offsets = 0;
     }
     return FIONA_OK;
 }

@@ -387,21 +387,111 @@ JobPlan build_jobs(const std::vector<OutWork> &work, uint32_t W, const Costs &k,
     return jp;
 }
 
-// Program words of a signed sum: n_plus | n_minus << 16, then each run as
-// 16-bit indices, two per word.
+// Form of the signed-sum programs in a schedule (tiled.h): 16-bit source
+// indices packed two per word, or one 32-bit byte offset (index * PB) per
+// source, each program starting on a 16-byte boundary.
+struct ProgForm {
+    bool offsets = false;
+    uint32_t PB = 0;  // bytes of one source tile pair
+};
+
+// Program words of a signed sum: n_plus | n_minus << 16, the runs and the
+// slot word (counts, then up to six 4-bit slot numbers, plus slots first).
+// A formation (`form_slot` >= 0) names the warp slot it fills: the word
+// before its program in the packed form, the third word of its program in
+// the offset form.
 void put_program(std::vector<uint32_t> &w, const std::vector<uint32_t> &plus, const std::vector<uint32_t> &minus,
-                 const std::vector<uint32_t> &plus_slots = {}, const std::vector<uint32_t> &minus_slots = {})
+                 const std::vector<uint32_t> &plus_slots, const std::vector<uint32_t> &minus_slots,
+                 const ProgForm &pf, int form_slot = -1)
 {
-    w.push_back((uint32_t)plus.size() | ((uint32_t)minus.size() << 16));
-    for (const auto *run : {&plus, &minus})
-        for (size_t i = 0; i < run->size(); i += 2)
-            w.push_back(run->at(i) | (i + 1 < run->size() ? run->at(i + 1) << 16 : 0u));
-    // the slot word: counts, then up to six 4-bit slot numbers (plus first)
     uint32_t sw = (uint32_t)plus_slots.size() | ((uint32_t)minus_slots.size() << 4);
     uint32_t j = 0;
     for (const auto *ss : {&plus_slots, &minus_slots})
         for (uint32_t sl : *ss) sw |= (sl & 15u) << (8 + 4 * j++);
+    const uint32_t h = (uint32_t)plus.size() | ((uint32_t)minus.size() << 16);
+    if (pf.offsets) {
+        while (w.size() % 4) w.push_back(0);
+        w.push_back(h);
+        w.push_back(sw);
+        w.push_back(form_slot >= 0 ? (uint32_t)form_slot : 0u);
+        w.push_back(0);
+        for (const auto *run : {&plus, &minus}) {
+            for (uint32_t s : *run) w.push_back(s * pf.PB);
+            while (w.size() % 4) w.push_back(0);
+        }
+        return;
+    }
+    if (form_slot >= 0) w.push_back((uint32_t)form_slot);
+    w.push_back(h);
+    for (const auto *run : {&plus, &minus})
+        for (size_t i = 0; i < run->size(); i += 2)
+            w.push_back(run->at(i) | (i + 1 < run->size() ? run->at(i + 1) << 16 : 0u));
     w.push_back(sw);
+}
+
+// A program decoded from schedule words (either form).
+struct ProgRead {
+    uint32_t np = 0, nm = 0;     // plus and minus run lengths
+    uint32_t sw = 0;             // slot word
+    uint32_t form_slot = 0;      // a formation's target slot
+    std::vector<uint32_t> src;   // the plus run's source indices, then the minus run's
+    size_t next = 0;             // word just past the program
+};
+
+// Decode the program at word p (a formation's, with its target slot, when
+// `formation`), reading no word at or past `end`; false if it does not fit,
+// is misaligned, or an offset is not a whole source.
+bool read_program(const std::vector<uint32_t> &w, size_t p, size_t end, const ProgForm &pf, bool formation,
+                  ProgRead &r)
+{
+    end = std::min(end, w.size());
+    r = ProgRead{};
+    if (pf.offsets) {
+        if (p % 4 || p + 4 > end || pf.PB == 0) return false;
+        r.np = w[p] & 0xffffu;
+        r.nm = w[p] >> 16;
+        r.sw = w[p + 1];
+        r.form_slot = w[p + 2];
+        if (!formation && w[p + 2]) return false;
+        p += 4;
+        for (uint32_t n : {r.np, r.nm}) {
+            const size_t padded = ((size_t)n + 3) & ~(size_t)3;
+            if (p + padded > end) return false;
+            for (uint32_t i = 0; i < n; ++i) {
+                if (w[p + i] % pf.PB) return false;
+                r.src.push_back(w[p + i] / pf.PB);
+            }
+            p += padded;
+        }
+        r.next = p;
+        return true;
+    }
+    if (formation) {
+        if (p >= end) return false;
+        r.form_slot = w[p++];
+    }
+    if (p >= end) return false;
+    r.np = w[p] & 0xffffu;
+    r.nm = w[p] >> 16;
+    ++p;
+    for (uint32_t n : {r.np, r.nm}) {
+        if (p + (n + 1) / 2 > end) return false;
+        for (uint32_t i = 0; i < n; ++i) r.src.push_back((w[p + i / 2] >> (16 * (i & 1))) & 0xffffu);
+        p += (n + 1) / 2;
+    }
+    if (p >= end) return false;
+    r.sw = w[p++];
+    r.next = p;
+    return true;
+}
+
+// The program form of a schedule, from its kernel arguments.
+ProgForm prog_form(const TiledArgs &a)
+{
+    ProgForm pf;
+    pf.offsets = a.src_offsets != 0;
+    pf.PB = a.src_bytes / (a.n_in + a.n_nodes + 1);
+    return pf;
 }
 
 // The whole schedule (see tiled.h).
@@ -417,7 +507,8 @@ void pad4(std::vector<uint32_t> &w)
 }
 
 Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const std::vector<Seg> &nodes, uint32_t W,
-             uint32_t mac_budget, uint32_t zero_index, uint32_t P, const std::vector<uint32_t> *warp_slots = nullptr)
+             uint32_t mac_budget, uint32_t zero_index, uint32_t P, const std::vector<uint32_t> *warp_slots = nullptr,
+             const ProgForm &pf = ProgForm{})
 {
     Sched sc;
     auto &w = sc.w;
@@ -426,8 +517,9 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
     sc.o_node_off = (uint32_t)w.size();
     w.resize(w.size() + nodes.size());
     for (size_t k = 0; k < nodes.size(); ++k) {
+        if (pf.offsets) pad4(w);
         w[sc.o_node_off + k] = (uint32_t)w.size();
-        put_program(w, nodes[k].plus, nodes[k].minus);
+        put_program(w, nodes[k].plus, nodes[k].minus, {}, {}, pf);
     }
     pad4(w);
     sc.o_warp = (uint32_t)w.size();
@@ -470,11 +562,9 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
             for (size_t p = first; k < segs.size() || r < raws.size(); ++p) {
                 if (p % P == 0 && k < segs.size() && seg_at[(p - b0) / P]) {
                     const Seg &sg = segs[k++];
-                    for (const Form &f : sg.forms) {
-                        segw[wi].push_back(f.slot);
-                        put_program(segw[wi], f.plus, f.minus, f.plus_slots, f.minus_slots);
-                    }
-                    put_program(segw[wi], sg.plus, sg.minus, sg.plus_slots, sg.minus_slots);
+                    for (const Form &f : sg.forms)
+                        put_program(segw[wi], f.plus, f.minus, f.plus_slots, f.minus_slots, pf, (int)f.slot);
+                    put_program(segw[wi], sg.plus, sg.minus, sg.plus_slots, sg.minus_slots, pf);
                     o.push_back((sg.scale_pt << kOpPtShift) | kOpSeg | (uint32_t)sg.forms.size());
                 } else {
                     o.push_back(raw_or_nop());  // a NOP while a SEG waits for its batch
@@ -529,7 +619,7 @@ Sched encode(const JobPlan &jp, const std::vector<uint32_t> &level_off, const st
         if (warp_slots) first += (*warp_slots)[wi];
         w.insert(w.end(), ops[wi].begin(), ops[wi].end());
     }
-    for (uint32_t wi = 0; wi < W; ++wi) {
+    for (uint32_t wi = 0; wi < W; ++wi) {  // (offset form: every program a multiple of four words)
         w[sc.o_warp + wi * kWarpTableWords + 2] = (uint32_t)w.size();
         w.insert(w.end(), segw[wi].begin(), segw[wi].end());
     }
@@ -984,18 +1074,14 @@ const char *check_tc(const std::vector<uint32_t> &w, const TiledArgs &a)
     for (uint32_t n = 0; n < a.tc_n; ++n) {
         std::vector<int> want(a.tc_k, 0);
         if (n < a.tc_groups) {  // the node program: plus run, minus run, inputs only
-            size_t p = w[a.o_node_off + n];
-            const uint32_t h = w[p++];
-            for (int sign : {1, -1}) {
-                const uint32_t cnt = sign > 0 ? (h & 0xffffu) : (h >> 16);
-                for (uint32_t i = 0; i < cnt; ++i) {
-                    const uint32_t idx = (w[p + i / 2] >> (16 * (i & 1))) & 0xffffu;
-                    if (idx >= a.n_in) return "tensor-core sums: a node reads a non-input";
-                    want[idx] += sign;
-                }
-                p += (cnt + 1) / 2;
+            ProgRead r;
+            if (!read_program(w, w[a.o_node_off + n], w.size(), prog_form(a), false, r))
+                return "tensor-core sums: node program";
+            for (uint32_t i = 0; i < r.np + r.nm; ++i) {
+                if (r.src[i] >= a.n_in) return "tensor-core sums: a node reads a non-input";
+                want[r.src[i]] += i < r.np ? 1 : -1;
             }
-            if (w[p] != 0) return "tensor-core sums: a node reads warp slots";
+            if (r.sw != 0) return "tensor-core sums: a node reads warp slots";
         }
         int cs = 0;
         uint32_t ab = 0;
@@ -1024,16 +1110,17 @@ const char *check_tc(const std::vector<uint32_t> &w, const TiledArgs &a)
 uint32_t count_addsub(const std::vector<uint32_t> &w, const TiledArgs &a, uint32_t W)
 {
     uint64_t n = 0;
-    auto program = [&](size_t &p) {  // operands of the program at word p; p is left past it
-        const uint32_t h = w[p++];
-        const uint32_t np = h & 0xffffu, nm = h >> 16;
-        p += (np + 1) / 2 + (nm + 1) / 2;
-        const uint32_t sw = w[p++];
-        return (uint64_t)np + nm + (sw & 15u) + ((sw >> 4) & 15u);
+    const ProgForm pf = prog_form(a);
+    // operands of the program at word p (a formation's when `form`); p is left past it
+    auto program = [&](size_t &p, bool form) -> uint64_t {
+        ProgRead r;
+        if (!read_program(w, p, w.size(), pf, form, r)) return 1;  // (check_schedule rejects the schedule)
+        p = r.next;
+        return (uint64_t)r.np + r.nm + (r.sw & 15u) + ((r.sw >> 4) & 15u);
     };
     for (uint32_t x = 0; x < a.n_nodes; ++x) {
         size_t p = w[a.o_node_off + x];
-        n += program(p) - 1;
+        n += program(p, false) - 1;
     }
     for (uint32_t wi = 0; wi < W; ++wi) {
         const size_t t = a.o_warp + (size_t)wi * kWarpTableWords;
@@ -1043,11 +1130,8 @@ uint32_t count_addsub(const std::vector<uint32_t> &w, const TiledArgs &a, uint32
         for (uint32_t f = 0; f < n_ops; ++f) {
             const uint32_t op = w[op0 + f];
             if (op & kOpSeg) {
-                for (uint32_t g = 0; g < (op & (kOpMaxSources - 1)); ++g) {
-                    ++sp;  // the slot
-                    n += program(sp) - 1;
-                }
-                const uint64_t k = program(sp);
+                for (uint32_t g = 0; g < (op & (kOpMaxSources - 1)); ++g) n += program(sp, true) - 1;
+                const uint64_t k = program(sp, false);
                 if (k) n += k - 1;
             }
             if (!(op & kOpNop)) ++products;
@@ -1096,29 +1180,23 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
         v = w[i];
         return true;
     };
-    // a signed-sum program at word `o` whose indices must be below `lim` and
-    // whose slot numbers below `slot_lim`
-    auto program = [&](size_t o, uint32_t lim, size_t end, size_t &next, uint32_t slot_lim) -> bool {
-        uint32_t h;
-        if (o >= end || !at(o, h)) return false;
-        const uint32_t np = h & 0xffffu, nm = h >> 16;
-        size_t p = o + 1;
-        for (uint32_t n : {np, nm}) {
-            for (uint32_t i = 0; i < n; i += 2) {
-                uint32_t x;
-                if (p >= end || !at(p, x)) return false;
-                if ((x & 0xffffu) >= lim) return false;
-                if (i + 1 < n && (x >> 16) >= lim) return false;
-                ++p;
-            }
-        }
-        uint32_t sw;
-        if (p >= end || !at(p, sw)) return false;
-        const uint32_t ns = (sw & 15u) + ((sw >> 4) & 15u);
-        if (ns > 6 || (ns < 6 && (sw >> (8 + 4 * ns)) != 0)) return false;
+    // a signed-sum program at word `o` (a formation's, whose target slot is
+    // below `slot_lim`, when `form`) whose indices must be below `lim` and
+    // whose slot numbers below `slot_lim`; in the offset form every offset a
+    // whole source and the program on a 16-byte boundary (read_program)
+    const ProgForm pf = prog_form(a);
+    if (pf.offsets && pf.PB != PB) return "program form";
+    auto program = [&](size_t o, uint32_t lim, size_t end, size_t &next, uint32_t slot_lim, bool form) -> bool {
+        ProgRead r;
+        if (!read_program(w, o, end, pf, form, r)) return false;
+        for (uint32_t x : r.src)
+            if (x >= lim) return false;
+        if (form && r.form_slot >= slot_lim) return false;
+        const uint32_t ns = (r.sw & 15u) + ((r.sw >> 4) & 15u);
+        if (ns > 6 || (ns < 6 && (r.sw >> (8 + 4 * ns)) != 0)) return false;
         for (uint32_t j = 0; j < ns; ++j)
-            if (((sw >> (8 + 4 * j)) & 15u) >= slot_lim) return false;
-        next = p + 1;
+            if (((r.sw >> (8 + 4 * j)) & 15u) >= slot_lim) return false;
+        next = r.next;
         return true;
     };
     // levels and node programs
@@ -1133,7 +1211,7 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
             uint32_t off;
             size_t next;
             // a node reads inputs and nodes of lower levels only
-            if (!at(a.o_node_off + x, off) || !program(off, a.n_in + w[a.o_level + l], a.o_warp, next, 0))
+            if (!at(a.o_node_off + x, off) || !program(off, a.n_in + w[a.o_level + l], a.o_warp, next, 0, false))
                 return "node program";
         }
     // warp streams
@@ -1164,12 +1242,10 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
             } else if (op & kOpSeg) {
                 size_t next;
                 for (uint32_t f = 0; f < (op & (kOpMaxSources - 1)); ++f) {  // formations into warp slots
-                    uint32_t slot;
-                    if (sp >= seg_end || !at(sp, slot) || slot >= n_wslots) return "formation slot";
-                    if (!program(sp + 1, n_src, seg_end, next, n_wslots)) return "formation program";
+                    if (!program(sp, n_src, seg_end, next, n_wslots, true)) return "formation program";
                     sp = next;
                 }
-                if (!program(sp, n_src, seg_end, next, n_wslots)) return "segment program";
+                if (!program(sp, n_src, seg_end, next, n_wslots, false)) return "segment program";
                 sp = next;
                 open = true;
             } else {
@@ -1231,24 +1307,23 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
     };
     std::vector<Expr> src(a.n_in + a.n_nodes + 1);  // + the zero tile
     for (uint32_t i = 0; i < a.n_in; ++i) src[i] = {{i, 1}};
-    // a run of n 16-bit indices from word p (each run starts on a new word)
-    auto run = [&](size_t &p, uint32_t n, Expr &e, int64_t f) {
-        for (uint32_t i = 0; i < n; ++i) add(e, src[(w[p + i / 2] >> (16 * (i & 1))) & 0xffffu], f);
-        p += (n + 1) / 2;
-    };
     std::vector<Expr> slot(std::max<uint32_t>(a.n_slots, 1));  // the current warp's slots
-    // a signed-sum program at word p; p is left past it
-    auto program = [&](size_t &p, Expr &e) {
-        const uint32_t h = w[p++];
-        run(p, h & 0xffffu, e, 1);
-        run(p, h >> 16, e, -1);
-        const uint32_t sw = w[p++];
-        const uint32_t nps = sw & 15u, ns = nps + ((sw >> 4) & 15u);
-        for (uint32_t j = 0; j < ns; ++j) add(e, slot[(sw >> (8 + 4 * j)) & 15u], j < nps ? 1 : -1);
+    const ProgForm pf = prog_form(a);
+    // a signed-sum program at word p (a formation's when `form`: its target
+    // slot goes to *fs); p is left past it (check_schedule has walked every
+    // program before)
+    auto program = [&](size_t &p, Expr &e, bool form, uint32_t *fs) {
+        ProgRead r;
+        if (!read_program(w, p, w.size(), pf, form, r)) return;
+        for (uint32_t i = 0; i < r.np + r.nm; ++i) add(e, src[r.src[i]], i < r.np ? 1 : -1);
+        const uint32_t nps = r.sw & 15u, ns = nps + ((r.sw >> 4) & 15u);
+        for (uint32_t j = 0; j < ns; ++j) add(e, slot[(r.sw >> (8 + 4 * j)) & 15u], j < nps ? 1 : -1);
+        if (fs) *fs = r.form_slot;
+        p = r.next;
     };
     for (uint32_t x = 0; x < a.n_nodes; ++x) {
         size_t p = w[a.o_node_off + x];
-        program(p, src[a.n_in + x]);
+        program(p, src[a.n_in + x], false, nullptr);
     }
     // (plaintext, input) -> coefficient, per output and partial slot
     using Map = std::map<std::pair<uint32_t, uint32_t>, int64_t>;
@@ -1266,13 +1341,13 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
             const uint32_t op = w[op0 + f], pt = op >> kOpPtShift;
             if (op & kOpSeg) {
                 for (uint32_t g = 0; g < (op & (kOpMaxSources - 1)); ++g) {
-                    const uint32_t sl = w[sp++];
+                    uint32_t sl = 0;
                     Expr u;
-                    program(sp, u);
+                    program(sp, u, true, &sl);
                     slot[sl] = std::move(u);
                 }
                 Expr e;
-                program(sp, e);
+                program(sp, e, false, nullptr);
                 for (auto &x : e) put(job, {pt, x.first}, x.second);
             } else if (!(op & kOpNop)) {
                 for (auto &x : src[op & (kOpMaxSources - 1)]) put(job, {pt, x.first}, x.second);
@@ -1305,8 +1380,10 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
 }  // namespace
 
 // kernel_tiled.cu
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem);
-int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr);
+// (kernel_tiled.cu; off: the variant whose signed-sum programs are in the offset form)
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off = false);
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr,
+                            bool off = false);
 // kernel_ws.cu
 int ws_kernel_attributes(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, cudaFuncAttributes *attr);
 int ws_configure_kernel(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, size_t smem);
@@ -1851,8 +1928,42 @@ int lower_tiled(fiona_plan *p)
         }
     }
     }  // !use_tc
-    best.smem = sc.w.size() * 4 + (size_t)(hp.n_in + lw.nodes.size() + 1) * PB * nbuf + (size_t)jp.n_part * PB +
-                (size_t)loc.n_slots * PB + 32;
+    auto smem_of = [&](const Sched &x) {
+        return x.w.size() * 4 + (size_t)(hp.n_in + lw.nodes.size() + 1) * PB * nbuf + (size_t)jp.n_part * PB +
+               (size_t)loc.n_slots * PB + 32;
+    };
+    // the signed-sum programs in the offset form (the kernel forms each
+    // source address with one addition: measured on the VGG layer, whose
+    // 1638 signed terms per tile dominate its index decoding), when the
+    // larger schedule still fits beside the regions and slots at the
+    // occupancy the shape was chosen for; otherwise (BERT, whose two source
+    // regions fill the shared memory) the packed indices.  FIONA_TILED_PACKED=1
+    // keeps the packed form (the same residues).
+    bool offsets = false;
+    if (!use_tc && !(getenv("FIONA_TILED_PACKED") && atoi(getenv("FIONA_TILED_PACKED")) > 0)) {
+        const Sched so = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(),
+                                best.P, loc.warp_slots.empty() ? nullptr : &loc.warp_slots, ProgForm{true, PB});
+        const size_t sm_off = smem_of(so);
+        // (and only when that kernel variant spills no more than the packed one)
+        cudaFuncAttributes attr{}, packed{};
+        bool ok = true;
+        if (!device) {
+            attr.numRegs = 128;
+            attr.sharedSizeBytes = 64;
+        } else {
+            ok = tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &attr, true) == FIONA_OK &&
+                 tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &packed, false) == FIONA_OK &&
+                 attr.localSizeBytes <= packed.localSizeBytes;
+        }
+        const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
+        if (ok && sm_off + attr.sharedSizeBytes <= smem_cap &&
+            per_sm / (sm_off + attr.sharedSizeBytes + 1024) >= std::max(best.ctas, 1u) &&
+            65536 / (best.W * 32 * regs) >= std::max(best.ctas, 1u)) {
+            sc = so;
+            offsets = true;
+        }
+    }
+    best.smem = smem_of(sc);
     TiledSchedule *ts = new (std::nothrow) TiledSchedule;
     if (!ts) return set_error(FIONA_ERR_NOMEM, "tiled schedule: host allocation");
     ts->C = best.C;
@@ -1905,6 +2016,7 @@ int lower_tiled(fiona_plan *p)
     }
     a.wait_ns = 2000000000ull;
     a.zero = 0;
+    a.src_offsets = offsets ? 1 : 0;
     if (const char *t = getenv("FIONA_TEST_TILED_TIMEOUT")) {  // test only: a copy wait that runs out
         if (atoi(t) > 0 && best.C == 1 && hp.n_in) {
             a.test_flags |= kTiledFlagExtraTx;
@@ -1925,7 +2037,7 @@ int lower_tiled(fiona_plan *p)
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
     }
     if (device) {
-        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, use_tc, ts->smem);
+        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, use_tc, ts->smem, offsets);
         if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
         if (rc != FIONA_OK) {
             cudaFree(ts->sched.blob);

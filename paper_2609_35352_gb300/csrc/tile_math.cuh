@@ -197,25 +197,105 @@ __device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32
     return wp;
 }
 
+// The same sum over a run of byte offsets (one 32-bit word per source: the
+// source's offset from the start of the region, so that its address is one
+// addition), the run starting on a 16-byte boundary and padded to a multiple
+// of four words.  K offsets per step, read with one or two vector loads, the
+// next step's requested before this step's additions (that request may read
+// words past the run, inside the dynamic shared memory as above, unused).
+// Returns the offset just past the padded run.
+template <int C, uint32_t TB>
+__device__ __forceinline__ uint32_t run_sum_offsets(const char *sm, uint32_t src, uint32_t wp, uint32_t n, V<C> &s0,
+                                                    V<C> &s1)
+{
+    constexpr uint32_t K = C == 1 ? 8 : 2;  // 2K loads of C words in flight
+    uint32_t k = 0;
+    if (n >= K) {
+        uint32_t o[K];
+        auto get = [&](uint32_t at) {
+            if constexpr (K == 8) {
+                const uint4 x = *reinterpret_cast<const uint4 *>(sm + at);
+                const uint4 y = *reinterpret_cast<const uint4 *>(sm + at + 16);
+                o[0] = x.x, o[1] = x.y, o[2] = x.z, o[3] = x.w, o[4] = y.x, o[5] = y.y, o[6] = y.z, o[7] = y.w;
+            } else {
+                const uint2 x = *reinterpret_cast<const uint2 *>(sm + at);
+                o[0] = x.x, o[1] = x.y;
+            }
+        };
+        get(wp);
+        for (; k + K <= n; k += K, wp += 4 * K) {
+            V<C> a[K], b[K];
+#pragma unroll
+            for (uint32_t j = 0; j < K; ++j) {
+                a[j] = lds<C>(sm, src + o[j]);
+                b[j] = lds<C>(sm, src + o[j] + TB);
+            }
+            get(wp + 4 * K);
+#pragma unroll
+            for (int x = 0; x < C; ++x) {
+#pragma unroll
+                for (uint32_t j = 0; j + 1 < K; j += 2) {  // three-input additions
+                    s0.x[x] = s0.x[x] + a[j].x[x] + a[j + 1].x[x];
+                    s1.x[x] = s1.x[x] + b[j].x[x] + b[j + 1].x[x];
+                }
+            }
+        }
+    }
+    for (; k + 2 <= n; k += 2, wp += 8) {
+        const uint2 w = *reinterpret_cast<const uint2 *>(sm + wp);
+        const V<C> a0 = lds<C>(sm, src + w.x), a1 = lds<C>(sm, src + w.y);
+        const V<C> b0 = lds<C>(sm, src + w.x + TB), b1 = lds<C>(sm, src + w.y + TB);
+#pragma unroll
+        for (int x = 0; x < C; ++x) {
+            s0.x[x] += a0.x[x] + a1.x[x];
+            s1.x[x] += b0.x[x] + b1.x[x];
+        }
+    }
+    if (k < n) {
+        const uint32_t o0 = src + *reinterpret_cast<const uint32_t *>(sm + wp);
+        const V<C> a0 = lds<C>(sm, o0), b0 = lds<C>(sm, o0 + TB);
+#pragma unroll
+        for (int x = 0; x < C; ++x) {
+            s0.x[x] += a0.x[x];
+            s1.x[x] += b0.x[x];
+        }
+        wp += 4;
+    }
+    return (wp + 15) & ~15u;  // the run started on a 16-byte boundary
+}
+
 // Signed sum of the program at byte offset `hdr`, both polys, as canonical
 // residues; SPLIT: the sources are in split form (else canonical, whatever
-// the arithmetic).  A program is n_plus | n_minus << 16, the plus run, the
-// minus run, then one slot word: n_plus_slots | n_minus_slots << 4 and up to
-// six 4-bit slot numbers from bit 8 (plus slots first).  A slot is a tile
-// pair of this warp's slot area at byte offset `slots` (this lane's words
-// of slot 0), holding a shared signed sum the warp formed earlier.  Returns
-// the offset just past the program.
+// the arithmetic).  A program starts with n_plus | n_minus << 16.  In the
+// packed form (`offsets` false) the plus run and the minus run of 16-bit
+// source indices follow, then one slot word: n_plus_slots | n_minus_slots
+// << 4 and up to six 4-bit slot numbers from bit 8 (plus slots first).  In
+// the offset form the slot word is the second word, the program's first four
+// words are a block of their own (the third holds a formation's target slot),
+// and each run is a run of source byte offsets padded to four words
+// (run_sum_offsets); every offset-form program starts on a 16-byte boundary.
+// A slot is a tile pair of this warp's slot area at byte offset `slots`
+// (this lane's words of slot 0), holding a shared signed sum the warp formed
+// earlier.  Returns the offset just past the program.
 template <bool SPLIT, int C, uint32_t TB>
 __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uint32_t hdr, uint32_t lim,
-                                               uint32_t slots, V<C> &o0, V<C> &o1)
+                                               uint32_t slots, V<C> &o0, V<C> &o1, bool offsets = false)
 {
     using A = Arith<SPLIT>;
     constexpr uint32_t PB = 2 * TB;
     const uint32_t h = *reinterpret_cast<const uint32_t *>(sm + hdr);
     V<C> p0{}, p1{}, m0{}, m1{};
-    uint32_t wp = run_sum<C, TB>(sm, src, hdr + 4, h & 0xffffu, p0, p1);
-    wp = run_sum<C, TB>(sm, src, wp, h >> 16, m0, m1);
-    const uint32_t sw = *reinterpret_cast<const uint32_t *>(sm + wp);
+    uint32_t next, sw;
+    if (offsets) {
+        sw = *reinterpret_cast<const uint32_t *>(sm + hdr + 4);
+        next = run_sum_offsets<C, TB>(sm, src, hdr + 16, h & 0xffffu, p0, p1);
+        next = run_sum_offsets<C, TB>(sm, src, next, h >> 16, m0, m1);
+    } else {
+        uint32_t wp = run_sum<C, TB>(sm, src, hdr + 4, h & 0xffffu, p0, p1);
+        wp = run_sum<C, TB>(sm, src, wp, h >> 16, m0, m1);
+        sw = *reinterpret_cast<const uint32_t *>(sm + wp);
+        next = wp + 4;
+    }
     const uint32_t nps = sw & 15u, ns = nps + ((sw >> 4) & 15u);
     for (uint32_t j = 0; j < ns; ++j) {
         const uint32_t o = slots + ((sw >> (8 + 4 * j)) & 15u) * PB;
@@ -234,7 +314,7 @@ __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uin
         o0.x[x] = A::signed_value(p0.x[x], m0.x[x], m);
         o1.x[x] = A::signed_value(p1.x[x], m1.x[x], m);
     }
-    return wp + 4;
+    return next;
 }
 
 }  // namespace tile

@@ -33,12 +33,21 @@
 //   node offsets    word offset of each node's program
 //   node programs   n_plus | n_minus << 16, then the plus then the minus
 //                   source indices, two 16-bit indices per word (each run
-//                   starts on a new word)
+//                   starts on a new word); or, in the offset form
+//                   (TiledArgs::src_offsets), a block of four words (the
+//                   header, the slot word, a formation's target slot, 0)
+//                   and the runs as one 32-bit word per source, its byte
+//                   offset s * 2T * 8 in the source region, each run padded
+//                   to a multiple of four words: the kernel then forms each
+//                   source's address with one addition instead of unpacking
+//                   and scaling an index
 //   warp table      per warp: op stream offset, op count (a multiple of the
 //                   prefetch depth), segment stream offset, target offset,
 //                   first warp slot (then padding to eight words)
 //   op streams      one word per operation (layout below)
 //   segment streams per SEG operation, in order: a program as above
+//                   (its formations first: a slot word and a program each,
+//                   or in the offset form a program holding its slot)
 //   target streams  per job: output index, or kPartBit | partial slot
 //   combine lists   per split output: its partial slots
 //   (tensor-core sums only) W as fp16 core matrices, then one fp32 constant
@@ -114,6 +123,7 @@ struct TiledArgs {
     uint64_t wait_ns;        // bound of the waits for input copies and for the contraction
     uint32_t test_flags;     // kTiledFlag* (0 outside tests)
     uint32_t zero;           // always 0, read at run time (rns::mac26)
+    uint32_t src_offsets;    // 1: programs in the offset form (source byte offsets), 0: packed indices
 };
 
 // Warp-specialised variant (kernel_ws.cu), two coefficients per lane.  The

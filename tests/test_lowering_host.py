@@ -72,6 +72,39 @@ def test_workloads_lower_exactly(name):
         assert plan.stats()["kernel"] == F.FIONA_KERNEL_TILED
 
 
+@pytest.mark.parametrize("packed", [False, True])
+def test_program_forms_lower_exactly(packed, monkeypatch):
+    """The signed-sum programs in both forms of the schedule: source byte
+    offsets (the default where the schedule fits) and 16-bit indices packed
+    two per word (FIONA_TILED_PACKED=1).  The schedule check walks each form
+    as the kernel reads it (alignment, whole-source offsets, formations'
+    target slots) and the symbolic check evaluates it against the plan's
+    terms; plan creation fails otherwise."""
+    if packed:
+        monkeypatch.setenv("FIONA_TILED_PACKED", "1")
+    forms = []
+    for seed in range(16):
+        rng = np.random.default_rng(9300 + seed)
+        shape = ["2,1,1", "1,2,1", "", "1,4,0"][seed % 4]
+        if shape:
+            monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+        else:
+            monkeypatch.delenv("FIONA_TILED_SHAPE", raising=False)
+        desc = random_layer(rng, big=seed % 3 == 2)
+        plan = lower(desc, 4096, int(rng.choice([40, 50, 59])), 2)
+        st = plan.stats()
+        if st["kernel"] == F.FIONA_KERNEL_TILED:
+            forms.append(st["source_offsets"])
+    # (a layer whose offset schedule does not fit in shared memory keeps the packed form)
+    if packed:
+        assert forms and all(f == 0 for f in forms), forms
+    else:
+        assert sum(forms) >= len(forms) // 2, forms
+    wl = W.make_workload("vgg")
+    st = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), wl.plan).stats()
+    assert st["source_offsets"] == (0 if packed else 1)
+
+
 def test_long_signed_runs_are_cut_and_still_exact():
     """One output whose signed run is far longer than the 64-word lazy-sum
     bound of narrow arithmetic (the lowering cuts it into pieces with the

@@ -59,6 +59,22 @@ def test_elementwise_parity_small(name, N, L, kernel):
     assert dl.ctx.device_check() == F.FIONA_OK
 
 
+@pytest.mark.parametrize("name,N,L", [("tiny-dag", None, None), ("vgg", 1024, 2), ("vit", 2048, 2),
+                                      ("bert-const", 1024, 1), ("overflow50", None, None)])
+def test_packed_programs_parity(name, N, L, monkeypatch):
+    """The tiled kernel with its signed-sum programs as packed 16-bit indices
+    (FIONA_TILED_PACKED=1; the form a schedule takes when the offset form
+    does not fit in shared memory) gives the same residues."""
+    monkeypatch.setenv("FIONA_TILED_PACKED", "1")
+    wl = W.make_workload(name, N=N, L=L)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel("tiled")
+    assert dl.plan.stats()["source_offsets"] == 0
+    dl.run()
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    assert np.array_equal(dl.outputs(), want)
+
+
 # Tiled shapes (coefficients per lane, warps, source regions[, most shared
 # sums kept (-1: the lowering's choice)[, operations per batch]]) chosen
 # through the lowering's override; every shape must give the same residues.
