@@ -1956,6 +1956,10 @@ int lower_tiled(fiona_plan *p)
                  attr.localSizeBytes <= packed.localSizeBytes;
         }
         const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
+        if (getenv("FIONA_TILED_DEBUG"))
+            fprintf(stderr, "offset form: ok=%d smem=%zu+%zu cap=%zu per_sm=%zu ctas=%u regs=%u local=%zu/%zu\n",
+                    (int)ok, sm_off, (size_t)attr.sharedSizeBytes, smem_cap, per_sm, best.ctas, regs,
+                    (size_t)attr.localSizeBytes, (size_t)packed.localSizeBytes);
         if (ok && sm_off + attr.sharedSizeBytes <= smem_cap &&
             per_sm / (sm_off + attr.sharedSizeBytes + 1024) >= std::max(best.ctas, 1u) &&
             65536 / (best.W * 32 * regs) >= std::max(best.ctas, 1u)) {

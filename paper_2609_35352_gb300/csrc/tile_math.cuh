@@ -200,7 +200,7 @@ __device__ __forceinline__ uint32_t run_sum(const char *sm, uint32_t src, uint32
 // The same sum over a run of byte offsets (one 32-bit word per source: the
 // source's offset from the start of the region, so that its address is one
 // addition), the run starting on a 16-byte boundary and padded to a multiple
-// of four words.  K offsets per step, read with one or two vector loads, the
+// of four words.  K offsets per step, read with one vector load, the
 // next step's requested before this step's additions (that request may read
 // words past the run, inside the dynamic shared memory as above, unused).
 // Returns the offset just past the padded run.
@@ -208,15 +208,16 @@ template <int C, uint32_t TB>
 __device__ __forceinline__ uint32_t run_sum_offsets(const char *sm, uint32_t src, uint32_t wp, uint32_t n, V<C> &s0,
                                                     V<C> &s1)
 {
-    constexpr uint32_t K = C == 1 ? 8 : 2;  // 2K loads of C words in flight
+    // 2K loads of C words in flight (measured on GB300 with one coefficient
+    // per lane: VGG 2.307 ms with K = 8, 2.274 ms with 4; with two, 2 beats 4)
+    constexpr uint32_t K = C == 1 ? 4 : 2;
     uint32_t k = 0;
     if (n >= K) {
         uint32_t o[K];
         auto get = [&](uint32_t at) {
-            if constexpr (K == 8) {
+            if constexpr (K == 4) {
                 const uint4 x = *reinterpret_cast<const uint4 *>(sm + at);
-                const uint4 y = *reinterpret_cast<const uint4 *>(sm + at + 16);
-                o[0] = x.x, o[1] = x.y, o[2] = x.z, o[3] = x.w, o[4] = y.x, o[5] = y.y, o[6] = y.z, o[7] = y.w;
+                o[0] = x.x, o[1] = x.y, o[2] = x.z, o[3] = x.w;
             } else {
                 const uint2 x = *reinterpret_cast<const uint2 *>(sm + at);
                 o[0] = x.x, o[1] = x.y;
