@@ -343,7 +343,7 @@ def measured_peak():
 
 KERNEL_FILES = {"direct": ["kernel_direct.cu", "rns.cuh"],
                 "tiled": ["kernel_tiled.cu", "kernel_tiled_off.cu", "tiled_kernel.cuh", "tiled.h", "lower_tiled.cpp",
-                          "rns.cuh", "tile_math.cuh", "async.cuh", "tc_signed.cuh", "tc_geometry.h"]}
+                          "rns.cuh", "tile_math.cuh", "async.cuh", "tc_signed.cuh", "tc_geometry.h", "../build.py"]}
 
 
 def kernel_source_hash(kernel: str) -> str:

@@ -24,6 +24,12 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O3",
          "--expt-relaxed-constexpr", "-I" + INCLUDE]
 
+# per-file ptxas settings: the tiled kernel's batch loop is sensitive to
+# register allocation; a higher register-usage level (documented ptxas
+# option, default 5) measured 1% faster on the VGG layer, 0.5% on ViT
+EXTRA = {"kernel_tiled.cu": ["-Xptxas", "-regUsageLevel=8"],
+         "kernel_tiled_off.cu": ["-Xptxas", "-regUsageLevel=8"]}
+
 LIBRARIES = {
     "libfiona.so": ["fiona_host.cpp", "lower_tiled.cpp", "plan_compile.cpp", "kernel_direct.cu",
                     "kernel_tiled.cu", "kernel_tiled_off.cu", "kernel_ws.cu", "rescale.cu", "encode.cu"],
@@ -76,7 +82,8 @@ def build(force: bool = False, verbose_ptxas: bool = False) -> dict:
             objs = [os.path.join(OUT, os.path.basename(s) + ".o") for s in srcs]
             jobs.append((target, paths, objs))
     with concurrent.futures.ThreadPoolExecutor(max_workers=max(2, os.cpu_count() or 2)) as ex:
-        futs = [ex.submit(_compile, s, o, extra) for (_, ps, os_) in jobs for s, o in zip(ps, os_)]
+        futs = [ex.submit(_compile, s, o, extra + EXTRA.get(os.path.basename(s), []))
+                for (_, ps, os_) in jobs for s, o in zip(ps, os_)]
         for f in futs:
             f.result()
     for target, _, objs in jobs:
