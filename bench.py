@@ -342,7 +342,7 @@ def measured_peak():
 
 
 KERNEL_FILES = {"direct": ["kernel_direct.cu", "rns.cuh"],
-                "tiled": ["kernel_tiled.cu", "kernel_tiled_off.cu", "tiled_kernel.cuh", "tiled.h", "lower_tiled.cpp",
+                "tiled": ["kernel_tiled.cu", "kernel_tiled_off.cu", "kernel_tiled_w12.cu", "tiled_kernel.cuh", "tiled.h", "lower_tiled.cpp",
                           "rns.cuh", "tile_math.cuh", "async.cuh", "tc_signed.cuh", "tc_geometry.h", "../build.py"]}
 
 

@@ -28,11 +28,12 @@ FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", 
 # register allocation; a higher register-usage level (documented ptxas
 # option, default 5) measured 1% faster on the VGG layer, 0.5% on ViT
 EXTRA = {"kernel_tiled.cu": ["-Xptxas", "-regUsageLevel=8"],
-         "kernel_tiled_off.cu": ["-Xptxas", "-regUsageLevel=8"]}
+         "kernel_tiled_off.cu": ["-Xptxas", "-regUsageLevel=8"],
+         "kernel_tiled_w12.cu": ["-Xptxas", "-regUsageLevel=8"]}
 
 LIBRARIES = {
     "libfiona.so": ["fiona_host.cpp", "lower_tiled.cpp", "plan_compile.cpp", "kernel_direct.cu",
-                    "kernel_tiled.cu", "kernel_tiled_off.cu", "kernel_ws.cu", "rescale.cu", "encode.cu"],
+                    "kernel_tiled.cu", "kernel_tiled_off.cu", "kernel_tiled_w12.cu", "kernel_ws.cu", "rescale.cu", "encode.cu"],
     "libfiona_workload.so": ["workload_fill.cu", "mul_roof.cu"],
 }
 

@@ -5,6 +5,9 @@
 
 // kernel_tiled_off.cu: the variant with programs in the offset form, or null
 void *tiled_select_offsets(int C, bool narrow, uint32_t P, bool kc);
+// kernel_tiled_w12.cu: the 12-warp variants (two coefficients per lane,
+// narrow moduli, batches of 8)
+void *tiled_select_w12(bool kc, bool off);
 
 namespace {
 
@@ -29,9 +32,11 @@ void *select_ptr_16(int C, bool narrow)
 
 // KC: the variant that reads constant plaintexts (operations marked kOpConst);
 // TC: the signed sums on the tensor cores (one coefficient per lane, narrow
-// moduli, batches of 16); off: signed-sum programs in the offset form
-void *select_ptr(int C, bool narrow, uint32_t P, bool kc, bool tc = false, bool off = false)
+// moduli, batches of 16); off: signed-sum programs in the offset form; w12:
+// the variant for CTAs of at most 12 warps
+void *select_ptr(int C, bool narrow, uint32_t P, bool kc, bool tc = false, bool off = false, bool w12 = false)
 {
+    if (w12) return C == 2 && narrow && P == 8 && !tc ? tiled_select_w12(kc, off) : nullptr;
     if (off) return tc ? nullptr : tiled_select_offsets(C, narrow, P, kc);
     if (tc) {
         if (C != 1 || !narrow || P != 16) return nullptr;
@@ -45,20 +50,21 @@ void *select_ptr(int C, bool narrow, uint32_t P, bool kc, bool tc = false, bool 
 
 }  // namespace
 
-int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr, bool off)
+int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr, bool off,
+                            bool w12)
 {
-    if (!select_ptr(C, narrow, P, kc, tc, off))
+    if (!select_ptr(C, narrow, P, kc, tc, off, w12))
         return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
-    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc, tc, off));
+    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc, tc, off, w12));
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attributes: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
 
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off)
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off, bool w12)
 {
-    if (!select_ptr(C, narrow, P, kc, tc, off))
+    if (!select_ptr(C, narrow, P, kc, tc, off, w12))
         return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
-    cudaError_t e = cudaFuncSetAttribute(select_ptr(C, narrow, P, kc, tc, off),
+    cudaError_t e = cudaFuncSetAttribute(select_ptr(C, narrow, P, kc, tc, off, w12),
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attribute: %s", cudaGetErrorString(e));
     return FIONA_OK;
@@ -126,7 +132,7 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     dim3 grid(std::min(tiles, resident));
     dim3 block(ts->warps * 32);
     cudaStream_t s = (cudaStream_t)stream;
-    void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const, ts->tc, a.src_offsets != 0);
+    void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const, ts->tc, a.src_offsets != 0, ts->w12);
     if (!fn) return set_error(FIONA_ERR_INTERNAL, "tiled kernel: no variant for the schedule's shape");
     CUtensorMap tm;  // read by the kernels with one coefficient per lane only
     memset(&tm, 0, sizeof(tm));

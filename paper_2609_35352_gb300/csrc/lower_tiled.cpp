@@ -1381,9 +1381,10 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
 
 // kernel_tiled.cu
 // (kernel_tiled.cu; off: the variant whose signed-sum programs are in the offset form)
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off = false);
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off = false,
+                           bool w12 = false);
 int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr,
-                            bool off = false);
+                            bool off = false, bool w12 = false);
 // kernel_ws.cu
 int ws_kernel_attributes(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, cudaFuncAttributes *attr);
 int ws_configure_kernel(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, size_t smem);
@@ -1651,6 +1652,7 @@ int lower_tiled(fiona_plan *p)
         uint32_t W = 0, P = 8;
         double pad = 0;               // share of padding operations
         bool dbl = false;
+        bool w12 = false;             // the variant for CTAs of at most 12 warps
         uint32_t keep = 0, ctas = 0;  // shared sums requested (top of the ranking)
         size_t smem = 0;
         double est = 0;
@@ -1672,8 +1674,19 @@ int lower_tiled(fiona_plan *p)
         } else if (tiled_kernel_attributes(C, narrow, batch, has_const, false, &attr) != FIONA_OK) {
             continue;
         }
-        const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
+        // the variant for CTAs of at most 12 warps (two coefficients per
+        // lane, narrow moduli, batches of 8): more registers a thread
+        cudaFuncAttributes attr12{};
+        bool has12 = C == 2 && batch == 8 && narrow;
+        if (has12 && !device) {
+            attr12.numRegs = 168;
+            attr12.sharedSizeBytes = 64;
+        } else if (has12) {
+            has12 = tiled_kernel_attributes(C, narrow, batch, has_const, false, &attr12, false, true) == FIONA_OK;
+        }
         for (uint32_t W : {16u, 12u, 8u, 4u, 2u, 1u}) {
+            const bool w12 = has12 && W <= 12;
+            const uint32_t regs = (std::max(w12 ? attr12.numRegs : attr.numRegs, 1) + 7) & ~7;
             // one or two warps only when the tuning override asks for them
             if (W < 4) {
                 const char *env = getenv("FIONA_TILED_SHAPE");
@@ -1746,29 +1759,37 @@ int lower_tiled(fiona_plan *p)
                 for (uint32_t wi = 0; wi < W; ++wi) n_ops += sc.w[sc.o_warp + wi * kWarpTableWords + 1];
                 s.pad = n_ops ? 1.0 - (double)sc.pt_ops / (double)n_ops : 0.0;
                 s.dbl = dbl;
+                s.w12 = w12;
                 s.keep = hi;
                 s.ctas = ctas;
                 s.smem = smem - attr.sharedSizeBytes;
                 s.est = rounds * per_round;
                 shapes.push_back(s);
                 if (getenv("FIONA_TILED_DEBUG"))
-                    fprintf(stderr, "C=%d P=%u W=%u dbl=%d keep=%u sched=%zu parts=%u smem=%zu ctas=%u pad=%.2f est=%.0f\n",
-                            C, batch, W, (int)dbl, s.keep, sc.w.size() * 4, jp.n_part, smem, ctas, s.pad, s.est);
+                    fprintf(stderr,
+                            "C=%d P=%u W=%u dbl=%d w12=%d keep=%u sched=%zu parts=%u smem=%zu ctas=%u pad=%.2f est=%.0f\n",
+                            C, batch, W, (int)dbl, (int)w12, s.keep, sc.w.size() * 4, jp.n_part, smem, ctas, s.pad,
+                            s.est);
             }
         }
     }
     if (shapes.empty()) return set_error(FIONA_ERR_ARG, "tiled kernel: the input tiles do not fit in shared memory");
     // Ranking (from shape sweeps of the layer workloads): a second source
     // region first (the next tile's inputs arrive during this one), then
-    // resident warps up to 16 per SM, then 2 coefficients per lane (half the
+    // resident warps up to 16 per SM (12 warps of the 12-warp variant count
+    // as 16: their deeper plaintext queues keep as many HBM reads in flight
+    // as 16 warps with 4), then 2 coefficients per lane (half the
     // per-operation overhead per coefficient), then more CTAs per SM (their
-    // per-tile phases overlap), then batches of 4 with 2 coefficients per
-    // lane and of 16, then 8, with one (BERT and ViT ran faster with 4; VGG
-    // with 16, its deeper plaintext queue keeping more HBM reads in flight),
-    // then the cost estimate.
+    // per-tile phases overlap), then, with 2 coefficients per lane, the
+    // 12-warp variant with batches of 8, batches of 4, and of 8, and with
+    // one, batches of 16, then 8 (measured: BERT, one CTA per SM, 5.998 ms
+    // with 12 warps x 8 against 6.049 ms with 16 x 4; ViT faster with two
+    // CTAs of 8 warps x 4; VGG with 16, its deeper plaintext queue keeping
+    // more HBM reads in flight), then the cost estimate.
     auto key = [](const Shape &s) {
-        const int pref = s.C == 2 ? (s.P == 4 ? 2 : 1) : (s.P == 16 ? 2 : s.P == 8 ? 1 : 0);
-        return std::make_tuple(s.dbl ? 1 : 0, std::min<uint32_t>(s.ctas * s.W, 16), s.C, s.ctas, pref, -s.est);
+        const int pref = s.C == 2 ? (s.w12 && s.P == 8 ? 3 : s.P == 4 ? 2 : 1) : (s.P == 16 ? 2 : s.P == 8 ? 1 : 0);
+        const uint32_t resident = s.w12 && s.W == 12 ? 16 : std::min<uint32_t>(s.ctas * s.W, 16);
+        return std::make_tuple(s.dbl ? 1 : 0, resident, s.C, s.ctas, pref, -s.est);
     };
     Shape best = *std::max_element(shapes.begin(), shapes.end(),
                                    [&](const Shape &a, const Shape &b) { return key(a) < key(b); });
@@ -1951,8 +1972,9 @@ int lower_tiled(fiona_plan *p)
             attr.numRegs = 128;
             attr.sharedSizeBytes = 64;
         } else {
-            ok = tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &attr, true) == FIONA_OK &&
-                 tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &packed, false) == FIONA_OK &&
+            ok = tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &attr, true, best.w12) == FIONA_OK &&
+                 tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &packed, false, best.w12) ==
+                     FIONA_OK &&
                  attr.localSizeBytes <= packed.localSizeBytes;
         }
         const uint32_t regs = (std::max(attr.numRegs, 1) + 7) & ~7;
@@ -1979,6 +2001,7 @@ int lower_tiled(fiona_plan *p)
     ts->smem = best.smem;
     ts->ctas_per_sm = best.ctas;
     ts->tc = use_tc;
+    ts->w12 = best.w12 && !use_tc;
     // (the group sums of the tensor-core variant are not shared sums: every
     // shared sum is expanded into them)
     ts->nodes_kept = use_tc ? 0 : (uint32_t)lw.nodes.size() + loc.formed;
@@ -2041,7 +2064,7 @@ int lower_tiled(fiona_plan *p)
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
     }
     if (device) {
-        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, use_tc, ts->smem, offsets);
+        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, use_tc, ts->smem, offsets, ts->w12);
         if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
         if (rc != FIONA_OK) {
             cudaFree(ts->sched.blob);

@@ -193,6 +193,7 @@ struct TiledSchedule {
     DeviceSchedule sched;
     TiledArgs args{};          // device pointers (data pointers unset)
     bool tc = false;           // the scale groups' signed sums run on the tensor cores (args.tc_groups)
+    bool w12 = false;          // the variant built for CTAs of at most 12 warps (kernel_tiled_w12.cu)
     bool ws = false;           // the warp-specialised kernel runs this plan
     uint32_t ring = 0;         // its plaintext ring depth D (groups of P slots per warp)
     WsArgs ws_args{};

@@ -158,9 +158,11 @@ __device__ __forceinline__ uint64_t evict_first_policy()
 }
 
 // OFF: the schedule's signed-sum programs are in the offset form (tiled.h;
-// TiledArgs::src_offsets), each source address one addition
-template <int C, bool NARROW, uint32_t P, bool KC, bool TC = false, bool OFF = false>
-__global__ void __launch_bounds__(kTiledMaxWarps * 32)
+// TiledArgs::src_offsets), each source address one addition.  WB: the most
+// warps a CTA of this variant runs (fewer warps leave each thread more
+// registers: the variants with 12 warps and 8-deep plaintext queues)
+template <int C, bool NARROW, uint32_t P, bool KC, bool TC = false, bool OFF = false, uint32_t WB = kTiledMaxWarps>
+__global__ void __launch_bounds__(WB * 32)
     tiled_kernel(const TiledArgs a, const __grid_constant__ CUtensorMap tm_in)
 {
     static_assert(!TC || (C == 1 && NARROW), "tensor-core sums: one coefficient per lane, narrow moduli");

@@ -79,8 +79,10 @@ def test_packed_programs_parity(name, N, L, monkeypatch):
 # sums kept (-1: the lowering's choice)[, operations per batch]]) chosen
 # through the lowering's override; every shape must give the same residues.
 # A fourth field forces the shared sums in play (0: all expanded), a fifth
-# selects batches of 4.
-SHAPES = ["2,16,0", "2,8,1", "1,16,1", "1,4,0", "2,12,1,0", "1,8,0,3", "2,8,1,-1,4", "1,16,0,2,4"]
+# selects batches of 4 (or 8: "2,12,1,-1,8" and "2,8,1,-1,8" take the
+# variant built for CTAs of at most 12 warps, two coefficients per lane).
+SHAPES = ["2,16,0", "2,8,1", "1,16,1", "1,4,0", "2,12,1,0", "1,8,0,3", "2,8,1,-1,4", "1,16,0,2,4", "2,12,1,-1,8",
+          "2,8,1,-1,8"]
 SHAPE_CASES = [("tiny-dag", None, None), ("vit", 2048, 2), ("bert", 1024, 1), ("bert-const", 1024, 1),
                ("vgg", 1024, 2),
                ("overflow60", None, None), ("overflow50", None, None)]
