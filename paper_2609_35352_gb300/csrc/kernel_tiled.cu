@@ -1,6 +1,7 @@
 // kernel_tiled.cu -- launch of the tiled evaluation kernel (tiled_kernel.cuh)
 // and its variants with packed signed-sum programs; the variants whose
-// programs are in the offset form are built in kernel_tiled_off.cu.
+// programs are in the offset form are built in kernel_tiled_off.cu, those
+// for CTAs of at most 12 warps in kernel_tiled_w12.cu.
 #include "tiled_kernel.cuh"
 
 // kernel_tiled_off.cu: the variant with programs in the offset form, or null

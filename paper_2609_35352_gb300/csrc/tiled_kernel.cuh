@@ -1,6 +1,7 @@
 // tiled_kernel.cuh -- the tiled evaluation kernel of the hybrid linear layer
-// (instantiated by kernel_tiled.cu and, in the offset form of its signed-sum
-// programs, by kernel_tiled_off.cu: two translation units built in parallel).
+// (instantiated by kernel_tiled.cu; its variants with signed-sum programs in
+// the offset form by kernel_tiled_off.cu, and those for CTAs of at most 12
+// warps by kernel_tiled_w12.cu: translation units built in parallel).
 //
 // A persistent CTA walks (limb l, coefficient tile) pairs, T = 32*C
 // coefficients per tile, all outputs per tile.  Shared memory holds the
@@ -22,7 +23,9 @@
 //  2. The materialised shared signed sums (Sec. 4.2 "Sharing Signed Sums")
 //     are formed once per tile, level by level, into the same region.
 //  3. Each warp runs its operation stream (tiled.h): per scale group a
-//     signed sum over sources, formed before the batch its product opens,
+//     signed sum over sources (their shared-memory offsets read from the
+//     schedule, or packed 16-bit indices where the larger schedule does not
+//     fit), formed before the batch its product opens,
 //     then one product by gamma (Sec. 4.2 "Grouping Reconstruction
 //     Operations"); per raw term a PMult-MAC of a
 //     plaintext tile and a source.  Plaintext tiles go from HBM straight to
