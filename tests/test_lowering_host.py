@@ -105,6 +105,33 @@ def test_program_forms_lower_exactly(packed, monkeypatch):
     assert st["source_offsets"] == (0 if packed else 1)
 
 
+def test_twelve_warp_variant_only_where_warps_balance():
+    """The shape ranking takes the 12-warp variant (two coefficients per
+    lane, batches of 8) for BERT, whose 96 outputs load 12 warps evenly and
+    whose source regions leave room for one CTA per SM, and keeps 16 warps
+    for the first 72 inputs of the VGG layer (16 outputs: 12 warps would
+    carry two outputs on four of them) and two CTAs of 8 warps for ViT."""
+    def shape(plan, wl):
+        st = F.Plan(F.Context(wl.N, wl.moduli, device=F.FIONA_DEVICE_NONE), plan).stats()
+        return st["tile_coeffs"], st["warps_per_cta"], st["ctas_per_sm"]
+    bert = W.make_workload("bert")
+    assert shape(bert.plan, bert) == (64, 12, 1)
+    vit = W.make_workload("vit")
+    assert shape(vit.plan, vit) == (64, 8, 2)
+    vgg = W.make_workload("vgg")
+    p = vgg.plan
+    rows, offs = [], [0]
+    for j in range(p.n_out):
+        t = p.terms[p.term_offsets[j]:p.term_offsets[j + 1]]
+        t = t[t["input"] < 72]
+        rows.append(t)
+        offs.append(offs[-1] + len(t))
+    half = W.Plan(n_in=72, n_out=p.n_out, n_pt=p.n_pt, term_offsets=np.array(offs, np.uint32),
+                  terms=np.concatenate(rows), group_scale_pt=p.group_scale_pt, group_output=p.group_output,
+                  node_offsets=p.node_offsets, children=p.children, uses=p.uses)
+    assert shape(half, vgg) == (64, 16, 1)
+
+
 def test_long_signed_runs_are_cut_and_still_exact():
     """One output whose signed run is far longer than the 64-word lazy-sum
     bound of narrow arithmetic (the lowering cuts it into pieces with the
