@@ -608,7 +608,8 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> None:
                        "shared_sums_formed": stats["nodes_materialized"],
                        "addsub_executed": stats.get("addsub_executed"),
                        "tensor_core_sums": stats.get("tensor_core_sums"),
-                       "source_offsets": stats.get("source_offsets")},
+                       "source_offsets": stats.get("source_offsets"),
+                       "const_raw_all": stats.get("const_raw_all")},
         }
         print(json.dumps(line), flush=True)
     plan.close()

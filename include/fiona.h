@@ -167,7 +167,9 @@ typedef struct fiona_plan_stats_t {
                                      offsets (one addition per source address), 0 if 16-bit
                                      indices packed two per word (used when the larger offset
                                      schedule does not fit in shared memory)                   */
-    uint32_t reserved;
+    uint32_t const_raw_all;       /* TILED: 1 if every raw plaintext of the plan is constant and
+                                     the kernel variant for that case runs (no per-operation test
+                                     of the plaintext's kind after a batch's first operation)   */
 } fiona_plan_stats_t;
 
 /* Create a context for ring dimension N (a power of two, 2^10 <= N <= 2^17)

@@ -583,6 +583,7 @@ static int select_kernel(fiona_plan *p, int which)
         s.addsub_executed = p->tiled->addsub;
         s.tensor_core_sums = p->tiled->tc ? p->tiled->args.tc_groups : 0;
         s.source_offsets = p->tiled->args.src_offsets;
+        s.const_raw_all = p->tiled->args.kc_all;
     } else {
         s.kernel = FIONA_KERNEL_DIRECT;
         s.tile_coeffs = 256;
@@ -593,6 +594,7 @@ static int select_kernel(fiona_plan *p, int which)
         s.addsub_executed = (uint32_t)std::min<uint64_t>(s.addsub_flat, 0xffffffffu);
         s.tensor_core_sums = 0;
         s.source_offsets = 0;
+        s.const_raw_all = 0;
     }
     return FIONA_OK;
 }

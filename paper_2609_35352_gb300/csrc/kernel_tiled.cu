@@ -8,7 +8,7 @@
 void *tiled_select_offsets(int C, bool narrow, uint32_t P, bool kc);
 // kernel_tiled_w12.cu: the 12-warp variants (two coefficients per lane,
 // narrow moduli, batches of 8)
-void *tiled_select_w12(bool kc, bool off);
+void *tiled_select_w12(bool kc, bool off, bool ka);
 
 namespace {
 
@@ -34,10 +34,12 @@ void *select_ptr_16(int C, bool narrow)
 // KC: the variant that reads constant plaintexts (operations marked kOpConst);
 // TC: the signed sums on the tensor cores (one coefficient per lane, narrow
 // moduli, batches of 16); off: signed-sum programs in the offset form; w12:
-// the variant for CTAs of at most 12 warps
-void *select_ptr(int C, bool narrow, uint32_t P, bool kc, bool tc = false, bool off = false, bool w12 = false)
+// the variant for CTAs of at most 12 warps; ka: every raw plaintext constant
+void *select_ptr(int C, bool narrow, uint32_t P, bool kc, bool tc = false, bool off = false, bool w12 = false,
+                 bool ka = false)
 {
-    if (w12) return C == 2 && narrow && P == 8 && !tc ? tiled_select_w12(kc, off) : nullptr;
+    if (w12) return C == 2 && narrow && P == 8 && !tc ? tiled_select_w12(kc, off, ka) : nullptr;
+    if (ka) return nullptr;  // (built for the 12-warp shape only)
     if (off) return tc ? nullptr : tiled_select_offsets(C, narrow, P, kc);
     if (tc) {
         if (C != 1 || !narrow || P != 16) return nullptr;
@@ -52,20 +54,21 @@ void *select_ptr(int C, bool narrow, uint32_t P, bool kc, bool tc = false, bool 
 }  // namespace
 
 int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr, bool off,
-                            bool w12)
+                            bool w12, bool ka)
 {
-    if (!select_ptr(C, narrow, P, kc, tc, off, w12))
+    if (!select_ptr(C, narrow, P, kc, tc, off, w12, ka))
         return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
-    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc, tc, off, w12));
+    cudaError_t e = cudaFuncGetAttributes(attr, select_ptr(C, narrow, P, kc, tc, off, w12, ka));
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attributes: %s", cudaGetErrorString(e));
     return FIONA_OK;
 }
 
-int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off, bool w12)
+int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off, bool w12,
+                           bool ka)
 {
-    if (!select_ptr(C, narrow, P, kc, tc, off, w12))
+    if (!select_ptr(C, narrow, P, kc, tc, off, w12, ka))
         return set_error(FIONA_ERR_ARG, "tiled kernel: no variant with C=%d, P=%u", C, P);
-    cudaError_t e = cudaFuncSetAttribute(select_ptr(C, narrow, P, kc, tc, off, w12),
+    cudaError_t e = cudaFuncSetAttribute(select_ptr(C, narrow, P, kc, tc, off, w12, ka),
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return set_error(FIONA_ERR_CUDA, "tiled kernel attribute: %s", cudaGetErrorString(e));
     return FIONA_OK;
@@ -133,7 +136,8 @@ int launch_tiled(const fiona_plan *p, void *stream, const uint64_t *in, const ui
     dim3 grid(std::min(tiles, resident));
     dim3 block(ts->warps * 32);
     cudaStream_t s = (cudaStream_t)stream;
-    void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const, ts->tc, a.src_offsets != 0, ts->w12);
+    void *fn = select_ptr(ts->C, ts->narrow, ts->batch, ts->has_const, ts->tc, a.src_offsets != 0, ts->w12,
+                          a.kc_all != 0);
     if (!fn) return set_error(FIONA_ERR_INTERNAL, "tiled kernel: no variant for the schedule's shape");
     CUtensorMap tm;  // read by the kernels with one coefficient per lane only
     memset(&tm, 0, sizeof(tm));

@@ -1236,6 +1236,7 @@ const char *check_schedule(const std::vector<uint32_t> &w, const TiledArgs &a, u
             // every operation loads a plaintext tile, NOPs included
             if ((op >> kOpPtShift) >= std::max<uint32_t>(n_pt, 1)) return "plaintext index";
             if ((op & kOpConst) && (op & kOpSeg)) return "SEG marked CONST";
+            if (a.kc_all && pos != 0 && !(op & (kOpNop | kOpConst))) return "RAW read as constant";
             if (op & kOpNop) {
                 if (op & kOpSeg) return "SEG marked NOP";
                 if ((op & (kOpMaxSources - 1)) != zero) return "NOP source";
@@ -1382,9 +1383,9 @@ const char *check_linear_map(const std::vector<uint32_t> &w, const TiledArgs &a,
 // kernel_tiled.cu
 // (kernel_tiled.cu; off: the variant whose signed-sum programs are in the offset form)
 int tiled_configure_kernel(int C, bool narrow, uint32_t P, bool kc, bool tc, size_t smem, bool off = false,
-                           bool w12 = false);
+                           bool w12 = false, bool ka = false);
 int tiled_kernel_attributes(int C, bool narrow, uint32_t P, bool kc, bool tc, cudaFuncAttributes *attr,
-                            bool off = false, bool w12 = false);
+                            bool off = false, bool w12 = false, bool ka = false);
 // kernel_ws.cu
 int ws_kernel_attributes(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, cudaFuncAttributes *attr);
 int ws_configure_kernel(bool narrow, uint32_t P, bool kc, uint32_t W, uint32_t D, size_t smem);
@@ -1966,6 +1967,15 @@ int lower_tiled(fiona_plan *p)
     // occupancy the shape was chosen for; otherwise (BERT, whose two source
     // regions fill the shared memory) the packed indices.  FIONA_TILED_PACKED=1
     // keeps the packed form (the same residues).
+    // every raw plaintext constant (the bert-const layers): the 12-warp
+    // shape has a kernel variant that reads every operation after a batch's
+    // first as constant, without a per-operation test (a SEG only opens a
+    // batch).  FIONA_TILED_KC_MIXED=1 keeps the per-operation test.
+    bool kc_all = false;
+    if (has_const && best.w12 && !use_tc && !(getenv("FIONA_TILED_KC_MIXED") && atoi(getenv("FIONA_TILED_KC_MIXED")) > 0)) {
+        kc_all = true;
+        for (const fiona_term &t : hp.terms) kc_all &= t.kind != FIONA_TERM_RAW;
+    }
     bool offsets = false;
     if (!use_tc && !(getenv("FIONA_TILED_PACKED") && atoi(getenv("FIONA_TILED_PACKED")) > 0)) {
         const Sched so = encode(jp, lw.level_off, lw.nodes, best.W, mac_budget, hp.n_in + (uint32_t)lw.nodes.size(),
@@ -1978,8 +1988,9 @@ int lower_tiled(fiona_plan *p)
             attr.numRegs = 128;
             attr.sharedSizeBytes = 64;
         } else {
-            ok = tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &attr, true, best.w12) == FIONA_OK &&
-                 tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &packed, false, best.w12) ==
+            ok = tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &attr, true, best.w12, kc_all) ==
+                     FIONA_OK &&
+                 tiled_kernel_attributes(best.C, narrow, best.P, has_const, false, &packed, false, best.w12, kc_all) ==
                      FIONA_OK &&
                  attr.localSizeBytes <= packed.localSizeBytes;
         }
@@ -2050,6 +2061,7 @@ int lower_tiled(fiona_plan *p)
     a.wait_ns = 2000000000ull;
     a.zero = 0;
     a.src_offsets = offsets ? 1 : 0;
+    a.kc_all = kc_all ? 1 : 0;
     if (const char *t = getenv("FIONA_TEST_TILED_TIMEOUT")) {  // test only: a copy wait that runs out
         if (atoi(t) > 0 && best.C == 1 && hp.n_in) {
             a.test_flags |= kTiledFlagExtraTx;
@@ -2070,7 +2082,7 @@ int lower_tiled(fiona_plan *p)
         return set_error(FIONA_ERR_INTERNAL, "tiled schedule check failed: %s", why);
     }
     if (device) {
-        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, use_tc, ts->smem, offsets, ts->w12);
+        int rc = tiled_configure_kernel(best.C, narrow, best.P, has_const, use_tc, ts->smem, offsets, ts->w12, kc_all);
         if (rc == FIONA_OK) rc = upload_blob(ts, sc.w);
         if (rc != FIONA_OK) {
             cudaFree(ts->sched.blob);

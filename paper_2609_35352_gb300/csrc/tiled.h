@@ -124,6 +124,8 @@ struct TiledArgs {
     uint32_t test_flags;     // kTiledFlag* (0 outside tests)
     uint32_t zero;           // always 0, read at run time (rns::mac26)
     uint32_t src_offsets;    // 1: programs in the offset form (source byte offsets), 0: packed indices
+    uint32_t kc_all;         // 1: every raw term's plaintext is constant (KA variant): operations after
+                             // a batch's first are read as constant, so none of them may be a non-constant RAW
 };
 
 // Warp-specialised variant (kernel_ws.cu), two coefficients per lane.  The

@@ -163,13 +163,18 @@ __device__ __forceinline__ uint64_t evict_first_policy()
 // OFF: the schedule's signed-sum programs are in the offset form (tiled.h;
 // TiledArgs::src_offsets), each source address one addition.  WB: the most
 // warps a CTA of this variant runs (fewer warps leave each thread more
-// registers: the variants with 12 warps and 8-deep plaintext queues)
-template <int C, bool NARROW, uint32_t P, bool KC, bool TC = false, bool OFF = false, uint32_t WB = kTiledMaxWarps>
+// registers: the variants with 12 warps and 8-deep plaintext queues).  KA
+// (with KC): every raw term of the plan has a constant plaintext, so every
+// operation after a batch's first is constant or padding (a SEG only opens
+// a batch): only the first operation of a batch tells its kind at run time
+template <int C, bool NARROW, uint32_t P, bool KC, bool TC = false, bool OFF = false, uint32_t WB = kTiledMaxWarps,
+          bool KA = false>
 __global__ void __launch_bounds__(WB * 32)
     tiled_kernel(const TiledArgs a, const __grid_constant__ CUtensorMap tm_in)
 {
     static_assert(!TC || (C == 1 && NARROW), "tensor-core sums: one coefficient per lane, narrow moduli");
     static_assert(!(TC && OFF), "tensor-core sums: packed programs");
+    static_assert(!KA || KC, "every raw plaintext constant: the constant-plaintext variant");
     using A = Arith<NARROW>;
     using Acc = typename A::Acc;
     static_assert(P % 4 == 0, "operation words are read four at a time");
@@ -267,8 +272,9 @@ __global__ void __launch_bounds__(WB * 32)
     // for a CONST operation in the limb at `lbase` (with stride 0 and the
     // schedule's own address for both when there is no next tile: a
     // harmless valid load)
-    auto fetch = [&](const char *base, const char *lbase, uint32_t stride, uint32_t w) -> V<C> {
-        const char *b = KC && (w & kOpConst) ? lbase : base;
+    // (`i`: the operation's position in its batch)
+    auto fetch = [&](const char *base, const char *lbase, uint32_t stride, uint32_t w, uint32_t i) -> V<C> {
+        const char *b = KC && ((KA && i > 0) || (w & kOpConst)) ? lbase : base;
         return ldg_stream<C>(reinterpret_cast<const uint64_t *>(b + (uint64_t)(w >> kOpPtShift) * stride), pol);
     };
     V<C> r[P];
@@ -280,7 +286,7 @@ __global__ void __launch_bounds__(WB * 32)
         const char *l0 = cur_ptl ? cur_lb : b0;
         const uint32_t s0 = cur_ptl ? stride_bytes : 0;
 #pragma unroll
-        for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, l0, s0, op_word(op0 + 4 * i));
+        for (uint32_t i = 0; i < P; ++i) r[i] = fetch(b0, l0, s0, op_word(op0 + 4 * i), i);
     }
 
     // start the copies of tile `t`'s inputs into region `reg`: thread 0's
@@ -566,11 +572,12 @@ __global__ void __launch_bounds__(WB * 32)
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
                     // a CONST plaintext is its limb's residue 0 at every coefficient
-                    const uint64_t g = A::operand((KC && x > 0 && (op & kOpConst)) ? r[i].x[0] : r[i].x[x]);
+                    const bool cst = KC && x > 0 && ((KA && i > 0) || (op & kOpConst));
+                    const uint64_t g = A::operand(cst ? r[i].x[0] : r[i].x[x]);
                     A::mac(acc[0][x], g, s0.x[x], zero);
                     A::mac(acc[1][x], g, s1.x[x], zero);
                 }
-                r[i] = fetch(nb, nlb, ns, nwi);
+                r[i] = fetch(nb, nlb, ns, nwi, i);
             }
             if (cw4.w & kOpLast) finish();  // the batch's last word
         }

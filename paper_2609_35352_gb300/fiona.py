@@ -67,8 +67,7 @@ class PlanStats(ctypes.Structure):
         [(n, ctypes.c_uint32) for n in (
             "N", "L", "n_in", "n_out", "n_pt", "n_groups", "tile_coeffs", "warps_per_cta",
             "smem_bytes", "ctas_per_sm", "kernel", "nodes_materialized", "addsub_executed",
-                  "tensor_core_sums", "source_offsets")] + \
-        [("reserved", ctypes.c_uint32)]
+                  "tensor_core_sums", "source_offsets", "const_raw_all")]
 
     def as_dict(self) -> Dict[str, int]:
         return {n: int(getattr(self, n)) for n, _ in self._fields_ if n != "reserved"}

@@ -75,6 +75,26 @@ def test_packed_programs_parity(name, N, L, monkeypatch):
     assert np.array_equal(dl.outputs(), want)
 
 
+@pytest.mark.parametrize("mixed", [False, True])
+@pytest.mark.parametrize("N,L", [(1024, 2), (4096, 1)])
+def test_all_constant_plaintexts_parity(N, L, mixed, monkeypatch):
+    """A layer whose every raw plaintext is constant (bert-const) on the
+    12-warp shape: the kernel variant that reads every operation after a
+    batch's first as constant, and (FIONA_TILED_KC_MIXED=1) the one that
+    tests each operation, give the same residues as the oracle."""
+    monkeypatch.setenv("FIONA_TILED_SHAPE", "2,12,1,-1,8")
+    if mixed:
+        monkeypatch.setenv("FIONA_TILED_KC_MIXED", "1")
+    wl = W.make_workload("bert-const", N=N, L=L)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel("tiled")
+    st = dl.plan.stats()
+    assert st["warps_per_cta"] == 12 and st["const_raw_all"] == (0 if mixed else 1)
+    dl.run()
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    assert np.array_equal(dl.outputs(), want)
+
+
 # Tiled shapes (coefficients per lane, warps, source regions[, most shared
 # sums kept (-1: the lowering's choice)[, operations per batch]]) chosen
 # through the lowering's override; every shape must give the same residues.
