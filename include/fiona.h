@@ -48,7 +48,10 @@
 extern "C" {
 #endif
 
-#define FIONA_ABI_VERSION 3
+/* 4: fiona_plan_stats_t's last two words report the signed-sum program form
+ * (source_offsets) and the all-constant-plaintext kernel variant
+ * (const_raw_all); the structure's size is unchanged (they were reserved). */
+#define FIONA_ABI_VERSION 4
 
 typedef struct fiona_ctx fiona_ctx;   /* N, RNS moduli, per-limb constants on one device */
 typedef struct fiona_plan fiona_plan; /* one validated, lowered linear layer */

@@ -36,7 +36,7 @@ def test_library_exports_every_declared_symbol(header, path):
         assert hasattr(lib, n), n
     if header == "fiona.h":
         assert set(F.EXPORTED) <= set(names)
-        assert F.lib().fiona_abi_version() == 3
+        assert F.lib().fiona_abi_version() == 4
 
 
 def ctx_none(N=1024, bits=40, L=3):
