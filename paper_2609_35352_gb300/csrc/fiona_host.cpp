@@ -127,6 +127,10 @@ static LimbConst limb_constants(uint64_t q)
     c.mu_hi = (uint64_t)(mu >> 64);
     c.mu_lo = (uint64_t)mu;
     c.mu64 = ~(uint64_t)0 / q;     // floor(2^64 / q) for odd q
+    uint32_t k = 0;
+    while (k < 64 && (q >> k)) ++k;  // bit length of q
+    c.km1 = k - 1;
+    c.mk = k + 63 < 128 ? (uint64_t)(((u128)1 << (k + 63)) / q) : 0;  // (used for q < 2^52: k + 63 < 116)
     return c;
 }
 

@@ -20,6 +20,15 @@
 //
 // reduce64: for x < 2^64, qe = hi(x * mu64) is floor(x/q) or one less, the
 // same argument with 2^64 in place of 2^128.
+//
+// reduce_k: for a k-bit q (2^(k-1) < q < 2^k) and x < 2^(k+63), with
+//   A  = floor(x / 2^(k-1))       (below 2^64)
+//   mk = floor(2^(k+63) / q)      (below 2^64, since q > 2^(k-1)),
+// qe = floor(A * mk / 2^64) satisfies x/q - 2 < qe <= x/q: writing
+// A = x/2^(k-1) - e1 and mk = 2^(k+63)/q - e2 with 0 <= e1, e2 < 1,
+//   x/q - A*mk/2^64 <= e1 * 2^(k-1)/q + e2 * x/2^(k+63) < 1 + 1,
+// so r = x - qe*q lies in [0, 3q): two conditional subtractions.  One
+// 64x64 high product replaces the five partial products of reduce128.
 #pragma once
 #include <stdint.h>
 
@@ -28,6 +37,8 @@ struct LimbConst {
     uint64_t mu_hi;
     uint64_t mu_lo;
     uint64_t mu64;
+    uint64_t mk;   // floor(2^(k+63) / q), k = bit length of q (reduce_k)
+    uint64_t km1;  // k - 1
 };
 
 #if defined(__CUDACC__)
@@ -154,7 +165,20 @@ __device__ __forceinline__ void mac26(uint64_t &lo, uint64_t &x, uint64_t &hi, u
     hi += p2;
 }
 
-// lo + (x - lo - hi) * 2^26 + hi * 2^52 mod q (below 2^116)
+// x1 * 2^64 + x0 mod q for a value below 2^(k+63) (see reduce_k above)
+__device__ __forceinline__ uint64_t reduce_k(uint64_t x0, uint64_t x1, const LimbConst &m)
+{
+    const uint32_t s = (uint32_t)m.km1;  // 1 <= k - 1 <= 51
+    const uint64_t A = (x0 >> s) | (x1 << (64 - s));
+    const uint64_t qe = __umul64hi(A, m.mk);
+    uint64_t r = x0 - qe * m.q;  // the true remainder is below 3q < 2^64
+    r = r >= m.q ? r - m.q : r;
+    return r >= m.q ? r - m.q : r;
+}
+
+// lo + (x - lo - hi) * 2^26 + hi * 2^52 mod q: the value of at most 1023
+// products of residues below q < 2^52 (kNarrowMacBudget), so below
+// 2^10 q^2 < 2^(2k+10) <= 2^(k+63), which reduce_k takes
 __device__ __forceinline__ uint64_t reduce26(uint64_t lo, uint64_t x, uint64_t hi, const LimbConst &m)
 {
     const uint64_t mid = x - lo - hi;
@@ -165,7 +189,7 @@ __device__ __forceinline__ uint64_t reduce26(uint64_t lo, uint64_t x, uint64_t h
         "addc.u64   %1, %1, %5;"
         : "+l"(x0), "+l"(x1)
         : "l"(mid << 26), "l"(mid >> 38), "l"(hi << 52), "l"(hi >> 12));
-    return reduce128(x0, x1, m);
+    return reduce_k(x0, x1, m);
 }
 
 }  // namespace rns

@@ -16,6 +16,8 @@ __device__ __forceinline__ LimbConst load_limb(uint32_t addr)
     LimbConst m;
     asm volatile("ld.shared.v2.u64 {%0, %1}, [%2];" : "=l"(m.q), "=l"(m.mu_hi) : "r"(addr));
     asm volatile("ld.shared.v2.u64 {%0, %1}, [%2+16];" : "=l"(m.mu_lo), "=l"(m.mu64) : "r"(addr));
+    // (not volatile: dropped where only the first four are used)
+    asm("ld.shared.v2.u64 {%0, %1}, [%2+32];" : "=l"(m.mk), "=l"(m.km1) : "r"(addr));
     return m;
 }
 
