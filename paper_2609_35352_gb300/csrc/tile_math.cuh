@@ -102,6 +102,13 @@ struct Arith<false> {
     {
         return rns::sub_mod(rns::reduce64(p, m), rns::reduce64(mm, m), m.q);
     }
+    // the same for narrow moduli (q < 2^52): P and M are sums of at most 64
+    // run terms and six slot terms, each below q, so P + 128q - M is positive
+    // and below 2^60: one reduction
+    __device__ static uint64_t signed_value_narrow(uint64_t p, uint64_t mm, const LimbConst &m)
+    {
+        return rns::reduce64(p + 128 * m.q - mm, m);
+    }
 };
 
 // q < 2^52: every factor in split form (sources split in shared memory or
@@ -280,7 +287,8 @@ __device__ __forceinline__ uint32_t run_sum_offsets(const char *sm, uint32_t src
 // A slot is a tile pair of this warp's slot area at byte offset `slots`
 // (this lane's words of slot 0), holding a shared signed sum the warp formed
 // earlier.  Returns the offset just past the program.
-template <bool SPLIT, int C, uint32_t TB>
+// NC: canonical sources with narrow moduli (Arith<false>::signed_value_narrow).
+template <bool SPLIT, int C, uint32_t TB, bool NC = false>
 __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uint32_t hdr, uint32_t lim,
                                                uint32_t slots, V<C> &o0, V<C> &o1, bool offsets = false)
 {
@@ -314,8 +322,13 @@ __device__ __forceinline__ uint32_t signed_sum(const char *sm, uint32_t src, uin
     const LimbConst m = load_limb(lim);
 #pragma unroll
     for (int x = 0; x < C; ++x) {
-        o0.x[x] = A::signed_value(p0.x[x], m0.x[x], m);
-        o1.x[x] = A::signed_value(p1.x[x], m1.x[x], m);
+        if constexpr (NC && !SPLIT) {
+            o0.x[x] = Arith<false>::signed_value_narrow(p0.x[x], m0.x[x], m);
+            o1.x[x] = Arith<false>::signed_value_narrow(p1.x[x], m1.x[x], m);
+        } else {
+            o0.x[x] = A::signed_value(p0.x[x], m0.x[x], m);
+            o1.x[x] = A::signed_value(p1.x[x], m1.x[x], m);
+        }
     }
     return next;
 }

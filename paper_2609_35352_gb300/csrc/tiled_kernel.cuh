@@ -446,7 +446,7 @@ __global__ void __launch_bounds__(WB * 32)
         for (uint32_t lev = 0; lev < a.n_levels; ++lev) {
             for (uint32_t x = sw[a.o_level + lev] + warp; x < sw[a.o_level + lev + 1]; x += n_warps) {
                 V<C> u0, u1;
-                signed_sum<SPLIT, C, TB>(sm, src, sw[a.o_node_off + x] * 4, lim, 0, u0, u1, offsets);
+                signed_sum<SPLIT, C, TB, NARROW && !SPLIT>(sm, src, sw[a.o_node_off + x] * 4, lim, 0, u0, u1, offsets);
                 if constexpr (SPLIT) {  // stored in the sources' form
 #pragma unroll
                     for (int x2 = 0; x2 < C; ++x2) {
@@ -522,7 +522,7 @@ __global__ void __launch_bounds__(WB * 32)
                     // third word in the offset form
                     const uint32_t dst = slots + sw[(sp >> 2) + (offsets ? 2 : 0)] * PB;
                     V<C> u0, u1;
-                    sp = signed_sum<SPLIT, C, TB>(sm, src, offsets ? sp : sp + 4, lim, slots, u0, u1, offsets);
+                    sp = signed_sum<SPLIT, C, TB, NARROW && !SPLIT>(sm, src, offsets ? sp : sp + 4, lim, slots, u0, u1, offsets);
                     if constexpr (SPLIT) {  // stored in the sources' form
 #pragma unroll
                         for (int x = 0; x < C; ++x) {
@@ -533,7 +533,7 @@ __global__ void __launch_bounds__(WB * 32)
                     sts<C>(sm, dst, u0);
                     sts<C>(sm, dst + TB, u1);
                 }
-                sp = signed_sum<SPLIT, C, TB>(sm, src, sp, lim, slots, g0, g1, offsets);
+                sp = signed_sum<SPLIT, C, TB, NARROW && !SPLIT>(sm, src, sp, lim, slots, g0, g1, offsets);
 #pragma unroll
                 for (int x = 0; x < C; ++x) {
                     g0.x[x] = A::operand(g0.x[x]);
