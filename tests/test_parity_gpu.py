@@ -264,6 +264,32 @@ def test_boundary_residues():
         assert np.array_equal(dl.outputs(), want), kernel
 
 
+@pytest.mark.parametrize("kernel,shape", [("direct", None), ("tiled", None), ("tiled", "2,16,0"),
+                                          ("tiled", "1,16,1"), ("tiled", "2,12,1,-1,8")])
+@pytest.mark.parametrize("bits", [51, 52])
+def test_widest_narrow_moduli(bits, kernel, shape, monkeypatch):
+    """The radix-2^26 arithmetic at the widest moduli it takes (every q below
+    2^52, high digits up to 2^26 - 1): every residue q - 1, and more products
+    and signed terms per output than the lazy bounds allow between
+    reductions, so that every accumulator comes near its bound; one and two
+    coefficients per lane, the 12-warp variant, and the direct kernel."""
+    if shape:
+        monkeypatch.setenv("FIONA_TILED_SHAPE", shape)
+    wl = W.make_workload("overflow50", bits=bits)
+    assert all(int(q).bit_length() == bits for q in wl.moduli)
+    dl = DeviceLayer(wl)
+    dl.plan.select_kernel(kernel)
+    st = dl.plan.stats()
+    if shape:
+        f = [int(v) for v in shape.split(",")]
+        assert (st["tile_coeffs"], st["warps_per_cta"]) == (32 * f[0], f[1])
+    dl.run()
+    want = oracle.linear_eval(wl.plan, wl.moduli, dl.X, dl.P)
+    mism = np.argwhere(dl.outputs() != want)
+    assert mism.shape[0] == 0, "first mismatches (j, c, l, k): %s" % mism[:5].tolist()
+    assert dl.ctx.device_check() == F.FIONA_OK
+
+
 FULL = ["wsum-pmult", "wsum-ternary", "wsum-hybrid", "vgg", "vit", "bert", "bert-const"]
 
 
