@@ -37,7 +37,10 @@
  * negative = failure) and leaves its out-arguments untouched on failure.
  * fiona_last_error() returns a one-line description of the most recent
  * failure in the calling thread.  No entry point synchronises the device,
- * except where stated.
+ * except where stated.  A call that works on a context's device makes it the
+ * current device for the call's duration and restores the caller's device
+ * on return; if it cannot select it, the call returns FIONA_ERR_CUDA having
+ * enqueued nothing.
  */
 #ifndef FIONA_H
 #define FIONA_H

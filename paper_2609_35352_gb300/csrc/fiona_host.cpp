@@ -615,6 +615,7 @@ extern "C" int fiona_device_check(const fiona_ctx *ctx, void *stream)
     if (ctx->device == FIONA_DEVICE_NONE)
         return set_error(FIONA_ERR_NODEVICE, "device_check: validation-only context");
     DeviceGuard g(ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "device_check: cannot select device %d", ctx->device);
     cudaStream_t s = (cudaStream_t)stream;
     int flag = 0;
     cudaError_t e = cudaStreamSynchronize(s);
@@ -829,6 +830,7 @@ extern "C" int fiona_linear_eval(const fiona_plan *p, void *stream, const uint64
     if (rc) return rc;
     if (p->hp.n_out == 0) return FIONA_OK;
     DeviceGuard g(p->ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "linear_eval: cannot select device %d", p->ctx->device);
     return launch_range(p, stream, in, pt, out, 0, p->ctx->L, p->ctx->L);
 }
 
@@ -842,6 +844,7 @@ extern "C" int fiona_linear_eval_level(const fiona_plan *p, void *stream, uint32
     if (rc) return rc;
     if (p->hp.n_out == 0) return FIONA_OK;
     DeviceGuard g(p->ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "linear_eval_level: cannot select device %d", p->ctx->device);
     return launch_range(p, stream, in, pt, out, 0, L_eval, L_eval);
 }
 
@@ -905,6 +908,7 @@ extern "C" int fiona_linear_eval_host(const fiona_plan *p, void *stream, const u
     if (const int rc = check_host_args(p, h_in, d_pt, h_out, d_in, d_out)) return rc;
     if (p->hp.n_out == 0) return FIONA_OK;
     DeviceGuard g(p->ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "linear_eval_host: cannot select device %d", p->ctx->device);
     cudaStream_t s = (cudaStream_t)stream;
     const int rc = eval_host_enqueue(p, s, h_in, d_pt, h_out, d_in, d_out, true);
     // whatever was queued completes before the call returns
@@ -925,6 +929,7 @@ extern "C" int fiona_linear_eval_host_async(const fiona_plan *p, void *stream, c
     if (const int rc = check_host_args(p, h_in, d_pt, h_out, d_in, d_out)) return rc;
     if (p->hp.n_out == 0) return FIONA_OK;
     DeviceGuard g(p->ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "linear_eval_host_async: cannot select device %d", p->ctx->device);
     return eval_host_enqueue(p, (cudaStream_t)stream, h_in, d_pt, h_out, d_in, d_out, false);
 }
 
@@ -935,6 +940,7 @@ extern "C" int fiona_linear_eval_host_join(const fiona_plan *p, void *stream)
         return set_error(FIONA_ERR_NODEVICE, "linear_eval_host_join: validation-only context");
     if (p->hp.n_out == 0) return FIONA_OK;
     DeviceGuard g(p->ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "linear_eval_host_join: cannot select device %d", p->ctx->device);
     const uint32_t chunks = std::min<uint32_t>(p->ctx->L, fiona_plan::kHostChunks);
     // the output copies run in order on one stream: the last chunk's is the last
     const cudaError_t e = cudaStreamWaitEvent((cudaStream_t)stream, (cudaEvent_t)p->ev_out[chunks - 1], 0);
@@ -996,6 +1002,7 @@ extern "C" int fiona_rescale(const fiona_ctx *ctx, void *stream, uint32_t L_cur,
     int rc = check_rescale_args(ctx, L_cur, count, polys, out, "rescale");
     if (rc) return rc;
     DeviceGuard g(ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "rescale: cannot select device %d", ctx->device);
     return launch_rescale(ctx, stream, L_cur, count, polys, out, flags & FIONA_RESCALE_ROUND);
 }
 
@@ -1014,6 +1021,7 @@ extern "C" int fiona_linear_eval_rescale(const fiona_plan *p, void *stream, uint
         return set_error(FIONA_ERR_ARG, "linear_eval_rescale: output overlaps the inputs");
     if (p->hp.n_out == 0) return FIONA_OK;
     DeviceGuard g(p->ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "linear_eval_rescale: cannot select device %d", p->ctx->device);
     rc = launch_range(p, stream, in, pt, work, 0, L_eval, L_eval);
     if (rc) return rc;
     return launch_rescale(p->ctx, stream, L_eval, count, work, out, flags & FIONA_RESCALE_ROUND);
@@ -1067,6 +1075,7 @@ extern "C" int fiona_ckks_embed(const fiona_ctx *ctx, void *stream, uint64_t cou
     int rc = check_embed_args(ctx, count, slots, scale, coeffs, work, "ckks_embed");
     if (rc || count == 0) return rc;
     DeviceGuard g(ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "ckks_embed: cannot select device %d", ctx->device);
     return launch_embed(ctx, stream, count, slots, scale, coeffs, work);
 }
 
@@ -1076,6 +1085,7 @@ extern "C" int fiona_encode_coeffs(const fiona_ctx *ctx, void *stream, uint32_t 
     int rc = check_encode_coeff_args(ctx, L_cur, count, coeffs, out, "encode_coeffs");
     if (rc || count == 0) return rc;
     DeviceGuard g(ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "encode_coeffs: cannot select device %d", ctx->device);
     return launch_encode_coeffs(ctx, stream, L_cur, count, coeffs, out);
 }
 
@@ -1092,6 +1102,7 @@ extern "C" int fiona_encode(const fiona_ctx *ctx, void *stream, uint32_t L_cur, 
     }
     if (rc || count == 0) return rc;
     DeviceGuard g(ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "encode: cannot select device %d", ctx->device);
     rc = launch_embed(ctx, stream, count, slots, scale, coeffs, work);
     if (rc) return rc;
     return launch_encode_coeffs(ctx, stream, L_cur, count, coeffs, out);
@@ -1107,5 +1118,6 @@ extern "C" int fiona_check_residues(const fiona_ctx *ctx, void *stream, const ui
     if (!data || ((uintptr_t)data & 15))
         return set_error(FIONA_ERR_ARG, "check_residues: null or misaligned data");
     DeviceGuard g(ctx->device);
+    if (!g.ok) return set_error(FIONA_ERR_CUDA, "check_residues: cannot select device %d", ctx->device);
     return launch_check_residues(ctx, stream, data, count);
 }
